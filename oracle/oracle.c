@@ -1,0 +1,255 @@
+/*
+ * fp64 CPU oracle for the VMamba SS2D selective scan and its channel-mean
+ * variant VMeanba (arXiv 2412.16602).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the test suite, the smoke check and the
+ * CPU-baseline leg of the benchmark may load this code.  It shares no code,
+ * header, table or helper with the CUDA library; it is written as plain,
+ * sequential loops in double precision, straight from the paper:
+ *
+ *   cross-scan / cross-merge ....... App. A, "VMamba" paragraph (SS2D = cross-scan,
+ *                                     selective scan per direction, cross-merge)
+ *   discretisation ................. App. A, Eq. 4 (Abar = exp(Delta A); Bbar)
+ *   selection (softplus of Delta) .. App. A, Eq. 6 (Delta = softplus(Parameter + s_Delta(u)))
+ *   recurrence ..................... App. A, Eq. 3 (h_t = Abar h_{t-1} + Bbar u_t, y_t = C h_t + D u_t)
+ *   channel mean (VMeanba) ......... Sec. 2.2, Eq. 9 (y = T^-1(Mamba(T(Abar, Bbar u, C))),
+ *                                     T = mean over the inner channel axis, T^-1 = broadcast)
+ *
+ * Readings of points the paper leaves open (each is listed in the design notes):
+ *   - scan directions: 0 row-major, 1 column-major, 2 = reverse of 0, 3 = reverse of 1;
+ *     merge sums ((dir0 + dir2) + (dir1 + dir3)).
+ *   - Bbar: Euler form Delta*B by default (b_mode 0); b_mode 1 is the exact
+ *     zero-order hold (exp(Delta A) - 1) / A * B, reading Eq. 4's "exp(Delta A - I)"
+ *     as the intended exp(Delta A) - I.
+ *   - initial state h_{-1} = 0.
+ *   - softplus(x) = log(1 + e^x), evaluated as max(x,0) + log1p(e^{-|x|}) (exact, no cut-off).
+ *   - channel mean: Abar is averaged after the exponential, the mean runs per
+ *     (batch, direction) over the D channels; C has no channel axis; the skip
+ *     term is per channel (skip_mode 0) or the channel mean of D*u (skip_mode 1).
+ *
+ * Layouts (row-major): x, out [B][D][H][W]; u, delta, y [B][K][D][L]; Bs, Cs
+ * [B][K][N][L]; A [K*D][N]; Dskip, bias [K*D]; ybar [B][K][L]; L = H*W; the
+ * per-channel parameter index is c = k*D + d.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORACLE_B_EULER 0
+#define ORACLE_B_ZOH 1
+#define ORACLE_SKIP_PER_CHANNEL 0
+#define ORACLE_SKIP_MEAN 1
+
+/* Eq. 6: tau_Delta = softplus. */
+static double softplus(double x) { return fmax(x, 0.0) + log1p(exp(-fabs(x))); }
+
+/* Eq. 4, discretised input weight Bbar for one state (scalar A, B). */
+static double discretise_b(double delta, double a, double b, int b_mode) {
+    if (b_mode == ORACLE_B_ZOH && a != 0.0)
+        return expm1(delta * a) / a * b;  /* (Delta A)^-1 (exp(Delta A) - 1) Delta B */
+    return delta * b;                     /* Euler: Delta B */
+}
+
+/* ---------------------------------------------------------------- cross-scan */
+
+/* Position of map pixel (h, w) in the sequence of direction k. */
+static long seq_pos(int k, long h, long w, long H, long W) {
+    long L = H * W;
+    switch (k) {
+    case 0: return h * W + w;                /* row-major */
+    case 1: return w * H + h;                /* column-major */
+    case 2: return L - 1 - (h * W + w);      /* row-major, reversed */
+    default: return L - 1 - (w * H + h);     /* column-major, reversed */
+    }
+}
+
+void oracle_cross_scan(const double* x, double* xs, long B, long D, long H, long W) {
+    long L = H * W;
+    for (long b = 0; b < B; ++b)
+        for (long d = 0; d < D; ++d) {
+            const double* plane = x + (b * D + d) * L;
+            for (int k = 0; k < 4; ++k) {
+                double* seq = xs + ((b * 4 + k) * D + d) * L;
+                for (long h = 0; h < H; ++h)
+                    for (long w = 0; w < W; ++w)
+                        seq[seq_pos(k, h, w, H, W)] = plane[h * W + w];
+            }
+        }
+}
+
+void oracle_cross_merge(const double* ys, double* out, long B, long D, long H, long W) {
+    long L = H * W;
+    for (long b = 0; b < B; ++b)
+        for (long d = 0; d < D; ++d) {
+            const double* s0 = ys + ((b * 4 + 0) * D + d) * L;
+            const double* s1 = ys + ((b * 4 + 1) * D + d) * L;
+            const double* s2 = ys + ((b * 4 + 2) * D + d) * L;
+            const double* s3 = ys + ((b * 4 + 3) * D + d) * L;
+            double* plane = out + (b * D + d) * L;
+            for (long h = 0; h < H; ++h)
+                for (long w = 0; w < W; ++w)
+                    plane[h * W + w] = (s0[seq_pos(0, h, w, H, W)] + s2[seq_pos(2, h, w, H, W)]) +
+                                       (s1[seq_pos(1, h, w, H, W)] + s3[seq_pos(3, h, w, H, W)]);
+        }
+}
+
+/* ------------------------------------------------------------ problem struct */
+
+typedef struct {
+    const double *u, *delta, *A, *Bs, *Cs, *Dskip, *bias;
+    double *y, *ybar;
+    long B, K, D, N, L;
+    int softplus_on, b_mode, skip_mode;
+} problem;
+
+/* ------------------------------------------------------- full selective scan */
+
+/* One channel row (b, k, d): Eq. 6 softplus, Eq. 4 discretisation, Eq. 3 recurrence. */
+static void full_row(const problem* p, long b, long k, long d, double* h) {
+    long L = p->L, N = p->N, c = k * p->D + d;
+    const double* u = p->u + ((b * p->K + k) * p->D + d) * L;
+    const double* dl = p->delta + ((b * p->K + k) * p->D + d) * L;
+    const double* Bk = p->Bs + (b * p->K + k) * N * L;
+    const double* Ck = p->Cs + (b * p->K + k) * N * L;
+    const double* A = p->A + c * N;
+    double* y = p->y + ((b * p->K + k) * p->D + d) * L;
+    for (long n = 0; n < N; ++n) h[n] = 0.0;
+    for (long t = 0; t < L; ++t) {
+        double v = dl[t] + p->bias[c];
+        double delta = p->softplus_on ? softplus(v) : v;
+        double acc = 0.0;
+        for (long n = 0; n < N; ++n) {
+            double abar = exp(delta * A[n]);
+            double bbar = discretise_b(delta, A[n], Bk[n * L + t], p->b_mode);
+            h[n] = abar * h[n] + bbar * u[t];
+            acc += Ck[n * L + t] * h[n];
+        }
+        y[t] = acc + p->Dskip[c] * u[t];
+    }
+}
+
+/* --------------------------------------------------- channel-mean (VMeanba) */
+
+/* One sequence (b, k): T = channel mean of (Abar, Bbar u, C), one-channel
+ * Mamba recurrence on the means, T^-1 = broadcast to every channel. */
+static void mean_seq(const problem* p, long b, long k, double* h, double* abar, double* bubar) {
+    long L = p->L, N = p->N, D = p->D;
+    const double* u = p->u + (b * p->K + k) * D * L;
+    const double* dl = p->delta + (b * p->K + k) * D * L;
+    const double* Bk = p->Bs + (b * p->K + k) * N * L;
+    const double* Ck = p->Cs + (b * p->K + k) * N * L;
+    double* y = p->y + (b * p->K + k) * D * L;
+    for (long n = 0; n < N; ++n) h[n] = 0.0;
+    for (long t = 0; t < L; ++t) {
+        /* T: mean over the channel axis of the discretised inputs */
+        for (long n = 0; n < N; ++n) { abar[n] = 0.0; bubar[n] = 0.0; }
+        double du_sum = 0.0;
+        for (long d = 0; d < D; ++d) {
+            long c = k * D + d;
+            double v = dl[d * L + t] + p->bias[c];
+            double delta = p->softplus_on ? softplus(v) : v;
+            for (long n = 0; n < N; ++n) {
+                abar[n] += exp(delta * p->A[c * N + n]);
+                bubar[n] += discretise_b(delta, p->A[c * N + n], Bk[n * L + t], p->b_mode) * u[d * L + t];
+            }
+            du_sum += p->Dskip[c] * u[d * L + t];
+        }
+        for (long n = 0; n < N; ++n) { abar[n] /= (double)D; bubar[n] /= (double)D; }
+        /* Mamba on the reduced (one-channel) inputs; C has no channel axis */
+        double ybar = 0.0;
+        for (long n = 0; n < N; ++n) {
+            h[n] = abar[n] * h[n] + bubar[n];
+            ybar += Ck[n * L + t] * h[n];
+        }
+        if (p->ybar) p->ybar[(b * p->K + k) * L + t] = ybar;
+        /* T^-1: broadcast to every channel, then the skip term */
+        for (long d = 0; d < D; ++d) {
+            long c = k * D + d;
+            double skip = p->skip_mode == ORACLE_SKIP_MEAN ? du_sum / (double)D : p->Dskip[c] * u[d * L + t];
+            y[d * L + t] = ybar + skip;
+        }
+    }
+}
+
+/* --------------------------------------------------------------- threading */
+
+typedef struct {
+    const problem* p;
+    int mean;
+    long first, last; /* work items [first, last) */
+} job;
+
+static void* run_job(void* arg) {
+    const job* j = (const job*)arg;
+    const problem* p = j->p;
+    long N = p->N;
+    double* scratch = (double*)malloc(sizeof(double) * 3 * (size_t)(N > 0 ? N : 1));
+    if (!scratch) return (void*)1;
+    for (long i = j->first; i < j->last; ++i) {
+        if (j->mean) {
+            long b = i / p->K, k = i % p->K;
+            mean_seq(p, b, k, scratch, scratch + N, scratch + 2 * N);
+        } else {
+            long d = i % p->D, bk = i / p->D;
+            full_row(p, bk / p->K, bk % p->K, d, scratch);
+        }
+    }
+    free(scratch);
+    return NULL;
+}
+
+/* Split the independent work items over nthreads threads (rows for the full
+ * path, (batch, direction) sequences for the mean path).  Returns 0 on success. */
+static int run(const problem* p, int mean, int nthreads) {
+    long items = mean ? p->B * p->K : p->B * p->K * p->D;
+    if (items <= 0) return 0;
+    if (nthreads < 1) nthreads = 1;
+    if (nthreads > items) nthreads = (int)items;
+    pthread_t* th = (pthread_t*)malloc(sizeof(pthread_t) * (size_t)nthreads);
+    job* jobs = (job*)malloc(sizeof(job) * (size_t)nthreads);
+    if (!th || !jobs) { free(th); free(jobs); return 1; }
+    int rc = 0;
+    for (int i = 0; i < nthreads; ++i) {
+        jobs[i].p = p;
+        jobs[i].mean = mean;
+        jobs[i].first = items * i / nthreads;
+        jobs[i].last = items * (i + 1) / nthreads;
+    }
+    int started = 0;
+    for (int i = 1; i < nthreads; ++i, ++started)
+        if (pthread_create(&th[i], NULL, run_job, &jobs[i]) != 0) { rc = 1; break; }
+    if (run_job(&jobs[0]) != NULL) rc = 1;
+    for (int i = 1; i <= started; ++i) {
+        void* r = NULL;
+        pthread_join(th[i], &r);
+        if (r != NULL) rc = 1;
+    }
+    free(th);
+    free(jobs);
+    return rc;
+}
+
+int oracle_selective_scan(const double* u, const double* delta, const double* A, const double* Bs,
+                          const double* Cs, const double* Dskip, const double* bias, double* y,
+                          long B, long K, long D, long N, long L, int softplus_on, int b_mode,
+                          int nthreads) {
+    problem p = {u, delta, A, Bs, Cs, Dskip, bias, y, NULL, B, K, D, N, L, softplus_on, b_mode,
+                 ORACLE_SKIP_PER_CHANNEL};
+    return run(&p, 0, nthreads);
+}
+
+int oracle_mean_scan(const double* u, const double* delta, const double* A, const double* Bs,
+                     const double* Cs, const double* Dskip, const double* bias, double* y,
+                     double* ybar, long B, long K, long D, long N, long L, int softplus_on,
+                     int b_mode, int skip_mode, int nthreads) {
+    problem p = {u, delta, A, Bs, Cs, Dskip, bias, y, ybar, B, K, D, N, L, softplus_on, b_mode,
+                 skip_mode};
+    return run(&p, 1, nthreads);
+}
+
+/* Eq. 6 softplus, exposed so that tests can pin it against known values. */
+void oracle_softplus(const double* x, double* out, long n) {
+    for (long i = 0; i < n; ++i) out[i] = softplus(x[i]);
+}

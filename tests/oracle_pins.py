@@ -1,0 +1,375 @@
+"""Pins of the fp64 oracle against facts the paper and the mathematics fix.
+
+Each ``pin_*`` takes an ``oracle.Oracle`` and raises AssertionError when the
+oracle disagrees with a closed form, a hand-worked case, an invariant or a
+brute-force unrolling.  None of them re-types the oracle's own loops: the
+expected values come from a different formulation (closed forms, explicit
+O(L^2) products, algebraic identities, permutation facts).
+
+``test_oracle_pins.py`` runs them on the real oracle; ``test_oracle_mutants.py``
+runs them on copies of oracle.c with planted mistakes and requires that every
+mistake trips at least one pin.
+"""
+from __future__ import annotations
+
+import math
+import os
+
+import numpy as np
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+LN2 = 0.6931471805599453
+
+
+def _close(a, b, rtol=1e-12, atol=1e-14, what=""):
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    if a.shape != b.shape:
+        raise AssertionError(f"{what}: shape {a.shape} != {b.shape}")
+    if not np.allclose(a, b, rtol=rtol, atol=atol):
+        err = np.max(np.abs(a - b))
+        raise AssertionError(f"{what}: max abs diff {err:.3e}")
+
+
+def _rand_problem(rng, B=1, K=2, D=3, N=4, L=7, draw_scale=0.5):
+    u = rng.standard_normal((B, K, D, L))
+    draw = draw_scale * rng.standard_normal((B, K, D, L))
+    A = -rng.uniform(0.5, 3.0, size=(K * D, N))
+    Bs = rng.standard_normal((B, K, N, L))
+    Cs = rng.standard_normal((B, K, N, L))
+    Dskip = rng.uniform(0.5, 1.5, size=K * D)
+    bias = rng.uniform(-3.0, 0.5, size=K * D)
+    return u, draw, A, Bs, Cs, Dskip, bias
+
+
+def _np_softplus(x):
+    # independent evaluation for building test expectations (log(1 + e^x))
+    return np.logaddexp(0.0, x)
+
+
+# ------------------------------------------------------------------ softplus
+
+
+def pin_softplus_special_values(orc):
+    """Eq. 6 tau = softplus: softplus(0) = ln 2; softplus(x) - softplus(-x) = x;
+    softplus(x) -> x for large x and -> e^x for very negative x."""
+    _close(orc.softplus([0.0]), [LN2], what="softplus(0)")
+    x = np.linspace(-30, 30, 121)
+    _close(orc.softplus(x) - orc.softplus(-x), x, rtol=1e-12, atol=1e-12, what="odd part")
+    _close(orc.softplus([800.0]), [800.0], what="large x")
+    _close(orc.softplus([-50.0]), [math.exp(-50.0)], rtol=1e-12, atol=0.0, what="small x")
+    if not np.all(np.diff(orc.softplus(x)) > 0):
+        raise AssertionError("softplus not increasing")
+
+
+# ------------------------------------------------------- cross-scan / merge
+
+
+def load_cross_scan_2x3():
+    path = os.path.join(GOLDEN, "cross_scan_2x3.txt")
+    rows = [ln.split() for ln in open(path) if ln.strip() and not ln.startswith("#")]
+    x = np.array([float(v) for v in rows[0]]).reshape(2, 3)
+    seqs = np.array([[float(v) for v in r] for r in rows[1:5]])
+    return x, seqs
+
+
+def pin_cross_scan_hand_worked(orc):
+    """App. A, VMamba: the 2x3 map unfolded along the four directions (worked by hand)."""
+    x, seqs = load_cross_scan_2x3()
+    xs = orc.cross_scan(x[None, None])
+    _close(xs[0, :, 0, :], seqs, rtol=0, atol=0, what="2x3 cross-scan")
+
+
+def pin_cross_scan_permutation_facts(orc):
+    """Direction 0 is the map read row by row, direction 1 the transposed map read
+    row by row, directions 2 and 3 are 0 and 1 reversed; every direction is a
+    permutation of the map."""
+    rng = np.random.default_rng(11)
+    for (H, W) in [(3, 5), (4, 4), (1, 6), (6, 1), (7, 7)]:
+        x = rng.standard_normal((2, 3, H, W))
+        xs = orc.cross_scan(x)
+        _close(xs[:, 0], x.reshape(2, 3, H * W), rtol=0, atol=0, what="dir0")
+        _close(xs[:, 1], np.swapaxes(x, -1, -2).reshape(2, 3, H * W), rtol=0, atol=0, what="dir1")
+        _close(xs[:, 2], xs[:, 0, :, ::-1], rtol=0, atol=0, what="dir2")
+        _close(xs[:, 3], xs[:, 1, :, ::-1], rtol=0, atol=0, what="dir3")
+        for k in range(4):
+            _close(np.sort(xs[:, k], axis=-1), np.sort(x.reshape(2, 3, -1), axis=-1),
+                   rtol=0, atol=0, what="permutation")
+
+
+def pin_merge_inverts_scan(orc):
+    """Each direction visits every pixel once, so merging the unfolded map gives 4x exactly."""
+    rng = np.random.default_rng(12)
+    for (H, W) in [(2, 3), (5, 4), (7, 7), (1, 9)]:
+        x = rng.standard_normal((2, 3, H, W))
+        _close(orc.cross_merge(orc.cross_scan(x), H, W), 4.0 * x, rtol=0, atol=0, what="merge(scan)")
+
+
+def pin_merge_one_hot(orc):
+    """A single 1 at sequence position l of direction k lands on the pixel that
+    direction visits at step l; merge of independent per-direction sequences."""
+    H, W = 3, 4
+    L = H * W
+    for k in range(4):
+        for l in range(L):
+            ys = np.zeros((1, 4, 1, L))
+            ys[0, k, 0, l] = 1.0
+            out = orc.cross_merge(ys, H, W)[0, 0]
+            ll = l if k < 2 else L - 1 - l
+            h, w = (ll // W, ll % W) if k % 2 == 0 else (ll % H, ll // H)
+            exp = np.zeros((H, W))
+            exp[h, w] = 1.0
+            _close(out, exp, rtol=0, atol=0, what=f"one-hot k={k} l={l}")
+
+
+# ------------------------------------------------------------ full scan
+
+
+def pin_scan_L1_closed_form(orc):
+    """At L = 1 with h_{-1} = 0: y_0 = u (delta sum_n C_n B_n + D), independent of A (Euler);
+    with zero-order hold y_0 = u (sum_n C_n B_n (e^{delta A_n} - 1)/A_n + D)."""
+    rng = np.random.default_rng(13)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, L=1)
+    B, K, D, L = u.shape
+    c = np.arange(K * D).reshape(K, D)
+    delta = _np_softplus(draw[..., 0] + bias[c][None])           # [B, K, D]
+    cb = np.einsum("bknl,bknl->bk", Cs, Bs)                       # sum_n C_n B_n
+    exp = u[..., 0] * (delta * cb[:, :, None] + Dskip[c][None])
+    _close(orc.selective_scan(u, draw, A, Bs, Cs, Dskip, bias)[..., 0], exp, what="L=1 euler")
+    Ar = A.reshape(K, D, -1)[None]                                # [1, K, D, N]
+    z = np.expm1(delta[..., None] * Ar) / Ar                      # (e^{delta A} - 1) / A
+    zoh = np.einsum("bkn,bkdn->bkd", Cs[..., 0] * Bs[..., 0], z)
+    exp_z = u[..., 0] * (zoh + Dskip[c][None])
+    _close(orc.selective_scan(u, draw, A, Bs, Cs, Dskip, bias, b_mode=1)[..., 0], exp_z,
+           what="L=1 zoh")
+
+
+def pin_scan_L2_hand_expansion(orc):
+    """y_1 = sum_n C_{1,n} (e^{delta_1 A_n} delta_0 B_{0,n} u_0 + delta_1 B_{1,n} u_1) + D u_1."""
+    rng = np.random.default_rng(14)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, B=1, K=1, D=1, N=3, L=2)
+    d0 = _np_softplus(draw[0, 0, 0, 0] + bias[0])
+    d1 = _np_softplus(draw[0, 0, 0, 1] + bias[0])
+    u0, u1 = u[0, 0, 0]
+    y1 = 0.0
+    for n in range(3):
+        y1 += Cs[0, 0, n, 1] * (math.exp(d1 * A[0, n]) * d0 * Bs[0, 0, n, 0] * u0
+                               + d1 * Bs[0, 0, n, 1] * u1)
+    y1 += Dskip[0] * u1
+    y = orc.selective_scan(u, draw, A, Bs, Cs, Dskip, bias)
+    _close(y[0, 0, 0, 1], y1, what="L=2")
+
+
+def pin_scan_geometric_sum(orc):
+    """N = 1, constant delta, B = C = u = 1: y_t = delta (1 - a^{t+1}) / (1 - a) + D, a = e^{delta A}."""
+    L = 40
+    for Aval, raw in [(-1.0, -2.0), (-0.3, 0.7), (-5.0, -6.0)]:
+        u = np.ones((1, 1, 1, L))
+        draw = np.full((1, 1, 1, L), raw)
+        A = np.array([[Aval]])
+        Bs = np.ones((1, 1, 1, L))
+        Cs = np.ones((1, 1, 1, L))
+        Dskip = np.array([0.25])
+        bias = np.array([0.1])
+        delta = _np_softplus(raw + 0.1)
+        a = math.exp(delta * Aval)
+        t = np.arange(L)
+        exp = delta * (1.0 - a ** (t + 1)) / (1.0 - a) + 0.25
+        _close(orc.selective_scan(u, draw, A, Bs, Cs, Dskip, bias)[0, 0, 0], exp, rtol=1e-11,
+               what="geometric sum")
+
+
+def brute_force_full(u, draw, A, Bs, Cs, Dskip, bias, b_mode=0):
+    """Explicit unrolled sum y_t = sum_n C_{t,n} sum_{s<=t} (prod_{r=s+1..t} Abar_{r,n}) Bbar_{s,n} u_s + D u_t."""
+    B, K, D, L = u.shape
+    N = Bs.shape[2]
+    y = np.zeros_like(u)
+    for b in range(B):
+        for k in range(K):
+            for d in range(D):
+                c = k * D + d
+                delta = [_np_softplus(draw[b, k, d, t] + bias[c]) for t in range(L)]
+                for t in range(L):
+                    acc = 0.0
+                    for n in range(N):
+                        inner = 0.0
+                        for s in range(t + 1):
+                            prod = 1.0
+                            for r in range(s + 1, t + 1):
+                                prod *= math.exp(delta[r] * A[c, n])
+                            if b_mode == 1:
+                                bb = math.expm1(delta[s] * A[c, n]) / A[c, n] * Bs[b, k, n, s]
+                            else:
+                                bb = delta[s] * Bs[b, k, n, s]
+                            inner += prod * bb * u[b, k, d, s]
+                        acc += Cs[b, k, n, t] * inner
+                    y[b, k, d, t] = acc + Dskip[c] * u[b, k, d, t]
+    return y
+
+
+def pin_scan_brute_force(orc):
+    """Brute-force O(L^2) unrolling of Eq. 3 on tiny random inputs (both B-bar forms)."""
+    rng = np.random.default_rng(15)
+    args = _rand_problem(rng, B=2, K=2, D=3, N=4, L=9)
+    _close(orc.selective_scan(*args), brute_force_full(*args), rtol=1e-11, atol=1e-12,
+           what="brute force euler")
+    _close(orc.selective_scan(*args, b_mode=1), brute_force_full(*args, b_mode=1), rtol=1e-11,
+           atol=1e-12, what="brute force zoh")
+
+
+def pin_scan_memoryless_limit(orc):
+    """Large Delta drives Abar = e^{delta A} to 0: y_t = u_t (delta_t sum_n C_{t,n} B_{t,n} + D)."""
+    rng = np.random.default_rng(16)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, L=6)
+    draw = 60.0 + rng.uniform(0, 1, size=draw.shape)
+    B, K, D, L = u.shape
+    c = np.arange(K * D).reshape(K, D)
+    delta = _np_softplus(draw + bias[c][None, :, :, None])
+    cb = np.einsum("bknl,bknl->bkl", Cs, Bs)
+    exp = u * (delta * cb[:, :, None, :] + Dskip[c][None, :, :, None])
+    _close(orc.selective_scan(u, draw, A, Bs, Cs, Dskip, bias), exp, rtol=1e-12, what="memoryless")
+
+
+def pin_scan_linear_and_causal(orc):
+    """For fixed Delta, B, C the scan is linear in u, and y_t does not depend on u_s for s > t."""
+    rng = np.random.default_rng(17)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, L=12)
+    u2 = rng.standard_normal(u.shape)
+    y1 = orc.selective_scan(u, draw, A, Bs, Cs, Dskip, bias)
+    y2 = orc.selective_scan(u2, draw, A, Bs, Cs, Dskip, bias)
+    y12 = orc.selective_scan(2.0 * u - 3.0 * u2, draw, A, Bs, Cs, Dskip, bias)
+    _close(y12, 2.0 * y1 - 3.0 * y2, rtol=1e-10, atol=1e-11, what="linearity")
+    u3 = u.copy()
+    u3[..., 7:] += 5.0
+    y3 = orc.selective_scan(u3, draw, A, Bs, Cs, Dskip, bias)
+    _close(y3[..., :7], y1[..., :7], rtol=0, atol=0, what="causality")
+    if np.allclose(y3[..., 7:], y1[..., 7:]):
+        raise AssertionError("later outputs ignore the perturbation")
+
+
+def pin_scan_zoh_euler_limit(orc):
+    """As A -> 0 the zero-order-hold Bbar = (e^{delta A} - 1)/A B tends to the Euler delta B."""
+    rng = np.random.default_rng(18)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, L=8)
+    A = A * 1e-9
+    ye = orc.selective_scan(u, draw, A, Bs, Cs, Dskip, bias, b_mode=0)
+    yz = orc.selective_scan(u, draw, A, Bs, Cs, Dskip, bias, b_mode=1)
+    _close(yz, ye, rtol=1e-7, atol=1e-8, what="zoh->euler")
+
+
+def pin_scan_softplus_off(orc):
+    """With the softplus switched off Delta = raw + bias is used as is (L = 1 closed form)."""
+    rng = np.random.default_rng(19)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, B=1, K=1, D=2, N=3, L=1)
+    draw = np.abs(draw) + 0.1
+    bias = np.abs(bias)
+    delta = draw[0, 0, :, 0] + bias
+    cb = float(np.sum(Cs[0, 0, :, 0] * Bs[0, 0, :, 0]))
+    exp = u[0, 0, :, 0] * (delta * cb + Dskip)
+    y = orc.selective_scan(u, draw, A, Bs, Cs, Dskip, bias, softplus_on=False)
+    _close(y[0, 0, :, 0], exp, what="softplus off")
+
+
+# ------------------------------------------------------------ channel mean
+
+
+def pin_mean_equals_full_on_identical_channels(orc):
+    """Eq. 9 loses nothing when every channel of a direction carries the same inputs."""
+    rng = np.random.default_rng(20)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, B=2, K=2, D=4, N=3, L=10)
+    u[:] = u[:, :, :1]
+    draw[:] = draw[:, :, :1]
+    K, D = 2, 4
+    A = np.repeat(A.reshape(K, D, -1)[:, :1], D, axis=1).reshape(K * D, -1)
+    Dskip = np.repeat(Dskip.reshape(K, D)[:, :1], D, axis=1).reshape(-1)
+    bias = np.repeat(bias.reshape(K, D)[:, :1], D, axis=1).reshape(-1)
+    yf = orc.selective_scan(u, draw, A, Bs, Cs, Dskip, bias)
+    ym, _ = orc.mean_scan(u, draw, A, Bs, Cs, Dskip, bias)
+    _close(ym, yf, rtol=1e-12, atol=1e-13, what="identical channels")
+
+
+def pin_mean_equals_full_at_D1(orc):
+    """With one channel the channel mean is the identity."""
+    rng = np.random.default_rng(21)
+    args = _rand_problem(rng, B=2, K=3, D=1, N=4, L=11)
+    _close(orc.mean_scan(*args)[0], orc.selective_scan(*args), rtol=1e-12, atol=1e-13, what="D=1")
+
+
+def brute_force_mean(u, draw, A, Bs, Cs, Dskip, bias, b_mode=0):
+    """ybar by explicit unrolling of the one-channel system built from the channel means
+    Abar_{t,n} = mean_d e^{delta_{d,t} A_{c,n}}, (Bbar u)_{t,n} = mean_d Bbar_{d,t,n} u_{d,t}."""
+    B, K, D, L = u.shape
+    N = Bs.shape[2]
+    ybar = np.zeros((B, K, L))
+    for b in range(B):
+        for k in range(K):
+            cidx = k * D + np.arange(D)
+            delta = _np_softplus(draw[b, k] + bias[cidx][:, None])           # [D, L]
+            Abar = np.exp(delta[:, :, None] * A[cidx][:, None, :]).mean(0)   # [L, N]
+            if b_mode == 1:
+                bb = np.expm1(delta[:, :, None] * A[cidx][:, None, :]) / A[cidx][:, None, :]
+                bb = bb * Bs[b, k].T[None]
+            else:
+                bb = delta[:, :, None] * Bs[b, k].T[None]
+            BUbar = (bb * u[b, k][:, :, None]).mean(0)                       # [L, N]
+            for t in range(L):
+                acc = 0.0
+                for n in range(N):
+                    inner = 0.0
+                    for s in range(t + 1):
+                        inner += np.prod(Abar[s + 1:t + 1, n]) * BUbar[s, n]
+                    acc += Cs[b, k, n, t] * inner
+                ybar[b, k, t] = acc
+    return ybar
+
+
+def pin_mean_brute_force(orc):
+    """ybar equals the brute-force unrolling of the averaged system, and y = ybar + D_c u
+    (T^-1 broadcast + per-channel skip) on every channel."""
+    rng = np.random.default_rng(22)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, B=2, K=2, D=5, N=3, L=8, draw_scale=1.5)
+    ym, yb = orc.mean_scan(u, draw, A, Bs, Cs, Dskip, bias)
+    _close(yb, brute_force_mean(u, draw, A, Bs, Cs, Dskip, bias), rtol=1e-11, atol=1e-12,
+           what="ybar brute force")
+    K, D = 2, 5
+    skip = Dskip.reshape(K, D)[None, :, :, None] * u
+    _close(ym, yb[:, :, None, :] + skip, rtol=1e-12, atol=1e-13, what="broadcast + skip")
+    ymz, ybz = orc.mean_scan(u, draw, A, Bs, Cs, Dskip, bias, b_mode=1)
+    _close(ybz, brute_force_mean(u, draw, A, Bs, Cs, Dskip, bias, b_mode=1), rtol=1e-11,
+           atol=1e-12, what="ybar brute force zoh")
+
+
+def pin_mean_L2_averages_after_exp(orc):
+    """Hand expansion at L = 2 of the reduced system: ybar_1 = sum_n C_{1,n}
+    (mean_d e^{delta_{d,1} A_{c,n}} mean_d delta_{d,0} B_{0,n} u_{d,0} + mean_d delta_{d,1} B_{1,n} u_{d,1}).
+    Two channels with very different Delta separate mean-of-exp from exp-of-mean."""
+    D, N = 2, 2
+    u = np.array([[[[1.0, 0.5], [2.0, -1.0]]]])
+    draw = np.array([[[[0.0, -4.0], [0.0, 3.0]]]])
+    A = np.array([[-1.0, -2.0], [-1.5, -0.5]])
+    Bs = np.array([[[[0.3, -0.7], [1.1, 0.4]]]])
+    Cs = np.array([[[[0.9, 1.3], [-0.2, 0.8]]]])
+    Dskip = np.array([0.0, 0.0])
+    bias = np.array([0.0, 0.0])
+    dl = _np_softplus(draw[0, 0])  # [D, L]
+    yb1 = 0.0
+    for n in range(N):
+        abar1 = np.mean([math.exp(dl[d, 1] * A[d, n]) for d in range(D)])
+        bu0 = np.mean([dl[d, 0] * Bs[0, 0, n, 0] * u[0, 0, d, 0] for d in range(D)])
+        bu1 = np.mean([dl[d, 1] * Bs[0, 0, n, 1] * u[0, 0, d, 1] for d in range(D)])
+        yb1 += Cs[0, 0, n, 1] * (abar1 * bu0 + bu1)
+    _, yb = orc.mean_scan(u, draw, A, Bs, Cs, Dskip, bias)
+    _close(yb[0, 0, 1], yb1, what="mean L=2")
+
+
+def pin_mean_skip_mean_mode(orc):
+    """skip_mode MEAN: y = ybar + mean_d(D_c u_d), the same value on every channel."""
+    rng = np.random.default_rng(23)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, B=1, K=2, D=4, N=2, L=5)
+    ym, yb = orc.mean_scan(u, draw, A, Bs, Cs, Dskip, bias, skip_mode=1)
+    skip = (Dskip.reshape(2, 4)[None, :, :, None] * u).mean(axis=2)
+    _close(ym, np.broadcast_to((yb + skip)[:, :, None, :], ym.shape), rtol=1e-12, atol=1e-13,
+           what="skip mean")
+
+
+ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

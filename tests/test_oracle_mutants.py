@@ -1,0 +1,55 @@
+"""Planted mistakes in a copy of the oracle must each trip at least one pin.
+
+Each mutant is a one-place textual change to oracle.c (a dropped term, a wrong
+sign, a wrong or transposed index, a wrong operand), compiled on the CPU into
+a temporary library; the real oracle is never touched.
+"""
+import os
+
+import pytest
+
+import oracle
+from tests.oracle_pins import ALL_PINS
+
+MUTANTS = {
+    "drop_skip_term": ("y[t] = acc + p->Dskip[c] * u[t];", "y[t] = acc;"),
+    "wrong_sign_in_abar": ("double abar = exp(delta * A[n]);", "double abar = exp(-delta * A[n]);"),
+    "C_replaced_by_B": ("acc += Ck[n * L + t] * h[n];", "acc += Bk[n * L + t] * h[n];"),
+    "input_without_u": ("h[n] = abar * h[n] + bbar * u[t];", "h[n] = abar * h[n] + bbar;"),
+    "bias_dropped": ("double v = dl[t] + p->bias[c];", "double v = dl[t];"),
+    "bias_wrong_channel": ("double v = dl[t] + p->bias[c];", "double v = dl[t] + p->bias[d];"),
+    "softplus_wrong_branch": ("log1p(exp(-fabs(x)))", "log1p(exp(-x))"),
+    "nonzero_initial_state": ("for (long n = 0; n < N; ++n) h[n] = 0.0;\n    for (long t = 0; t < L; ++t) {\n        double v",
+                              "for (long n = 0; n < N; ++n) h[n] = 1.0;\n    for (long t = 0; t < L; ++t) {\n        double v"),
+    "zoh_missing_delta": ("return expm1(delta * a) / a * b;", "return expm1(delta * a) / (delta * a) * b;"),
+    "column_major_as_row_major": ("case 1: return w * H + h;", "case 1: return h * W + w;"),
+    "reverse_off_by_one": ("case 2: return L - 1 - (h * W + w);", "case 2: return (L - (h * W + w)) % L;"),
+    "merge_wrong_direction": ("(s0[seq_pos(0, h, w, H, W)] + s2[seq_pos(2, h, w, H, W)])",
+                              "(s0[seq_pos(0, h, w, H, W)] + s2[seq_pos(3, h, w, H, W)])"),
+    "mean_sum_not_mean": ("abar[n] /= (double)D; bubar[n] /= (double)D;", "bubar[n] /= (double)D;"),
+    "mean_wrong_channel_A": ("abar[n] += exp(delta * p->A[c * N + n]);",
+                             "abar[n] += exp(delta * p->A[(k * D) * N + n]);"),
+    "mean_skip_wrong_channel": (": p->Dskip[c] * u[d * L + t];", ": p->Dskip[k * D] * u[d * L + t];"),
+    "mean_output_before_update": ("h[n] = abar[n] * h[n] + bubar[n];\n            ybar += Ck[n * L + t] * h[n];",
+                                  "ybar += Ck[n * L + t] * h[n];\n            h[n] = abar[n] * h[n] + bubar[n];"),
+    "mean_bu_without_u": ("p->b_mode) * u[d * L + t];", "p->b_mode);"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name, tmp_path):
+    old, new = MUTANTS[name]
+    src = open(oracle.SOURCE).read()
+    assert src.count(old) == 1, f"mutation site for {name} not found exactly once"
+    mpath = os.path.join(tmp_path, f"oracle_{name}.c")
+    with open(mpath, "w") as f:
+        f.write(src.replace(old, new))
+    lib = oracle.compile_c(mpath, os.path.join(tmp_path, f"liboracle_{name}.so"))
+    mutant = oracle.Oracle(lib)
+    caught = []
+    for pin in ALL_PINS:
+        try:
+            pin(mutant)
+        except AssertionError:
+            caught.append(pin.__name__)
+    assert caught, f"no pin catches mutant {name}"
