@@ -1,0 +1,403 @@
+#!/usr/bin/env python3
+"""Benchmark of the SS2D selective-scan hot path (full and VMeanba channel-mean).
+
+One step = one SS2D pass over one synthetic batch, both paths:
+    cross-scan x -> xs;  full scan xs -> y_full;  channel-mean scan xs -> y_mean;
+    cross-merge y_full -> out_full;  cross-merge y_mean -> out_mean
+all through the C ABI of libvmb.  The default workload is the VMamba-T
+stage-1 scan at batch 1 (D=192, N=16, 56x56, fp32).
+
+Prints ONE JSON line (rank 0).  `value` is the step's algorithmic HBM bytes
+(sum over its five kernels) per second of device time, with inputs resident
+in HBM and L2 flushed before every step; `e2e` is the same metric with the
+inputs copied from pinned host memory and both outputs copied back inside
+the timed region.  `--impl reference` times the fp64 CPU oracle on the same
+workload instead.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads  # noqa: E402
+
+METRIC = ("selective-scan HBM GB/s and (B·K·D·L)/s, full vs channel-mean, "
+          "% of GB300 HBM peak")
+DEFAULT_WORKLOAD = workloads.STAGE1_B1
+FALLBACK_HBM_GBS = 6800.0
+KERNELS = ["cross_scan", "full_scan", "mean_scan", "cross_merge_full", "cross_merge_mean"]
+SOURCES = {"full_scan": "full_scan.cu", "mean_scan": "mean_scan.cu", "cross_scan": "cross_scan_merge.cu",
+           "cross_merge_full": "cross_scan_merge.cu", "cross_merge_mean": "cross_scan_merge.cu"}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    return ap.parse_args()
+
+
+def kernel_bytes(wl: workloads.Workload) -> dict:
+    return {"cross_scan": wl.csm_bytes(), "full_scan": wl.scan_bytes(), "mean_scan": wl.scan_bytes(),
+            "cross_merge_full": wl.csm_bytes(), "cross_merge_mean": wl.csm_bytes()}
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def src_hash(kernel: str) -> str:
+    p = os.path.join(ROOT, "paper_2412_16602_gb300", "csrc", SOURCES[kernel])
+    with open(p, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def committed_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current source of that kernel (else None)."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    want = src_hash(kernel)
+    for line in open(path):
+        if line.startswith("#") or not line.strip():
+            continue
+        kv = dict(tok.split("=", 1) for tok in line.split() if "=" in tok)
+        if kv.get("kernel") == kernel and kv.get("workload") == workload and kv.get("src_sha") == want:
+            return float(kv["dram_bytes_per_launch"])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = []
+        for line in (self.out or "").splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+
+
+def oracle_step(inp, nthreads):
+    import oracle
+    oracle.ss2d_full(inp, nthreads=nthreads)
+    oracle.ss2d_mean(inp, nthreads=nthreads)
+
+
+def time_oracle(inp, target_s=10.0, max_steps=None):
+    """Run whole oracle steps until about target_s seconds have passed."""
+    import oracle
+    nth = oracle.default_threads()
+    times = []
+    t_end = time.perf_counter() + target_s
+    while True:
+        t0 = time.perf_counter()
+        oracle_step(inp, nth)
+        times.append(time.perf_counter() - t0)
+        if time.perf_counter() >= t_end or (max_steps and len(times) >= max_steps):
+            break
+    return times, nth
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+
+class Step:
+    """Pre-marshalled C-ABI calls of one SS2D step (pointers, shapes, stream)."""
+
+    def __init__(self, vmb, wl, g, outs, stream_handle):
+        self.vmb = vmb
+        lib = vmb.lib
+        self.lib = lib
+        B, D, N, H, W = wl.B, wl.D, wl.N, wl.H, wl.W
+        K = 4
+        dt = vmb.VMB_BF16 if wl.dtype == "bf16" else vmb.VMB_F32
+        P = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
+        s = ctypes.c_void_p(stream_handle)
+        fl = vmb.VMB_FLAG_SOFTPLUS
+        wsf = outs["ws_full"]
+        wsm = outs["ws_mean"]
+        self.calls = [
+            ("cross_scan", lib.vmb_cross_scan, (P(g["x"]), P(outs["xs"]), B, D, H, W, dt, s)),
+            ("full_scan", lib.vmb_selective_scan_fwd,
+             (P(outs["xs"]), P(g["draw"]), P(g["A"]), P(g["Bs"]), P(g["Cs"]), P(g["Dskip"]), P(g["bias"]),
+              P(outs["yf"]), B, K, D, N, H, W, fl, dt, P(wsf), wsf.numel(), s)),
+            ("mean_scan", lib.vmb_mean_scan_fwd,
+             (P(outs["xs"]), P(g["draw"]), P(g["A"]), P(g["Bs"]), P(g["Cs"]), P(g["Dskip"]), P(g["bias"]),
+              P(outs["ym"]), ctypes.c_void_p(0), B, K, D, N, H, W, fl, dt, P(wsm), wsm.numel(), s)),
+            ("cross_merge_full", lib.vmb_cross_merge, (P(outs["yf"]), P(outs["of"]), B, D, H, W, dt, s)),
+            ("cross_merge_mean", lib.vmb_cross_merge, (P(outs["ym"]), P(outs["om"]), B, D, H, W, dt, s)),
+        ]
+
+    def run(self, events=None):
+        for i, (name, fn, args) in enumerate(self.calls):
+            st = fn(*args)
+            if st != 0:
+                raise RuntimeError(f"{name}: {self.vmb.status_string(st)}")
+            if events is not None:
+                events[i + 1].record()
+
+
+def run_ours(args, wl, rank, world, local_rank):
+    import torch
+    import paper_2412_16602_gb300 as vmb
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    inp = workloads.make_inputs(wl, seed=wl.seed + 7919 * rank)
+    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    host = {}
+    for k, v in inp.arrays().items():
+        t = torch.from_numpy(np.ascontiguousarray(v))
+        if k in ("x", "draw", "Bs", "Cs"):
+            t = t.to(tdt)
+        host[k] = t.pin_memory()
+    g = {k: v.to(dev) for k, v in host.items()}
+    B, D, N, H, W, L = wl.B, wl.D, wl.N, wl.H, wl.W, wl.L
+    outs = {
+        "xs": torch.empty((B, 4, D, L), dtype=tdt, device=dev),
+        "yf": torch.empty((B, 4, D, L), dtype=tdt, device=dev),
+        "ym": torch.empty((B, 4, D, L), dtype=tdt, device=dev),
+        "of": torch.empty((B, D, H, W), dtype=tdt, device=dev),
+        "om": torch.empty((B, D, H, W), dtype=tdt, device=dev),
+        "ws_full": torch.zeros(vmb.vmb_scan_workspace_bytes(0, B, 4, D, N, H, W, tdt), dtype=torch.uint8, device=dev),
+        "ws_mean": torch.zeros(vmb.vmb_scan_workspace_bytes(1, B, 4, D, N, H, W, tdt), dtype=torch.uint8, device=dev),
+    }
+    stream = torch.cuda.current_stream()
+    step = Step(vmb, wl, g, outs, stream.cuda_stream)
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.float32, device=dev)
+
+    def prelude():
+        flush.fill_(1.0)           # evict the inputs from L2
+        torch.cuda._sleep(100000)  # let the host enqueue the whole step before the GPU reaches it
+
+    for _ in range(args.warmup):
+        prelude()
+        step.run()
+    torch.cuda.synchronize()
+    if vmb.vmb_read_status(outs["ws_full"]) != 0 or vmb.vmb_read_status(outs["ws_mean"]) != 0:
+        raise RuntimeError("device error word set during warm-up")
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(KERNELS) + 1)] for _ in range(args.steps)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clk:
+        for i in range(args.steps):
+            prelude()
+            evs[i][0].record()
+            step.run(evs[i])
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    if vmb.vmb_read_status(outs["ws_full"]) != 0 or vmb.vmb_read_status(outs["ws_mean"]) != 0:
+        raise RuntimeError("device error word set during the timed steps")
+    per_kernel = {k: [] for k in KERNELS}
+    step_ms = []
+    for e in evs:
+        step_ms.append(e[0].elapsed_time(e[-1]))
+        for j, k in enumerate(KERNELS):
+            per_kernel[k].append(e[j].elapsed_time(e[j + 1]))
+    total_ms = float(sum(step_ms))
+
+    # ---- end-to-end leg: pinned host inputs -> device -> step -> host outputs
+    out_host = {"of": torch.empty(outs["of"].shape, dtype=tdt).pin_memory(),
+                "om": torch.empty(outs["om"].shape, dtype=tdt).pin_memory()}
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    d2h = sum(t.numel() * t.element_size() for t in out_host.values())
+
+    def e2e_step():
+        for k, t in host.items():
+            g[k].copy_(t, non_blocking=True)
+        step.run()
+        out_host["of"].copy_(outs["of"], non_blocking=True)
+        out_host["om"].copy_(outs["om"], non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    e0.record()
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e1.record()
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+
+    res = {"total_ms": total_ms, "step_ms": step_ms, "per_kernel": per_kernel, "e2e_ms": e2e_ms,
+           "h2d": h2d, "d2h": d2h, "clocks": clk.summary()}
+    if world > 1:
+        t = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        res["total_ms"], res["e2e_ms"] = float(t[0]), float(t[1])
+    return res, inp
+
+
+def main():
+    args = parse()
+    wl = workloads.WORKLOADS[args.workload]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    step_bytes = sum(kernel_bytes(wl).values())
+    elems = wl.scan_elements()
+    config = {"workload": wl.name, "B": wl.B, "K": 4, "D": wl.D, "N": wl.N, "H": wl.H, "W": wl.W, "L": wl.L,
+              "storage": wl.dtype, "sigma": wl.sigma, "l2": "flushed before every step (2x L2 write)",
+              "step": "cross_scan + full_scan + mean_scan + 2 x cross_merge"}
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        inp = workloads.make_inputs(wl)
+        import oracle
+        for _ in range(min(args.warmup, 1)):
+            oracle_step(inp, oracle.default_threads())
+        times = []
+        nth = oracle.default_threads()
+        for _ in range(args.steps):
+            t0 = time.perf_counter()
+            oracle_step(inp, nth)
+            times.append(time.perf_counter() - t0)
+        ms = 1e3 * sum(times) / len(times)
+        v = step_bytes / (ms / 1e3) / 1e9
+        line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "GB/s", "n_gpus": args.gpus,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config,
+                "elements_per_s": 2 * elems / (ms / 1e3),
+                "cpu_baseline": {"value": v, "unit": "GB/s", "cores": nth, "kind": "oracle",
+                                 "sample": f"whole {wl.name} step per timed step (full + mean paths)"},
+                "e2e": {"value": v, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return
+
+    if world > 1:
+        import torch
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    res, inp = run_ours(args, wl, rank, world, local_rank)
+    if rank != 0:
+        if world > 1:
+            import torch
+            torch.distributed.destroy_process_group()
+        return
+
+    ms = res["total_ms"] / args.steps
+    value = world * step_bytes / (ms / 1e3) / 1e9
+    kb = kernel_bytes(wl)
+    peak, peak_src = measured_peaks()
+    per = {}
+    for k in KERNELS:
+        avg = statistics.mean(res["per_kernel"][k])
+        per[k] = {"us": avg * 1e3, "gbs": kb[k] / (avg / 1e3) / 1e9, "frac_of_peak": kb[k] / (avg / 1e3) / 1e9 / peak}
+    dominant = max(KERNELS, key=lambda k: statistics.mean(res["per_kernel"][k]))
+    dom_ms = statistics.mean(res["per_kernel"][dominant])
+    achieved = kb[dominant] / (dom_ms / 1e3) / 1e9
+    traffic = committed_traffic(dominant, wl.name)
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded; shared map + per-channel noise)",
+        "config": config,
+        "elements_per_s": world * 2 * elems / (ms / 1e3),
+        "frac_of_peak": value / peak,
+        "full": {"us": per["full_scan"]["us"], "gbs": per["full_scan"]["gbs"],
+                 "elements_per_s": elems / (per["full_scan"]["us"] / 1e6),
+                 "frac_of_peak": per["full_scan"]["frac_of_peak"]},
+        "mean": {"us": per["mean_scan"]["us"], "gbs": per["mean_scan"]["gbs"],
+                 "elements_per_s": elems / (per["mean_scan"]["us"] / 1e6),
+                 "frac_of_peak": per["mean_scan"]["frac_of_peak"]},
+        "mean_speedup_over_full": per["full_scan"]["us"] / per["mean_scan"]["us"],
+        "kernels": per,
+        "roofline": {"kernel": dominant, "bound": "hbm", "achieved": achieved, "peak": peak,
+                     "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)" if peak_src == "measured"
+                     else "fallback 6.8 TB/s", "unit": "GB/s", "frac": achieved / peak,
+                     "algorithmic_bytes_per_launch": kb[dominant], "traffic": traffic},
+        "gpu_launches": len(KERNELS) * args.steps,
+        "clocks": res["clocks"],
+        "e2e": {"value": world * step_bytes / (res["e2e_ms"] / args.e2e_steps / 1e3) / 1e9, "unit": "GB/s",
+                "ms_per_step": res["e2e_ms"] / args.e2e_steps,
+                "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"]},
+    }
+    if not args.no_cpu_baseline and world >= 1 and rank == 0:
+        times, nth = time_oracle(inp, target_s=10.0)
+        cms = 1e3 * statistics.mean(times)
+        line["cpu_baseline"] = {"value": step_bytes / (cms / 1e3) / 1e9, "unit": "GB/s", "cores": nth,
+                                "kind": "oracle", "ms_per_step": cms,
+                                "sample": f"{len(times)} whole {wl.name} steps (full + mean paths), ~10 s"}
+    print(json.dumps(line))
+    if world > 1:
+        import torch
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,171 @@
+/*
+ * vmb.h - C ABI of the GB300 (sm_103a) library for the VMamba SS2D selective
+ * scan and its channel-mean variant VMeanba (arXiv 2412.16602).
+ *
+ * The SS2D module (App. A, "VMamba" paragraph) is cross-scan -> selective scan
+ * per direction -> cross-merge.  The selective scan is the discretised,
+ * input-dependent state space model of App. A, Eqs. 3, 4 and 6.  VMeanba
+ * (Sec. 2.2, Eq. 9) replaces the scan's inputs (Abar, Bbar u, C) by their mean
+ * over the inner channel axis, runs one recurrence, and broadcasts the result
+ * back to every channel.
+ *
+ * Conventions shared by every call
+ *   - All tensor pointers are caller-owned DEVICE memory, dense row-major.
+ *     The library allocates nothing and keeps no global state; scratch memory
+ *     (the look-back workspace of the scans) is passed in by the caller.
+ *   - Every call only validates its arguments and enqueues kernels on
+ *     `stream`; it never synchronises (except vmb_read_status) and never
+ *     throws or aborts.  Validation errors return before any launch, with no
+ *     side effects.  A failed launch returns VMB_ERR_CUDA.
+ *   - Shapes: B batch, K scan directions, D inner channels (d_inner), N state
+ *     size (d_state), H x W the feature map, L = H*W the sequence length.
+ *     A zero B, K, D, H or W is an empty problem: the call returns VMB_OK and
+ *     launches nothing.  Negative sizes, or sizes whose element counts do
+ *     not fit in int64, return VMB_ERR_INVALID_ARG.
+ *   - dtype is the storage type of x/xs/u/delta/Bs/Cs/y/out (fp32 or bf16);
+ *     A, Dskip and delta_bias are always fp32; arithmetic and the scan state
+ *     are always fp32.  bf16 outputs are rounded to nearest even.
+ *   - Pointers must be aligned to their element size (VMB_ERR_MISALIGNED
+ *     otherwise).  16-byte aligned rows take the vectorised load path; other
+ *     layouts take an element-wise path that gives the same results.
+ *   - Outputs must not alias inputs.
+ *   - Calls are thread-safe.  Scan calls that share one workspace must not
+ *     overlap in time (order them on one stream).
+ */
+#ifndef VMB_H
+#define VMB_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    VMB_OK = 0,
+    VMB_ERR_INVALID_ARG = 1, /* null pointer, bad size or flag */
+    VMB_ERR_MISALIGNED = 2,  /* pointer not aligned to its element size (workspace: 256 B) */
+    VMB_ERR_UNSUPPORTED = 3, /* valid request this build does not implement (e.g. N > 16) */
+    VMB_ERR_WORKSPACE = 4,   /* workspace missing or smaller than vmb_scan_workspace_bytes() */
+    VMB_ERR_CUDA = 5,        /* a CUDA runtime call or kernel launch failed */
+    VMB_ERR_TIMEOUT = 6,     /* device side: a look-back wait gave up (read via vmb_read_status) */
+    VMB_ERR_BOUNDS = 7       /* device side: an index check failed (bounds-checked builds only) */
+} vmb_status;
+
+typedef enum { VMB_F32 = 0, VMB_BF16 = 1 } vmb_dtype;
+
+/* Scan flags (bitwise OR). */
+#define VMB_FLAG_SOFTPLUS 0x1u  /* delta = softplus(delta_raw + delta_bias) (Eq. 6); else raw + bias */
+#define VMB_FLAG_B_ZOH 0x2u     /* Bbar = (exp(delta A) - 1) / A * B, zero-order hold (Eq. 4);
+                                   else the Euler form Bbar = delta * B */
+#define VMB_FLAG_SKIP_MEAN 0x4u /* vmb_mean_scan_fwd only: skip term = mean_d(Dskip_c u_d),
+                                   broadcast; else per channel Dskip_c * u_d */
+/* Test hook, never set in production: the first L-chunk of every sequence of
+ * a multi-chunk scan does not publish its state, so that the look-back waits
+ * of its successors run out (bounded, about 0.2 s) and the call reports
+ * VMB_ERR_TIMEOUT through vmb_read_status.  No effect on single-chunk plans. */
+#define VMB_FLAG_TEST_SUPPRESS_PUBLISH 0x40000000u
+
+/* Scan path selector for vmb_scan_workspace_bytes. */
+#define VMB_PATH_FULL 0
+#define VMB_PATH_MEAN 1
+
+/*
+ * vmb_cross_scan - SS2D cross-scan (App. A, "VMamba": unfold the H x W map
+ * along four directions into four 1-D sequences).
+ *   x   [B, D, H, W]       input map
+ *   xs  [B, 4, D, L]       output sequences: direction 0 reads the map row by
+ *                          row, 1 column by column, 2 and 3 are 0 and 1 reversed:
+ *     xs[b,0,d,l] = x[b,d,l/W,l%W]      xs[b,1,d,l] = x[b,d,l%H,l/H]
+ *     xs[b,2,d,l] = xs[b,0,d,L-1-l]     xs[b,3,d,l] = xs[b,1,d,L-1-l]
+ * A pure permutation: results are bit-exact copies of x.
+ */
+vmb_status vmb_cross_scan(const void* x, void* xs, int B, int D, int H, int W, vmb_dtype dtype,
+                          cudaStream_t stream);
+
+/*
+ * vmb_cross_merge - SS2D cross-merge (App. A, "VMamba": merge the four
+ * sequence sets back into the 2-D map).
+ *   ys  [B, 4, D, L]       per-direction outputs
+ *   out [B, D, H, W]       out[b,d,h,w] = (ys0[p0] + ys2[p2]) + (ys1[p1] + ys3[p3]),
+ *                          p0 = h*W + w, p1 = w*H + h, p2 = L-1-p0, p3 = L-1-p1,
+ *                          summed in fp32 in exactly this order.
+ */
+vmb_status vmb_cross_merge(const void* ys, void* out, int B, int D, int H, int W,
+                           vmb_dtype dtype, cudaStream_t stream);
+
+/*
+ * vmb_scan_workspace_bytes - bytes of zero-initialised device workspace that
+ * vmb_selective_scan_fwd (path VMB_PATH_FULL) or vmb_mean_scan_fwd
+ * (VMB_PATH_MEAN) needs for this problem on the current device.  Always >= 256
+ * (the status header).  The workspace holds the status word and the
+ * chunk-carry exchange of the L-chunked scans.
+ *
+ * The workspace must be zero-filled once before its first use (cudaMemset or
+ * a zeros tensor); afterwards every call leaves it ready for the next one.
+ * Returns 0 for invalid arguments.
+ */
+size_t vmb_scan_workspace_bytes(int path, int B, int K, int D, int N, int H, int W,
+                                vmb_dtype dtype);
+
+/*
+ * vmb_selective_scan_fwd - full-channel selective scan over K directions
+ * (App. A: selection Eq. 6, discretisation Eq. 4, recurrence Eq. 3), with the
+ * discretisation fused into the scan:
+ *   c = k*D + d,  delta_t = softplus(delta[b,k,d,t] + delta_bias[c])
+ *   h_n(-1) = 0,  h_n(t) = exp(delta_t A[c,n]) h_n(t-1) + Bbar_n(t) u[b,k,d,t]
+ *   y[b,k,d,t] = sum_n Cs[b,k,n,t] h_n(t) + Dskip[c] u[b,k,d,t]
+ *   u, delta, y [B, K, D, L] (dtype);  Bs, Cs [B, K, N, L] (dtype)
+ *   A [K*D, N], Dskip [K*D], delta_bias [K*D] (fp32)
+ *   flags: VMB_FLAG_SOFTPLUS | VMB_FLAG_B_ZOH
+ *   workspace: >= vmb_scan_workspace_bytes(VMB_PATH_FULL, ...) bytes, 256-B
+ *   aligned, zero-filled before first use.
+ * Supports 1 <= N <= 16 (VMB_ERR_UNSUPPORTED above) and any K >= 1.
+ */
+vmb_status vmb_selective_scan_fwd(const void* u, const void* delta, const float* A, const void* Bs,
+                                  const void* Cs, const float* Dskip, const float* delta_bias,
+                                  void* y, int B, int K, int D, int N, int H, int W,
+                                  unsigned flags, vmb_dtype dtype, void* workspace,
+                                  size_t workspace_bytes, cudaStream_t stream);
+
+/*
+ * vmb_mean_scan_fwd - VMeanba channel-mean scan (Sec. 2.2, Eq. 9:
+ * y = T^-1(Mamba(T(Abar, Bbar u, C)))), T the mean over the D channels of one
+ * (batch, direction), T^-1 the broadcast back to every channel:
+ *   Abar_n(t)    = (1/D) sum_d exp(delta_{d,t} A[c_d,n])      (mean after the exp)
+ *   (Bbar u)_n(t)= (1/D) sum_d Bbar_{d,n}(t) u[b,k,d,t]
+ *   h_n(t) = Abar_n(t) h_n(t-1) + (Bbar u)_n(t),  ybar(t) = sum_n Cs[b,k,n,t] h_n(t)
+ *   y[b,k,d,t] = ybar(t) + Dskip[c] u[b,k,d,t]      (VMB_FLAG_SKIP_MEAN:
+ *                ybar(t) + (1/D) sum_d Dskip[c_d] u[b,k,d,t])
+ * Same arguments as vmb_selective_scan_fwd, plus
+ *   ybar [B, K, L] fp32 device pointer, or NULL: optional copy of ybar.
+ * The recurrence runs once per (b, k) instead of once per (b, k, d).
+ */
+vmb_status vmb_mean_scan_fwd(const void* u, const void* delta, const float* A, const void* Bs,
+                             const void* Cs, const float* Dskip, const float* delta_bias, void* y,
+                             float* ybar, int B, int K, int D, int N, int H, int W, unsigned flags,
+                             vmb_dtype dtype, void* workspace, size_t workspace_bytes,
+                             cudaStream_t stream);
+
+/*
+ * vmb_read_status - synchronise `stream`, then return and clear the device
+ * error word of `workspace` (VMB_OK, VMB_ERR_TIMEOUT or VMB_ERR_BOUNDS).  A
+ * device-side error leaves the outputs of that call undefined but the CUDA
+ * context usable.  Returns VMB_ERR_CUDA if the synchronisation fails.
+ */
+vmb_status vmb_read_status(void* workspace, cudaStream_t stream);
+
+/* Static description of a status code (never NULL). */
+const char* vmb_status_string(vmb_status status);
+
+/* Library version: major*10000 + minor*100 + patch. */
+int vmb_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VMB_H */

@@ -1,0 +1,292 @@
+// cross_scan_merge.cu - SS2D cross-scan and cross-merge (App. A, "VMamba") for sm_103a.
+//
+// cross-scan: x[B,D,H,W] -> xs[B,4,D,L].  A CTA stages ppc whole maps (planes)
+// in shared memory with a padded row stride, then writes the four direction
+// rows of every plane: 0 row-major, 1 column-major, 2 and 3 the reverses of 0
+// and 1.  Global loads and stores are 16-byte vectors when rows are 16-byte
+// aligned; the padding keeps the column-major reads free of bank conflicts.
+//
+// cross-merge: ys[B,4,D,L] -> out[B,D,H,W], out = (ys0[p0] + ys2[p2]) +
+// (ys1[p1] + ys3[p3]) in fp32 in that order.  Directions 0 and 2 are read
+// straight from global memory in output order (2 reversed); directions 1 and
+// 3 are staged in shared memory keyed by (w, h) so the transposed reads are
+// conflict-free.
+//
+// Index arithmetic uses division by invariant integers via multiply-high
+// (Granlund & Montgomery, "Division by invariant integers using
+// multiplication", PLDI 1994, round-up variant), valid for dividends < 2^31.
+#include "vmb_common.cuh"
+#include "vmb_internal.h"
+
+namespace vmb {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr size_t kMaxSmem = 200 * 1024;
+
+struct FastDiv {
+    unsigned d, m, s;
+};
+FastDiv make_fastdiv(unsigned d) {
+    unsigned s = 0;
+    while ((1ull << s) < d) ++s;
+    const unsigned long long m = ((1ull << 32) * ((1ull << s) - d)) / d + 1;
+    return {d, (unsigned)m, s};
+}
+__device__ __forceinline__ unsigned fdiv(unsigned n, FastDiv f) { return (__umulhi(n, f.m) + n) >> f.s; }
+
+struct CsmParams {
+    const void* in;
+    void* out;
+    int D, H, W, L;
+    long long planes;  // B * D
+    int ppc;           // planes per CTA
+    int vec;
+    FastDiv fL, fW, fH, fD;
+};
+
+template <typename T>
+union Vec {
+    uint4 v;
+    T e[16 / sizeof(T)];
+};
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) cross_scan_kernel(const CsmParams p) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    T* sp = reinterpret_cast<T*>(smem_raw);  // [ppc][H][W+1]
+    constexpr int VE = 16 / sizeof(T);
+    const T* x = static_cast<const T*>(p.in);
+    T* xs = static_cast<T*>(p.out);
+    const int L = p.L, W = p.W, H = p.H, WP = p.W + 1;
+    const long long p0 = (long long)blockIdx.x * p.ppc;
+    const int np = (int)min((long long)p.ppc, p.planes - p0);
+    const unsigned n = (unsigned)(np * L);
+    const T* src = x + p0 * L;
+    // stage the planes
+    if (p.vec) {
+        for (unsigned i = threadIdx.x * VE; i < n; i += kThreads * VE) {
+            Vec<T> v;
+            v.v = *reinterpret_cast<const uint4*>(src + i);
+#pragma unroll
+            for (int q = 0; q < VE; ++q) {
+                const unsigned e = i + q;
+                const unsigned j = fdiv(e, p.fL), r = e - j * L;
+                const unsigned h = fdiv(r, p.fW), w = r - h * W;
+                sp[(j * H + h) * WP + w] = v.e[q];
+            }
+        }
+    } else {
+        for (unsigned e = threadIdx.x; e < n; e += kThreads) {
+            const unsigned j = fdiv(e, p.fL), r = e - j * L;
+            const unsigned h = fdiv(r, p.fW), w = r - h * W;
+            sp[(j * H + h) * WP + w] = src[e];
+        }
+    }
+    __syncthreads();
+    // write the four direction rows of every staged plane
+#pragma unroll 1
+    for (int kd = 0; kd < 4; ++kd) {
+        const bool rev = kd >= 2, colmajor = kd & 1;
+        if (p.vec) {
+            for (unsigned i = threadIdx.x * VE; i < n; i += kThreads * VE) {
+                const unsigned j = fdiv(i, p.fL), l = i - j * L;
+                const long long pi = p0 + j;
+                const unsigned b = fdiv((unsigned)pi, p.fD), d = (unsigned)pi - b * p.D;
+                Vec<T> v;
+#pragma unroll
+                for (int q = 0; q < VE; ++q) {
+                    const unsigned m = rev ? L - 1 - (l + q) : l + q;
+                    unsigned h, w;
+                    if (colmajor) {
+                        w = fdiv(m, p.fH);
+                        h = m - w * H;
+                    } else {
+                        h = fdiv(m, p.fW);
+                        w = m - h * W;
+                    }
+                    v.e[q] = sp[(j * H + h) * WP + w];
+                }
+                *reinterpret_cast<uint4*>(xs + (((long long)b * 4 + kd) * p.D + d) * L + l) = v.v;
+            }
+        } else {
+            for (unsigned i = threadIdx.x; i < n; i += kThreads) {
+                const unsigned j = fdiv(i, p.fL), l = i - j * L;
+                const long long pi = p0 + j;
+                const unsigned b = fdiv((unsigned)pi, p.fD), d = (unsigned)pi - b * p.D;
+                const unsigned m = rev ? L - 1 - l : l;
+                unsigned h, w;
+                if (colmajor) {
+                    w = fdiv(m, p.fH);
+                    h = m - w * H;
+                } else {
+                    h = fdiv(m, p.fW);
+                    w = m - h * W;
+                }
+                xs[(((long long)b * 4 + kd) * p.D + d) * L + l] = sp[(j * H + h) * WP + w];
+            }
+        }
+    }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) cross_merge_kernel(const CsmParams p) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int L = p.L, W = p.W, H = p.H, HP = p.H + 1;
+    const long long p0 = (long long)blockIdx.x * p.ppc;
+    const int np = (int)min((long long)p.ppc, p.planes - p0);
+    T* s1 = reinterpret_cast<T*>(smem_raw);  // [ppc][W][H+1], keyed by (w, h)
+    T* s3 = s1 + (size_t)p.ppc * W * HP;
+    constexpr int VE = 16 / sizeof(T);
+    const T* ys = static_cast<const T*>(p.in);
+    T* out = static_cast<T*>(p.out);
+    const unsigned n = (unsigned)(np * L);
+    auto row = [&](long long pi, int kd) {
+        const unsigned b = fdiv((unsigned)pi, p.fD), d = (unsigned)pi - b * p.D;
+        return ys + (((long long)b * 4 + kd) * p.D + d) * L;
+    };
+    // stage directions 1 and 3
+    for (int kd = 1; kd <= 3; kd += 2) {
+        T* dst = kd == 1 ? s1 : s3;
+        const bool rev = kd == 3;
+        if (p.vec) {
+            for (unsigned i = threadIdx.x * VE; i < n; i += kThreads * VE) {
+                const unsigned j = fdiv(i, p.fL), l = i - j * L;
+                Vec<T> v;
+                v.v = *reinterpret_cast<const uint4*>(row(p0 + j, kd) + l);
+#pragma unroll
+                for (int q = 0; q < VE; ++q) {
+                    const unsigned m = rev ? L - 1 - (l + q) : l + q;  // column-major position
+                    const unsigned w = fdiv(m, p.fH), h = m - w * H;
+                    dst[(j * W + w) * HP + h] = v.e[q];
+                }
+            }
+        } else {
+            for (unsigned i = threadIdx.x; i < n; i += kThreads) {
+                const unsigned j = fdiv(i, p.fL), l = i - j * L;
+                const unsigned m = rev ? L - 1 - l : l;
+                const unsigned w = fdiv(m, p.fH), h = m - w * H;
+                dst[(j * W + w) * HP + h] = row(p0 + j, kd)[l];
+            }
+        }
+    }
+    __syncthreads();
+    // out[h, w] = (ys0[hW+w] + ys2[L-1-(hW+w)]) + (ys1[wH+h] + ys3[L-1-(wH+h)])
+    if (p.vec) {
+        for (unsigned i = threadIdx.x * VE; i < n; i += kThreads * VE) {
+            const unsigned j = fdiv(i, p.fL), pos = i - j * L;
+            const long long pi = p0 + j;
+            Vec<T> v0, v2, o;
+            v0.v = *reinterpret_cast<const uint4*>(row(pi, 0) + pos);
+            v2.v = *reinterpret_cast<const uint4*>(row(pi, 2) + (L - VE - pos));  // reversed block
+#pragma unroll
+            for (int q = 0; q < VE; ++q) {
+                const unsigned pq = pos + q;
+                const unsigned h = fdiv(pq, p.fW), w = pq - h * W;
+                const unsigned si = (j * W + w) * HP + h;
+                const float a = io<T>::cvt(v0.e[q]) + io<T>::cvt(v2.e[VE - 1 - q]);
+                const float c = io<T>::cvt(s1[si]) + io<T>::cvt(s3[si]);
+                o.e[q] = io<T>::to(a + c);
+            }
+            *reinterpret_cast<uint4*>(out + pi * L + pos) = o.v;
+        }
+    } else {
+        for (unsigned i = threadIdx.x; i < n; i += kThreads) {
+            const unsigned j = fdiv(i, p.fL), pos = i - j * L;
+            const long long pi = p0 + j;
+            const unsigned h = fdiv(pos, p.fW), w = pos - h * W;
+            const unsigned si = (j * W + w) * HP + h;
+            const float a = io<T>::cvt(row(pi, 0)[pos]) + io<T>::cvt(row(pi, 2)[L - 1 - pos]);
+            const float c = io<T>::cvt(s1[si]) + io<T>::cvt(s3[si]);
+            out[pi * L + pos] = io<T>::to(a + c);
+        }
+    }
+}
+
+// Planes too large for shared memory: one thread per element, plain gathers.
+template <typename T>
+__global__ void cross_scan_direct(const T* x, T* xs, int D, int H, int W, long long total) {
+    const long long L = (long long)H * W;
+    for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total; e += (long long)gridDim.x * blockDim.x) {
+        const long long l = e % L, row = e / L;  // row = (b*4 + kd)*D + d
+        const long long d = row % D, bk = row / D, kd = bk % 4, b = bk / 4;
+        const long long m = kd >= 2 ? L - 1 - l : l;
+        const long long h = (kd & 1) ? m % H : m / W;
+        const long long w = (kd & 1) ? m / H : m % W;
+        xs[e] = x[((b * D + d) * H + h) * W + w];
+    }
+}
+
+template <typename T>
+__global__ void cross_merge_direct(const T* ys, T* out, int D, int H, int W, long long total) {
+    const long long L = (long long)H * W;
+    for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total; e += (long long)gridDim.x * blockDim.x) {
+        const long long pos = e % L, pl = e / L, d = pl % D, b = pl / D;
+        const long long h = pos / W, w = pos % W, p1 = w * H + h;
+        const T* r = ys + (b * 4 * D + d) * L;
+        const long long st = (long long)D * L;
+        const float a = io<T>::cvt(r[pos]) + io<T>::cvt(r[2 * st + L - 1 - pos]);
+        const float c = io<T>::cvt(r[st + p1]) + io<T>::cvt(r[3 * st + L - 1 - p1]);
+        out[e] = io<T>::to(a + c);
+    }
+}
+
+template <typename T>
+vmb_status launch_csm(bool merge, const void* in, void* outp, int B, int D, int H, int W, cudaStream_t stream) {
+    const int L = H * W;
+    const long long planes = (long long)B * D;
+    const size_t es = sizeof(T);
+    const size_t per_plane = merge ? 2 * (size_t)W * (H + 1) * es : (size_t)H * (W + 1) * es;
+    const bool small_enough = per_plane <= kMaxSmem && planes < (1ll << 31) &&
+                              (long long)L * 4 < (1ll << 31);
+    if (!small_enough) {
+        const long long total = merge ? planes * L : planes * 4 * L;
+        const int grid = (int)std::min<long long>((total + kThreads - 1) / kThreads, 152ll * 32);
+        if (merge)
+            cross_merge_direct<T><<<grid, kThreads, 0, stream>>>(static_cast<const T*>(in), static_cast<T*>(outp), D, H, W, total);
+        else
+            cross_scan_direct<T><<<grid, kThreads, 0, stream>>>(static_cast<const T*>(in), static_cast<T*>(outp), D, H, W, total);
+        return cudaGetLastError() == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+    }
+    // about 8K elements per CTA, bounded by shared memory
+    int ppc = (int)std::max<long long>(1, 8192 / L);
+    while (ppc > 1 && (size_t)ppc * per_plane > kMaxSmem) --ppc;
+    if (ppc > planes) ppc = (int)planes;
+    CsmParams p{};
+    p.in = in;
+    p.out = outp;
+    p.D = D;
+    p.H = H;
+    p.W = W;
+    p.L = L;
+    p.planes = planes;
+    p.ppc = ppc;
+    const auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
+    p.vec = ((size_t)L * es % 16 == 0) && al16(in) && al16(outp);
+    p.fL = make_fastdiv((unsigned)L);
+    p.fW = make_fastdiv((unsigned)W);
+    p.fH = make_fastdiv((unsigned)H);
+    p.fD = make_fastdiv((unsigned)D);
+    const size_t smem = (size_t)ppc * per_plane;
+    const void* fn = merge ? reinterpret_cast<const void*>(&cross_merge_kernel<T>)
+                           : reinterpret_cast<const void*>(&cross_scan_kernel<T>);
+    if (smem > 48 * 1024 && cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem) != cudaSuccess)
+        return VMB_ERR_CUDA;
+    const unsigned grid = (unsigned)((planes + ppc - 1) / ppc);
+    void* args[] = {&p};
+    return cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, stream) == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+}
+
+}  // namespace
+
+vmb_status launch_cross_scan(const void* x, void* xs, int B, int D, int H, int W, vmb_dtype dt, cudaStream_t stream) {
+    return dt == VMB_BF16 ? launch_csm<__nv_bfloat16>(false, x, xs, B, D, H, W, stream)
+                          : launch_csm<float>(false, x, xs, B, D, H, W, stream);
+}
+
+vmb_status launch_cross_merge(const void* ys, void* out, int B, int D, int H, int W, vmb_dtype dt, cudaStream_t stream) {
+    return dt == VMB_BF16 ? launch_csm<__nv_bfloat16>(true, ys, out, B, D, H, W, stream)
+                          : launch_csm<float>(true, ys, out, B, D, H, W, stream);
+}
+
+}  // namespace vmb

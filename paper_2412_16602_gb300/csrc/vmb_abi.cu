@@ -1,0 +1,195 @@
+// vmb_abi.cu - the extern "C" entry points of libvmb (declared in include/vmb.h):
+// argument validation, plan and workspace sizing, launch on the caller's stream.
+#include <limits.h>
+
+#include <mutex>
+
+#include "vmb_common.cuh"
+#include "vmb_internal.h"
+
+namespace vmb {
+
+int device_sm_count() {
+    static std::mutex mu;
+    static int cache[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    std::lock_guard<std::mutex> g(mu);
+    if (dev >= 0 && dev < 64 && cache[dev] > 0) return cache[dev];
+    int n = 1;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) n = 1;
+    if (dev >= 0 && dev < 64) cache[dev] = n;
+    return n;
+}
+
+namespace {
+
+bool mul_ok(long long a, long long b, long long* out) {
+    if (a < 0 || b < 0) return false;
+    if (a != 0 && b > LLONG_MAX / a) return false;
+    *out = a * b;
+    return true;
+}
+
+bool count(long long* out, std::initializer_list<long long> dims) {
+    long long v = 1;
+    for (long long d : dims)
+        if (!mul_ok(v, d, &v)) return false;
+    *out = v;
+    return true;
+}
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+size_t esize(vmb_dtype dt) { return dt == VMB_BF16 ? 2 : 4; }
+
+bool dtype_ok(vmb_dtype dt) { return dt == VMB_F32 || dt == VMB_BF16; }
+
+constexpr unsigned kKnownFlags =
+    VMB_FLAG_SOFTPLUS | VMB_FLAG_B_ZOH | VMB_FLAG_SKIP_MEAN | VMB_FLAG_TEST_SUPPRESS_PUBLISH;
+
+// Shared checks of the cross-scan / cross-merge calls.  *empty is set for a
+// problem with no elements.
+vmb_status check_csm(const void* in, const void* out, int B, int D, int H, int W, vmb_dtype dt, bool* empty) {
+    if (!dtype_ok(dt) || B < 0 || D < 0 || H < 0 || W < 0) return VMB_ERR_INVALID_ARG;
+    long long n4 = 0;
+    if (!count(&n4, {B, 4, D, H, W})) return VMB_ERR_INVALID_ARG;
+    *empty = n4 == 0;
+    if (*empty) return VMB_OK;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    if (!in || !out) return VMB_ERR_INVALID_ARG;
+    if (!aligned(in, esize(dt)) || !aligned(out, esize(dt))) return VMB_ERR_MISALIGNED;
+    return VMB_OK;
+}
+
+vmb_status check_scan(const ScanArgs& a, bool mean, bool* empty) {
+    if (!dtype_ok(a.dtype)) return VMB_ERR_INVALID_ARG;
+    if (a.B < 0 || a.K < 0 || a.D < 0 || a.N < 0 || a.L < 0) return VMB_ERR_INVALID_ARG;
+    if (a.flags & ~kKnownFlags) return VMB_ERR_INVALID_ARG;
+    if (!mean && (a.flags & VMB_FLAG_SKIP_MEAN)) return VMB_ERR_INVALID_ARG;
+    long long n = 0, nbc = 0;
+    if (!count(&n, {a.B, a.K, a.D, a.L}) || !count(&nbc, {a.B, a.K, a.N > 0 ? a.N : 1, a.L}))
+        return VMB_ERR_INVALID_ARG;
+    *empty = n == 0;
+    if (*empty) return VMB_OK;
+    if (a.N < 1) return VMB_ERR_INVALID_ARG;
+    if (a.N > 16) return VMB_ERR_UNSUPPORTED;
+    long long grid_rows = 0;
+    if (!count(&grid_rows, {a.B, a.K, a.D}) || grid_rows > INT_MAX / 2) return VMB_ERR_UNSUPPORTED;
+    if (!a.u || !a.delta || !a.A || !a.Bs || !a.Cs || !a.Dskip || !a.bias || !a.y) return VMB_ERR_INVALID_ARG;
+    const size_t es = esize(a.dtype);
+    if (!aligned(a.u, es) || !aligned(a.delta, es) || !aligned(a.Bs, es) || !aligned(a.Cs, es) ||
+        !aligned(a.y, es) || !aligned(a.A, 4) || !aligned(a.Dskip, 4) || !aligned(a.bias, 4) ||
+        (a.ybar && !aligned(a.ybar, 4)))
+        return VMB_ERR_MISALIGNED;
+    return VMB_OK;
+}
+
+vmb_status run_scan(ScanArgs& a, bool mean, cudaStream_t stream) {
+    bool empty = false;
+    vmb_status s = check_scan(a, mean, &empty);
+    if (s != VMB_OK || empty) return s;
+    if (!a.ws) return VMB_ERR_WORKSPACE;
+    if (!aligned(a.ws, 256)) return VMB_ERR_MISALIGNED;
+    ScanPlan plan{};
+    s = mean ? plan_mean(a, &plan) : plan_full(a, &plan);
+    if (s != VMB_OK) return s;
+    if (a.ws_bytes < plan.ws_bytes) return VMB_ERR_WORKSPACE;
+    return mean ? launch_mean(a, plan, stream) : launch_full(a, plan, stream);
+}
+
+}  // namespace
+}  // namespace vmb
+
+using namespace vmb;
+
+extern "C" {
+
+vmb_status vmb_cross_scan(const void* x, void* xs, int B, int D, int H, int W, vmb_dtype dtype, cudaStream_t stream) {
+    bool empty = false;
+    vmb_status s = check_csm(x, xs, B, D, H, W, dtype, &empty);
+    if (s != VMB_OK || empty) return s;
+    return launch_cross_scan(x, xs, B, D, H, W, dtype, stream);
+}
+
+vmb_status vmb_cross_merge(const void* ys, void* out, int B, int D, int H, int W, vmb_dtype dtype, cudaStream_t stream) {
+    bool empty = false;
+    vmb_status s = check_csm(ys, out, B, D, H, W, dtype, &empty);
+    if (s != VMB_OK || empty) return s;
+    return launch_cross_merge(ys, out, B, D, H, W, dtype, stream);
+}
+
+size_t vmb_scan_workspace_bytes(int path, int B, int K, int D, int N, int H, int W, vmb_dtype dtype) {
+    if (path != VMB_PATH_FULL && path != VMB_PATH_MEAN) return 0;
+    if (H < 0 || W < 0 || (long long)H * W > INT_MAX) return 0;
+    ScanArgs a{};
+    a.B = B;
+    a.K = K;
+    a.D = D;
+    a.N = N;
+    a.L = H * W;
+    a.dtype = dtype;
+    // shape-only validation: stand-in non-null, aligned pointers
+    static const float dummy[4] = {0, 0, 0, 0};
+    a.u = a.delta = a.Bs = a.Cs = dummy;
+    a.A = a.Dskip = a.bias = dummy;
+    a.y = const_cast<float*>(dummy);
+    bool empty = false;
+    if (check_scan(a, path == VMB_PATH_MEAN, &empty) != VMB_OK) return 0;
+    if (empty) return 256;
+    ScanPlan plan{};
+    if ((path == VMB_PATH_MEAN ? plan_mean(a, &plan) : plan_full(a, &plan)) != VMB_OK) return 0;
+    return plan.ws_bytes;
+}
+
+vmb_status vmb_selective_scan_fwd(const void* u, const void* delta, const float* A, const void* Bs, const void* Cs,
+                                  const float* Dskip, const float* delta_bias, void* y, int B, int K, int D, int N,
+                                  int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,
+                                  size_t workspace_bytes, cudaStream_t stream) {
+    if (H < 0 || W < 0) return VMB_ERR_INVALID_ARG;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    ScanArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, y, nullptr, B, K, D, N, H * W, flags, dtype, workspace, workspace_bytes};
+    return run_scan(a, false, stream);
+}
+
+vmb_status vmb_mean_scan_fwd(const void* u, const void* delta, const float* A, const void* Bs, const void* Cs,
+                             const float* Dskip, const float* delta_bias, void* y, float* ybar, int B, int K, int D,
+                             int N, int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,
+                             size_t workspace_bytes, cudaStream_t stream) {
+    if (H < 0 || W < 0) return VMB_ERR_INVALID_ARG;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    ScanArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, y, ybar, B, K, D, N, H * W, flags, dtype, workspace, workspace_bytes};
+    return run_scan(a, true, stream);
+}
+
+vmb_status vmb_read_status(void* workspace, cudaStream_t stream) {
+    if (!workspace) return VMB_ERR_INVALID_ARG;
+    if (!aligned(workspace, 256)) return VMB_ERR_MISALIGNED;
+    WsHeader* hdr = static_cast<WsHeader*>(workspace);
+    unsigned err = 0;
+    if (cudaMemcpyAsync(&err, &hdr->err, sizeof(err), cudaMemcpyDeviceToHost, stream) != cudaSuccess)
+        return VMB_ERR_CUDA;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return VMB_ERR_CUDA;
+    if (err == 0) return VMB_OK;
+    if (cudaMemsetAsync(&hdr->err, 0, sizeof(unsigned), stream) != cudaSuccess) return VMB_ERR_CUDA;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return VMB_ERR_CUDA;
+    return (err & kErrTimeout) ? VMB_ERR_TIMEOUT : VMB_ERR_BOUNDS;
+}
+
+const char* vmb_status_string(vmb_status s) {
+    switch (s) {
+    case VMB_OK: return "ok";
+    case VMB_ERR_INVALID_ARG: return "invalid argument";
+    case VMB_ERR_MISALIGNED: return "misaligned pointer";
+    case VMB_ERR_UNSUPPORTED: return "unsupported problem";
+    case VMB_ERR_WORKSPACE: return "workspace missing or too small";
+    case VMB_ERR_CUDA: return "CUDA error";
+    case VMB_ERR_TIMEOUT: return "device wait timed out";
+    case VMB_ERR_BOUNDS: return "device bounds check failed";
+    }
+    return "unknown status";
+}
+
+int vmb_version(void) { return 100; }
+
+}  // extern "C"

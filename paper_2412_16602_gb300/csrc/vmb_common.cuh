@@ -1,0 +1,167 @@
+// vmb_common.cuh - device helpers shared by the sm_103a kernels of libvmb:
+// storage-type conversion, the fp32 fast math of the discretisation, and the
+// bounded decoupled look-back used to carry the scan state across L-chunks.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace vmb {
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+// ------------------------------------------------------------ storage types
+
+template <typename T> struct io;
+template <> struct io<float> {
+    static __device__ __forceinline__ float ld(const float* p) { return *p; }
+    static __device__ __forceinline__ float cvt(float v) { return v; }
+    static __device__ __forceinline__ float to(float v) { return v; }
+};
+template <> struct io<__nv_bfloat16> {
+    static __device__ __forceinline__ float ld(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+    static __device__ __forceinline__ float cvt(__nv_bfloat16 v) { return __bfloat162float(v); }
+    // round to nearest even
+    static __device__ __forceinline__ __nv_bfloat16 to(float v) { return __float2bfloat16_rn(v); }
+};
+
+// ------------------------------------------------------------------- math
+
+// 2^x on the MUFU pipe (ex2.approx, flush-to-zero).  Relative error about
+// 2^-22 over the range the scan uses; the parity tests bound its effect.
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ float rcp(float x) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// softplus(v) = log(1 + e^v) (Eq. 6, tau_Delta), written as
+// max(v, 0) + log1p(e^-|v|).  log1p(e) for e in (0, 1] uses the series
+// log1p(e) = 2 atanh(z) = 2 z (1 + z^2/3 + z^4/5 + ...), z = e / (2 + e) <= 1/3
+// (Abramowitz & Stegun 4.1.27), truncated after z^12/13: truncation error below
+// (1/3)^14 / 15 ~ 1.4e-8 relative, so the result keeps the relative accuracy of
+// e^-|v| even where log1p(e) is tiny.  No cut-off for large |v|.
+__device__ __forceinline__ float softplus(float v) {
+    float e = ex2(-fabsf(v) * kLog2e);
+    float z = e * rcp(2.0f + e);
+    float w = z * z;
+    float p = 1.0f / 13.0f;
+    p = fmaf(p, w, 1.0f / 11.0f);
+    p = fmaf(p, w, 1.0f / 9.0f);
+    p = fmaf(p, w, 1.0f / 7.0f);
+    p = fmaf(p, w, 1.0f / 5.0f);
+    p = fmaf(p, w, 1.0f / 3.0f);
+    p = fmaf(p, w, 1.0f);
+    return fmaxf(v, 0.0f) + 2.0f * z * p;
+}
+
+// ------------------------------------------------------ memory-model helpers
+
+__device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_release(unsigned* p, unsigned v) {
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned ld_relaxed(const unsigned* p) {
+    unsigned v;
+    asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ float ld_cg(const float* p) { return __ldcg(p); }
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// ------------------------------------------------------- workspace / look-back
+
+// Status header at the start of every scan workspace (256 bytes).
+struct WsHeader {
+    unsigned ticket;     // next CTA ticket of the running launch
+    unsigned done;       // CTAs of the running launch that have finished
+    unsigned gen;        // launch generation: tags the chunk flags of one launch
+    unsigned err;        // error bits (kErrTimeout, kErrBounds), cleared by vmb_read_status
+    unsigned err_seq;    // first sequence / chunk whose wait gave up (diagnostics)
+    unsigned err_chunk;
+    unsigned pad[58];
+};
+static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
+
+constexpr unsigned kErrTimeout = 1u;
+constexpr unsigned kErrBounds = 2u;
+constexpr unsigned kFlagAggregate = 1u;  // chunk aggregate published
+constexpr unsigned kFlagInclusive = 2u;  // chunk inclusive prefix (end state) published
+constexpr uint64_t kWaitLimitNs = 200ull * 1000ull * 1000ull;  // 0.2 s per wait
+
+__device__ __forceinline__ unsigned flag_word(unsigned gen, unsigned kind) {
+    return ((gen & 0x3FFFFFFFu) << 2) | kind;
+}
+
+// Spin (one thread) until `flag` carries this launch's generation, or give up.
+// Returns kFlagAggregate / kFlagInclusive, or 0 when the wait ran out or another
+// CTA already reported an error (then every later wait returns at once).
+__device__ __forceinline__ unsigned wait_flag(const unsigned* flag, unsigned gen, WsHeader* hdr,
+                                              unsigned seq, unsigned chunk) {
+    const unsigned tag = gen & 0x3FFFFFFFu;
+    uint64_t t0 = 0;
+    unsigned ns = 32;
+    for (unsigned it = 0;; ++it) {
+        unsigned f = ld_acquire(flag);
+        if ((f >> 2) == tag && (f & 3u)) return f & 3u;
+        if ((it & 15u) == 0) {
+            if (ld_relaxed(&hdr->err)) return 0;
+            uint64_t now = globaltimer_ns();
+            if (it == 0) t0 = now;
+            else if (now - t0 > kWaitLimitNs) {
+                if (atomicOr(&hdr->err, kErrTimeout) == 0) {
+                    hdr->err_seq = seq;
+                    hdr->err_chunk = chunk;
+                }
+                return 0;
+            }
+        }
+        __nanosleep(ns);
+        if (ns < 1024) ns <<= 1;
+    }
+}
+
+// Called by thread 0 of every CTA of a look-back launch once the CTA is done
+// with the workspace: the last CTA resets the ticket and completion counters
+// and advances the generation, leaving the workspace ready for the next launch.
+__device__ __forceinline__ void finish_launch(WsHeader* hdr, unsigned total_ctas) {
+    __threadfence();
+    unsigned prev = atomicAdd(&hdr->done, 1u);
+    if (prev == total_ctas - 1) {
+        __threadfence();
+        hdr->ticket = 0;
+        hdr->done = 0;
+        atomicAdd(&hdr->gen, 1u);
+        __threadfence();
+    }
+}
+
+// --------------------------------------------------------- async copies
+
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem, int src_bytes) {
+    unsigned s = (unsigned)__cvta_generic_to_shared(smem);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(s), "l"(gmem), "r"(src_bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+}  // namespace vmb

@@ -1,0 +1,75 @@
+// vmb_internal.h - host-side plumbing between the C ABI (vmb_abi.cu) and the
+// kernel launchers (cross_scan_merge.cu, full_scan.cu, mean_scan.cu).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "vmb.h"
+
+namespace vmb {
+
+// One scan problem as the ABI received it (shapes already validated).
+struct ScanArgs {
+    const void* u;
+    const void* delta;
+    const float* A;
+    const void* Bs;
+    const void* Cs;
+    const float* Dskip;
+    const float* bias;
+    void* y;
+    float* ybar;  // mean path only (may be null)
+    int B, K, D, N, L;
+    unsigned flags;
+    vmb_dtype dtype;
+    void* ws;
+    size_t ws_bytes;
+};
+
+// Execution plan of an L-chunked scan: how the (sequence, chunk) grid is cut
+// and how much workspace its look-back needs.  Deterministic for a given
+// problem, build and device, so that the workspace query and the launch agree.
+struct ScanPlan {
+    int np;            // padded state count (1, 2, 4, 8, 16)
+    int tile_rows;     // channels per CTA (full path) or 0 (mean path)
+    int tiles_per_bk;  // channel tiles per (b, k)   (full path)
+    int n_seq;         // independent sequences: channel tiles (full) or (b, k) pairs (mean)
+    int n_chunks;      // chunks along L per sequence
+    int chunk_len;     // steps per chunk (a multiple of the stage length)
+    size_t state_floats;  // floats of one chunk's published state (per array)
+    size_t ws_bytes;      // total workspace bytes
+};
+
+inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Workspace layout: [header 256 B][flags n_seq*n_chunks u32][agg_P][agg_H][inc_H]
+struct WsLayout {
+    size_t flags_off, aggP_off, aggH_off, incH_off, total;
+};
+inline WsLayout ws_layout(const ScanPlan& p) {
+    WsLayout w;
+    size_t slots = (size_t)p.n_seq * (size_t)p.n_chunks;
+    w.flags_off = 256;
+    w.aggP_off = align_up(w.flags_off + slots * 4, 256);
+    size_t arr = align_up(slots * p.state_floats * 4, 256);
+    w.aggH_off = w.aggP_off + arr;
+    w.incH_off = w.aggH_off + arr;
+    w.total = w.incH_off + arr;
+    if (p.n_chunks <= 1) w.total = 256;  // single-chunk plans only use the header
+    return w;
+}
+
+int device_sm_count();
+
+vmb_status plan_full(const ScanArgs& a, ScanPlan* plan);
+vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan);
+vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream);
+vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream);
+vmb_status launch_cross_scan(const void* x, void* xs, int B, int D, int H, int W, vmb_dtype dt,
+                             cudaStream_t stream);
+vmb_status launch_cross_merge(const void* ys, void* out, int B, int D, int H, int W, vmb_dtype dt,
+                              cudaStream_t stream);
+
+}  // namespace vmb

@@ -1,0 +1,258 @@
+"""Python binding of libvmb (include/vmb.h): argument marshalling only.
+
+Every function has the name of the C entry point it calls and takes torch
+CUDA tensors; it checks shapes and dtypes, allocates outputs with torch when
+none are given, and passes raw device pointers plus the current CUDA stream
+to the library.  All arithmetic runs in the library's kernels: there is no
+fallback, and a missing library raises at import.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libvmb.so")
+
+VMB_OK = 0
+VMB_ERR_INVALID_ARG = 1
+VMB_ERR_MISALIGNED = 2
+VMB_ERR_UNSUPPORTED = 3
+VMB_ERR_WORKSPACE = 4
+VMB_ERR_CUDA = 5
+VMB_ERR_TIMEOUT = 6
+VMB_ERR_BOUNDS = 7
+
+VMB_F32 = 0
+VMB_BF16 = 1
+
+VMB_FLAG_SOFTPLUS = 0x1
+VMB_FLAG_B_ZOH = 0x2
+VMB_FLAG_SKIP_MEAN = 0x4
+VMB_FLAG_TEST_SUPPRESS_PUBLISH = 0x40000000
+
+VMB_PATH_FULL = 0
+VMB_PATH_MEAN = 1
+
+EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb_selective_scan_fwd",
+           "vmb_mean_scan_fwd", "vmb_read_status", "vmb_status_string", "vmb_version"]
+
+
+class VmbError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+
+
+def _load() -> ctypes.CDLL:
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is not built: run `python -c \"import __graft_entry__ as g; g.build()\"`")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i, u, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint, ctypes.c_size_t
+    lib.vmb_cross_scan.argtypes = [vp, vp, i, i, i, i, i, vp]
+    lib.vmb_cross_merge.argtypes = [vp, vp, i, i, i, i, i, vp]
+    lib.vmb_scan_workspace_bytes.argtypes = [i, i, i, i, i, i, i, i]
+    lib.vmb_scan_workspace_bytes.restype = sz
+    lib.vmb_selective_scan_fwd.argtypes = [vp] * 8 + [i] * 6 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_fwd.argtypes = [vp] * 9 + [i] * 6 + [u, i, vp, sz, vp]
+    lib.vmb_read_status.argtypes = [vp, vp]
+    lib.vmb_status_string.argtypes = [i]
+    lib.vmb_status_string.restype = ctypes.c_char_p
+    lib.vmb_version.argtypes = []
+    for name in ["vmb_cross_scan", "vmb_cross_merge", "vmb_selective_scan_fwd", "vmb_mean_scan_fwd",
+                 "vmb_read_status", "vmb_version"]:
+        getattr(lib, name).restype = i
+    return lib
+
+
+lib = _load()
+
+
+def status_string(status: int) -> str:
+    return lib.vmb_status_string(int(status)).decode()
+
+
+def vmb_status_string(status: int) -> str:
+    return status_string(status)
+
+
+def vmb_version() -> int:
+    return lib.vmb_version()
+
+
+def _check(status: int, where: str):
+    if status != VMB_OK:
+        raise VmbError(status, where)
+
+
+def _dtype_code(t: torch.dtype) -> int:
+    if t == torch.float32:
+        return VMB_F32
+    if t == torch.bfloat16:
+        return VMB_BF16
+    raise TypeError(f"unsupported dtype {t} (float32 or bfloat16)")
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else ctypes.c_void_p(0)
+
+
+def _dev(t: torch.Tensor, name: str):
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+# ---------------------------------------------------------------- cross-scan / merge
+
+
+def vmb_cross_scan(x: torch.Tensor, xs: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """x [B, D, H, W] -> xs [B, 4, D, H*W] (bit-exact permutation)."""
+    _dev(x, "x")
+    B, D, H, W = x.shape
+    if xs is None:
+        xs = torch.empty((B, 4, D, H * W), dtype=x.dtype, device=x.device)
+    _dev(xs, "xs")
+    if xs.shape != (B, 4, D, H * W) or xs.dtype != x.dtype:
+        raise ValueError("xs must be [B, 4, D, H*W] with the dtype of x")
+    _check(lib.vmb_cross_scan(_ptr(x), _ptr(xs), B, D, H, W, _dtype_code(x.dtype), _stream(stream)),
+           "vmb_cross_scan")
+    return xs
+
+
+def vmb_cross_merge(ys: torch.Tensor, H: int, W: int, out: torch.Tensor | None = None,
+                    stream=None) -> torch.Tensor:
+    """ys [B, 4, D, H*W] -> out [B, D, H, W]."""
+    _dev(ys, "ys")
+    B, K, D, L = ys.shape
+    if K != 4 or L != H * W:
+        raise ValueError("ys must be [B, 4, D, H*W]")
+    if out is None:
+        out = torch.empty((B, D, H, W), dtype=ys.dtype, device=ys.device)
+    _dev(out, "out")
+    if out.shape != (B, D, H, W) or out.dtype != ys.dtype:
+        raise ValueError("out must be [B, D, H, W] with the dtype of ys")
+    _check(lib.vmb_cross_merge(_ptr(ys), _ptr(out), B, D, H, W, _dtype_code(ys.dtype), _stream(stream)),
+           "vmb_cross_merge")
+    return out
+
+
+# ---------------------------------------------------------------- scans
+
+
+def vmb_scan_workspace_bytes(path: int, B: int, K: int, D: int, N: int, H: int, W: int,
+                             dtype: torch.dtype = torch.float32) -> int:
+    return int(lib.vmb_scan_workspace_bytes(path, B, K, D, N, H, W, _dtype_code(dtype)))
+
+
+class Workspace:
+    """A zero-initialised device workspace that grows on demand (one per device).
+
+    The library keeps a workspace ready for the next call by itself; only a
+    newly allocated buffer needs zero-filling, which torch.zeros does."""
+
+    def __init__(self):
+        self._bufs = {}
+        self._lock = threading.Lock()
+
+    def get(self, nbytes: int, device: torch.device) -> torch.Tensor:
+        key = (device.type, device.index)
+        with self._lock:
+            buf = self._bufs.get(key)
+            if buf is None or buf.numel() < nbytes:
+                n = max(nbytes, 256)
+                n = (n + 255) // 256 * 256
+                buf = torch.zeros(n, dtype=torch.uint8, device=device)
+                self._bufs[key] = buf
+            return buf
+
+
+_default_ws = Workspace()
+
+
+def _scan_shapes(u, delta, A, Bs, Cs, Dskip, delta_bias, H, W):
+    for t, n in [(u, "u"), (delta, "delta"), (A, "A"), (Bs, "Bs"), (Cs, "Cs"), (Dskip, "Dskip"),
+                 (delta_bias, "delta_bias")]:
+        _dev(t, n)
+    B, K, D, L = u.shape
+    N = Bs.shape[2]
+    if L != H * W:
+        raise ValueError("u must be [B, K, D, H*W]")
+    if delta.shape != u.shape or Bs.shape != (B, K, N, L) or Cs.shape != (B, K, N, L):
+        raise ValueError("delta [B,K,D,L], Bs and Cs [B,K,N,L] expected")
+    if len({u.dtype, delta.dtype, Bs.dtype, Cs.dtype}) != 1:
+        raise ValueError("u, delta, Bs, Cs must share one dtype")
+    if A.shape != (K * D, N) or Dskip.shape != (K * D,) or delta_bias.shape != (K * D,):
+        raise ValueError("A [K*D, N], Dskip [K*D], delta_bias [K*D] expected")
+    if A.dtype != torch.float32 or Dskip.dtype != torch.float32 or delta_bias.dtype != torch.float32:
+        raise ValueError("A, Dskip, delta_bias must be float32")
+    return B, K, D, N, L
+
+
+def vmb_selective_scan_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, H: int, W: int, *,
+                           y=None, flags: int = VMB_FLAG_SOFTPLUS, workspace=None,
+                           stream=None) -> torch.Tensor:
+    """Full-channel selective scan: y [B, K, D, H*W] (dtype of u)."""
+    B, K, D, N, L = _scan_shapes(u, delta, A, Bs, Cs, Dskip, delta_bias, H, W)
+    if y is None:
+        y = torch.empty_like(u)
+    _dev(y, "y")
+    if y.shape != u.shape or y.dtype != u.dtype:
+        raise ValueError("y must match u")
+    ws_bytes = vmb_scan_workspace_bytes(VMB_PATH_FULL, B, K, D, N, H, W, u.dtype)
+    if workspace is None:
+        workspace = _default_ws.get(ws_bytes, u.device)
+    _check(lib.vmb_selective_scan_fwd(_ptr(u), _ptr(delta), _ptr(A), _ptr(Bs), _ptr(Cs), _ptr(Dskip),
+                                      _ptr(delta_bias), _ptr(y), B, K, D, N, H, W, flags,
+                                      _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
+                                      _stream(stream)), "vmb_selective_scan_fwd")
+    return y
+
+
+def vmb_mean_scan_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, H: int, W: int, *,
+                      y=None, ybar=None, want_ybar: bool = False, flags: int = VMB_FLAG_SOFTPLUS,
+                      workspace=None, stream=None):
+    """VMeanba channel-mean scan: returns (y [B, K, D, L], ybar [B, K, L] fp32 or None)."""
+    B, K, D, N, L = _scan_shapes(u, delta, A, Bs, Cs, Dskip, delta_bias, H, W)
+    if y is None:
+        y = torch.empty_like(u)
+    _dev(y, "y")
+    if y.shape != u.shape or y.dtype != u.dtype:
+        raise ValueError("y must match u")
+    if ybar is None and want_ybar:
+        ybar = torch.empty((B, K, L), dtype=torch.float32, device=u.device)
+    if ybar is not None:
+        _dev(ybar, "ybar")
+        if ybar.shape != (B, K, L) or ybar.dtype != torch.float32:
+            raise ValueError("ybar must be float32 [B, K, L]")
+    ws_bytes = vmb_scan_workspace_bytes(VMB_PATH_MEAN, B, K, D, N, H, W, u.dtype)
+    if workspace is None:
+        workspace = _default_ws.get(ws_bytes, u.device)
+    _check(lib.vmb_mean_scan_fwd(_ptr(u), _ptr(delta), _ptr(A), _ptr(Bs), _ptr(Cs), _ptr(Dskip),
+                                 _ptr(delta_bias), _ptr(y), _ptr(ybar), B, K, D, N, H, W, flags,
+                                 _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
+                                 _stream(stream)), "vmb_mean_scan_fwd")
+    return y, ybar
+
+
+def vmb_read_status(workspace=None, device=None, stream=None) -> int:
+    """Synchronise and return (then clear) the device error word of a workspace."""
+    if workspace is None:
+        dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+        workspace = _default_ws.get(256, dev)
+    return int(lib.vmb_read_status(_ptr(workspace), _stream(stream)))
+
+
+def default_workspace(device=None) -> torch.Tensor:
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    return _default_ws.get(256, dev)

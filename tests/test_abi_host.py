@@ -1,0 +1,107 @@
+"""The C ABI without a GPU: the library loads, exports what include/vmb.h
+declares, and rejects invalid arguments before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "vmb.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2412_16602_gb300 import _build
+    path = _build.build()
+    lib = ctypes.CDLL(path)
+    vp, i, u, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint, ctypes.c_size_t
+    lib.vmb_cross_scan.argtypes = [vp, vp, i, i, i, i, i, vp]
+    lib.vmb_cross_merge.argtypes = [vp, vp, i, i, i, i, i, vp]
+    lib.vmb_scan_workspace_bytes.argtypes = [i] * 8
+    lib.vmb_scan_workspace_bytes.restype = sz
+    lib.vmb_selective_scan_fwd.argtypes = [vp] * 8 + [i] * 6 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_fwd.argtypes = [vp] * 9 + [i] * 6 + [u, i, vp, sz, vp]
+    lib.vmb_status_string.argtypes = [i]
+    lib.vmb_status_string.restype = ctypes.c_char_p
+    lib.vmb_read_status.argtypes = [vp, vp]
+    return lib
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(vmb_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_four_calls():
+    names = declared_functions()
+    for n in ["vmb_cross_scan", "vmb_selective_scan_fwd", "vmb_mean_scan_fwd", "vmb_cross_merge"]:
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), f"{name} declared in vmb.h but not exported"
+
+
+def test_status_strings(lib):
+    for s in range(8):
+        assert lib.vmb_status_string(s)
+    assert lib.vmb_status_string(99) == b"unknown status"
+    assert lib.vmb_version() >= 100
+
+
+FAKE = 0x10000  # never dereferenced: validation fails before any device access
+S = 0  # null stream
+
+
+def scan_call(lib, fn, *, ptrs=None, B=1, K=4, D=8, N=16, H=4, W=4, flags=1, dtype=0,
+              ws=0x100000, ws_bytes=1 << 20, mean=False):
+    p = [FAKE] * 8 if ptrs is None else ptrs
+    if mean:
+        return fn(*p[:8], 0, B, K, D, N, H, W, flags, dtype, ws, ws_bytes, S)
+    return fn(*p[:8], B, K, D, N, H, W, flags, dtype, ws, ws_bytes, S)
+
+
+def test_cross_scan_validation(lib):
+    assert lib.vmb_cross_scan(FAKE, FAKE, -1, 4, 4, 4, 0, S) == 1        # negative size
+    assert lib.vmb_cross_scan(0, FAKE, 1, 4, 4, 4, 0, S) == 1            # null input
+    assert lib.vmb_cross_scan(FAKE, FAKE, 1, 4, 4, 4, 7, S) == 1         # bad dtype
+    assert lib.vmb_cross_scan(FAKE + 2, FAKE, 1, 4, 4, 4, 0, S) == 2     # fp32 misaligned
+    assert lib.vmb_cross_scan(FAKE + 2, FAKE, 1, 4, 4, 4, 1, S) != 2     # bf16: 2-byte aligned is fine
+    assert lib.vmb_cross_scan(0, 0, 0, 4, 4, 4, 0, S) == 0               # empty problem: no launch
+    assert lib.vmb_cross_merge(FAKE, 0, 1, 4, 4, 4, 0, S) == 1
+    assert lib.vmb_cross_merge(0, 0, 2, 3, 0, 5, 0, S) == 0
+
+
+@pytest.mark.parametrize("mean", [False, True])
+def test_scan_validation(lib, mean):
+    fn = lib.vmb_mean_scan_fwd if mean else lib.vmb_selective_scan_fwd
+    assert scan_call(lib, fn, B=-1, mean=mean) == 1
+    assert scan_call(lib, fn, N=0, mean=mean) == 1
+    assert scan_call(lib, fn, N=17, mean=mean) == 3                      # unsupported state size
+    assert scan_call(lib, fn, flags=0x100, mean=mean) == 1               # unknown flag
+    assert scan_call(lib, fn, dtype=5, mean=mean) == 1
+    assert scan_call(lib, fn, ptrs=[FAKE] * 7 + [0], mean=mean) == 1     # null output
+    assert scan_call(lib, fn, ptrs=[FAKE + 2] + [FAKE] * 7, mean=mean) == 2  # misaligned fp32
+    assert scan_call(lib, fn, ws=0, mean=mean) == 4                      # no workspace
+    assert scan_call(lib, fn, ws=FAKE + 16, mean=mean) == 2              # workspace not 256-B aligned
+    assert scan_call(lib, fn, ptrs=[0] * 8, B=0, ws=0, mean=mean) == 0   # empty problem
+    assert scan_call(lib, fn, ptrs=[0] * 8, H=0, ws=0, mean=mean) == 0
+
+
+def test_skip_mean_flag_is_mean_only(lib):
+    assert scan_call(lib, lib.vmb_selective_scan_fwd, flags=0x5) == 1
+
+
+def test_workspace_query_invalid_and_empty(lib):
+    assert lib.vmb_scan_workspace_bytes(7, 1, 4, 8, 16, 4, 4, 0) == 0
+    assert lib.vmb_scan_workspace_bytes(0, 1, 4, 8, 17, 4, 4, 0) == 0
+    assert lib.vmb_scan_workspace_bytes(0, -1, 4, 8, 16, 4, 4, 0) == 0
+    assert lib.vmb_scan_workspace_bytes(1, 0, 4, 8, 16, 4, 4, 0) == 256
+
+
+def test_read_status_rejects_null(lib):
+    assert lib.vmb_read_status(0, 0) == 1
+    assert lib.vmb_read_status(FAKE + 8, 0) == 2

@@ -1,0 +1,170 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle.
+
+Index work (cross-scan) is compared bit for bit; floating-point outputs within
+rel-L2 <= 1e-5 and max-abs <= 1e-4 max|y| (fp32 storage) or rel-L2 <= 1e-2
+(bf16 storage).  Shapes span several tiles and chunks and ragged tails.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+from tests.parity import check, to_device, to_numpy
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():  # pragma: no cover - collected on CPU, skipped by marker
+    pytest.skip("needs a GPU", allow_module_level=True)
+
+import paper_2412_16602_gb300 as vmb  # noqa: E402
+
+DEV = torch.device("cuda", 0)
+
+
+def gpu_step(inp, flags=vmb.VMB_FLAG_SOFTPLUS, mean_flags=None):
+    g = to_device(inp, DEV)
+    wl = inp.wl
+    xs = vmb.vmb_cross_scan(g["x"])
+    yf = vmb.vmb_selective_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W,
+                                    flags=flags)
+    ym, ybar = vmb.vmb_mean_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W,
+                                     want_ybar=True, flags=flags if mean_flags is None else mean_flags)
+    of = vmb.vmb_cross_merge(yf, wl.H, wl.W)
+    om = vmb.vmb_cross_merge(ym, wl.H, wl.W)
+    assert vmb.vmb_read_status() == vmb.VMB_OK
+    return {k: v for k, v in dict(xs=xs, yf=yf, ym=ym, ybar=ybar, of=of, om=om).items()}
+
+
+SHAPES = [
+    # (B, D, N, H, W, dtype)
+    (1, 192, 16, 14, 14, "f32"),     # the small SS2D workload
+    (2, 40, 16, 9, 11, "f32"),       # ragged channel tile, odd L = 99 (element-wise path)
+    (1, 70, 16, 32, 40, "f32"),      # L = 1280: several stages and L-chunks
+    (3, 33, 5, 7, 7, "f32"),         # odd N (padded states), L = 49
+    (2, 64, 1, 12, 16, "f32"),       # N = 1
+    (2, 24, 8, 8, 8, "f32"),         # N = 8
+    (1, 48, 3, 5, 13, "bf16"),       # bf16, odd L
+    (2, 96, 16, 16, 16, "bf16"),     # bf16, aligned rows
+    (1, 8, 16, 64, 64, "f32"),       # few channels, long sequence: many chunks
+]
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=[f"B{s[0]}_D{s[1]}_N{s[2]}_{s[3]}x{s[4]}_{s[5]}" for s in SHAPES])
+def test_ss2d_parity(shape):
+    B, D, N, H, W, dt = shape
+    wl = workloads.small_case(B=B, D=D, N=N, H=H, W=W, dtype=dt, seed=100 + D + N)
+    inp = workloads.make_inputs(wl)
+    out = gpu_step(inp)
+    u_ref, yf_ref, of_ref = oracle.ss2d_full(inp)
+    _, ym_ref, ybar_ref, om_ref = oracle.ss2d_mean(inp)
+    xs = to_numpy(out["xs"])
+    assert np.array_equal(xs, u_ref), "cross-scan must be bit-exact"
+    check(to_numpy(out["yf"]), yf_ref, dt, "full y")
+    check(to_numpy(out["of"]), of_ref, dt, "full merged")
+    check(to_numpy(out["ym"]), ym_ref, dt, "mean y")
+    check(to_numpy(out["ybar"]), ybar_ref, "f32" if dt == "f32" else "bf16", "mean ybar")
+    check(to_numpy(out["om"]), om_ref, dt, "mean merged")
+
+
+@pytest.mark.parametrize("flags", [0, vmb.VMB_FLAG_SOFTPLUS | vmb.VMB_FLAG_B_ZOH, vmb.VMB_FLAG_B_ZOH])
+def test_flag_variants(flags):
+    wl = workloads.small_case(B=1, D=50, N=16, H=10, W=12, seed=5)
+    inp = workloads.make_inputs(wl)
+    if not flags & vmb.VMB_FLAG_SOFTPLUS:
+        inp.bias[:] = np.abs(inp.bias)          # keep delta = raw + bias positive without softplus
+        inp.draw[:] = np.abs(inp.draw) * 0.05
+    out = gpu_step(inp, flags=flags)
+    kw = dict(softplus_on=bool(flags & vmb.VMB_FLAG_SOFTPLUS), b_mode=1 if flags & vmb.VMB_FLAG_B_ZOH else 0)
+    _, yf_ref, _ = oracle.ss2d_full(inp, **kw)
+    _, ym_ref, ybar_ref, _ = oracle.ss2d_mean(inp, **kw)
+    check(to_numpy(out["yf"]), yf_ref, "f32", "full y")
+    check(to_numpy(out["ym"]), ym_ref, "f32", "mean y")
+
+
+def test_skip_mean_mode():
+    wl = workloads.small_case(B=2, D=30, N=4, H=6, W=8, seed=6)
+    inp = workloads.make_inputs(wl)
+    out = gpu_step(inp, mean_flags=vmb.VMB_FLAG_SOFTPLUS | vmb.VMB_FLAG_SKIP_MEAN)
+    _, ym_ref, _, _ = oracle.ss2d_mean(inp, skip_mode=oracle.SKIP_MEAN)
+    check(to_numpy(out["ym"]), ym_ref, "f32", "mean y (skip mean)")
+
+
+def test_merge_exact_on_integers():
+    """With integer-valued inputs every partial sum is exact: the merge is bit-exact."""
+    rng = np.random.default_rng(9)
+    for (B, D, H, W) in [(2, 3, 5, 7), (1, 4, 8, 8), (3, 2, 1, 9)]:
+        ys = rng.integers(-1000, 1000, size=(B, 4, D, H * W)).astype(np.float32)
+        got = vmb.vmb_cross_merge(torch.from_numpy(ys).to(DEV), H, W).cpu().numpy()
+        assert np.array_equal(got.astype(np.float64), oracle.cross_merge(ys, H, W))
+
+
+def test_misaligned_views_take_element_path():
+    """Tensors starting 4 bytes into an allocation are valid (element-wise path)."""
+    wl = workloads.small_case(B=1, D=20, N=16, H=8, W=8, seed=8)
+    inp = workloads.make_inputs(wl)
+    g = to_device(inp, DEV)
+
+    def shifted(t):
+        buf = torch.empty(t.numel() + 1, dtype=t.dtype, device=DEV)
+        v = buf[1:].view(t.shape)
+        v.copy_(t)
+        return v
+
+    xs = vmb.vmb_cross_scan(shifted(g["x"]), shifted(torch.empty((1, 4, 20, 64), device=DEV)))
+    y = shifted(torch.empty_like(xs))
+    vmb.vmb_selective_scan_fwd(xs, shifted(g["draw"]), g["A"], shifted(g["Bs"]), shifted(g["Cs"]), g["Dskip"],
+                               g["bias"], 8, 8, y=y)
+    _, yf_ref, _ = oracle.ss2d_full(inp)
+    check(to_numpy(y), yf_ref, "f32", "full y (misaligned)")
+
+
+def test_empty_problem_is_a_noop():
+    x = torch.empty((0, 4, 5, 5), device=DEV)
+    assert vmb.vmb_cross_scan(x).shape == (0, 4, 4, 25)
+
+
+def test_workspace_reuse_over_many_calls():
+    """The look-back workspace stays consistent over repeated chunked calls."""
+    wl = workloads.small_case(B=1, D=16, N=16, H=40, W=40, seed=10)
+    inp = workloads.make_inputs(wl)
+    g = to_device(inp, DEV)
+    xs = vmb.vmb_cross_scan(g["x"])
+    ref = None
+    for _ in range(20):
+        y = vmb.vmb_selective_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], 40, 40)
+        ym, _ = vmb.vmb_mean_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], 40, 40)
+        if ref is None:
+            ref = (y.clone(), ym.clone())
+        else:
+            assert torch.equal(y, ref[0]) and torch.equal(ym, ref[1]), "results must be deterministic"
+    assert vmb.vmb_read_status() == vmb.VMB_OK
+
+
+@pytest.mark.parametrize("mean", [False, True])
+def test_lookback_wait_times_out_cleanly(mean):
+    """A chunk that never publishes makes its successors' bounded waits run out:
+    the call reports VMB_ERR_TIMEOUT and the context and workspace stay usable."""
+    wl = workloads.small_case(B=1, D=16, N=16, H=48, W=48, seed=11)
+    inp = workloads.make_inputs(wl)
+    g = to_device(inp, DEV)
+    xs = vmb.vmb_cross_scan(g["x"])
+    ws = torch.zeros(vmb.vmb_scan_workspace_bytes(1 if mean else 0, 1, 4, 16, 16, 48, 48) + 256,
+                     dtype=torch.uint8, device=DEV)
+    args = (xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], 48, 48)
+    flags = vmb.VMB_FLAG_SOFTPLUS | vmb.VMB_FLAG_TEST_SUPPRESS_PUBLISH
+    if mean:
+        vmb.vmb_mean_scan_fwd(*args, flags=flags, workspace=ws)
+    else:
+        vmb.vmb_selective_scan_fwd(*args, flags=flags, workspace=ws)
+    assert vmb.vmb_read_status(ws) == vmb.VMB_ERR_TIMEOUT
+    assert vmb.vmb_read_status(ws) == vmb.VMB_OK  # cleared
+    # the same workspace works again
+    if mean:
+        y, _ = vmb.vmb_mean_scan_fwd(*args, workspace=ws)
+        _, ref, _, _ = oracle.ss2d_mean(inp)
+    else:
+        y = vmb.vmb_selective_scan_fwd(*args, workspace=ws)
+        _, ref, _ = oracle.ss2d_full(inp)
+    assert vmb.vmb_read_status(ws) == vmb.VMB_OK
+    check(to_numpy(y), ref, "f32", "after timeout")
