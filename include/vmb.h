@@ -151,6 +151,32 @@ vmb_status vmb_mean_scan_fwd(const void* u, const void* delta, const float* A, c
                              cudaStream_t stream);
 
 /*
+ * vmb_selective_scan_fwd_noalloc - vmb_selective_scan_fwd for callers that
+ * cannot allocate device memory (for example plugin code inside a framework
+ * whose memory pool owns the device and forbids allocations of its own, or a
+ * serving loop that must not allocate once it runs).  The paper has no
+ * counterpart; this is a deployment convenience.
+ *   Same arguments and results as vmb_selective_scan_fwd, without the
+ *   workspace: the chunk-exchange scratch is a 16 MiB array built into the
+ *   library, which every GPU that loads libvmb holds until the process exits.
+ *   The call allocates nothing.
+ *   Returns VMB_ERR_WORKSPACE when the problem's plan needs more than 16 MiB of
+ *   scratch (vmb_scan_workspace_bytes(VMB_PATH_FULL, ...) > 16 MiB).
+ *   The first call made with a given device current looks up the array's
+ *   device address on that device; make that first call before any stream
+ *   capture.  Each call first clears the part of the array that must start at
+ *   zero (an asynchronous memset on `stream`).  All calls share the one array
+ *   per device, so calls that overlap in time on the GPU (other streams, other
+ *   host threads) race and must be serialised by the caller.  Device-side wait
+ *   timeouts have no readback for this entry point.
+ */
+vmb_status vmb_selective_scan_fwd_noalloc(const void* u, const void* delta, const float* A,
+                                          const void* Bs, const void* Cs, const float* Dskip,
+                                          const float* delta_bias, void* y, int B, int K, int D,
+                                          int N, int H, int W, unsigned flags, vmb_dtype dtype,
+                                          cudaStream_t stream);
+
+/*
  * vmb_read_status - synchronise `stream`, then return and clear the device
  * error word of `workspace` (VMB_OK, VMB_ERR_TIMEOUT or VMB_ERR_BOUNDS).  A
  * device-side error leaves the outputs of that call undefined but the CUDA
