@@ -53,6 +53,8 @@ def parse():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--batch", type=int, default=None,
+                    help="override the workload's batch size (smaller captures for profiling)")
     return ap.parse_args()
 
 
@@ -306,6 +308,8 @@ def run_ours(args, wl, rank, world, local_rank):
 def main():
     args = parse()
     wl = workloads.WORKLOADS[args.workload]
+    if args.batch is not None:
+        wl = wl.replace(B=args.batch, name=f"{wl.name}@batch{args.batch}")
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

@@ -1,25 +1,29 @@
 // full_scan.cu - full-channel selective scan (App. A, Eqs. 3, 4, 6) for sm_103a.
 //
-// One CTA owns a tile of DT = 256/G channels of one (batch, direction) and one
-// chunk of the sequence.  Each thread owns one channel and NG = NP/G of its
-// NP states (G threads per channel, adjacent lanes).  The CTA streams its
-// chunk through shared memory in stages of kTS steps (cp.async, double
-// buffered); a conversion pass turns each stage into fp32, applies the
-// softplus of Eq. 6 once per element, and transposes B and C to [t][n] so a
-// thread reads its states as one vector.  Discretisation (Eq. 4) happens in
-// registers: Abar = 2^(delta * A log2 e) on the MUFU pipe, Bbar u = delta u B.
-// The per-channel output y = sum_n C_n h_n + D u is reduced across the G lanes
-// with a transposed butterfly (lane g ends with step t0+g), staged in shared
-// memory and written back with 16-byte stores.
+// One CTA owns a tile of DT channels of one (batch, direction) and one chunk
+// of the sequence.  G adjacent lanes share a channel, each owning NG = NP/G of
+// its NP states (G = 1, 2 or 4, picked by the planner from the available row
+// parallelism).  The chunk streams through shared memory in stages of TS
+// steps (cp.async, double buffered, u and delta rows padded so that the
+// per-channel 128-bit reads are free of bank conflicts).  In registers, per
+// step: delta = softplus(raw + bias) (Eq. 6, computed once per element, the G
+// lanes of a channel splitting the steps and sharing by shuffle), Abar =
+// 2^(delta A log2 e) on the MUFU pipe, Bbar u = delta u B (Eq. 4), h = Abar h
+// + Bbar u and y = C.h + D u (Eq. 3).  B and C are transposed to [t][n] per stage so a lane
+// reads its states as 128-bit vectors.  y is reduced across the G lanes by a
+// transposed butterfly, staged in shared memory and written with 16-byte
+// stores.
 //
 // Long sequences with few channels are cut into L-chunks that run in
 // parallel.  Chunks after the first run twice: a first pass computes the
-// chunk's aggregate (P = prod Abar, H = end state from h = 0) and publishes
-// it; a decoupled look-back over the predecessors' aggregates and inclusive
-// end states gives the carry-in state; the second pass recomputes the chunk
-// from that state and writes y.  The first chunk of a sequence runs once and
-// publishes its end state.  Chunk order is fixed by a ticket counter so that a
-// CTA only ever waits on CTAs that started before it; every wait is bounded.
+// chunk's aggregate (S = sum of delta, so prod Abar_n = 2^(A_n log2 e S), and
+// H = end state from h = 0) and publishes it; a decoupled look-back finds the
+// carry-in state; the second pass recomputes the chunk from that state and
+// writes y.  Chunk order follows a ticket counter, so a CTA only waits on
+// CTAs that started before it; every wait is bounded.
+#include <stdlib.h>
+#include <string.h>
+
 #include <mutex>
 #include <type_traits>
 
@@ -28,8 +32,6 @@
 
 namespace vmb {
 namespace {
-
-constexpr int kStages = 2;
 
 struct FullParams {
     const void* u;
@@ -43,67 +45,110 @@ struct FullParams {
     int K, D, N, L;
     int softplus_on;
     int tiles_per_bk, n_tiles, n_chunks, chunk_len;
-    int vec;       // rows are 16-byte aligned: cp.async 16-byte path
+    int vec;       // rows are 16-byte aligned: cp.async 16-byte path and vector stores
     int suppress;  // test hook: chunk 0 does not publish
     WsHeader* hdr;
     unsigned* flags;
-    float* aggP;
+    float* aggP;   // per chunk: sum of delta per channel (DT floats, rest unused)
     float* aggH;
     float* incH;
 };
 
 __host__ __device__ constexpr size_t a16(size_t v) { return (v + 15) / 16 * 16; }
 
-// Tile shape per state split G: 64 channels x 32-step stages when four lanes
-// share a channel (N = 16), 128 channels x 16-step stages otherwise, so that
-// a CTA's shared memory stays near 60 KB and three or more CTAs fit per SM.
-template <typename T, int NP, int G>
+// Tile shape: G lanes per channel, DT channels per CTA, TS steps per stage
+// (0: one 16-byte chunk per row), NSTG stages in the cp.async ring, and the
+// CTAs per SM the register budget is sized for.
+template <int G_, int DT_, int TS_, int NSTG_, int MINB_ = 1>
+struct Shape {
+    static constexpr int G = G_, DT = DT_, TS = TS_, NSTG = NSTG_, MINB = MINB_;
+};
+
+template <typename T, int NP, class SH>
 struct Layout {
-    static constexpr int DT = G == 4 ? 64 : 128;
+    static constexpr int G = SH::G, DT = SH::DT, NSTG = SH::NSTG, MINB = SH::MINB;
+    static constexpr int TS = SH::TS ? SH::TS : 16 / (int)sizeof(T);
     static constexpr int THREADS = DT * G;
-    static constexpr int TS = G == 4 ? 32 : 16;
-    static constexpr int TSF = TS + 1;
-    static constexpr int RAW = (2 * DT + 2 * NP) * TS;  // elements per raw stage
-    static constexpr size_t raw_bytes = a16((size_t)kStages * RAW * sizeof(T));
-    static constexpr size_t uf_off = raw_bytes;
-    static constexpr size_t df_off = uf_off + (size_t)DT * TSF * 4;
-    static constexpr size_t bf_off = a16(df_off + (size_t)DT * TSF * 4);
-    static constexpr size_t cf_off = bf_off + (size_t)TS * NP * 4;
-    static constexpr size_t ys_off = a16(cf_off + (size_t)TS * NP * 4);
-    static constexpr size_t bias_off = a16(ys_off + (size_t)DT * TS * sizeof(T));
-    static constexpr size_t bytes = bias_off + (size_t)DT * 4;
+    static constexpr int PAD = 16 / (int)sizeof(T);  // one 16-byte chunk of row padding
+    static constexpr int RS = TS + PAD;               // raw row stride (elements)
+    static constexpr int SLOT = (2 * DT + 2 * NP) * RS;
+    static constexpr size_t raw_bytes = a16((size_t)NSTG * SLOT * sizeof(T));
+    static constexpr size_t bf_off = raw_bytes;                      // 2 slots of [TS][NP] fp32
+    static constexpr size_t cf_off = bf_off + (size_t)2 * TS * NP * 4;
+    static constexpr size_t bytes = cf_off + (size_t)2 * TS * NP * 4;
+    static_assert(TS % 4 == 0 && NP % G == 0 && THREADS % 32 == 0 && NSTG >= 3, "tile shape");
     static_assert(bytes <= 100 * 1024, "full-scan tile must leave room for two CTAs per SM");
 };
 
-// Sum of yp[j] over the G lanes of one channel; lane g returns the sum for j = g.
-template <int G>
-__device__ __forceinline__ float reduce_lanes(const float (&yp)[G], int g) {
-    if constexpr (G == 1) {
-        return yp[0];
-    } else if constexpr (G == 2) {
-        float keep = g ? yp[1] : yp[0];
-        float send = g ? yp[0] : yp[1];
-        return keep + __shfl_xor_sync(0xffffffffu, send, 1);
+// Four consecutive elements of one row as fp32 (16-byte / 8-byte aligned reads).
+__device__ __forceinline__ void load4(const float* p, float (&v)[4]) {
+    const float4 q = *reinterpret_cast<const float4*>(p);
+    v[0] = q.x;
+    v[1] = q.y;
+    v[2] = q.z;
+    v[3] = q.w;
+}
+__device__ __forceinline__ void load4(const __nv_bfloat16* p, float (&v)[4]) {
+    const uint2 q = *reinterpret_cast<const uint2*>(p);
+    v[0] = __uint_as_float(q.x << 16);
+    v[1] = __uint_as_float(q.x & 0xffff0000u);
+    v[2] = __uint_as_float(q.y << 16);
+    v[3] = __uint_as_float(q.y & 0xffff0000u);
+}
+
+// NG consecutive fp32 values from shared memory (16-byte aligned when NG >= 4).
+template <int NG>
+__device__ __forceinline__ void load_states(const float* p, float (&v)[NG]) {
+    if constexpr (NG % 4 == 0) {
+#pragma unroll
+        for (int i = 0; i < NG; i += 4) {
+            const float4 q = *reinterpret_cast<const float4*>(p + i);
+            v[i] = q.x;
+            v[i + 1] = q.y;
+            v[i + 2] = q.z;
+            v[i + 3] = q.w;
+        }
     } else {
-        static_assert(G == 4, "G in {1, 2, 4}");
-        const bool hi = g & 2;
-        float k0 = hi ? yp[2] : yp[0], k1 = hi ? yp[3] : yp[1];
-        float s0 = hi ? yp[0] : yp[2], s1 = hi ? yp[1] : yp[3];
-        k0 += __shfl_xor_sync(0xffffffffu, s0, 2);
-        k1 += __shfl_xor_sync(0xffffffffu, s1, 2);
-        const bool odd = g & 1;
-        float kk = odd ? k1 : k0, ss = odd ? k0 : k1;
-        return kk + __shfl_xor_sync(0xffffffffu, ss, 1);
+#pragma unroll
+        for (int i = 0; i < NG; ++i) v[i] = p[i];
     }
 }
 
-template <typename T, int NP, int G, bool WITH_C>
-__device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t row0, size_t bcrow0,
-                                           int nrows, int l0) {
-    using LY = Layout<T, NP, G>;
-    constexpr int DT = LY::DT;
-    constexpr int kTS = LY::TS;
-    constexpr int kThreads = LY::THREADS;
+__device__ __forceinline__ float sel4(const float (&v)[4], int j) {
+    return j == 0 ? v[0] : j == 1 ? v[1] : j == 2 ? v[2] : v[3];
+}
+
+// Store n consecutive outputs of one row (n = 4, 2 or 1), vectorised when aligned.
+template <typename T, int NV>
+__device__ __forceinline__ void store_row(T* dst, const float (&v)[NV], int nvalid_here, bool vec) {
+    if (vec && nvalid_here >= NV) {
+        if constexpr (sizeof(T) == 4 && NV == 4) {
+            *reinterpret_cast<float4*>(dst) = make_float4(v[0], v[1], v[2], v[3]);
+            return;
+        } else if constexpr (sizeof(T) == 4 && NV == 2) {
+            *reinterpret_cast<float2*>(dst) = make_float2(v[0], v[1]);
+            return;
+        } else if constexpr (sizeof(T) == 2 && NV == 4) {
+            const unsigned lo = __bfloat16_as_ushort(io<T>::to(v[0])) | ((unsigned)__bfloat16_as_ushort(io<T>::to(v[1])) << 16);
+            const unsigned hi = __bfloat16_as_ushort(io<T>::to(v[2])) | ((unsigned)__bfloat16_as_ushort(io<T>::to(v[3])) << 16);
+            *reinterpret_cast<uint2*>(dst) = make_uint2(lo, hi);
+            return;
+        } else if constexpr (sizeof(T) == 2 && NV == 2) {
+            *reinterpret_cast<unsigned*>(dst) =
+                __bfloat16_as_ushort(io<T>::to(v[0])) | ((unsigned)__bfloat16_as_ushort(io<T>::to(v[1])) << 16);
+            return;
+        }
+    }
+#pragma unroll
+    for (int j = 0; j < NV; ++j)
+        if (j < nvalid_here) dst[j] = io<T>::to(v[j]);
+}
+
+template <typename T, int NP, class SH, bool WITH_C>
+__device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t row0, size_t bcrow0, int nrows,
+                                           int l0) {
+    using LY = Layout<T, NP, SH>;
+    constexpr int DT = LY::DT, kTS = LY::TS, RS = LY::RS, kThreads = LY::THREADS;
     constexpr int VE = 16 / sizeof(T);  // elements per 16-byte chunk
     constexpr int CPR = kTS / VE;       // chunks per stage row
     const T* u = static_cast<const T*>(p.u);
@@ -111,6 +156,7 @@ __device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t r
     const T* Bs = static_cast<const T*>(p.Bs);
     const T* Cs = static_cast<const T*>(p.Cs);
     const int L = p.L;
+    T* dB = dst + 2 * DT * RS;
     if (p.vec) {
         constexpr int nU = DT * CPR, nB = NP * CPR;
         constexpr int total = 2 * nU + (WITH_C ? 2 : 1) * nB;
@@ -118,24 +164,21 @@ __device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t r
             const T* src;
             T* d;
             bool ok;
-            int r, ch;
             if (i < 2 * nU) {
                 const int j = i < nU ? i : i - nU;
-                r = j / CPR;
-                ch = j % CPR;
+                const int r = j / CPR, ch = j % CPR;
                 const T* base = i < nU ? u : dl;
                 ok = r < nrows && l0 + ch * VE < L;
                 src = ok ? base + ((row0 + r) * (size_t)L + l0 + ch * VE) : base;
-                d = dst + (i < nU ? 0 : DT * kTS) + r * kTS + ch * VE;
+                d = dst + (i < nU ? 0 : DT * RS) + r * RS + ch * VE;
             } else {
                 const int i2 = i - 2 * nU;
                 const int j = i2 < nB ? i2 : i2 - nB;
-                r = j / CPR;
-                ch = j % CPR;
+                const int r = j / CPR, ch = j % CPR;
                 const T* base = i2 < nB ? Bs : Cs;
                 ok = r < p.N && l0 + ch * VE < L;
                 src = ok ? base + ((bcrow0 + r) * (size_t)L + l0 + ch * VE) : base;
-                d = dst + 2 * DT * kTS + (i2 < nB ? 0 : NP * kTS) + r * kTS + ch * VE;
+                d = dB + (i2 < nB ? 0 : NP * RS) + r * RS + ch * VE;
             }
             cp_async16(d, src, ok ? 16 : 0);
         }
@@ -149,35 +192,30 @@ __device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t r
                 const int r = j / kTS, t = j % kTS;
                 const T* base = i < nU ? u : dl;
                 if (r < nrows && l0 + t < L) v = base[(row0 + r) * (size_t)L + l0 + t];
+                dst[(i < nU ? 0 : DT * RS) + r * RS + t] = v;
             } else {
                 const int i2 = i - 2 * nU;
                 const int j = i2 < nB ? i2 : i2 - nB;
                 const int r = j / kTS, t = j % kTS;
                 const T* base = i2 < nB ? Bs : Cs;
                 if (r < p.N && l0 + t < L) v = base[(bcrow0 + r) * (size_t)L + l0 + t];
+                dB[(i2 < nB ? 0 : NP * RS) + r * RS + t] = v;
             }
-            dst[i] = v;
         }
     }
 }
 
-template <typename T, int NP, int G, bool ZOH>
-__global__ void __launch_bounds__(Layout<T, NP, G>::THREADS) full_scan_kernel(const FullParams p) {
-    using LY = Layout<T, NP, G>;
-    constexpr int kThreads = LY::THREADS;
-    constexpr int kTS = LY::TS;
+template <typename T, int NP, class SH, bool ZOH>
+__global__ void __launch_bounds__(Layout<T, NP, SH>::THREADS, Layout<T, NP, SH>::MINB)
+    full_scan_kernel(const FullParams p) {
+    using LY = Layout<T, NP, SH>;
+    constexpr int kThreads = LY::THREADS, kTS = LY::TS, RS = LY::RS, SLOT = LY::SLOT, DT = LY::DT;
+    constexpr int G = LY::G, NSTG = LY::NSTG;
     constexpr int NG = NP / G;
-    constexpr int DT = LY::DT;
-    constexpr int TSF = LY::TSF;
-    constexpr int RAW = LY::RAW;
     extern __shared__ __align__(16) unsigned char smem[];
     T* raw = reinterpret_cast<T*>(smem);
-    float* uf = reinterpret_cast<float*>(smem + LY::uf_off);
-    float* df = reinterpret_cast<float*>(smem + LY::df_off);
     float* bfm = reinterpret_cast<float*>(smem + LY::bf_off);
     float* cfm = reinterpret_cast<float*>(smem + LY::cf_off);
-    T* ys = reinterpret_cast<T*>(smem + LY::ys_off);
-    float* s_bias = reinterpret_cast<float*>(smem + LY::bias_off);
     __shared__ unsigned s_misc[2];
 
     const int tid = threadIdx.x;
@@ -215,9 +253,7 @@ __global__ void __launch_bounds__(Layout<T, NP, G>::THREADS) full_scan_kernel(co
     const size_t row0 = (size_t)bk * p.D + d0;
     const size_t bcrow0 = (size_t)bk * p.N;
 
-    for (int i = tid; i < DT; i += kThreads) s_bias[i] = i < nrows ? p.bias[(size_t)k * p.D + d0 + i] : 0.0f;
-
-    float A2[NG], Ar[NG], h[NG], P[NG];
+    float A2[NG], Ar[NG], h[NG];
 #pragma unroll
     for (int i = 0; i < NG; ++i) {
         const int n = g * NG + i;
@@ -225,131 +261,141 @@ __global__ void __launch_bounds__(Layout<T, NP, G>::THREADS) full_scan_kernel(co
         A2[i] = a * kLog2e;
         Ar[i] = a;
         h[i] = 0.0f;
-        P[i] = 1.0f;
     }
     const float dsk = cval ? p.Dskip[(size_t)k * p.D + d] : 0.0f;
+    const float bias = cval ? p.bias[(size_t)k * p.D + d] : 0.0f;
     const int l_begin = chunk * p.chunk_len;
     const int l_end = min(p.L, l_begin + p.chunk_len);
     const int nst = (l_end - l_begin + kTS - 1) / kTS;
-    __syncthreads();
+    T* yrow = static_cast<T*>(p.y) + (row0 + c) * (size_t)p.L;
+    float ssum = 0.0f;  // sum of delta over the chunk (first pass)
 
-    // One pass over the chunk.  PH2 = false: aggregate only (h from 0, P = prod Abar).
+    // One pass over the chunk.  PH2 = false: aggregate only (h from 0, S).
     // PH2 = true: recurrence from the carried-in h, output y.
+    // Ring of NSTG raw stages, prefetch distance NSTG - 1; B and C of stage s+1
+    // are transposed to [t][n] while stage s is computed; one barrier per stage.
+    // Steps past the end of the sequence (last stage only) run on zero-filled
+    // inputs; their outputs are not stored and the final state is not used.
     auto pass = [&](auto ph2_tag) {
         constexpr bool PH2 = decltype(ph2_tag)::value;
-        load_stage<T, NP, G, PH2>(p, raw, row0, bcrow0, nrows, l_begin);
-        cp_async_commit();
+        auto transpose = [&](int st) {
+            const T* rb = raw + (st % NSTG) * SLOT + 2 * DT * RS;
+            const T* rc = rb + NP * RS;
+            float* bo = bfm + (st & 1) * kTS * NP;
+            float* co = cfm + (st & 1) * kTS * NP;
+            for (int i = tid; i < NP * kTS; i += kThreads) {
+                const int n = i % NP, t = i / NP;
+                bo[t * NP + n] = io<T>::cvt(rb[n * RS + t]);
+                if constexpr (PH2) co[t * NP + n] = io<T>::cvt(rc[n * RS + t]);
+            }
+        };
+#pragma unroll
+        for (int q = 0; q < NSTG - 1; ++q) {
+            if (q < nst) load_stage<T, NP, SH, PH2>(p, raw + q * SLOT, row0, bcrow0, nrows, l_begin + q * kTS);
+            cp_async_commit();
+        }
+        cp_async_wait<NSTG - 2>();
+        __syncthreads();
+        transpose(0);
         for (int s = 0; s < nst; ++s) {
             const int l0 = l_begin + s * kTS;
-            if (s + 1 < nst) load_stage<T, NP, G, PH2>(p, raw + ((s + 1) & 1) * RAW, row0, bcrow0, nrows, l0 + kTS);
+            const int nvalid = min(kTS, l_end - l0);
+            cp_async_wait<NSTG - 3>();  // stages <= s+1 have landed
+            __syncthreads();
+            if (s + NSTG - 1 < nst)
+                load_stage<T, NP, SH, PH2>(p, raw + ((s + NSTG - 1) % NSTG) * SLOT, row0, bcrow0, nrows,
+                                           l0 + (NSTG - 1) * kTS);
             cp_async_commit();
-            cp_async_wait<1>();
-            __syncthreads();
-            // ---- conversion: fp32, softplus(delta + bias), B/C transposed to [t][n]
-            {
-                const T* ru = raw + (s & 1) * RAW;
-                const T* rd = ru + DT * kTS;
-                const T* rb = rd + DT * kTS;
-                const T* rc = rb + NP * kTS;
-                const int nvalid = min(kTS, l_end - l0);
-                for (int i = tid; i < DT * kTS; i += kThreads) {
-                    const int r = i / kTS, t = i % kTS;
-                    const bool ok = r < nrows && t < nvalid;
-                    const float v = io<T>::cvt(rd[i]) + s_bias[r];
-                    const float dv = p.softplus_on ? softplus(v) : v;
-                    uf[r * TSF + t] = ok ? io<T>::cvt(ru[i]) : 0.0f;
-                    df[r * TSF + t] = ok ? dv : 0.0f;
-                }
-                for (int i = tid; i < NP * kTS; i += kThreads) {
-                    const int n = i / kTS, t = i % kTS;
-                    const bool ok = n < p.N && t < nvalid;
-                    bfm[t * NP + n] = ok ? io<T>::cvt(rb[i]) : 0.0f;
-                    if constexpr (PH2) cfm[t * NP + n] = ok ? io<T>::cvt(rc[i]) : 0.0f;
-                }
-            }
-            __syncthreads();
-            // ---- recurrence over the stage
+            if (s + 1 < nst) transpose(s + 1);
+            const T* ru = raw + (s % NSTG) * SLOT;
+            const T* rd = ru + DT * RS;
+            const float* bst = bfm + (s & 1) * kTS * NP;
+            const float* cst = cfm + (s & 1) * kTS * NP;
 #pragma unroll 1
-            for (int t0 = 0; t0 < kTS; t0 += G) {
-                float yp[G];
+            for (int t0 = 0; t0 < kTS; t0 += 4) {
+                float u4[4], r4[4], dl4[4];
+                load4(ru + c * RS + t0, u4);
+                load4(rd + c * RS + t0, r4);
+                // softplus once per element; the G lanes of a channel split the steps
+                if constexpr (G == 1) {
 #pragma unroll
-                for (int j = 0; j < G; ++j) {
+                    for (int j = 0; j < 4; ++j) {
+                        const float v = r4[j] + bias;
+                        dl4[j] = p.softplus_on ? softplus(v) : v;
+                    }
+                } else if constexpr (G == 2) {
+                    const float va = (g ? r4[1] : r4[0]) + bias, vb = (g ? r4[3] : r4[2]) + bias;
+                    const float a = p.softplus_on ? softplus(va) : va;
+                    const float b = p.softplus_on ? softplus(vb) : vb;
+                    const float oa = __shfl_xor_sync(0xffffffffu, a, 1);
+                    const float ob = __shfl_xor_sync(0xffffffffu, b, 1);
+                    dl4[0] = g ? oa : a;
+                    dl4[1] = g ? a : oa;
+                    dl4[2] = g ? ob : b;
+                    dl4[3] = g ? b : ob;
+                } else {
+                    const float v = sel4(r4, g) + bias;
+                    const float a = p.softplus_on ? softplus(v) : v;
+                    const int base = (threadIdx.x & 31) & ~3;
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) dl4[j] = __shfl_sync(0xffffffffu, a, base + j);
+                }
+                float yp[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
                     const int t = t0 + j;
-                    const float dlt = df[c * TSF + t];
-                    const float uu = uf[c * TSF + t];
+                    const float dlt = dl4[j];
+                    const float uu = u4[j];
+                    if constexpr (!PH2) ssum += (t < nvalid) ? dlt : 0.0f;
                     const float du = dlt * uu;
                     float Bv[NG], Cv[NG];
+                    load_states<NG>(bst + t * NP + g * NG, Bv);
+                    if constexpr (PH2) load_states<NG>(cst + t * NP + g * NG, Cv);
+                    // scalar FP32 (on GB300 the packed f32x2 forms issue slower in this
+                    // MUFU-heavy mix); four accumulators keep the y chain short
+                    float ya[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
                     for (int i = 0; i < NG; ++i) {
-                        Bv[i] = bfm[t * NP + g * NG + i];
-                        if constexpr (PH2) Cv[i] = cfm[t * NP + g * NG + i];
-                    }
-                    float ya = 0.0f, yb = 0.0f;
-                    if constexpr (!ZOH && NG % 2 == 0) {
-#pragma unroll
-                        for (int i = 0; i < NG; i += 2) {
-                            const float2 x = __fmul2_rn(make_float2(dlt, dlt), make_float2(A2[i], A2[i + 1]));
-                            const float2 a = make_float2(ex2(x.x), ex2(x.y));
-                            const float2 bb = __fmul2_rn(make_float2(du, du), make_float2(Bv[i], Bv[i + 1]));
-                            const float2 hh = __ffma2_rn(a, make_float2(h[i], h[i + 1]), bb);
-                            h[i] = hh.x;
-                            h[i + 1] = hh.y;
-                            if constexpr (PH2) {
-                                const float2 acc = __ffma2_rn(make_float2(Cv[i], Cv[i + 1]), hh, make_float2(ya, yb));
-                                ya = acc.x;
-                                yb = acc.y;
-                            } else {
-                                const float2 pp = __fmul2_rn(make_float2(P[i], P[i + 1]), a);
-                                P[i] = pp.x;
-                                P[i + 1] = pp.y;
-                            }
+                        float a, bb;
+                        if constexpr (ZOH) {
+                            const float em1 = expm1f(dlt * Ar[i]);
+                            a = 1.0f + em1;
+                            bb = (Ar[i] != 0.0f ? em1 / Ar[i] : dlt) * Bv[i] * uu;
+                        } else {
+                            a = ex2(dlt * A2[i]);
+                            bb = du * Bv[i];
                         }
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < NG; ++i) {
-                            float a, bb;
-                            if constexpr (ZOH) {
-                                const float em1 = expm1f(dlt * Ar[i]);
-                                a = 1.0f + em1;
-                                bb = (Ar[i] != 0.0f ? em1 / Ar[i] : dlt) * Bv[i] * uu;
-                            } else {
-                                a = ex2(dlt * A2[i]);
-                                bb = du * Bv[i];
-                            }
-                            h[i] = fmaf(a, h[i], bb);
-                            if constexpr (PH2) {
-                                if (i & 1) yb = fmaf(Cv[i], h[i], yb);
-                                else ya = fmaf(Cv[i], h[i], ya);
-                            } else {
-                                P[i] *= a;
-                            }
-                        }
+                        h[i] = fmaf(a, h[i], bb);
+                        if constexpr (PH2) ya[i & 3] = fmaf(Cv[i], h[i], ya[i & 3]);
                     }
-                    yp[j] = ya + yb;
+                    yp[j] = (ya[0] + ya[1]) + (ya[2] + ya[3]);
                 }
                 if constexpr (PH2) {
-                    const float r = reduce_lanes<G>(yp, g);
-                    const int t = t0 + g;
-                    ys[c * kTS + t] = io<T>::to(fmaf(dsk, uf[c * TSF + t], r));
-                }
-            }
-            // ---- write the stage's outputs
-            if constexpr (PH2) {
-                __syncthreads();
-                T* y = static_cast<T*>(p.y);
-                const int nvalid = min(kTS, l_end - l0);
-                if (p.vec) {
-                    constexpr int VE = 16 / sizeof(T), CPR = kTS / VE;
-                    for (int i = tid; i < DT * CPR; i += kThreads) {
-                        const int r = i / CPR, ch = i % CPR;
-                        if (r < nrows && ch * VE < nvalid)
-                            *reinterpret_cast<uint4*>(y + (row0 + r) * (size_t)p.L + l0 + ch * VE) =
-                                *reinterpret_cast<const uint4*>(ys + r * kTS + ch * VE);
-                    }
-                } else {
-                    for (int i = tid; i < DT * kTS; i += kThreads) {
-                        const int r = i / kTS, t = i % kTS;
-                        if (r < nrows && t < nvalid) y[(row0 + r) * (size_t)p.L + l0 + t] = ys[i];
+                    // y = sum over the channel's lanes + D u, stored straight from registers
+                    if constexpr (G == 1) {
+                        float o[4];
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) o[j] = fmaf(dsk, u4[j], yp[j]);
+                        if (cval) store_row<T, 4>(yrow + l0 + t0, o, nvalid - t0, p.vec);
+                    } else if constexpr (G == 2) {
+                        // lane g keeps steps 2g and 2g+1
+                        const float k0 = g ? yp[2] : yp[0], k1 = g ? yp[3] : yp[1];
+                        const float s0 = g ? yp[0] : yp[2], s1 = g ? yp[1] : yp[3];
+                        float o[2];
+                        o[0] = fmaf(dsk, g ? u4[2] : u4[0], k0 + __shfl_xor_sync(0xffffffffu, s0, 1));
+                        o[1] = fmaf(dsk, g ? u4[3] : u4[1], k1 + __shfl_xor_sync(0xffffffffu, s1, 1));
+                        if (cval) store_row<T, 2>(yrow + l0 + t0 + 2 * g, o, nvalid - t0 - 2 * g, p.vec);
+                    } else {
+                        const bool hi = g & 2;
+                        float k0 = hi ? yp[2] : yp[0], k1 = hi ? yp[3] : yp[1];
+                        const float s0 = hi ? yp[0] : yp[2], s1 = hi ? yp[1] : yp[3];
+                        k0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+                        k1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+                        const bool odd = g & 1;
+                        const float kk = odd ? k1 : k0, ss = odd ? k0 : k1;
+                        float o[1];
+                        o[0] = fmaf(dsk, sel4(u4, g), kk + __shfl_xor_sync(0xffffffffu, ss, 1));
+                        if (cval) store_row<T, 1>(yrow + l0 + t0 + g, o, nvalid - t0 - g, false);
                     }
                 }
             }
@@ -363,32 +409,24 @@ __global__ void __launch_bounds__(Layout<T, NP, G>::THREADS) full_scan_kernel(co
     if (chunked && chunk > 0) {
         pass(std::false_type{});
         const size_t slot = (size_t)tile * p.n_chunks + chunk;
+        if (g == 0) p.aggP[slot * sfl + c] = ssum;
 #pragma unroll
-        for (int i = 0; i < NG; ++i) {
-            p.aggP[slot * sfl + my_off + i] = P[i];
-            p.aggH[slot * sfl + my_off + i] = h[i];
-        }
+        for (int i = 0; i < NG; ++i) p.aggH[slot * sfl + my_off + i] = h[i];
         __threadfence();
         __syncthreads();
         if (tid == 0) st_release(&p.flags[slot], flag_word(gen, kFlagAggregate));
         // Decoupled look-back: walk back until a predecessor's inclusive state is
         // published, then fold the aggregates after it left to right,
-        // h <- P_m h + H_m.  Every inclusive state is defined by this same left
-        // fold from chunk 0, so the carry is bit-identical whichever predecessor
-        // the walk stops at (results do not depend on scheduling).
-        int found = -1;
-        for (int j = chunk - 1; j >= 0; --j) {
-            const size_t sj = (size_t)tile * p.n_chunks + j;
-            if (tid == 0) s_misc[0] = wait_flag(&p.flags[sj], gen, p.hdr, (unsigned)tile, (unsigned)j);
-            __syncthreads();
-            const unsigned kind = s_misc[0];
-            __syncthreads();
-            if (kind == kFlagInclusive) {
-                found = j;
-                break;
-            }
-            if (kind != kFlagAggregate) break;  // wait gave up: error already recorded
+        // h <- 2^(A_n log2 e S_m) h + H_m.  Every inclusive state is defined by
+        // this same left fold from chunk 0, so the carry is bit-identical
+        // whichever predecessor the walk stops at (results do not depend on
+        // scheduling).
+        if (tid < 32) {
+            const int f = lookback_find(p.flags + (size_t)tile * p.n_chunks, chunk, gen, p.hdr, (unsigned)tile);
+            if (tid == 0) s_misc[0] = (unsigned)f;
         }
+        __syncthreads();
+        const int found = (int)s_misc[0];
         float RH[NG];
 #pragma unroll
         for (int i = 0; i < NG; ++i) RH[i] = 0.0f;
@@ -398,15 +436,16 @@ __global__ void __launch_bounds__(Layout<T, NP, G>::THREADS) full_scan_kernel(co
             for (int i = 0; i < NG; ++i) RH[i] = ld_cg(&p.incH[sf * sfl + my_off + i]);
             for (int m = found + 1; m < chunk; ++m) {
                 const size_t sm = (size_t)tile * p.n_chunks + m;
+                const float sm_s = ld_cg(&p.aggP[sm * sfl + c]);
 #pragma unroll
                 for (int i = 0; i < NG; ++i)
-                    RH[i] = fmaf(ld_cg(&p.aggP[sm * sfl + my_off + i]), RH[i], ld_cg(&p.aggH[sm * sfl + my_off + i]));
+                    RH[i] = fmaf(ex2(A2[i] * sm_s), RH[i], ld_cg(&p.aggH[sm * sfl + my_off + i]));
             }
         }
-        // inclusive end state of this chunk = P * h_in + H
+        // inclusive end state of this chunk
 #pragma unroll
         for (int i = 0; i < NG; ++i) {
-            p.incH[slot * sfl + my_off + i] = fmaf(P[i], RH[i], h[i]);
+            p.incH[slot * sfl + my_off + i] = fmaf(ex2(A2[i] * ssum), RH[i], h[i]);
             h[i] = RH[i];
         }
         __threadfence();
@@ -435,39 +474,49 @@ __global__ void __launch_bounds__(Layout<T, NP, G>::THREADS) full_scan_kernel(co
 struct KernelInfo {
     const void* fn;
     size_t smem;
-    int G;
-    int DT;
-    int threads;
-    int ts;
+    int G, DT, threads, ts;
 };
 
-template <typename T, int NP, int G, bool ZOH>
+template <typename T, int NP, class SH, bool ZOH>
 KernelInfo info_for() {
-    using LY = Layout<T, NP, G>;
-    const void* fn = reinterpret_cast<const void*>(&full_scan_kernel<T, NP, G, ZOH>);
+    using LY = Layout<T, NP, SH>;
+    const void* fn = reinterpret_cast<const void*>(&full_scan_kernel<T, NP, SH, ZOH>);
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [&] {
         attr_err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LY::bytes);
     });
-    if (attr_err != cudaSuccess) return {nullptr, 0, G, LY::DT, LY::THREADS, LY::TS};
-    return {fn, LY::bytes, G, LY::DT, LY::THREADS, LY::TS};
+    return {attr_err == cudaSuccess ? fn : nullptr, LY::bytes, LY::G, LY::DT, LY::THREADS, LY::TS};
 }
 
+// Tile shapes per padded state count, in order of preference (fewest lanes
+// per channel first).  The zero-order-hold variant uses the first shape.
+int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 5; }
+
 template <typename T, bool ZOH>
-KernelInfo pick_np(int np) {
+KernelInfo pick_t(int np, int shape) {
+    if (ZOH) shape = 0;
     switch (np) {
-    case 1: return info_for<T, 1, 1, ZOH>();
-    case 2: return info_for<T, 2, 1, ZOH>();
-    case 4: return info_for<T, 4, 1, ZOH>();
-    case 8: return info_for<T, 8, 2, ZOH>();
-    default: return info_for<T, 16, 4, ZOH>();
+    case 1: return info_for<T, 1, Shape<1, 128, 16, 3>, ZOH>();
+    case 2: return info_for<T, 2, Shape<1, 128, 16, 3>, ZOH>();
+    case 4: return info_for<T, 4, Shape<1, 128, 16, 3>, ZOH>();
+    case 8:
+        if (shape == 1) return info_for<T, 8, Shape<2, 64, 16, 3>, false>();
+        return info_for<T, 8, Shape<1, 128, 8, 3>, ZOH>();
+    default:
+        switch (shape) {
+        case 1: return info_for<T, 16, Shape<2, 128, 8, 3>, false>();
+        case 2: return info_for<T, 16, Shape<2, 64, 16, 3>, false>();
+        case 3: return info_for<T, 16, Shape<4, 64, 16, 3>, false>();
+        case 4: return info_for<T, 16, Shape<4, 32, 32, 3>, false>();
+        default: return info_for<T, 16, Shape<1, 128, 0, 3, 7>, ZOH>();
+        }
     }
 }
 
-KernelInfo pick(vmb_dtype dt, int np, bool zoh) {
-    if (dt == VMB_BF16) return zoh ? pick_np<__nv_bfloat16, true>(np) : pick_np<__nv_bfloat16, false>(np);
-    return zoh ? pick_np<float, true>(np) : pick_np<float, false>(np);
+KernelInfo pick(vmb_dtype dt, int np, int shape, bool zoh) {
+    if (dt == VMB_BF16) return zoh ? pick_t<__nv_bfloat16, true>(np, shape) : pick_t<__nv_bfloat16, false>(np, shape);
+    return zoh ? pick_t<float, true>(np, shape) : pick_t<float, false>(np, shape);
 }
 
 int pad_states(int N) {
@@ -476,37 +525,80 @@ int pad_states(int N) {
     return np;
 }
 
+// Optional tuning override "shape[,chunks]" from the environment
+// (VMB_FULL_PLAN), used to sweep tile shapes; unset in normal use.
+bool env_plan(int* shape, int* chunks) {
+    const char* e = getenv("VMB_FULL_PLAN");
+    if (!e || !*e) return false;
+    *shape = atoi(e);
+    const char* comma = strchr(e, ',');
+    *chunks = comma ? atoi(comma + 1) : 0;
+    return true;
+}
+
 }  // namespace
 
 vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     if (a.N < 1 || a.N > 16) return VMB_ERR_UNSUPPORTED;
     const int np = pad_states(a.N);
-    KernelInfo ki = pick(a.dtype, np, (a.flags & VMB_FLAG_B_ZOH) != 0);
-    if (!ki.fn) return VMB_ERR_CUDA;
-    int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ki.fn, ki.threads, ki.smem) != cudaSuccess)
-        return VMB_ERR_CUDA;
-    if (per_sm < 1) per_sm = 1;
-    const long long resident = (long long)per_sm * device_sm_count();
+    const bool zoh = (a.flags & VMB_FLAG_B_ZOH) != 0;
+    const long long rows = (long long)a.B * a.K * a.D;
+    const int sms = device_sm_count();
+    const int nshapes = zoh ? 1 : shape_count(np);
+    // The first shape (fewest lanes per channel) whose grid fills the GPU;
+    // otherwise the most parallel shape, cutting L into chunks if even that
+    // leaves SMs idle.
+    int chosen = nshapes - 1, forced_chunks = 0;
+    bool fits = false;
+    long long resident_ctas = 0;
+    KernelInfo ki{};
+    int env_shape = 0;
+    const bool forced = env_plan(&env_shape, &forced_chunks) && !zoh;
+    for (int sh = 0; sh < nshapes; ++sh) {
+        if (forced && sh != env_shape % nshapes) continue;
+        ki = pick(a.dtype, np, sh, zoh);
+        if (!ki.fn) return VMB_ERR_CUDA;
+        int per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ki.fn, ki.threads, ki.smem) != cudaSuccess)
+            return VMB_ERR_CUDA;
+        resident_ctas = (long long)(per_sm < 1 ? 1 : per_sm) * sms;
+        const long long capacity = resident_ctas * ki.threads;
+        chosen = sh;
+        if (forced) {
+            fits = forced_chunks <= 1;
+            break;
+        }
+        if (rows * ki.G * 4 >= capacity * 3) {
+            fits = true;
+            break;
+        }
+    }
+    if (!forced && !fits) {  // the most parallel shape, and keep it if it is close to a full wave
+        ki = pick(a.dtype, np, chosen, zoh);
+        int per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ki.fn, ki.threads, ki.smem) != cudaSuccess)
+            return VMB_ERR_CUDA;
+        resident_ctas = (long long)(per_sm < 1 ? 1 : per_sm) * sms;
+        fits = rows * ki.G * 5 >= resident_ctas * ki.threads * 2;
+    }
     ScanPlan p{};
     p.np = np;
+    p.split = chosen;
     p.tile_rows = ki.DT;
     p.tiles_per_bk = (a.D + ki.DT - 1) / ki.DT;
     p.n_seq = a.B * a.K * p.tiles_per_bk;
-    // Cut L only when the channel tiles alone cannot fill the GPU; keep chunks
-    // at least 128 steps long so the look-back traffic stays small.
-    const int kTS = ki.ts;
     int n_chunks = 1;
-    if (p.n_seq < resident) {
-        const long long want = (resident + p.n_seq - 1) / p.n_seq;
-        const long long max_chunks = (a.L + 127) / 128;
+    if (forced && forced_chunks > 1) {
+        n_chunks = forced_chunks;
+    } else if (!fits && p.n_seq < resident_ctas) {
+        const long long want = (resident_ctas + p.n_seq - 1) / p.n_seq;
+        const long long max_chunks = (a.L + 63) / 64;  // chunks of at least 64 steps
         n_chunks = (int)(want < max_chunks ? want : max_chunks);
         if (n_chunks < 1) n_chunks = 1;
     }
     int chunk_len = (a.L + n_chunks - 1) / n_chunks;
-    chunk_len = (chunk_len + kTS - 1) / kTS * kTS;
-    n_chunks = (a.L + chunk_len - 1) / chunk_len;
-    p.n_chunks = n_chunks;
+    chunk_len = (chunk_len + ki.ts - 1) / ki.ts * ki.ts;
+    p.n_chunks = (a.L + chunk_len - 1) / chunk_len;
     p.chunk_len = chunk_len;
     p.state_floats = (size_t)ki.DT * np;
     p.ws_bytes = ws_layout(p).total;
@@ -515,7 +607,7 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
 }
 
 vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream) {
-    KernelInfo ki = pick(a.dtype, plan.np, (a.flags & VMB_FLAG_B_ZOH) != 0);
+    KernelInfo ki = pick(a.dtype, plan.np, plan.split, (a.flags & VMB_FLAG_B_ZOH) != 0);
     if (!ki.fn) return VMB_ERR_CUDA;
     const size_t es = a.dtype == VMB_BF16 ? 2 : 4;
     FullParams p{};

@@ -4,23 +4,27 @@
 // over the D channels of one (batch, direction), the recurrence runs once on
 // the averages, and T^-1 broadcasts its output back to every channel.
 //
-// One CTA owns one (batch, direction) and one chunk of TC steps.
-//   A. Channel reduction, fused into the load: the chunk's u and delta are
-//      streamed through shared memory in sub-tiles of kDS channels (cp.async,
-//      double buffered); each element gets its softplus once; thread (t, g, s)
-//      accumulates sum_d 2^(delta_{d,t} A_{c,n} log2 e) for its NG states n
-//      over its share s of the channels, and sum_d delta_{d,t} u_{d,t}.  Abar
-//      is averaged after the exponential (Eq. 9 averages Abar itself).
-//   B. The one-channel recurrence on the averages: micro-chunks of 8 steps per
-//      (state, micro-chunk) thread, a serial combine over the micro-chunks, a
-//      decoupled look-back over the preceding chunks of the same (batch,
-//      direction) for the carry-in state, then the exact states and
-//      ybar_t = sum_n C_{t,n} h_{t,n}.
+// One CTA owns one (batch, direction) and one chunk of TC steps; thread (t, s)
+// owns step t of the chunk and every S-th channel.
+//   A. Channel reduction, fused into the load: each thread reads delta and u of
+//      its channels at its step straight from global memory (the lanes of a
+//      warp cover consecutive steps, so every load is a coalesced 32-wide row
+//      segment), applies the softplus of Eq. 6 once per element, and
+//      accumulates sum_d 2^(delta_{d,t} A_{c,n} log2 e) for every state n and
+//      sum_d delta_{d,t} u_{d,t}.  Abar is averaged after the exponential
+//      (Eq. 9 averages Abar itself); Bbar u = B_n mean_d(delta_d u_d).
+//   B. The partial sums of the S channel groups are added in shared memory; the
+//      one-channel recurrence runs on the averages in micro-chunks of 8 steps
+//      per (state, micro-chunk) thread with a serial combine, a decoupled
+//      look-back over the preceding chunks of the same (batch, direction)
+//      gives the carry-in state, and ybar_t = sum_n C_{t,n} h_{t,n}.
 //   C. Broadcast + skip: y[d, t] = ybar_t + Dskip_c u[d, t] for every channel,
-//      written with 16-byte stores (u is read again; it is still in L2).
+//      coalesced along t (u is read again; it is still in L2).
 // The recurrence and the C.h work run once per (b, k) instead of once per
 // (b, k, d); the exponentials of Abar stay per (b, k, d, n) because the mean
 // is taken after them.
+#include <stdlib.h>
+
 #include <mutex>
 
 #include "vmb_common.cuh"
@@ -30,8 +34,7 @@ namespace vmb {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kDS = 32;     // channels per reduction sub-tile
-constexpr int kMC = 8;      // steps per micro-chunk of the local scan
+constexpr int kMC = 8;  // steps per micro-chunk of the local scan
 
 struct MeanParams {
     const void* u;
@@ -46,7 +49,6 @@ struct MeanParams {
     int K, D, N, L;
     int softplus_on, skip_mean;
     int n_chunks, chunk_len, n_seq;
-    int vec;
     int suppress;
     WsHeader* hdr;
     unsigned* flags;
@@ -55,65 +57,56 @@ struct MeanParams {
     float* incH;
 };
 
-__host__ __device__ constexpr size_t a16(size_t v) { return (v + 15) / 16 * 16; }
-
-template <typename T, int NP, int TC>
+template <int NP, int TC, bool ZOH>
 struct MLayout {
-    static constexpr int NG = NP < 4 ? NP : 4;
-    static constexpr int G = NP / NG;
-    static constexpr int ITEMS = TC * G;             // (t, g) reduction items
-    static constexpr int S = kThreads / ITEMS;       // channel splits
-    static constexpr int TCF = TC + 1;
-    static constexpr int RAW = 2 * kDS * TC;         // u + delta sub-tile
-    static constexpr size_t raw_bytes = a16((size_t)2 * RAW * sizeof(T));
-    static constexpr size_t dlf_off = raw_bytes;
-    static constexpr size_t uf_off = dlf_off + (size_t)kDS * TCF * 4;
-    static constexpr size_t a2_off = a16(uf_off + (size_t)kDS * TCF * 4);
-    static constexpr size_t ar_off = a2_off + (size_t)kDS * NP * 4;
-    static constexpr size_t dsk_off = ar_off + (size_t)kDS * NP * 4;
-    static constexpr size_t bias_off = dsk_off + (size_t)kDS * 4;
-    static constexpr size_t red_off = a16(bias_off + (size_t)kDS * 4);     // [S][TC][NP] x 2
-    static constexpr size_t redu_off = red_off + (size_t)2 * S * TC * NP * 4;  // [S][TC] x 2
-    static constexpr size_t abar_off = a16(redu_off + (size_t)2 * S * TC * 4);
-    static constexpr size_t bubar_off = abar_off + (size_t)TC * NP * 4;
-    static constexpr size_t bf_off = bubar_off + (size_t)TC * NP * 4;
-    static constexpr size_t cf_off = bf_off + (size_t)TC * NP * 4;
-    static constexpr size_t mc_off = cf_off + (size_t)TC * NP * 4;          // [4][TC/kMC][NP]
-    static constexpr size_t ybar_off = mc_off + (size_t)4 * (TC / kMC) * NP * 4;
-    static constexpr size_t dsu_off = ybar_off + (size_t)TC * 4;
-    static constexpr size_t hin_off = dsu_off + (size_t)TC * 4;
-    static constexpr size_t bytes = hin_off + (size_t)NP * 4;
-    static_assert(S >= 1 && kThreads % ITEMS == 0, "items must divide the block");
+    static constexpr int S = kThreads / TC;  // channel groups
+    static constexpr int NMC = TC / kMC;
+    static constexpr int CG = 256;           // channels whose A / bias / Dskip are staged at a time
+    // shared memory (floats)
+    static constexpr int red = 0;                               // [S][TC][NP] partial sums of Abar
+    static constexpr int redb = red + S * TC * NP;              // [S][TC][NP] partial sums of Bbar u (ZOH)
+    static constexpr int redu = redb + (ZOH ? S * TC * NP : 0); // [S][TC] sums of delta u
+    static constexpr int reds = redu + S * TC;                  // [S][TC] sums of Dskip u (skip mean)
+    static constexpr int abar = reds + S * TC;                  // [TC][NP]
+    static constexpr int bubar = abar + TC * NP;                // [TC][NP]
+    static constexpr int bf = bubar + TC * NP;                  // [TC][NP]
+    static constexpr int cf = bf + TC * NP;                     // [TC][NP]
+    static constexpr int mc = cf + TC * NP;                     // [4][NMC][NP]
+    static constexpr int ybar = mc + 4 * NMC * NP;              // [TC]
+    static constexpr int dsu = ybar + TC;                       // [TC]
+    static constexpr int hin = dsu + TC;                        // [NP]
+    static constexpr int a2 = (hin + NP + 3) / 4 * 4;           // [CG][NP] A * log2 e (raw A for ZOH)
+    static constexpr int bias = a2 + CG * NP;                   // [CG]
+    static constexpr int dsk = bias + CG;                       // [CG]
+    static constexpr size_t bytes = (size_t)(dsk + CG) * 4;
+    static_assert(kThreads % TC == 0 && TC % 32 == 0, "a warp covers 32 consecutive steps");
+    static_assert(NP * NMC <= kThreads, "local scan mapping");
     static_assert(bytes <= 100 * 1024, "mean-scan tile must leave room for two CTAs per SM");
-    static_assert(TC % kMC == 0 && NP * (TC / kMC) <= kThreads, "local scan mapping");
 };
 
 template <typename T, int NP, int TC, bool ZOH>
 __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p) {
-    using LY = MLayout<T, NP, TC>;
-    constexpr int NG = LY::NG, G = LY::G, S = LY::S, TCF = LY::TCF, RAW = LY::RAW;
-    constexpr int NMC = TC / kMC;
-    extern __shared__ __align__(16) unsigned char smem[];
-    T* raw = reinterpret_cast<T*>(smem);
-    float* dlf = reinterpret_cast<float*>(smem + LY::dlf_off);
-    float* uf = reinterpret_cast<float*>(smem + LY::uf_off);
-    float* s_a2 = reinterpret_cast<float*>(smem + LY::a2_off);
-    float* s_ar = reinterpret_cast<float*>(smem + LY::ar_off);
-    float* s_dsk = reinterpret_cast<float*>(smem + LY::dsk_off);
-    float* s_bias = reinterpret_cast<float*>(smem + LY::bias_off);
-    float* red = reinterpret_cast<float*>(smem + LY::red_off);
-    float* redu = reinterpret_cast<float*>(smem + LY::redu_off);
-    float* abar = reinterpret_cast<float*>(smem + LY::abar_off);
-    float* bubar = reinterpret_cast<float*>(smem + LY::bubar_off);
-    float* bfm = reinterpret_cast<float*>(smem + LY::bf_off);
-    float* cfm = reinterpret_cast<float*>(smem + LY::cf_off);
-    float* mcP = reinterpret_cast<float*>(smem + LY::mc_off);
+    using LY = MLayout<NP, TC, ZOH>;
+    constexpr int S = LY::S, NMC = LY::NMC, CG = LY::CG;
+    extern __shared__ __align__(16) float sm[];
+    float* red = sm + LY::red;
+    float* redb = sm + LY::redb;
+    float* redu = sm + LY::redu;
+    float* reds = sm + LY::reds;
+    float* abar = sm + LY::abar;
+    float* bubar = sm + LY::bubar;
+    float* bfm = sm + LY::bf;
+    float* cfm = sm + LY::cf;
+    float* mcP = sm + LY::mc;
     float* mcH = mcP + NMC * NP;
     float* exP = mcH + NMC * NP;
     float* exH = exP + NMC * NP;
-    float* s_ybar = reinterpret_cast<float*>(smem + LY::ybar_off);
-    float* s_dsu = reinterpret_cast<float*>(smem + LY::dsu_off);
-    float* s_hin = reinterpret_cast<float*>(smem + LY::hin_off);
+    float* s_ybar = sm + LY::ybar;
+    float* s_dsu = sm + LY::dsu;
+    float* s_hin = sm + LY::hin;
+    float* s_a2 = sm + LY::a2;
+    float* s_bias = sm + LY::bias;
+    float* s_dsk = sm + LY::dsk;
     __shared__ unsigned s_misc[2];
 
     const int tid = threadIdx.x;
@@ -149,6 +142,7 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
     const size_t bcrow0 = (size_t)seq * N;  // first row of Bs/Cs
     const T* u = static_cast<const T*>(p.u);
     const T* dlr = static_cast<const T*>(p.dl);
+    const float* Ak = p.A + (size_t)k * D * N;
 
     // B and C of the chunk, transposed to [t][n]
     for (int i = tid; i < NP * TC; i += kThreads) {
@@ -160,121 +154,105 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
     }
 
     // ---------------------------------------------------------------- phase A
-    const int item = tid % LY::ITEMS;
-    const int sidx = tid / LY::ITEMS;
-    const int rt = item % TC;  // step of this reduction item
-    const int rg = item / TC;  // state group of this reduction item
-    float acc[NG], accb[NG];
+    const int rt = tid % TC;  // step of this thread
+    const int sg = tid / TC;  // channel group of this thread
+    const bool tv = rt < nvalid;
+    float acc[NP], accb[NP];
 #pragma unroll
-    for (int i = 0; i < NG; ++i) {
-        acc[i] = 0.0f;
-        accb[i] = 0.0f;
+    for (int n = 0; n < NP; ++n) {
+        acc[n] = 0.0f;
+        accb[n] = 0.0f;
     }
     float sdu = 0.0f, sdsu = 0.0f;
-
-    const int nsub = (D + kDS - 1) / kDS;
-    auto load_sub = [&](int st, T* dst) {
-        const int r0 = st * kDS;
-        const int nr = min(kDS, D - r0);
-        if (p.vec) {
-            constexpr int VE = 16 / sizeof(T), CPR = TC / VE;
-            for (int i = tid; i < 2 * kDS * CPR; i += kThreads) {
-                const int which = i / (kDS * CPR);
-                const int j = i % (kDS * CPR);
-                const int r = j / CPR, ch = j % CPR;
-                const T* base = which ? dlr : u;
-                const bool ok = r < nr && ch * VE < nvalid;
-                const T* src = ok ? base + (urow0 + r0 + r) * (size_t)L + l0 + ch * VE : base;
-                cp_async16(dst + which * kDS * TC + r * TC + ch * VE, src, ok ? 16 : 0);
-            }
-        } else {
-            for (int i = tid; i < 2 * kDS * TC; i += kThreads) {
-                const int which = i / (kDS * TC);
-                const int j = i % (kDS * TC);
-                const int r = j / TC, t = j % TC;
-                const T* base = which ? dlr : u;
-                T v = T(0.0f);
-                if (r < nr && t < nvalid) v = base[(urow0 + r0 + r) * (size_t)L + l0 + t];
-                dst[i] = v;
-            }
-        }
-    };
-
-    load_sub(0, raw);
-    cp_async_commit();
-    for (int st = 0; st < nsub; ++st) {
-        if (st + 1 < nsub) load_sub(st + 1, raw + ((st + 1) & 1) * RAW);
-        cp_async_commit();
-        cp_async_wait<1>();
-        const int r0 = st * kDS;
-        const int nr = min(kDS, D - r0);
-        // per-channel tables of the sub-tile
-        for (int i = tid; i < kDS * NP; i += kThreads) {
+    // Channel groups of CG: stage the group's A (times log2 e), bias and Dskip in
+    // shared memory, then every thread reduces its channels of the group with the
+    // delta and u of the next kPF channels already in flight.
+    constexpr int kPF = 8;
+    const size_t col = (size_t)l0 + (tv ? rt : 0);
+    const T* dcol = dlr + urow0 * (size_t)L + col;
+    const T* ucol = u + urow0 * (size_t)L + col;
+    for (int g0 = 0; g0 < D; g0 += CG) {
+        const int gn = min(CG, D - g0);
+        __syncthreads();  // previous group's tables are no longer read
+        for (int i = tid; i < CG * NP; i += kThreads) {
             const int r = i / NP, n = i % NP;
-            const float a = (r < nr && n < N) ? p.A[((size_t)k * D + r0 + r) * N + n] : 0.0f;
-            s_a2[i] = a * kLog2e;
-            s_ar[i] = a;
+            const float av = (r < gn && n < N) ? Ak[(size_t)(g0 + r) * N + n] : 0.0f;
+            s_a2[i] = ZOH ? av : av * kLog2e;
         }
-        for (int i = tid; i < kDS; i += kThreads) {
-            s_bias[i] = i < nr ? p.bias[(size_t)k * D + r0 + i] : 0.0f;
-            s_dsk[i] = i < nr ? p.Dskip[(size_t)k * D + r0 + i] : 0.0f;
+        for (int i = tid; i < CG; i += kThreads) {
+            s_bias[i] = i < gn ? p.bias[(size_t)k * D + g0 + i] : 0.0f;
+            s_dsk[i] = i < gn ? p.Dskip[(size_t)k * D + g0 + i] : 0.0f;
         }
         __syncthreads();
-        // conversion: softplus once per element
-        {
-            const T* ru = raw + (st & 1) * RAW;
-            const T* rd = ru + kDS * TC;
-            for (int i = tid; i < kDS * TC; i += kThreads) {
-                const int r = i / TC, t = i % TC;
-                const bool ok = r < nr && t < nvalid;
-                const float v = io<T>::cvt(rd[i]) + s_bias[r];
+        if (!tv) continue;
+        float vd[kPF], vu[kPF];
+#pragma unroll
+        for (int q = 0; q < kPF; ++q) {
+            const int d = sg + q * S;
+            vd[q] = d < gn ? io<T>::ld(dcol + (size_t)(g0 + d) * L) : 0.0f;
+            vu[q] = d < gn ? io<T>::ld(ucol + (size_t)(g0 + d) * L) : 0.0f;
+        }
+        for (int d0 = sg; d0 < gn; d0 += kPF * S) {
+            float nd[kPF], nu[kPF];
+#pragma unroll
+            for (int q = 0; q < kPF; ++q) {
+                const int d = d0 + (q + kPF) * S;
+                nd[q] = d < gn ? io<T>::ld(dcol + (size_t)(g0 + d) * L) : 0.0f;
+                nu[q] = d < gn ? io<T>::ld(ucol + (size_t)(g0 + d) * L) : 0.0f;
+            }
+#pragma unroll
+            for (int q = 0; q < kPF; ++q) {
+                const int d = d0 + q * S;
+                if (d >= gn) break;
+                const float v = vd[q] + s_bias[d];
+                const float uv = vu[q];
                 const float dv = p.softplus_on ? softplus(v) : v;
-                dlf[r * TCF + t] = ok ? dv : 0.0f;
-                uf[r * TCF + t] = ok ? io<T>::cvt(ru[i]) : 0.0f;
-            }
-        }
-        __syncthreads();
-        // reduction over this thread's channels of the sub-tile
-        for (int r = sidx; r < nr; r += S) {
-            const float dv = dlf[r * TCF + rt];
-            const float uv = uf[r * TCF + rt];
-            const float* a2 = s_a2 + r * NP + rg * NG;
-            if constexpr (ZOH) {
-                const float* ar = s_ar + r * NP + rg * NG;
+                const float* a2 = s_a2 + d * NP;  // broadcast reads: every lane has the same d
+                if constexpr (ZOH) {
 #pragma unroll
-                for (int i = 0; i < NG; ++i) {
-                    const float em1 = expm1f(dv * ar[i]);
-                    acc[i] += 1.0f + em1;
-                    accb[i] = fmaf(ar[i] != 0.0f ? em1 / ar[i] : dv, uv, accb[i]);
+                    for (int n = 0; n < NP; ++n) {
+                        const float an = a2[n];
+                        const float em1 = expm1f(dv * an);
+                        acc[n] += 1.0f + em1;
+                        accb[n] = fmaf(an != 0.0f ? em1 / an : dv, uv, accb[n]);
+                    }
+                } else if constexpr (NP % 4 == 0) {
+#pragma unroll
+                    for (int n = 0; n < NP; n += 4) {
+                        const float4 qa = *reinterpret_cast<const float4*>(a2 + n);
+                        acc[n] += ex2(dv * qa.x);
+                        acc[n + 1] += ex2(dv * qa.y);
+                        acc[n + 2] += ex2(dv * qa.z);
+                        acc[n + 3] += ex2(dv * qa.w);
+                    }
+                } else {
+#pragma unroll
+                    for (int n = 0; n < NP; ++n) acc[n] += ex2(dv * a2[n]);
                 }
-            } else if constexpr (NG % 2 == 0) {
-#pragma unroll
-                for (int i = 0; i < NG; i += 2) {
-                    const float2 x = __fmul2_rn(make_float2(dv, dv), make_float2(a2[i], a2[i + 1]));
-                    const float2 e = make_float2(ex2(x.x), ex2(x.y));
-                    const float2 s2 = __fadd2_rn(make_float2(acc[i], acc[i + 1]), e);
-                    acc[i] = s2.x;
-                    acc[i + 1] = s2.y;
-                }
-            } else {
-#pragma unroll
-                for (int i = 0; i < NG; ++i) acc[i] += ex2(dv * a2[i]);
+                sdu = fmaf(dv, uv, sdu);
+                if (p.skip_mean) sdsu = fmaf(s_dsk[d], uv, sdsu);
             }
-            if (rg == 0) sdu = fmaf(dv, uv, sdu);
-            if (p.skip_mean && rg == G - 1) sdsu = fmaf(s_dsk[r], uv, sdsu);
+#pragma unroll
+            for (int q = 0; q < kPF; ++q) {
+                vd[q] = nd[q];
+                vu[q] = nu[q];
+            }
         }
     }
-    cp_async_wait<0>();
+    if (!tv) {
+        // steps past the end of the sequence: identity (Abar = 1, Bbar u = 0)
+#pragma unroll
+        for (int n = 0; n < NP; ++n) acc[n] = sg == 0 ? (float)D : 0.0f;
+    }
 
     // ---------------------------------------------------------------- phase B
-    // partial sums of the S channel splits -> averages
 #pragma unroll
-    for (int i = 0; i < NG; ++i) {
-        red[(sidx * TC + rt) * NP + rg * NG + i] = acc[i];
-        red[S * TC * NP + (sidx * TC + rt) * NP + rg * NG + i] = accb[i];
+    for (int n = 0; n < NP; ++n) {
+        red[(sg * TC + rt) * NP + n] = acc[n];
+        if constexpr (ZOH) redb[(sg * TC + rt) * NP + n] = accb[n];
     }
-    if (rg == 0) redu[sidx * TC + rt] = sdu;
-    if (rg == G - 1) redu[S * TC + sidx * TC + rt] = sdsu;
+    redu[sg * TC + rt] = sdu;
+    reds[sg * TC + rt] = sdsu;
     __syncthreads();
     const float invD = 1.0f / (float)D;
     for (int i = tid; i < TC * NP; i += kThreads) {
@@ -283,7 +261,7 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
 #pragma unroll
         for (int s = 0; s < S; ++s) {
             sa += red[s * TC * NP + i];
-            sb += red[S * TC * NP + s * TC * NP + i];
+            if constexpr (ZOH) sb += redb[s * TC * NP + i];
             su += redu[s * TC + t];
         }
         abar[i] = sa * invD;
@@ -292,7 +270,7 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
     for (int t = tid; t < TC; t += kThreads) {
         float sd = 0.0f;
 #pragma unroll
-        for (int s = 0; s < S; ++s) sd += redu[S * TC + s * TC + t];
+        for (int s = 0; s < S; ++s) sd += reds[s * TC + t];
         s_dsu[t] = sd * invD;
     }
     __syncthreads();
@@ -322,7 +300,6 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
             H = fmaf(mp, H, mcH[m * NP + n]);
             P *= mp;
         }
-        float hin = 0.0f;
         if (chunked) {
             const size_t slot = (size_t)seq * p.n_chunks + chunk;
             if (chunk == 0) {
@@ -335,7 +312,6 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
         }
         s_hin[n] = H;  // temporarily: the chunk's local end state
         mcP[n] = P;    // temporarily: the chunk's product (mcP is no longer needed)
-        (void)hin;
     }
     __syncthreads();
     if (chunked) {
@@ -346,24 +322,17 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
         if (chunk > 0) {
             // Decoupled look-back with a left fold after the inclusive state found
             // (bit-identical carry whichever predecessor the walk stops at).
-            int found = -1;
-            for (int j = chunk - 1; j >= 0; --j) {
-                const size_t sj = (size_t)seq * p.n_chunks + j;
-                if (tid == 0) s_misc[0] = wait_flag(&p.flags[sj], gen, p.hdr, (unsigned)seq, (unsigned)j);
-                __syncthreads();
-                const unsigned kind = s_misc[0];
-                __syncthreads();
-                if (kind == kFlagInclusive) {
-                    found = j;
-                    break;
-                }
-                if (kind != kFlagAggregate) break;
+            if (tid < 32) {
+                const int f = lookback_find(p.flags + (size_t)seq * p.n_chunks, chunk, gen, p.hdr, (unsigned)seq);
+                if (tid == 0) s_misc[0] = (unsigned)f;
             }
+            __syncthreads();
+            const int found = (int)s_misc[0];
             if (found >= 0 && tid < NP) {
                 RH = ld_cg(&p.incH[((size_t)seq * p.n_chunks + found) * NP + tid]);
                 for (int m = found + 1; m < chunk; ++m) {
-                    const size_t sm = (size_t)seq * p.n_chunks + m;
-                    RH = fmaf(ld_cg(&p.aggP[sm * NP + tid]), RH, ld_cg(&p.aggH[sm * NP + tid]));
+                    const size_t smi = (size_t)seq * p.n_chunks + m;
+                    RH = fmaf(ld_cg(&p.aggP[smi * NP + tid]), RH, ld_cg(&p.aggH[smi * NP + tid]));
                 }
             }
             if (tid < NP) {
@@ -401,31 +370,27 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
     __syncthreads();
 
     // ---------------------------------------------------------------- phase C
-    T* y = static_cast<T*>(p.y);
-    if (p.vec) {
-        constexpr int VE = 16 / sizeof(T), CPR = TC / VE;
-        for (int i = tid; i < D * CPR; i += kThreads) {
-            const int r = i / CPR, ch = i % CPR;
-            if (ch * VE >= nvalid) continue;
-            const size_t gi = (urow0 + r) * (size_t)L + l0 + ch * VE;
-            const float dsk = p.Dskip[(size_t)k * D + r];
-            union { uint4 v; T e[VE]; } in, out;
-            in.v = *reinterpret_cast<const uint4*>(u + gi);
+    if (tv) {
+        T* y = static_cast<T*>(p.y);
+        const size_t col = (size_t)l0 + rt;
+        const float yb = s_ybar[rt];
+        const float dsu = s_dsu[rt];
+        constexpr int kPF = 8;
+        for (int d0 = sg; d0 < D; d0 += kPF * S) {
+            float uv[kPF];
 #pragma unroll
-            for (int e = 0; e < VE; ++e) {
-                const int t = ch * VE + e;
-                const float skip = p.skip_mean ? s_dsu[t] : dsk * io<T>::cvt(in.e[e]);
-                out.e[e] = io<T>::to(s_ybar[t] + skip);
+            for (int q = 0; q < kPF; ++q) {
+                const int d = d0 + q * S;
+                uv[q] = (d < D && !p.skip_mean) ? io<T>::ld(u + (urow0 + d) * (size_t)L + col) : 0.0f;
             }
-            *reinterpret_cast<uint4*>(y + gi) = out.v;
-        }
-    } else {
-        for (int i = tid; i < D * TC; i += kThreads) {
-            const int r = i / TC, t = i % TC;
-            if (t >= nvalid) continue;
-            const size_t gi = (urow0 + r) * (size_t)L + l0 + t;
-            const float skip = p.skip_mean ? s_dsu[t] : p.Dskip[(size_t)k * D + r] * io<T>::ld(u + gi);
-            y[gi] = io<T>::to(s_ybar[t] + skip);
+#pragma unroll
+            for (int q = 0; q < kPF; ++q) {
+                const int d = d0 + q * S;
+                if (d < D) {
+                    const float skip = p.skip_mean ? dsu : __ldg(p.Dskip + (size_t)k * D + d) * uv[q];  // Dskip: 1 KB per 256 channels, L1-resident
+                    y[(urow0 + d) * (size_t)L + col] = io<T>::to(yb + skip);
+                }
+            }
         }
     }
 
@@ -444,7 +409,7 @@ struct KInfo {
 
 template <typename T, int NP, int TC, bool ZOH>
 KInfo minfo() {
-    using LY = MLayout<T, NP, TC>;
+    using LY = MLayout<NP, TC, ZOH>;
     const void* fn = reinterpret_cast<const void*>(&mean_scan_kernel<T, NP, TC, ZOH>);
     static std::once_flag once;
     static cudaError_t err = cudaSuccess;
@@ -458,8 +423,8 @@ KInfo minfo() {
 template <typename T, int NP, bool ZOH>
 KInfo pick_tc(int tc) {
     switch (tc) {
-    case 16: return minfo<T, NP, 16, ZOH>();
     case 32: return minfo<T, NP, 32, ZOH>();
+    case 128: return minfo<T, NP, 128, ZOH>();
     default: return minfo<T, NP, 64, ZOH>();
     }
 }
@@ -487,17 +452,21 @@ vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan) {
     int np = 1;
     while (np < a.N) np <<= 1;
     const bool zoh = (a.flags & VMB_FLAG_B_ZOH) != 0;
-    // Largest chunk length whose grid still fills the GPU (one CTA per (b, k, chunk)).
+    // Longest chunk whose grid still gives every SM a few CTAs
+    // (one CTA per (b, k, chunk)); VMB_MEAN_TC forces a chunk length (tuning).
     const long long seqs = (long long)a.B * a.K;
-    int tc = 16;
-    for (int cand : {64, 32, 16}) {
+    int tc = 32;
+    const char* e = getenv("VMB_MEAN_TC");
+    const int forced = e ? atoi(e) : 0;
+    for (int cand : {128, 64, 32}) {
+        if (forced && cand != forced) continue;
         KInfo ki = mpick(a.dtype, np, cand, zoh);
         if (!ki.fn) return VMB_ERR_CUDA;
         int per_sm = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ki.fn, kThreads, ki.smem) != cudaSuccess)
             return VMB_ERR_CUDA;
         const long long resident = (long long)(per_sm < 1 ? 1 : per_sm) * device_sm_count();
-        if (seqs * ((a.L + cand - 1) / cand) >= resident || cand == 16) {
+        if (forced || seqs * ((a.L + cand - 1) / cand) >= 2 * resident || cand == 32) {
             tc = cand;
             break;
         }
@@ -518,7 +487,6 @@ vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan) {
 vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream) {
     KInfo ki = mpick(a.dtype, plan.np, plan.chunk_len, (a.flags & VMB_FLAG_B_ZOH) != 0);
     if (!ki.fn) return VMB_ERR_CUDA;
-    const size_t es = a.dtype == VMB_BF16 ? 2 : 4;
     MeanParams p{};
     p.u = a.u;
     p.dl = a.delta;
@@ -538,8 +506,6 @@ vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     p.n_chunks = plan.n_chunks;
     p.chunk_len = plan.chunk_len;
     p.n_seq = plan.n_seq;
-    const auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
-    p.vec = ((size_t)a.L * es % 16 == 0) && al16(a.u) && al16(a.delta) && al16(a.y);
     p.suppress = (a.flags & VMB_FLAG_TEST_SUPPRESS_PUBLISH) ? 1 : 0;
     const WsLayout w = ws_layout(plan);
     unsigned char* ws = static_cast<unsigned char*>(a.ws);

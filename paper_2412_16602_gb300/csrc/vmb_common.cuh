@@ -108,28 +108,49 @@ __device__ __forceinline__ unsigned flag_word(unsigned gen, unsigned kind) {
     return ((gen & 0x3FFFFFFFu) << 2) | kind;
 }
 
-// Spin (one thread) until `flag` carries this launch's generation, or give up.
-// Returns kFlagAggregate / kFlagInclusive, or 0 when the wait ran out or another
-// CTA already reported an error (then every later wait returns at once).
-__device__ __forceinline__ unsigned wait_flag(const unsigned* flag, unsigned gen, WsHeader* hdr,
-                                              unsigned seq, unsigned chunk) {
+// Warp-wide look-back (call from one full warp; every lane gets the result).
+// Finds the nearest predecessor j < chunk whose inclusive state is published
+// such that every chunk in (j, chunk) has at least its aggregate published;
+// the lanes poll 32 predecessor flags per round.  Returns -1 when the wait ran
+// out or another CTA already reported an error.
+__device__ __forceinline__ int lookback_find(const unsigned* flags, int chunk, unsigned gen, WsHeader* hdr,
+                                             unsigned seq) {
     const unsigned tag = gen & 0x3FFFFFFFu;
-    uint64_t t0 = 0;
+    const int lane = threadIdx.x & 31;
+    int hi = chunk - 1;
+    const uint64_t t0 = globaltimer_ns();
     unsigned ns = 32;
     for (unsigned it = 0;; ++it) {
-        unsigned f = ld_acquire(flag);
-        if ((f >> 2) == tag && (f & 3u)) return f & 3u;
+        const int j = hi - lane;
+        unsigned kind = 0;
+        if (j >= 0) {
+            const unsigned f = ld_acquire(&flags[j]);
+            kind = ((f >> 2) == tag) ? (f & 3u) : 0u;
+        }
+        const unsigned inc = __ballot_sync(0xffffffffu, kind == kFlagInclusive);
+        const unsigned valid = __ballot_sync(0xffffffffu, kind != 0 || j < 0);
+        if (inc) {
+            const int l = __ffs(inc) - 1;
+            const unsigned need = l == 0 ? 0u : ((1u << l) - 1u);
+            if ((valid & need) == need) return hi - l;
+        } else if (valid == 0xffffffffu && hi >= 32) {
+            hi -= 32;  // the whole window has aggregates: look further back
+            continue;
+        }
         if ((it & 15u) == 0) {
-            if (ld_relaxed(&hdr->err)) return 0;
-            uint64_t now = globaltimer_ns();
-            if (it == 0) t0 = now;
-            else if (now - t0 > kWaitLimitNs) {
-                if (atomicOr(&hdr->err, kErrTimeout) == 0) {
-                    hdr->err_seq = seq;
-                    hdr->err_chunk = chunk;
+            unsigned stop = 0;
+            if (lane == 0) {
+                if (ld_relaxed(&hdr->err)) {
+                    stop = 1;
+                } else if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                    if (atomicOr(&hdr->err, kErrTimeout) == 0) {
+                        hdr->err_seq = seq;
+                        hdr->err_chunk = (unsigned)chunk;
+                    }
+                    stop = 1;
                 }
-                return 0;
             }
+            if (__shfl_sync(0xffffffffu, stop, 0)) return -1;
         }
         __nanosleep(ns);
         if (ns < 1024) ns <<= 1;

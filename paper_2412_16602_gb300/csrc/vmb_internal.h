@@ -33,6 +33,7 @@ struct ScanArgs {
 // problem, build and device, so that the workspace query and the launch agree.
 struct ScanPlan {
     int np;            // padded state count (1, 2, 4, 8, 16)
+    int split;         // tile-shape index (full path)
     int tile_rows;     // channels per CTA (full path) or 0 (mean path)
     int tiles_per_bk;  // channel tiles per (b, k)   (full path)
     int n_seq;         // independent sequences: channel tiles (full) or (b, k) pairs (mean)

@@ -168,3 +168,35 @@ def test_lookback_wait_times_out_cleanly(mean):
         _, ref, _ = oracle.ss2d_full(inp)
     assert vmb.vmb_read_status(ws) == vmb.VMB_OK
     check(to_numpy(y), ref, "f32", "after timeout")
+
+
+@pytest.mark.parametrize("plan", ["0", "1", "2", "3", "4", "0,3", "3,5", "4,2"])
+@pytest.mark.parametrize("dt", ["f32", "bf16"])
+def test_every_tile_shape(plan, dt, monkeypatch):
+    """Each tile shape of the full scan (and forced L-chunking) against the oracle."""
+    monkeypatch.setenv("VMB_FULL_PLAN", plan)
+    wl = workloads.small_case(B=1, D=72, N=16, H=24, W=28, dtype=dt, seed=21)
+    inp = workloads.make_inputs(wl)
+    g = to_device(inp, DEV)
+    xs = vmb.vmb_cross_scan(g["x"])
+    y = vmb.vmb_selective_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W)
+    assert vmb.vmb_read_status() == vmb.VMB_OK
+    _, ref, _ = oracle.ss2d_full(inp)
+    check(to_numpy(y), ref, dt, f"full y plan {plan}")
+
+
+@pytest.mark.parametrize("tc", ["32", "64", "128"])
+@pytest.mark.parametrize("dt", ["f32", "bf16"])
+def test_every_mean_chunk_length(tc, dt, monkeypatch):
+    """Each chunk length of the channel-mean scan against the oracle (ragged last chunk)."""
+    monkeypatch.setenv("VMB_MEAN_TC", tc)
+    wl = workloads.small_case(B=2, D=70, N=16, H=19, W=21, dtype=dt, seed=22)
+    inp = workloads.make_inputs(wl)
+    g = to_device(inp, DEV)
+    xs = vmb.vmb_cross_scan(g["x"])
+    y, yb = vmb.vmb_mean_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W,
+                                  want_ybar=True)
+    assert vmb.vmb_read_status() == vmb.VMB_OK
+    _, ref, ybar_ref, _ = oracle.ss2d_mean(inp)
+    check(to_numpy(y), ref, dt, f"mean y tc {tc}")
+    check(to_numpy(yb), ybar_ref, dt, f"mean ybar tc {tc}")
