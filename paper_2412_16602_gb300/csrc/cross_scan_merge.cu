@@ -6,6 +6,9 @@
 // and 1.  Global loads and stores are 16-byte vectors when rows are 16-byte
 // aligned; the padding keeps the column-major reads free of bank conflicts.
 //
+// Maps of 1024 pixels or more use band kernels instead: one CTA per band of
+// eight rows of one map (see below), which keeps batch-1 problems parallel.
+//
 // cross-merge: ys[B,4,D,L] -> out[B,D,H,W], out = (ys0[p0] + ys2[p2]) +
 // (ys1[p1] + ys3[p3]) in fp32 in that order.  Directions 0 and 2 are read
 // straight from global memory in output order (2 reversed); directions 1 and
@@ -203,6 +206,160 @@ __global__ void __launch_bounds__(kThreads) cross_merge_kernel(const CsmParams p
     }
 }
 
+// ---------------------------------------------------------------- band kernels
+// Maps of at least kBandMinL pixels: one CTA per band of kRB rows of one map, so
+// that even a batch-1 problem has enough CTAs.  Directions 0 and 2 of a band are
+// one contiguous run of the sequence; directions 1 and 3 are W runs of kRB
+// steps, written from a [kRB][W+1] shared tile.
+constexpr int kRB = 8;
+constexpr int kBandMinL = 1024;
+constexpr int kBandThreads = 128;
+
+struct BandParams {
+    const void* in;
+    void* out;
+    int D, H, W, L;
+    int nbands;  // bands per map
+    int vec;     // W and H multiples of the vector width, 16-byte aligned bases
+};
+
+template <typename T>
+__global__ void __launch_bounds__(kBandThreads) cross_scan_band_kernel(const BandParams p) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    T* tile = reinterpret_cast<T*>(smem_raw);  // [kRB][W+1]
+    constexpr int VE = 16 / sizeof(T);
+    const int W = p.W, H = p.H, L = p.L, WP = p.W + 1;
+    const long long plane = blockIdx.x / p.nbands;
+    const int band = blockIdx.x % p.nbands;
+    const int h0 = band * kRB;
+    const int rb = min(kRB, H - h0);
+    const int n = rb * W;
+    const long long b = plane / p.D, d = plane % p.D;
+    const T* src = static_cast<const T*>(p.in) + plane * L + (long long)h0 * W;
+    T* xs = static_cast<T*>(p.out);
+    T* row0 = xs + ((b * 4 + 0) * p.D + d) * L;
+    T* row1 = xs + ((b * 4 + 1) * p.D + d) * L;
+    T* row2 = xs + ((b * 4 + 2) * p.D + d) * L;
+    T* row3 = xs + ((b * 4 + 3) * p.D + d) * L;
+    if (p.vec) {
+        for (int e = threadIdx.x * VE; e < n; e += kBandThreads * VE) {
+            Vec<T> v, r;
+            v.v = *reinterpret_cast<const uint4*>(src + e);
+            const int j = e / W, w = e - j * W;  // a vector never crosses a row (W % VE == 0)
+#pragma unroll
+            for (int q = 0; q < VE; ++q) {
+                tile[j * WP + w + q] = v.e[q];
+                r.e[q] = v.e[VE - 1 - q];
+            }
+            *reinterpret_cast<uint4*>(row0 + (long long)h0 * W + e) = v.v;           // direction 0
+            *reinterpret_cast<uint4*>(row2 + L - (long long)h0 * W - e - VE) = r.v;  // direction 2
+        }
+    } else {
+        for (int e = threadIdx.x; e < n; e += kBandThreads) {
+            const T v = src[e];
+            const int j = e / W, w = e - j * W;
+            tile[j * WP + w] = v;
+            row0[(long long)h0 * W + e] = v;
+            row2[L - 1 - (long long)h0 * W - e] = v;
+        }
+    }
+    __syncthreads();
+    // directions 1 and 3: for each column w, the steps w*H + h0 .. w*H + h0 + rb - 1
+    if (p.vec && rb == kRB) {
+        constexpr int RV = kRB / VE;  // vectors per run
+        for (int i = threadIdx.x; i < W * RV; i += kBandThreads) {
+            const int w = i / RV, jv = (i - w * RV) * VE;
+            Vec<T> v, r;
+#pragma unroll
+            for (int q = 0; q < VE; ++q) {
+                v.e[q] = tile[(jv + q) * WP + w];
+                r.e[q] = tile[(jv + VE - 1 - q) * WP + w];
+            }
+            const long long pos = (long long)w * H + h0 + jv;
+            *reinterpret_cast<uint4*>(row1 + pos) = v.v;
+            *reinterpret_cast<uint4*>(row3 + L - pos - VE) = r.v;
+        }
+    } else {
+        for (int e = threadIdx.x; e < n; e += kBandThreads) {
+            const int w = e / rb, j = e - w * rb;
+            const T v = tile[j * WP + w];
+            const long long pos = (long long)w * H + h0 + j;
+            row1[pos] = v;
+            row3[L - 1 - pos] = v;
+        }
+    }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kBandThreads) cross_merge_band_kernel(const BandParams p) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const int W = p.W, H = p.H, L = p.L, WP = p.W + 1;
+    T* s1 = reinterpret_cast<T*>(smem_raw);  // [kRB][W+1]: ys1 at pixel (h0 + j, w)
+    T* s3 = s1 + kRB * WP;                     // [kRB][W+1]: ys3 at pixel (h0 + j, w)
+    constexpr int VE = 16 / sizeof(T);
+    const long long plane = blockIdx.x / p.nbands;
+    const int band = blockIdx.x % p.nbands;
+    const int h0 = band * kRB;
+    const int rb = min(kRB, H - h0);
+    const int n = rb * W;
+    const long long b = plane / p.D, d = plane % p.D;
+    const T* ys = static_cast<const T*>(p.in);
+    const T* row0 = ys + ((b * 4 + 0) * p.D + d) * L;
+    const T* row1 = ys + ((b * 4 + 1) * p.D + d) * L;
+    const T* row2 = ys + ((b * 4 + 2) * p.D + d) * L;
+    const T* row3 = ys + ((b * 4 + 3) * p.D + d) * L;
+    T* out = static_cast<T*>(p.out) + plane * L + (long long)h0 * W;
+    // stage directions 1 and 3 of the band's pixels
+    if (p.vec && rb == kRB) {
+        constexpr int RV = kRB / VE;
+        for (int i = threadIdx.x; i < W * RV; i += kBandThreads) {
+            const int w = i / RV, jv = (i - w * RV) * VE;
+            const long long pos = (long long)w * H + h0 + jv;
+            Vec<T> v1, v3;
+            v1.v = *reinterpret_cast<const uint4*>(row1 + pos);
+            v3.v = *reinterpret_cast<const uint4*>(row3 + L - pos - VE);
+#pragma unroll
+            for (int q = 0; q < VE; ++q) {
+                s1[(jv + q) * WP + w] = v1.e[q];
+                s3[(jv + q) * WP + w] = v3.e[VE - 1 - q];
+            }
+        }
+    } else {
+        for (int e = threadIdx.x; e < n; e += kBandThreads) {
+            const int w = e / rb, j = e - w * rb;
+            const long long pos = (long long)w * H + h0 + j;
+            s1[j * WP + w] = row1[pos];
+            s3[j * WP + w] = row3[L - 1 - pos];
+        }
+    }
+    __syncthreads();
+    // out = (ys0 + ys2) + (ys1 + ys3), in this order
+    if (p.vec) {
+        for (int e = threadIdx.x * VE; e < n; e += kBandThreads * VE) {
+            const int j = e / W, w = e - j * W;
+            const long long pos = (long long)h0 * W + e;
+            Vec<T> v0, v2, o;
+            v0.v = *reinterpret_cast<const uint4*>(row0 + pos);
+            v2.v = *reinterpret_cast<const uint4*>(row2 + L - pos - VE);
+#pragma unroll
+            for (int q = 0; q < VE; ++q) {
+                const float a = io<T>::cvt(v0.e[q]) + io<T>::cvt(v2.e[VE - 1 - q]);
+                const float c = io<T>::cvt(s1[j * WP + w + q]) + io<T>::cvt(s3[j * WP + w + q]);
+                o.e[q] = io<T>::to(a + c);
+            }
+            *reinterpret_cast<uint4*>(out + e) = o.v;
+        }
+    } else {
+        for (int e = threadIdx.x; e < n; e += kBandThreads) {
+            const int j = e / W, w = e - j * W;
+            const long long pos = (long long)h0 * W + e;
+            const float a = io<T>::cvt(row0[pos]) + io<T>::cvt(row2[L - 1 - pos]);
+            const float c = io<T>::cvt(s1[j * WP + w]) + io<T>::cvt(s3[j * WP + w]);
+            out[e] = io<T>::to(a + c);
+        }
+    }
+}
+
 // Planes too large for shared memory: one thread per element, plain gathers.
 template <typename T>
 __global__ void cross_scan_direct(const T* x, T* xs, int D, int H, int W, long long total) {
@@ -247,6 +404,29 @@ vmb_status launch_csm(bool merge, const void* in, void* outp, int B, int D, int 
         else
             cross_scan_direct<T><<<grid, kThreads, 0, stream>>>(static_cast<const T*>(in), static_cast<T*>(outp), D, H, W, total);
         return cudaGetLastError() == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+    }
+    if (L >= kBandMinL && (size_t)2 * kRB * (W + 1) * es <= kMaxSmem && planes * ((H + kRB - 1) / kRB) < (1ll << 31)) {
+        BandParams bp{};
+        bp.in = in;
+        bp.out = outp;
+        bp.D = D;
+        bp.H = H;
+        bp.W = W;
+        bp.L = L;
+        bp.nbands = (H + kRB - 1) / kRB;
+        const int VE = (int)(16 / es);
+        const auto a16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
+        bp.vec = (W % VE == 0) && (H % VE == 0) && a16(in) && a16(outp);
+        const size_t smem = (merge ? 2 : 1) * (size_t)kRB * (W + 1) * es;
+        const void* fn = merge ? reinterpret_cast<const void*>(&cross_merge_band_kernel<T>)
+                               : reinterpret_cast<const void*>(&cross_scan_band_kernel<T>);
+        if (smem > 48 * 1024 &&
+            cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem) != cudaSuccess)
+            return VMB_ERR_CUDA;
+        void* args[] = {&bp};
+        const unsigned nblk = (unsigned)(planes * bp.nbands);
+        return cudaLaunchKernel(fn, dim3(nblk), dim3(kBandThreads), args, smem, stream) == cudaSuccess ? VMB_OK
+                                                                                                        : VMB_ERR_CUDA;
     }
     // about 8K elements per CTA, bounded by shared memory
     int ppc = (int)std::max<long long>(1, 8192 / L);

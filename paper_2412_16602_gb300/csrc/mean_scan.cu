@@ -63,8 +63,8 @@ struct MLayout {
     static constexpr int NMC = TC / kMC;
     static constexpr int CG = 256;           // channels whose A / bias / Dskip are staged at a time
     // shared memory (floats)
-    static constexpr int red = 0;                               // [S][TC][NP] partial sums of Abar
-    static constexpr int redb = red + S * TC * NP;              // [S][TC][NP] partial sums of Bbar u (ZOH)
+    static constexpr int red = 0;                               // [S][NP][TC] partial sums of Abar
+    static constexpr int redb = red + S * TC * NP;              // [S][NP][TC] partial sums of Bbar u (ZOH)
     static constexpr int redu = redb + (ZOH ? S * TC * NP : 0); // [S][TC] sums of delta u
     static constexpr int reds = redu + S * TC;                  // [S][TC] sums of Dskip u (skip mean)
     static constexpr int abar = reds + S * TC;                  // [TC][NP]
@@ -171,6 +171,8 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
     const size_t col = (size_t)l0 + (tv ? rt : 0);
     const T* dcol = dlr + urow0 * (size_t)L + col;
     const T* ucol = u + urow0 * (size_t)L + col;
+    // u is read again by the broadcast pass: keep it in L2; delta streams through
+    const uint64_t keep = l2_evict_last(), stream = l2_evict_first();
     for (int g0 = 0; g0 < D; g0 += CG) {
         const int gn = min(CG, D - g0);
         __syncthreads();  // previous group's tables are no longer read
@@ -189,16 +191,16 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
 #pragma unroll
         for (int q = 0; q < kPF; ++q) {
             const int d = sg + q * S;
-            vd[q] = d < gn ? io<T>::ld(dcol + (size_t)(g0 + d) * L) : 0.0f;
-            vu[q] = d < gn ? io<T>::ld(ucol + (size_t)(g0 + d) * L) : 0.0f;
+            vd[q] = d < gn ? ld_hint(dcol + (size_t)(g0 + d) * L, stream) : 0.0f;
+            vu[q] = d < gn ? ld_hint(ucol + (size_t)(g0 + d) * L, keep) : 0.0f;
         }
         for (int d0 = sg; d0 < gn; d0 += kPF * S) {
             float nd[kPF], nu[kPF];
 #pragma unroll
             for (int q = 0; q < kPF; ++q) {
                 const int d = d0 + (q + kPF) * S;
-                nd[q] = d < gn ? io<T>::ld(dcol + (size_t)(g0 + d) * L) : 0.0f;
-                nu[q] = d < gn ? io<T>::ld(ucol + (size_t)(g0 + d) * L) : 0.0f;
+                nd[q] = d < gn ? ld_hint(dcol + (size_t)(g0 + d) * L, stream) : 0.0f;
+                nu[q] = d < gn ? ld_hint(ucol + (size_t)(g0 + d) * L, keep) : 0.0f;
             }
 #pragma unroll
             for (int q = 0; q < kPF; ++q) {
@@ -247,25 +249,25 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
 
     // ---------------------------------------------------------------- phase B
 #pragma unroll
-    for (int n = 0; n < NP; ++n) {
-        red[(sg * TC + rt) * NP + n] = acc[n];
-        if constexpr (ZOH) redb[(sg * TC + rt) * NP + n] = accb[n];
+    for (int n = 0; n < NP; ++n) {  // [S][NP][TC]: lanes (consecutive t) hit consecutive banks
+        red[(sg * NP + n) * TC + rt] = acc[n];
+        if constexpr (ZOH) redb[(sg * NP + n) * TC + rt] = accb[n];
     }
     redu[sg * TC + rt] = sdu;
     reds[sg * TC + rt] = sdsu;
     __syncthreads();
     const float invD = 1.0f / (float)D;
     for (int i = tid; i < TC * NP; i += kThreads) {
-        const int t = i / NP;
+        const int n = i / TC, t = i % TC;
         float sa = 0.0f, sb = 0.0f, su = 0.0f;
 #pragma unroll
         for (int s = 0; s < S; ++s) {
-            sa += red[s * TC * NP + i];
-            if constexpr (ZOH) sb += redb[s * TC * NP + i];
+            sa += red[(s * NP + n) * TC + t];
+            if constexpr (ZOH) sb += redb[(s * NP + n) * TC + t];
             su += redu[s * TC + t];
         }
-        abar[i] = sa * invD;
-        bubar[i] = bfm[i] * (ZOH ? sb : su) * invD;
+        abar[t * NP + n] = sa * invD;
+        bubar[t * NP + n] = bfm[t * NP + n] * (ZOH ? sb : su) * invD;
     }
     for (int t = tid; t < TC; t += kThreads) {
         float sd = 0.0f;
@@ -376,19 +378,20 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
         const float yb = s_ybar[rt];
         const float dsu = s_dsu[rt];
         constexpr int kPF = 8;
+        const uint64_t stream = l2_evict_first();
         for (int d0 = sg; d0 < D; d0 += kPF * S) {
             float uv[kPF];
 #pragma unroll
             for (int q = 0; q < kPF; ++q) {
                 const int d = d0 + q * S;
-                uv[q] = (d < D && !p.skip_mean) ? io<T>::ld(u + (urow0 + d) * (size_t)L + col) : 0.0f;
+                uv[q] = (d < D && !p.skip_mean) ? ld_hint(u + (urow0 + d) * (size_t)L + col, stream) : 0.0f;
             }
 #pragma unroll
             for (int q = 0; q < kPF; ++q) {
                 const int d = d0 + q * S;
                 if (d < D) {
                     const float skip = p.skip_mean ? dsu : __ldg(p.Dskip + (size_t)k * D + d) * uv[q];  // Dskip: 1 KB per 256 channels, L1-resident
-                    y[(urow0 + d) * (size_t)L + col] = io<T>::to(yb + skip);
+                    st_hint(y + (urow0 + d) * (size_t)L + col, yb + skip, stream);
                 }
             }
         }

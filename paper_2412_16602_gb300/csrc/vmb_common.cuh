@@ -172,6 +172,39 @@ __device__ __forceinline__ void finish_launch(WsHeader* hdr, unsigned total_ctas
     }
 }
 
+// ------------------------------------------------------ L2 eviction policies
+
+// Cache policies for loads/stores with an L2 eviction hint (sm_80+ createpolicy):
+// evict_last keeps data that is read again soon, evict_first streams data
+// through without displacing it.
+__device__ __forceinline__ uint64_t l2_evict_last() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint64_t l2_evict_first() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ float ld_hint(const float* p, uint64_t pol) {
+    float v;
+    asm volatile("ld.global.L2::cache_hint.f32 %0, [%1], %2;" : "=f"(v) : "l"(p), "l"(pol));
+    return v;
+}
+__device__ __forceinline__ float ld_hint(const __nv_bfloat16* p, uint64_t pol) {
+    unsigned short v;
+    asm volatile("ld.global.L2::cache_hint.b16 %0, [%1], %2;" : "=h"(v) : "l"(p), "l"(pol));
+    return __uint_as_float((unsigned)v << 16);
+}
+__device__ __forceinline__ void st_hint(float* p, float v, uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.f32 [%0], %1, %2;" ::"l"(p), "f"(v), "l"(pol) : "memory");
+}
+__device__ __forceinline__ void st_hint(__nv_bfloat16* p, float v, uint64_t pol) {
+    const unsigned short b = __bfloat16_as_ushort(__float2bfloat16_rn(v));
+    asm volatile("st.global.L2::cache_hint.b16 [%0], %1, %2;" ::"l"(p), "h"(b), "l"(pol) : "memory");
+}
+
 // --------------------------------------------------------- async copies
 
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem, int src_bytes) {

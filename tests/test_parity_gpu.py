@@ -47,6 +47,8 @@ SHAPES = [
     (1, 48, 3, 5, 13, "bf16"),       # bf16, odd L
     (2, 96, 16, 16, 16, "bf16"),     # bf16, aligned rows
     (1, 8, 16, 64, 64, "f32"),       # few channels, long sequence: many chunks
+    (1, 6, 4, 37, 29, "f32"),        # band cross-scan/merge: ragged last band, odd width (element path)
+    (2, 6, 4, 32, 40, "bf16"),       # band cross-scan/merge, bf16 vector path
 ]
 
 
