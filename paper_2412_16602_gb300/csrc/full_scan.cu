@@ -491,7 +491,7 @@ KernelInfo info_for() {
 
 // Tile shapes per padded state count, in order of preference (fewest lanes
 // per channel first).  The zero-order-hold variant uses the first shape.
-int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 5; }
+int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 7; }
 
 template <typename T, bool ZOH>
 KernelInfo pick_t(int np, int shape) {
@@ -509,6 +509,8 @@ KernelInfo pick_t(int np, int shape) {
         case 2: return info_for<T, 16, Shape<2, 64, 16, 3>, false>();
         case 3: return info_for<T, 16, Shape<4, 64, 16, 3>, false>();
         case 4: return info_for<T, 16, Shape<4, 32, 32, 3>, false>();
+        case 5: return info_for<T, 16, Shape<1, 64, 16, 3>, false>();
+        case 6: return info_for<T, 16, Shape<1, 32, 16, 3>, false>();
         default: return info_for<T, 16, Shape<1, 128, 0, 3, 7>, ZOH>();
         }
     }
@@ -538,64 +540,95 @@ bool env_plan(int* shape, int* chunks) {
 
 }  // namespace
 
+// Roles of the tile shapes of one padded state count: "wide" (one lane per
+// channel, 128 channels: cheapest per state update), "mid" (two lanes per
+// channel), and for sequences that must be cut into chunks "chunk_narrow"
+// (one lane per channel, 64 channels) and "chunk_wide" (widest split).
+struct ShapeRoles {
+    int wide, mid, chunk_narrow, chunk_wide;
+};
+ShapeRoles roles(int np) {
+    if (np >= 16) return {0, 2, 5, 3};
+    if (np == 8) return {0, 1, 0, 1};
+    return {0, 0, 0, 0};
+}
+
 vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     if (a.N < 1 || a.N > 16) return VMB_ERR_UNSUPPORTED;
     const int np = pad_states(a.N);
     const bool zoh = (a.flags & VMB_FLAG_B_ZOH) != 0;
     const long long rows = (long long)a.B * a.K * a.D;
     const int sms = device_sm_count();
-    const int nshapes = zoh ? 1 : shape_count(np);
-    // The first shape (fewest lanes per channel) whose grid fills the GPU;
-    // otherwise the most parallel shape, cutting L into chunks if even that
-    // leaves SMs idle.
-    int chosen = nshapes - 1, forced_chunks = 0;
-    bool fits = false;
-    long long resident_ctas = 0;
+    auto info = [&](int sh, KernelInfo* ki, long long* resident) -> vmb_status {
+        *ki = pick(a.dtype, np, sh, zoh);
+        if (!ki->fn) return VMB_ERR_CUDA;
+        int per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ki->fn, ki->threads, ki->smem) != cudaSuccess)
+            return VMB_ERR_CUDA;
+        *resident = (long long)(per_sm < 1 ? 1 : per_sm) * sms;
+        return VMB_OK;
+    };
+    // Rules measured on GB300 over the benchmark workloads: plenty of rows ->
+    // one lane per channel; a fair number -> two lanes; too few -> cut L into
+    // chunks, with one lane per channel when the chunks stay long (>= 256
+    // steps) and the widest split otherwise (chunks >= 128 steps).
+    int shape = 0, n_chunks = 1, forced_chunks = 0, env_shape = 0;
     KernelInfo ki{};
-    int env_shape = 0;
-    const bool forced = env_plan(&env_shape, &forced_chunks) && !zoh;
-    for (int sh = 0; sh < nshapes; ++sh) {
-        if (forced && sh != env_shape % nshapes) continue;
-        ki = pick(a.dtype, np, sh, zoh);
-        if (!ki.fn) return VMB_ERR_CUDA;
-        int per_sm = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ki.fn, ki.threads, ki.smem) != cudaSuccess)
-            return VMB_ERR_CUDA;
-        resident_ctas = (long long)(per_sm < 1 ? 1 : per_sm) * sms;
-        const long long capacity = resident_ctas * ki.threads;
-        chosen = sh;
-        if (forced) {
-            fits = forced_chunks <= 1;
-            break;
+    long long res = 0;
+    vmb_status st;
+    if (!zoh && env_plan(&env_shape, &forced_chunks)) {
+        shape = env_shape % shape_count(np);
+        if ((st = info(shape, &ki, &res)) != VMB_OK) return st;
+        n_chunks = forced_chunks > 1 ? forced_chunks : 1;
+    } else if (zoh) {
+        if ((st = info(0, &ki, &res)) != VMB_OK) return st;
+        const long long tiles = a.B * a.K * (long long)((a.D + ki.DT - 1) / ki.DT);
+        if (rows * 4 < res * ki.threads * 3 && tiles < res) {
+            const long long want = (res + tiles - 1) / tiles, mx = (a.L + 255) / 256;
+            n_chunks = (int)(want < mx ? want : mx);
         }
-        if (rows * ki.G * 4 >= capacity * 3) {
-            fits = true;
-            break;
+    } else {
+        const ShapeRoles r = roles(np);
+        if ((st = info(r.wide, &ki, &res)) != VMB_OK) return st;
+        shape = r.wide;
+        if (rows * 4 < res * ki.threads * 3) {
+            KernelInfo km{};
+            long long rm = 0;
+            if ((st = info(r.mid, &km, &rm)) != VMB_OK) return st;
+            if (rows * km.G * 2 >= rm * km.threads) {
+                shape = r.mid;
+                ki = km;
+                res = rm;
+            } else {
+                KernelInfo kn{};
+                long long rn = 0;
+                if ((st = info(r.chunk_narrow, &kn, &rn)) != VMB_OK) return st;
+                const long long tiles_n = a.B * a.K * (long long)((a.D + kn.DT - 1) / kn.DT);
+                const long long want_n = (2 * rn + tiles_n - 1) / tiles_n;
+                if (a.L / want_n >= 256) {
+                    shape = r.chunk_narrow;
+                    ki = kn;
+                    n_chunks = (int)want_n;
+                } else {
+                    KernelInfo kw{};
+                    long long rw = 0;
+                    if ((st = info(r.chunk_wide, &kw, &rw)) != VMB_OK) return st;
+                    const long long tiles_w = a.B * a.K * (long long)((a.D + kw.DT - 1) / kw.DT);
+                    const long long want_w = (rw + tiles_w - 1) / tiles_w, mx = (a.L + 127) / 128;
+                    shape = r.chunk_wide;
+                    ki = kw;
+                    n_chunks = (int)(want_w < mx ? want_w : mx);
+                }
+            }
         }
     }
-    if (!forced && !fits) {  // the most parallel shape, and keep it if it is close to a full wave
-        ki = pick(a.dtype, np, chosen, zoh);
-        int per_sm = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ki.fn, ki.threads, ki.smem) != cudaSuccess)
-            return VMB_ERR_CUDA;
-        resident_ctas = (long long)(per_sm < 1 ? 1 : per_sm) * sms;
-        fits = rows * ki.G * 5 >= resident_ctas * ki.threads * 2;
-    }
+    if (n_chunks < 1) n_chunks = 1;
     ScanPlan p{};
     p.np = np;
-    p.split = chosen;
+    p.split = shape;
     p.tile_rows = ki.DT;
     p.tiles_per_bk = (a.D + ki.DT - 1) / ki.DT;
     p.n_seq = a.B * a.K * p.tiles_per_bk;
-    int n_chunks = 1;
-    if (forced && forced_chunks > 1) {
-        n_chunks = forced_chunks;
-    } else if (!fits && p.n_seq < resident_ctas) {
-        const long long want = (resident_ctas + p.n_seq - 1) / p.n_seq;
-        const long long max_chunks = (a.L + 63) / 64;  // chunks of at least 64 steps
-        n_chunks = (int)(want < max_chunks ? want : max_chunks);
-        if (n_chunks < 1) n_chunks = 1;
-    }
     int chunk_len = (a.L + n_chunks - 1) / n_chunks;
     chunk_len = (chunk_len + ki.ts - 1) / ki.ts * ki.ts;
     p.n_chunks = (a.L + chunk_len - 1) / chunk_len;
