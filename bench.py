@@ -143,6 +143,32 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+# ----------------------------------------------------------------------------- ranks
+
+
+def rank_seed(wl: workloads.Workload, rank: int) -> int:
+    """Every rank draws its own batch (weak scaling: per-rank work is fixed)."""
+    return wl.seed + 7919 * rank
+
+
+def max_over_ranks(values, world: int, device=None):
+    """Element-wise max of a list of floats over all ranks (the step time of the
+    slowest rank); identity on one rank.  Only timings cross ranks: the path
+    itself has no exchange step."""
+    if world <= 1:
+        return list(values)
+    import torch
+    t = torch.tensor(list(values), dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
+def job_throughput(step_bytes: int, world: int, max_ms_per_step: float) -> float:
+    """Whole-job GB/s: every rank moves step_bytes per step; the job takes as
+    long as its slowest rank."""
+    return world * step_bytes / (max_ms_per_step / 1e3) / 1e9
+
+
 # ----------------------------------------------------------------------------- CPU oracle
 
 
@@ -212,7 +238,7 @@ def run_ours(args, wl, rank, world, local_rank):
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
-    inp = workloads.make_inputs(wl, seed=wl.seed + 7919 * rank)
+    inp = workloads.make_inputs(wl, seed=rank_seed(wl, rank))
     tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
     host = {}
     for k, v in inp.arrays().items():
@@ -298,10 +324,7 @@ def run_ours(args, wl, rank, world, local_rank):
 
     res = {"total_ms": total_ms, "step_ms": step_ms, "per_kernel": per_kernel, "e2e_ms": e2e_ms,
            "h2d": h2d, "d2h": d2h, "clocks": clk.summary()}
-    if world > 1:
-        t = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        res["total_ms"], res["e2e_ms"] = float(t[0]), float(t[1])
+    res["total_ms"], res["e2e_ms"] = max_over_ranks([total_ms, e2e_ms], world, dev)
     return res, inp
 
 
@@ -355,7 +378,7 @@ def main():
         return
 
     ms = res["total_ms"] / args.steps
-    value = world * step_bytes / (ms / 1e3) / 1e9
+    value = job_throughput(step_bytes, world, ms)
     kb = kernel_bytes(wl)
     peak, peak_src = measured_peaks()
     per = {}
@@ -387,7 +410,7 @@ def main():
                      "algorithmic_bytes_per_launch": kb[dominant], "traffic": traffic},
         "gpu_launches": len(KERNELS) * args.steps,
         "clocks": res["clocks"],
-        "e2e": {"value": world * step_bytes / (res["e2e_ms"] / args.e2e_steps / 1e3) / 1e9, "unit": "GB/s",
+        "e2e": {"value": job_throughput(step_bytes, world, res["e2e_ms"] / args.e2e_steps), "unit": "GB/s",
                 "ms_per_step": res["e2e_ms"] / args.e2e_steps,
                 "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"]},
     }
