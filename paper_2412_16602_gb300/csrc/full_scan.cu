@@ -469,6 +469,225 @@ __global__ void __launch_bounds__(Layout<T, NP, SH>::THREADS, Layout<T, NP, SH>:
     }
 }
 
+// ----------------------------------------------------------- lane-per-state variant
+// For problems with few channel rows (a batch-1 map): the 16 lanes of a
+// half-warp share one channel and each owns one of its 16 states, so a channel
+// row gets 16x the threads of the one-lane-per-channel tiles and a long
+// sequence needs few or no L-chunks.  Per step a lane does one state update;
+// delta and delta*u are computed once per step by one lane of the channel and
+// broadcast by shuffle; B and C are read from the stage rows as they landed
+// ([n][t], four steps per 128-bit read, no transpose); y is reduced over the 16
+// lanes by a transposed butterfly every 16 steps (lane n ends with step t0+n).
+using LanesShape = Shape<16, 16, 32, 3>;  // 16 lanes per channel, 16 channels, 32-step stages
+
+// Sum of v[0..CNT) over the lanes of a half-warp, transposed: after the four
+// levels lane n holds the sum for index n.
+template <int CNT, int M>
+__device__ __forceinline__ void reduce_level(float (&v)[16], bool up) {
+#pragma unroll
+    for (int i = 0; i < CNT / 2; ++i) {
+        const float keep = up ? v[i + CNT / 2] : v[i];
+        const float send = up ? v[i] : v[i + CNT / 2];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, M);
+    }
+}
+
+template <typename T, bool ZOH>
+__global__ void __launch_bounds__(256) full_scan_lanes_kernel(const FullParams p) {
+    using LY = Layout<T, 16, LanesShape>;
+    constexpr int kTS = LY::TS, RS = LY::RS, SLOT = LY::SLOT, DT = LY::DT, NSTG = LY::NSTG;
+    extern __shared__ __align__(16) unsigned char smem[];
+    T* raw = reinterpret_cast<T*>(smem);
+    __shared__ unsigned s_misc[2];
+
+    const int tid = threadIdx.x;
+    int tile, chunk;
+    unsigned gen = 0;
+    const bool chunked = p.n_chunks > 1;
+    if (chunked) {
+        if (tid == 0) {
+            s_misc[0] = atomicAdd(&p.hdr->ticket, 1u);
+            s_misc[1] = ld_relaxed(&p.hdr->gen);
+        }
+        __syncthreads();
+        const unsigned t = s_misc[0];
+        gen = s_misc[1];
+        if (t >= (unsigned)(p.n_tiles * p.n_chunks)) {  // workspace was not zero-filled
+            if (tid == 0) {
+                atomicOr(&p.hdr->err, kErrBounds);
+                finish_launch(p.hdr, (unsigned)(p.n_tiles * p.n_chunks));
+            }
+            return;
+        }
+        chunk = (int)(t / (unsigned)p.n_tiles);
+        tile = (int)(t % (unsigned)p.n_tiles);
+    } else {
+        tile = blockIdx.x;
+        chunk = 0;
+    }
+    const int bk = tile / p.tiles_per_bk;
+    const int d0 = (tile % p.tiles_per_bk) * DT;
+    const int k = bk % p.K;
+    const int lane = tid & 31;
+    const int c = (tid >> 5) * 2 + (lane >> 4);  // channel within the tile
+    const int n = lane & 15;                     // state owned by this lane
+    const int hb = lane & 16;                    // first lane of the channel's half-warp
+    const int d = d0 + c;
+    const bool cval = d < p.D;
+    const int nrows = min(DT, p.D - d0);
+    const size_t row0 = (size_t)bk * p.D + d0;
+    const size_t bcrow0 = (size_t)bk * p.N;
+    const float Ar = (cval && n < p.N) ? p.A[((size_t)k * p.D + d) * p.N + n] : 0.0f;
+    const float A2 = Ar * kLog2e;
+    const float dsk = cval ? p.Dskip[(size_t)k * p.D + d] : 0.0f;
+    const float bias = cval ? p.bias[(size_t)k * p.D + d] : 0.0f;
+    const int l_begin = chunk * p.chunk_len;
+    const int l_end = min(p.L, l_begin + p.chunk_len);
+    const int nst = (l_end - l_begin + kTS - 1) / kTS;
+    T* yrow = static_cast<T*>(p.y) + (row0 + c) * (size_t)p.L;
+    float h = 0.0f;
+    float ssum = 0.0f;  // this lane's share of the chunk's sum of delta (first pass)
+
+    auto pass = [&](auto ph2_tag) {
+        constexpr bool PH2 = decltype(ph2_tag)::value;
+#pragma unroll
+        for (int q = 0; q < NSTG - 1; ++q) {
+            if (q < nst) load_stage<T, 16, LanesShape, PH2>(p, raw + q * SLOT, row0, bcrow0, nrows, l_begin + q * kTS);
+            cp_async_commit();
+        }
+        for (int s = 0; s < nst; ++s) {
+            const int l0 = l_begin + s * kTS;
+            const int nvalid = min(kTS, l_end - l0);
+            cp_async_wait<NSTG - 2>();  // stage s has landed
+            __syncthreads();
+            if (s + NSTG - 1 < nst)
+                load_stage<T, 16, LanesShape, PH2>(p, raw + ((s + NSTG - 1) % NSTG) * SLOT, row0, bcrow0, nrows,
+                                                   l0 + (NSTG - 1) * kTS);
+            cp_async_commit();
+            const T* ru = raw + (s % NSTG) * SLOT + c * RS;
+            const T* rd = ru + DT * RS;
+            const T* rb = raw + (s % NSTG) * SLOT + 2 * DT * RS + n * RS;
+            const T* rc = rb + 16 * RS;
+#pragma unroll 1
+            for (int g0 = 0; g0 < kTS; g0 += 16) {
+                // this lane's own step g0 + n: delta and delta * u, once per element
+                const bool tv = g0 + n < nvalid;  // ragged tail: identity step (a = 1, b = 0)
+                const float uo = tv ? io<T>::cvt(ru[g0 + n]) : 0.0f;
+                const float vo = io<T>::cvt(rd[g0 + n]) + bias;
+                const float dlo = tv ? (p.softplus_on ? softplus(vo) : vo) : 0.0f;
+                const float duo = dlo * uo;
+                if constexpr (!PH2) ssum += dlo;
+                float Bv[16], Cv[16], yp[16];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    float t4[4];
+                    load4(rb + g0 + 4 * q, t4);
+                    Bv[4 * q] = t4[0];
+                    Bv[4 * q + 1] = t4[1];
+                    Bv[4 * q + 2] = t4[2];
+                    Bv[4 * q + 3] = t4[3];
+                    if constexpr (PH2) {
+                        load4(rc + g0 + 4 * q, t4);
+                        Cv[4 * q] = t4[0];
+                        Cv[4 * q + 1] = t4[1];
+                        Cv[4 * q + 2] = t4[2];
+                        Cv[4 * q + 3] = t4[3];
+                    }
+                }
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    const float dl = __shfl_sync(0xffffffffu, dlo, hb + j);
+                    float a, bb;
+                    if constexpr (ZOH) {
+                        const float uu = __shfl_sync(0xffffffffu, uo, hb + j);
+                        const float em1 = expm1f(dl * Ar);
+                        a = 1.0f + em1;
+                        bb = (Ar != 0.0f ? em1 / Ar : dl) * Bv[j] * uu;
+                    } else {
+                        const float du = __shfl_sync(0xffffffffu, duo, hb + j);
+                        a = ex2(dl * A2);
+                        bb = du * Bv[j];
+                    }
+                    h = fmaf(a, h, bb);
+                    if constexpr (PH2) yp[j] = Cv[j] * h;
+                }
+                if constexpr (PH2) {
+                    const bool u8 = n & 8, u4 = n & 4, u2 = n & 2, u1 = n & 1;
+                    reduce_level<16, 8>(yp, u8);
+                    reduce_level<8, 4>(yp, u4);
+                    reduce_level<4, 2>(yp, u2);
+                    reduce_level<2, 1>(yp, u1);
+                    if (cval && tv) yrow[l0 + g0 + n] = io<T>::to(fmaf(dsk, uo, yp[0]));
+                }
+            }
+        }
+        cp_async_wait<0>();
+        __syncthreads();
+    };
+
+    constexpr size_t sfl = (size_t)DT * 16;  // floats of one published state
+    const size_t my_off = (size_t)c * 16 + n;
+    if (chunked && chunk > 0) {
+        pass(std::false_type{});
+        // the channel's sum of delta over the chunk: add the 16 lanes' shares
+        float cs = ssum;
+#pragma unroll
+        for (int m = 8; m >= 1; m >>= 1) cs += __shfl_xor_sync(0xffffffffu, cs, m);
+        const size_t slot = (size_t)tile * p.n_chunks + chunk;
+        if (n == 0) p.aggP[slot * sfl + c] = cs;
+        p.aggH[slot * sfl + my_off] = h;
+        __threadfence();
+        __syncthreads();
+        if (tid == 0) st_release(&p.flags[slot], flag_word(gen, kFlagAggregate));
+        // decoupled look-back and left fold, as in full_scan_kernel
+        if (tid < 32) {
+            const int f = lookback_find(p.flags + (size_t)tile * p.n_chunks, chunk, gen, p.hdr, (unsigned)tile);
+            if (tid == 0) s_misc[0] = (unsigned)f;
+        }
+        __syncthreads();
+        const int found = (int)s_misc[0];
+        float RH = 0.0f;
+        if (found >= 0) {
+            // staged fold, as in full_scan_kernel
+            constexpr int kAgg = DT * 16 + DT;
+            constexpr int kFB = (int)((size_t)NSTG * SLOT * sizeof(T) / (kAgg * 4));
+            float* sa = reinterpret_cast<float*>(raw);
+            RH = ld_cg(&p.incH[((size_t)tile * p.n_chunks + found) * sfl + my_off]);
+            for (int m0 = found + 1; m0 < chunk; m0 += kFB) {
+                const int nb = min(kFB, chunk - m0);
+                for (int i = tid; i < nb * kAgg; i += 256) {
+                    const int q = i / kAgg, r = i % kAgg;
+                    const size_t sm = (size_t)tile * p.n_chunks + m0 + q;
+                    sa[i] = r < DT * 16 ? ld_cg(&p.aggH[sm * sfl + r]) : ld_cg(&p.aggP[sm * sfl + (r - DT * 16)]);
+                }
+                __syncthreads();
+                for (int q = 0; q < nb; ++q)
+                    RH = fmaf(ex2(A2 * sa[q * kAgg + DT * 16 + c]), RH, sa[q * kAgg + my_off]);
+                __syncthreads();
+            }
+        }
+        p.incH[slot * sfl + my_off] = fmaf(ex2(A2 * cs), RH, h);
+        h = RH;
+        __threadfence();
+        __syncthreads();
+        if (tid == 0) st_release(&p.flags[slot], flag_word(gen, kFlagInclusive));
+    }
+
+    pass(std::true_type{});
+
+    if (chunked) {
+        if (chunk == 0) {
+            const size_t slot = (size_t)tile * p.n_chunks;
+            p.incH[slot * sfl + my_off] = h;
+            __threadfence();
+            __syncthreads();
+            if (tid == 0 && !p.suppress) st_release(&p.flags[slot], flag_word(gen, kFlagInclusive));
+        }
+        __syncthreads();
+        if (tid == 0) finish_launch(p.hdr, (unsigned)(p.n_tiles * p.n_chunks));
+    }
+}
+
 // ------------------------------------------------------------------ host side
 
 struct KernelInfo {
@@ -489,9 +708,22 @@ KernelInfo info_for() {
     return {attr_err == cudaSuccess ? fn : nullptr, LY::bytes, LY::G, LY::DT, LY::THREADS, LY::TS};
 }
 
+template <typename T, bool ZOH>
+KernelInfo lanes_info() {
+    using LY = Layout<T, 16, LanesShape>;
+    const void* fn = reinterpret_cast<const void*>(&full_scan_lanes_kernel<T, ZOH>);
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [&] {
+        attr_err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LY::raw_bytes);
+    });
+    return {attr_err == cudaSuccess ? fn : nullptr, LY::raw_bytes, 16, LY::DT, 256, LY::TS};
+}
+
 // Tile shapes per padded state count, in order of preference (fewest lanes
 // per channel first).  The zero-order-hold variant uses the first shape.
-int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 7; }
+int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 8; }
+constexpr int kLanesShape = 7;  // index of the lane-per-state variant (N <= 16 padded to 16)
 
 template <typename T, bool ZOH>
 KernelInfo pick_t(int np, int shape) {
@@ -511,6 +743,7 @@ KernelInfo pick_t(int np, int shape) {
         case 4: return info_for<T, 16, Shape<4, 32, 32, 3>, false>();
         case 5: return info_for<T, 16, Shape<1, 64, 16, 3>, false>();
         case 6: return info_for<T, 16, Shape<1, 32, 16, 3>, false>();
+        case 7: return lanes_info<T, false>();
         default: return info_for<T, 16, Shape<1, 128, 0, 3, 7>, ZOH>();
         }
     }
@@ -591,7 +824,18 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
         const ShapeRoles r = roles(np);
         if ((st = info(r.wide, &ki, &res)) != VMB_OK) return st;
         shape = r.wide;
-        if (rows * 4 < res * ki.threads * 3) {
+        KernelInfo kl{};
+        long long rl = 0;
+        if (np == 16 && a.L <= 1024 && rows * 4 < res * ki.threads * 3) {
+            // short sequences with few rows: one lane per state, single pass
+            if ((st = info(kLanesShape, &kl, &rl)) != VMB_OK) return st;
+            if (rows * 16 <= rl * kl.threads) {
+                shape = kLanesShape;
+                ki = kl;
+                res = rl;
+            }
+        }
+        if (shape != kLanesShape && rows * 4 < res * ki.threads * 3) {
             KernelInfo km{};
             long long rm = 0;
             if ((st = info(r.mid, &km, &rm)) != VMB_OK) return st;

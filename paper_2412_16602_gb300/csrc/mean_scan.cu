@@ -330,11 +330,27 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
             }
             __syncthreads();
             const int found = (int)s_misc[0];
-            if (found >= 0 && tid < NP) {
-                RH = ld_cg(&p.incH[((size_t)seq * p.n_chunks + found) * NP + tid]);
-                for (int m = found + 1; m < chunk; ++m) {
-                    const size_t smi = (size_t)seq * p.n_chunks + m;
-                    RH = fmaf(ld_cg(&p.aggP[smi * NP + tid]), RH, ld_cg(&p.aggH[smi * NP + tid]));
+            if (found >= 0) {
+                // Fold the aggregates after the inclusive state left to right.  They are
+                // staged into shared memory (the partial-sum area, free by now) in
+                // batches with all loads in flight at once, then folded from there.
+                constexpr int kFB = (S * TC * NP) / (2 * NP);  // aggregates per batch
+                float* sP = red;
+                float* sH = red + kFB * NP;
+                if (tid < NP) RH = ld_cg(&p.incH[((size_t)seq * p.n_chunks + found) * NP + tid]);
+                for (int m0 = found + 1; m0 < chunk; m0 += kFB) {
+                    const int nb = min(kFB, chunk - m0);
+                    for (int i = tid; i < nb * NP; i += kThreads) {
+                        const size_t smi = (size_t)seq * p.n_chunks + m0 + i / NP;
+                        sP[i] = ld_cg(&p.aggP[smi * NP + i % NP]);
+                        sH[i] = ld_cg(&p.aggH[smi * NP + i % NP]);
+                    }
+                    __syncthreads();
+                    if (tid < NP) {
+#pragma unroll 8
+                        for (int q = 0; q < nb; ++q) RH = fmaf(sP[q * NP + tid], RH, sH[q * NP + tid]);
+                    }
+                    __syncthreads();
                 }
             }
             if (tid < NP) {
