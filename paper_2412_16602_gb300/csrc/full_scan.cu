@@ -144,11 +144,12 @@ __device__ __forceinline__ void store_row(T* dst, const float (&v)[NV], int nval
         if (j < nvalid_here) dst[j] = io<T>::to(v[j]);
 }
 
-template <typename T, int NP, class SH, bool WITH_C>
-__device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t row0, size_t bcrow0, int nrows,
-                                           int l0) {
-    using LY = Layout<T, NP, SH>;
-    constexpr int DT = LY::DT, kTS = LY::TS, RS = LY::RS, kThreads = LY::THREADS;
+// Copy kTS steps (from l0) of DT u and delta rows and of the NP B (and C) rows
+// into shared memory rows of stride RS: u at row 0, delta at row DT, B at 2 DT,
+// C at 2 DT + NP.  Rows and steps past the problem are zero-filled.
+template <typename T, int NP, int DT, int kTS, int RS, int kThreads, bool WITH_C, bool WITH_B = true>
+__device__ __forceinline__ void load_tile(const FullParams& p, T* dst, size_t row0, size_t bcrow0, int nrows,
+                                          int l0) {
     constexpr int VE = 16 / sizeof(T);  // elements per 16-byte chunk
     constexpr int CPR = kTS / VE;       // chunks per stage row
     const T* u = static_cast<const T*>(p.u);
@@ -159,7 +160,7 @@ __device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t r
     T* dB = dst + 2 * DT * RS;
     if (p.vec) {
         constexpr int nU = DT * CPR, nB = NP * CPR;
-        constexpr int total = 2 * nU + (WITH_C ? 2 : 1) * nB;
+        constexpr int total = 2 * nU + (WITH_B ? (WITH_C ? 2 : 1) * nB : 0);
         for (int i = threadIdx.x; i < total; i += kThreads) {
             const T* src;
             T* d;
@@ -184,7 +185,7 @@ __device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t r
         }
     } else {
         constexpr int nU = DT * kTS, nB = NP * kTS;
-        constexpr int total = 2 * nU + (WITH_C ? 2 : 1) * nB;
+        constexpr int total = 2 * nU + (WITH_B ? (WITH_C ? 2 : 1) * nB : 0);
         for (int i = threadIdx.x; i < total; i += kThreads) {
             T v = T(0.0f);
             if (i < 2 * nU) {
@@ -203,6 +204,13 @@ __device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t r
             }
         }
     }
+}
+
+template <typename T, int NP, class SH, bool WITH_C>
+__device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t row0, size_t bcrow0, int nrows,
+                                           int l0) {
+    using LY = Layout<T, NP, SH>;
+    load_tile<T, NP, LY::DT, LY::TS, LY::RS, LY::THREADS, WITH_C>(p, dst, row0, bcrow0, nrows, l0);
 }
 
 template <typename T, int NP, class SH, bool ZOH>
@@ -688,12 +696,352 @@ __global__ void __launch_bounds__(256) full_scan_lanes_kernel(const FullParams p
     }
 }
 
+// ------------------------------------------------------ three-launch chunked variant
+// For long sequences with few channel rows (a batch-1 map) the sequence is cut
+// into many short chunks of CL steps and the carry between chunks is resolved
+// by three launches instead of a look-back, so that no CTA waits on another:
+//   1. every chunk but the last computes its aggregate (S = sum of delta and
+//      H = end state from h = 0) from a tile holding the whole chunk in shared
+//      memory;
+//   2. one thread per (channel, state) folds the aggregates left to right,
+//      inc_m = 2^(A_n log2 e S_m) inc_{m-1} + H_m (the fold that defines the
+//      inclusive states of the look-back path, so both give the same bits);
+//   3. every chunk reruns its steps from the carried-in state inc_{m-1}, Eq. 3,
+//      and writes y.
+// One lane per channel owns all 16 states, the cheapest update per state; B and
+// C are read from their [n][t] rows four steps at a time (broadcast reads, no
+// transpose), so a step costs one 128-bit read per state and operand.
+template <int DT_, int CL_, int NS_, int MINB_>
+struct ChunkShape {
+    static constexpr int DT = DT_, CL = CL_, NS = NS_, MINB = MINB_;  // NS: load sub-stages per chunk
+};
+
+template <typename T, class CS>
+struct ChunkLayout {
+    static constexpr int DT = CS::DT, CL = CS::CL, NS = CS::NS, SUB = CL / NS, MINB = CS::MINB, NP = 16;
+    static constexpr int PAD = 16 / (int)sizeof(T);
+    static constexpr int RS = CL + PAD;           // row stride (elements); rows start 16-byte aligned
+    static constexpr int ROWS = 2 * DT;  // u, delta (B and C go to the fp32 area)
+    static constexpr size_t raw_bytes = a16((size_t)ROWS * RS * sizeof(T));
+    // fp32 delta after the softplus: in place of the raw delta rows for fp32
+    // storage, a separate [DT][CL + 4] area for bf16
+    static constexpr int FS = CL + 4;
+    static constexpr bool F32 = sizeof(T) == 4;
+    static constexpr size_t dl_off = F32 ? (size_t)DT * RS * 4 : raw_bytes;
+    // B and C as fp32 rows [2 NP][FS], converted once at load time (for bf16
+    // storage one conversion per element instead of one per element and channel)
+    static constexpr size_t bc_off = F32 ? raw_bytes : raw_bytes + (size_t)DT * FS * 4;
+    static constexpr size_t a2_off = bc_off + (size_t)2 * NP * FS * 4;
+    // A * log2 e per channel: [DT][16] with the four 16-byte quads of a row
+    // swizzled by (c >> 1) & 3, so eight consecutive channels read their quad q
+    // from distinct banks
+    static constexpr size_t bytes = a2_off + (size_t)DT * NP * 4;
+    static_assert(CL % NS == 0 && SUB % 8 == 0 && DT % 32 == 0 && NS <= 4, "chunk tile shape");
+    static_assert(sizeof(T) == 2 || RS == FS, "fp32 delta rows are rewritten in place");
+};
+
+// Programmatic dependent launch (sm_90+): let the next kernel of the stream be
+// scheduled now / wait until the previous kernel's writes are visible.  Both
+// are no-ops for a kernel launched without the programmatic attribute.
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Load of sub-stage `part` (steps part*SUB .. part*SUB+SUB-1) of the chunk
+// tile: thread i always copies 16-byte column i % CPR of rows i / CPR + k *
+// (DT / CPR), so the addresses advance by a fixed row stride.  Rows that are
+// not 16-byte aligned take the element-wise loader, all of it with part 0.
+template <typename T, class CS, bool WITH_C>
+__device__ __forceinline__ void load_chunk_part(const FullParams& p, T* dst, size_t row0, size_t bcrow0, int nrows,
+                                                int l0, int part) {
+    using LY = ChunkLayout<T, CS>;
+    constexpr int DT = LY::DT, CL = LY::CL, SUB = LY::SUB, RS = LY::RS, NP = 16;
+    const int L = p.L;
+    if (p.vec) {
+        constexpr int VE = 16 / (int)sizeof(T);
+        constexpr int CPR = SUB / VE;  // 16-byte chunks per row and sub-stage
+        constexpr int RPP = DT / CPR;  // rows per pass of the DT threads
+        static_assert(DT % CPR == 0, "tile loader mapping");
+        const int ch = threadIdx.x % CPR, r0 = threadIdx.x / CPR;
+        const int t = part * SUB + ch * VE;  // step within the chunk
+        const bool colok = l0 + t < L;
+        const T* u = static_cast<const T*>(p.u);
+        const T* dl = static_cast<const T*>(p.dl);
+        const size_t step = (size_t)RPP * L;
+        size_t off = (row0 + r0) * (size_t)L + l0 + t;
+#pragma unroll
+        for (int it = 0; it < DT / RPP; ++it, off += step) {
+            const int r = r0 + it * RPP;
+            const bool ok = colok && r < nrows;
+            cp_async16(dst + r * RS + t, ok ? u + off : u, ok ? 16 : 0);
+            cp_async16(dst + (DT + r) * RS + t, ok ? dl + off : dl, ok ? 16 : 0);
+        }
+    } else if (part == 0) {
+        load_tile<T, NP, DT, CL, RS, DT, WITH_C, false>(p, dst, row0, bcrow0, nrows, l0);
+    }
+}
+
+// B (and C) of the whole chunk read with plain 16-byte loads and stored as
+// fp32 rows [n][t] of stride FS (zero past the problem).
+template <typename T, class CS, bool WITH_C>
+__device__ __forceinline__ void load_chunk_bc_f32(const FullParams& p, float* fb, size_t bcrow0, int l0) {
+    using LY = ChunkLayout<T, CS>;
+    constexpr int DT = LY::DT, CL = LY::CL, FS = LY::FS, NP = 16;
+    const int L = p.L;
+    const T* Bs = static_cast<const T*>(p.Bs);
+    const T* Cs = static_cast<const T*>(p.Cs);
+    if (p.vec) {
+        constexpr int VE = 16 / (int)sizeof(T);
+        constexpr int CPR = CL / VE;  // 16-byte chunks per row
+        constexpr int total = (WITH_C ? 2 : 1) * NP * CPR;
+#pragma unroll
+        for (int i = threadIdx.x; i < total; i += DT) {
+            const int r = (i / CPR) % NP, ch = i % CPR, which = i / (NP * CPR);
+            const int l = l0 + ch * VE;
+            uint4 q = make_uint4(0u, 0u, 0u, 0u);
+            if (r < p.N && l < L) q = __ldg(reinterpret_cast<const uint4*>((which ? Cs : Bs) + (bcrow0 + r) * (size_t)L + l));
+            float* o = fb + (which * NP + r) * FS + ch * VE;
+            if constexpr (LY::F32) {
+                *reinterpret_cast<uint4*>(o) = q;
+            } else {
+                *reinterpret_cast<float4*>(o) = make_float4(__uint_as_float(q.x << 16), __uint_as_float(q.x & 0xffff0000u),
+                                                            __uint_as_float(q.y << 16), __uint_as_float(q.y & 0xffff0000u));
+                *reinterpret_cast<float4*>(o + 4) = make_float4(__uint_as_float(q.z << 16), __uint_as_float(q.z & 0xffff0000u),
+                                                                __uint_as_float(q.w << 16), __uint_as_float(q.w & 0xffff0000u));
+            }
+        }
+    } else {
+        constexpr int total = (WITH_C ? 2 : 1) * NP * CL;
+        for (int i = threadIdx.x; i < total; i += DT) {
+            const int r = (i / CL) % NP, t = i % CL, which = i / (NP * CL);
+            float v = 0.0f;
+            if (r < p.N && l0 + t < L) v = io<T>::ld((which ? Cs : Bs) + (bcrow0 + r) * (size_t)L + l0 + t);
+            fb[(which * NP + r) * FS + t] = v;
+        }
+    }
+}
+
+__device__ __forceinline__ void lds4_ordered(const float* p, float (&v)[4]) {
+    const unsigned a = (unsigned)__cvta_generic_to_shared(p);
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]) : "r"(a));
+}
+__device__ __forceinline__ float ex2_ordered(float x) {
+    float y;
+    asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ void cp_async_wait_upto(int n) {
+    switch (n) {
+    case 0: cp_async_wait<0>(); break;
+    case 1: cp_async_wait<1>(); break;
+    case 2: cp_async_wait<2>(); break;
+    default: cp_async_wait<3>(); break;
+    }
+}
+
+template <typename T, class CS, bool PH2>
+__global__ void __launch_bounds__(CS::DT, CS::MINB) full_chunk_kernel(const FullParams p) {
+    using LY = ChunkLayout<T, CS>;
+    constexpr int DT = LY::DT, CL = LY::CL, NS = LY::NS, SUB = LY::SUB, RS = LY::RS, FS = LY::FS, NP = 16;
+    extern __shared__ __align__(16) unsigned char smem[];
+    T* raw = reinterpret_cast<T*>(smem);
+    float* sdl = reinterpret_cast<float*>(smem + LY::dl_off);
+
+    pdl_launch_dependents();
+    const int c = threadIdx.x;  // channel within the tile
+    const int tile = blockIdx.x % p.n_tiles;
+    const int chunk = blockIdx.x / p.n_tiles;
+    const int bk = tile / p.tiles_per_bk;
+    const int d0 = (tile % p.tiles_per_bk) * DT;
+    const int k = bk % p.K;
+    const int d = d0 + c;
+    const bool cval = d < p.D;
+    const int nrows = min(DT, p.D - d0);
+    const size_t row0 = (size_t)bk * p.D + d0;
+    const size_t bcrow0 = (size_t)bk * p.N;
+    const int l0 = chunk * CL;
+    // every sub-stage in flight at once; each is computed as soon as it lands
+#pragma unroll
+    for (int part = 0; part < NS; ++part) {
+        load_chunk_part<T, CS, PH2>(p, raw, row0, bcrow0, nrows, l0, part);
+        cp_async_commit();
+    }
+    float* fbc = reinterpret_cast<float*>(smem + LY::bc_off);
+    load_chunk_bc_f32<T, CS, PH2>(p, fbc, bcrow0, l0);
+    const float bias = cval ? p.bias[(size_t)k * p.D + d] : 0.0f;
+    const float dsk = cval ? p.Dskip[(size_t)k * p.D + d] : 0.0f;
+    float* sa2 = reinterpret_cast<float*>(smem + LY::a2_off) + c * NP;  // this channel's row (own row only)
+    const int sw = (c >> 1) & 3;
+#pragma unroll
+    for (int q = 0; q < NP / 4; ++q) {
+        float a[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int n = 4 * q + i;
+            a[i] = (cval && n < p.N) ? p.A[((size_t)k * p.D + d) * p.N + n] * kLog2e : 0.0f;
+        }
+        *reinterpret_cast<float4*>(sa2 + 4 * (q ^ sw)) = make_float4(a[0], a[1], a[2], a[3]);
+    }
+    float h[NP];
+#pragma unroll
+    for (int n = 0; n < NP; ++n) h[n] = 0.0f;
+    constexpr size_t sfl = (size_t)DT * NP;  // floats of one chunk's state (aggP uses the first DT)
+    const size_t slot = (size_t)tile * p.n_chunks + chunk;
+
+    const T* ru = raw + c * RS;
+    const T* rd = raw + (DT + c) * RS;
+    const float* rb = fbc;
+    const float* rc = fbc + NP * FS;
+    float* fd = sdl + c * FS;
+    const int nvalid = min(CL, p.L - l0);
+    T* yrow = static_cast<T*>(p.y) + (row0 + c) * (size_t)p.L + l0;
+    float ssum = 0.0f;
+#pragma unroll 1
+    for (int part = 0; part < NS; ++part) {
+        cp_async_wait_upto(NS - 1 - part);
+        __syncthreads();
+        // delta = softplus(raw + bias) (Eq. 6) for this thread's channel over the
+        // sub-stage, once per element with every step independent, as fp32 rows
+#pragma unroll
+        for (int t0 = part * SUB; t0 < part * SUB + SUB; t0 += 4) {
+            float r4[4];
+            load4(rd + t0, r4);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float v = r4[j] + bias;
+                r4[j] = p.softplus_on ? softplus(v) : v;
+                if constexpr (!PH2) ssum += r4[j];  // every step of an aggregated chunk is in range
+            }
+            *reinterpret_cast<float4*>(fd + t0) = make_float4(r4[0], r4[1], r4[2], r4[3]);
+        }
+        if (PH2 && part == 0) {
+            pdl_wait();  // the carried-in states of launch 2
+            if (chunk > 0) {
+                const float4* src = reinterpret_cast<const float4*>(p.incH + (slot - 1) * sfl + (size_t)c * NP);
+#pragma unroll
+                for (int q = 0; q < NP / 4; ++q) {
+                    const float4 v = __ldcg(src + q);
+                    h[4 * q] = v.x;
+                    h[4 * q + 1] = v.y;
+                    h[4 * q + 2] = v.z;
+                    h[4 * q + 3] = v.w;
+                }
+            }
+        }
+#pragma unroll 1
+        for (int t0 = part * SUB; t0 < part * SUB + SUB; t0 += 4) {
+            float dl4[4], du4[4];
+            {
+                float u4[4];
+                load4(ru + t0, u4);
+                load4(fd + t0, dl4);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) du4[j] = dl4[j] * u4[j];
+            }
+            float ya[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+            for (int q = 0; q < NP / 4; ++q) {
+                float a2[4];
+                load4(sa2 + 4 * (q ^ sw), a2);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int n = 4 * q + i;
+                    // B, C reads and the exponentials as ordered (volatile) asm: left
+                    // free, the compiler hoists all 32 row reads of the block and runs
+                    // out of registers
+                    float b4[4], c4[4];
+                    lds4_ordered(rb + n * FS + t0, b4);
+                    if constexpr (PH2) lds4_ordered(rc + n * FS + t0, c4);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        h[n] = fmaf(ex2_ordered(dl4[j] * a2[i]), h[n], du4[j] * b4[j]);
+                        if constexpr (PH2) ya[j] = fmaf(c4[j], h[n], ya[j]);
+                    }
+                }
+            }
+            if constexpr (PH2) {
+                float u4[4], o[4];
+                load4(ru + t0, u4);  // read again rather than held across the state loop
+#pragma unroll
+                for (int j = 0; j < 4; ++j) o[j] = fmaf(dsk, u4[j], ya[j]);
+                if (cval) store_row<T, 4>(yrow + t0, o, nvalid - t0, p.vec);
+            }
+        }
+    }
+    if constexpr (!PH2) {
+        p.aggP[slot * sfl + c] = ssum;
+        float4* dst = reinterpret_cast<float4*>(p.aggH + slot * sfl + (size_t)c * NP);
+#pragma unroll
+        for (int q = 0; q < NP / 4; ++q) dst[q] = make_float4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
+    }
+}
+
+// Launch 2 of the chunked variant: one thread per (channel, state) folds the
+// chunk aggregates of its tile left to right.  The fold itself is a short FMA
+// chain; what costs is the latency of fetching the aggregates, so they are
+// read kCarryBatch chunks at a time with the next batch in flight while the
+// current one is folded (compile-time chunk stride: no per-load address math).
+constexpr int kCarryThreads = 128;  // 8 channels x 16 states
+constexpr int kCarryBatch = 16;
+
+template <int DT>
+__global__ void __launch_bounds__(kCarryThreads) full_carry_kernel(const FullParams p) {
+    constexpr int groups = DT / 8;
+    constexpr size_t sfl = (size_t)DT * 16;
+    pdl_launch_dependents();
+    const int tid = threadIdx.x;
+    const int tile = blockIdx.x / groups;
+    const int c = (blockIdx.x % groups) * 8 + (tid >> 4), n = tid & 15;
+    const int bk = tile / p.tiles_per_bk;
+    const int d = (tile % p.tiles_per_bk) * DT + c;
+    const int k = bk % p.K;
+    const float A2 = (d < p.D && n < p.N) ? p.A[((size_t)k * p.D + d) * p.N + n] * kLog2e : 0.0f;
+    const int M = p.n_chunks - 1;  // aggregates to fold: the last chunk's is never needed
+    const size_t base = (size_t)tile * p.n_chunks * sfl;
+    const float* sp = p.aggP + base + c;
+    const float* hp = p.aggH + base + (size_t)c * 16 + n;
+    float* ip = p.incH + base + (size_t)c * 16 + n;
+    float S[2][kCarryBatch], H[2][kCarryBatch];
+    auto fetch = [&](int m0, float(&s)[kCarryBatch], float(&hh)[kCarryBatch]) {
+#pragma unroll
+        for (int q = 0; q < kCarryBatch; ++q) {
+            if (m0 + q < M) {
+                s[q] = __ldcg(sp + (size_t)q * sfl);
+                hh[q] = __ldcg(hp + (size_t)q * sfl);
+            }
+        }
+        sp += kCarryBatch * sfl;
+        hp += kCarryBatch * sfl;
+    };
+    auto fold = [&](int m0, const float(&s)[kCarryBatch], const float(&hh)[kCarryBatch], float& RH) {
+#pragma unroll
+        for (int q = 0; q < kCarryBatch; ++q) {
+            if (m0 + q < M) {
+                RH = fmaf(ex2(A2 * s[q]), RH, hh[q]);
+                ip[(size_t)q * sfl] = RH;
+            }
+        }
+        ip += kCarryBatch * sfl;
+    };
+    float RH = 0.0f;
+    pdl_wait();  // the aggregates of launch 1
+    fetch(0, S[0], H[0]);
+    for (int m0 = 0; m0 < M; m0 += 2 * kCarryBatch) {
+        if (m0 + kCarryBatch < M) fetch(m0 + kCarryBatch, S[1], H[1]);
+        fold(m0, S[0], H[0], RH);
+        if (m0 + kCarryBatch >= M) break;
+        if (m0 + 2 * kCarryBatch < M) fetch(m0 + 2 * kCarryBatch, S[0], H[0]);
+        fold(m0 + kCarryBatch, S[1], H[1], RH);
+    }
+}
+
 // ------------------------------------------------------------------ host side
 
 struct KernelInfo {
-    const void* fn;
+    const void* fn;  // the kernel that writes y
     size_t smem;
     int G, DT, threads, ts;
+    const void* agg = nullptr;  // chunked variant: the aggregate kernel (launch 1)
 };
 
 template <typename T, int NP, class SH, bool ZOH>
@@ -720,10 +1068,28 @@ KernelInfo lanes_info() {
     return {attr_err == cudaSuccess ? fn : nullptr, LY::raw_bytes, 16, LY::DT, 256, LY::TS};
 }
 
+template <typename T, class CS>
+KernelInfo chunk_info() {
+    using LY = ChunkLayout<T, CS>;
+    const void* fa = reinterpret_cast<const void*>(&full_chunk_kernel<T, CS, false>);
+    const void* ff = reinterpret_cast<const void*>(&full_chunk_kernel<T, CS, true>);
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [&] {
+        attr_err = cudaFuncSetAttribute(fa, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LY::bytes);
+        if (attr_err == cudaSuccess)
+            attr_err = cudaFuncSetAttribute(ff, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LY::bytes);
+    });
+    const bool ok = attr_err == cudaSuccess;
+    return {ok ? ff : nullptr, LY::bytes, 1, LY::DT, LY::DT, LY::CL, ok ? fa : nullptr};
+}
+
 // Tile shapes per padded state count, in order of preference (fewest lanes
 // per channel first).  The zero-order-hold variant uses the first shape.
-int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 8; }
-constexpr int kLanesShape = 7;  // index of the lane-per-state variant (N <= 16 padded to 16)
+int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 11; }
+constexpr int kLanesShape = 7;   // index of the lane-per-state variant (N <= 16 padded to 16)
+constexpr int kChunkShape = 8;   // first index of the three-launch chunked variant (shapes 8, 9, 10)
+bool is_chunk_shape(int np, int shape) { return np == 16 && shape >= kChunkShape && shape < kChunkShape + 3; }
 
 template <typename T, bool ZOH>
 KernelInfo pick_t(int np, int shape) {
@@ -744,6 +1110,9 @@ KernelInfo pick_t(int np, int shape) {
         case 5: return info_for<T, 16, Shape<1, 64, 16, 3>, false>();
         case 6: return info_for<T, 16, Shape<1, 32, 16, 3>, false>();
         case 7: return lanes_info<T, false>();
+        case 8: return chunk_info<T, ChunkShape<64, 32, 2, 8>>();
+        case 9: return chunk_info<T, ChunkShape<128, 32, 2, 4>>();
+        case 10: return chunk_info<T, ChunkShape<64, 64, 4, 5>>();
         default: return info_for<T, 16, Shape<1, 128, 0, 3, 7>, ZOH>();
         }
     }
@@ -803,8 +1172,9 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     };
     // Rules measured on GB300 over the benchmark workloads: plenty of rows ->
     // one lane per channel; a fair number -> two lanes; too few -> cut L into
-    // chunks, with one lane per channel when the chunks stay long (>= 256
-    // steps) and the widest split otherwise (chunks >= 128 steps).
+    // chunks: 64-step chunks of the three-launch variant while they fit in two
+    // waves, else look-back chunks with one lane per channel when they stay
+    // long (>= 256 steps) and the widest split otherwise (>= 128 steps).
     int shape = 0, n_chunks = 1, forced_chunks = 0, env_shape = 0;
     KernelInfo ki{};
     long long res = 0;
@@ -839,10 +1209,24 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
             KernelInfo km{};
             long long rm = 0;
             if ((st = info(r.mid, &km, &rm)) != VMB_OK) return st;
+            KernelInfo kc{};
+            long long rc = 0;
+            long long chunk_ctas = 0;
+            if (np == 16) {
+                // few rows: the three-launch chunked variant while its grid of
+                // 64-step chunks fits in two waves (beyond that its aggregate
+                // traffic outweighs the look-back's second pass)
+                if ((st = info(kChunkShape + 2, &kc, &rc)) != VMB_OK) return st;
+                chunk_ctas = a.B * a.K * (long long)((a.D + kc.DT - 1) / kc.DT) * ((a.L + kc.ts - 1) / kc.ts);
+            }
             if (rows * km.G * 2 >= rm * km.threads) {
                 shape = r.mid;
                 ki = km;
                 res = rm;
+            } else if (np == 16 && chunk_ctas <= 2 * rc) {
+                shape = kChunkShape + 2;
+                ki = kc;
+                res = rc;
             } else {
                 KernelInfo kn{};
                 long long rn = 0;
@@ -866,6 +1250,7 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
             }
         }
     }
+    if (is_chunk_shape(np, shape)) n_chunks = (a.L + ki.ts - 1) / ki.ts;  // chunks of exactly ts steps
     if (n_chunks < 1) n_chunks = 1;
     ScanPlan p{};
     p.np = np;
@@ -881,6 +1266,24 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     p.ws_bytes = ws_layout(p).total;
     *plan = p;
     return VMB_OK;
+}
+
+// Launch that may begin while the previous kernel of the stream is still
+// running (programmatic stream serialization); the kernel orders its reads of
+// that kernel's results with griddepcontrol.wait.
+static cudaError_t launch_pdl(const void* fn, unsigned grid, int threads, size_t smem, void** args,
+                              cudaStream_t stream) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3((unsigned)threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelExC(&cfg, fn, args);
 }
 
 vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream) {
@@ -917,6 +1320,19 @@ vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     p.incH = reinterpret_cast<float*>(ws + w.incH_off);
     const unsigned grid = (unsigned)(plan.n_seq * plan.n_chunks);
     void* args[] = {&p};
+    if (is_chunk_shape(plan.np, plan.split) && plan.n_chunks > 1) {
+        // launches 1 and 2 of the chunked variant: aggregates, then the carry fold
+        if (!ki.agg) return VMB_ERR_CUDA;
+        const unsigned grid_agg = (unsigned)(plan.n_seq * (plan.n_chunks - 1));
+        cudaError_t e = cudaLaunchKernel(ki.agg, dim3(grid_agg), dim3(ki.threads), args, ki.smem, stream);
+        if (e != cudaSuccess) return VMB_ERR_CUDA;
+        const unsigned grid_carry = (unsigned)(plan.n_seq * (ki.DT / 8));
+        const void* carry = ki.DT == 128 ? reinterpret_cast<const void*>(&full_carry_kernel<128>)
+                                         : reinterpret_cast<const void*>(&full_carry_kernel<64>);
+        if (launch_pdl(carry, grid_carry, kCarryThreads, 0, args, stream) != cudaSuccess) return VMB_ERR_CUDA;
+        // launch 3 loads its tile and applies the softplus before it waits for the carry
+        return launch_pdl(ki.fn, grid, ki.threads, ki.smem, args, stream) == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+    }
     cudaError_t e = cudaLaunchKernel(ki.fn, dim3(grid), dim3(ki.threads), args, ki.smem, stream);
     return e == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
 }

@@ -172,7 +172,8 @@ def test_lookback_wait_times_out_cleanly(mean):
     check(to_numpy(y), ref, "f32", "after timeout")
 
 
-@pytest.mark.parametrize("plan", ["0", "1", "2", "3", "4", "5", "6", "7", "0,3", "3,5", "4,2", "5,4", "6,7", "7,3", "7,6"])
+@pytest.mark.parametrize("plan", ["0", "1", "2", "3", "4", "5", "6", "7", "8", "9", "10", "0,3", "3,5", "4,2", "5,4",
+                                  "6,7", "7,3", "7,6"])
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
 def test_every_tile_shape(plan, dt, monkeypatch):
     """Each tile shape of the full scan (and forced L-chunking) against the oracle."""
@@ -185,6 +186,35 @@ def test_every_tile_shape(plan, dt, monkeypatch):
     assert vmb.vmb_read_status() == vmb.VMB_OK
     _, ref, _ = oracle.ss2d_full(inp)
     check(to_numpy(y), ref, dt, f"full y plan {plan}")
+
+
+CHUNKED_CASES = [
+    # (B, D, N, H, W, dtype)
+    (1, 72, 16, 20, 30, "f32"),   # L = 600: ragged last chunk, ragged channel tile, vector rows
+    (1, 72, 16, 23, 29, "f32"),   # L = 667: element-wise rows
+    (2, 40, 12, 17, 19, "bf16"),  # padded states, odd L, bf16
+    (2, 64, 16, 16, 24, "bf16"),  # bf16 vector rows
+    (1, 24, 16, 5, 5, "f32"),     # one chunk only: no aggregate or carry launch
+]
+
+
+@pytest.mark.parametrize("plan", ["8", "9", "10"])
+@pytest.mark.parametrize("case", CHUNKED_CASES, ids=[f"B{s[0]}_D{s[1]}_N{s[2]}_{s[3]}x{s[4]}_{s[5]}"
+                                                     for s in CHUNKED_CASES])
+def test_chunked_full_scan(plan, case, monkeypatch):
+    """The three-launch chunked full scan (aggregates, carry fold, rerun) against the oracle."""
+    monkeypatch.setenv("VMB_FULL_PLAN", plan)
+    B, D, N, H, W, dt = case
+    wl = workloads.small_case(B=B, D=D, N=N, H=H, W=W, dtype=dt, seed=31 + D)
+    inp = workloads.make_inputs(wl)
+    g = to_device(inp, DEV)
+    xs = vmb.vmb_cross_scan(g["x"])
+    y = vmb.vmb_selective_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W)
+    y2 = vmb.vmb_selective_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W)
+    assert vmb.vmb_read_status() == vmb.VMB_OK
+    _, ref, _ = oracle.ss2d_full(inp)
+    check(to_numpy(y), ref, dt, f"chunked full y plan {plan}")
+    assert torch.equal(y, y2), "the chunked scan must be deterministic"
 
 
 @pytest.mark.parametrize("tc", ["32", "64", "128"])
