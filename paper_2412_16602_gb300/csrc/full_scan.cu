@@ -708,19 +708,20 @@ __global__ void __launch_bounds__(256) full_scan_lanes_kernel(const FullParams p
 //      inclusive states of the look-back path, so both give the same bits);
 //   3. every chunk reruns its steps from the carried-in state inc_{m-1}, Eq. 3,
 //      and writes y.
-// One lane per channel owns all 16 states, the cheapest update per state; B and
-// C are read from their [n][t] rows four steps at a time (broadcast reads, no
-// transpose), so a step costs one 128-bit read per state and operand.
-template <int DT_, int CL_, int NS_, int MINB_>
+// G lanes per channel (1 or 2) own 16 / G of its states each; B and C are read
+// from fp32 [n][t] rows four steps at a time (broadcast reads, no transpose),
+// so a step costs one 128-bit read per state and operand.
+template <int G_, int DT_, int CL_, int NS_, int MINB_>
 struct ChunkShape {
-    static constexpr int DT = DT_, CL = CL_, NS = NS_, MINB = MINB_;  // NS: load sub-stages per chunk
+    static constexpr int G = G_, DT = DT_, CL = CL_, NS = NS_, MINB = MINB_;  // NS: load sub-stages per chunk
 };
 
 template <typename T, class CS>
 struct ChunkLayout {
-    static constexpr int DT = CS::DT, CL = CS::CL, NS = CS::NS, SUB = CL / NS, MINB = CS::MINB, NP = 16;
+    static constexpr int G = CS::G, DT = CS::DT, CL = CS::CL, NS = CS::NS, SUB = CL / NS, MINB = CS::MINB, NP = 16;
+    static constexpr int THREADS = G * DT, NG = NP / G;
     static constexpr int PAD = 16 / (int)sizeof(T);
-    static constexpr int RS = CL + PAD;           // row stride (elements); rows start 16-byte aligned
+    static constexpr int RS = CL + PAD;  // row stride (elements); rows start 16-byte aligned
     static constexpr int ROWS = 2 * DT;  // u, delta (B and C go to the fp32 area)
     static constexpr size_t raw_bytes = a16((size_t)ROWS * RS * sizeof(T));
     // fp32 delta after the softplus: in place of the raw delta rows for fp32
@@ -732,11 +733,13 @@ struct ChunkLayout {
     // storage one conversion per element instead of one per element and channel)
     static constexpr size_t bc_off = F32 ? raw_bytes : raw_bytes + (size_t)DT * FS * 4;
     static constexpr size_t a2_off = bc_off + (size_t)2 * NP * FS * 4;
-    // A * log2 e per channel: [DT][16] with the four 16-byte quads of a row
-    // swizzled by (c >> 1) & 3, so eight consecutive channels read their quad q
-    // from distinct banks
-    static constexpr size_t bytes = a2_off + (size_t)DT * NP * 4;
-    static_assert(CL % NS == 0 && SUB % 8 == 0 && DT % 32 == 0 && NS <= 4, "chunk tile shape");
+    // G = 1: A * log2 e per channel in shared memory, [DT][16] with the four
+    // 16-byte quads of a row swizzled by (c >> 1) & 3 so that eight consecutive
+    // channels read their quad q from distinct banks (in registers it would
+    // not leave room for the 16 states); G = 2 keeps its 8 values in registers
+    static constexpr size_t bytes = a2_off + (G == 1 ? (size_t)DT * NP * 4 : 0);
+    static_assert(CL % NS == 0 && SUB % (4 * G) == 0 && DT % 32 == 0 && NS <= 4 && (G == 1 || G == 2),
+                  "chunk tile shape");
     static_assert(sizeof(T) == 2 || RS == FS, "fp32 delta rows are rewritten in place");
 };
 
@@ -746,21 +749,22 @@ struct ChunkLayout {
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
-// Load of sub-stage `part` (steps part*SUB .. part*SUB+SUB-1) of the chunk
-// tile: thread i always copies 16-byte column i % CPR of rows i / CPR + k *
-// (DT / CPR), so the addresses advance by a fixed row stride.  Rows that are
-// not 16-byte aligned take the element-wise loader, all of it with part 0.
-template <typename T, class CS, bool WITH_C>
-__device__ __forceinline__ void load_chunk_part(const FullParams& p, T* dst, size_t row0, size_t bcrow0, int nrows,
-                                                int l0, int part) {
+// Load of sub-stage `part` (steps part*SUB .. part*SUB+SUB-1) of the u and
+// delta rows of the chunk tile: thread i always copies 16-byte column i % CPR
+// of rows i / CPR + k * (THREADS / CPR), so the addresses advance by a fixed
+// row stride.  Rows that are not 16-byte aligned take the element-wise loader,
+// all of it with part 0.
+template <typename T, class CS>
+__device__ __forceinline__ void load_chunk_part(const FullParams& p, T* dst, size_t row0, int nrows, int l0,
+                                                int part) {
     using LY = ChunkLayout<T, CS>;
-    constexpr int DT = LY::DT, CL = LY::CL, SUB = LY::SUB, RS = LY::RS, NP = 16;
+    constexpr int DT = LY::DT, CL = LY::CL, SUB = LY::SUB, RS = LY::RS, NP = 16, THREADS = LY::THREADS;
     const int L = p.L;
     if (p.vec) {
         constexpr int VE = 16 / (int)sizeof(T);
-        constexpr int CPR = SUB / VE;  // 16-byte chunks per row and sub-stage
-        constexpr int RPP = DT / CPR;  // rows per pass of the DT threads
-        static_assert(DT % CPR == 0, "tile loader mapping");
+        constexpr int CPR = SUB / VE;       // 16-byte chunks per row and sub-stage
+        constexpr int RPP = THREADS / CPR;  // rows per pass of the CTA
+        static_assert(THREADS % CPR == 0 && DT % RPP == 0, "tile loader mapping");
         const int ch = threadIdx.x % CPR, r0 = threadIdx.x / CPR;
         const int t = part * SUB + ch * VE;  // step within the chunk
         const bool colok = l0 + t < L;
@@ -776,7 +780,7 @@ __device__ __forceinline__ void load_chunk_part(const FullParams& p, T* dst, siz
             cp_async16(dst + (DT + r) * RS + t, ok ? dl + off : dl, ok ? 16 : 0);
         }
     } else if (part == 0) {
-        load_tile<T, NP, DT, CL, RS, DT, WITH_C, false>(p, dst, row0, bcrow0, nrows, l0);
+        load_tile<T, NP, DT, CL, RS, THREADS, false, false>(p, dst, row0, 0, nrows, l0);
     }
 }
 
@@ -785,7 +789,7 @@ __device__ __forceinline__ void load_chunk_part(const FullParams& p, T* dst, siz
 template <typename T, class CS, bool WITH_C>
 __device__ __forceinline__ void load_chunk_bc_f32(const FullParams& p, float* fb, size_t bcrow0, int l0) {
     using LY = ChunkLayout<T, CS>;
-    constexpr int DT = LY::DT, CL = LY::CL, FS = LY::FS, NP = 16;
+    constexpr int CL = LY::CL, FS = LY::FS, NP = 16, THREADS = LY::THREADS;
     const int L = p.L;
     const T* Bs = static_cast<const T*>(p.Bs);
     const T* Cs = static_cast<const T*>(p.Cs);
@@ -794,7 +798,7 @@ __device__ __forceinline__ void load_chunk_bc_f32(const FullParams& p, float* fb
         constexpr int CPR = CL / VE;  // 16-byte chunks per row
         constexpr int total = (WITH_C ? 2 : 1) * NP * CPR;
 #pragma unroll
-        for (int i = threadIdx.x; i < total; i += DT) {
+        for (int i = threadIdx.x; i < total; i += THREADS) {
             const int r = (i / CPR) % NP, ch = i % CPR, which = i / (NP * CPR);
             const int l = l0 + ch * VE;
             uint4 q = make_uint4(0u, 0u, 0u, 0u);
@@ -811,7 +815,7 @@ __device__ __forceinline__ void load_chunk_bc_f32(const FullParams& p, float* fb
         }
     } else {
         constexpr int total = (WITH_C ? 2 : 1) * NP * CL;
-        for (int i = threadIdx.x; i < total; i += DT) {
+        for (int i = threadIdx.x; i < total; i += THREADS) {
             const int r = (i / CL) % NP, t = i % CL, which = i / (NP * CL);
             float v = 0.0f;
             if (r < p.N && l0 + t < L) v = io<T>::ld((which ? Cs : Bs) + (bcrow0 + r) * (size_t)L + l0 + t);
@@ -840,15 +844,16 @@ __device__ __forceinline__ void cp_async_wait_upto(int n) {
 }
 
 template <typename T, class CS, bool PH2>
-__global__ void __launch_bounds__(CS::DT, CS::MINB) full_chunk_kernel(const FullParams p) {
+__global__ void __launch_bounds__(ChunkLayout<T, CS>::THREADS, CS::MINB) full_chunk_kernel(const FullParams p) {
     using LY = ChunkLayout<T, CS>;
-    constexpr int DT = LY::DT, CL = LY::CL, NS = LY::NS, SUB = LY::SUB, RS = LY::RS, FS = LY::FS, NP = 16;
+    constexpr int G = LY::G, NG = LY::NG, DT = LY::DT, CL = LY::CL, NS = LY::NS, SUB = LY::SUB, RS = LY::RS,
+                  FS = LY::FS, NP = 16;
     extern __shared__ __align__(16) unsigned char smem[];
     T* raw = reinterpret_cast<T*>(smem);
     float* sdl = reinterpret_cast<float*>(smem + LY::dl_off);
 
     pdl_launch_dependents();
-    const int c = threadIdx.x;  // channel within the tile
+    const int c = threadIdx.x / G, g = threadIdx.x % G;  // channel within the tile, lane of the channel
     const int tile = blockIdx.x % p.n_tiles;
     const int chunk = blockIdx.x / p.n_tiles;
     const int bk = tile / p.tiles_per_bk;
@@ -863,47 +868,58 @@ __global__ void __launch_bounds__(CS::DT, CS::MINB) full_chunk_kernel(const Full
     // every sub-stage in flight at once; each is computed as soon as it lands
 #pragma unroll
     for (int part = 0; part < NS; ++part) {
-        load_chunk_part<T, CS, PH2>(p, raw, row0, bcrow0, nrows, l0, part);
+        load_chunk_part<T, CS>(p, raw, row0, nrows, l0, part);
         cp_async_commit();
     }
     float* fbc = reinterpret_cast<float*>(smem + LY::bc_off);
     load_chunk_bc_f32<T, CS, PH2>(p, fbc, bcrow0, l0);
     const float bias = cval ? p.bias[(size_t)k * p.D + d] : 0.0f;
     const float dsk = cval ? p.Dskip[(size_t)k * p.D + d] : 0.0f;
-    float* sa2 = reinterpret_cast<float*>(smem + LY::a2_off) + c * NP;  // this channel's row (own row only)
+    const float* Ad = p.A + ((size_t)k * p.D + d) * p.N;
+    float A2r[G == 1 ? 1 : NG];  // G = 2: this lane's A * log2 e
+    float* sa2 = reinterpret_cast<float*>(smem + LY::a2_off) + c * NP;  // G = 1: this channel's row (own row only)
     const int sw = (c >> 1) & 3;
+    if constexpr (G == 1) {
 #pragma unroll
-    for (int q = 0; q < NP / 4; ++q) {
-        float a[4];
+        for (int q = 0; q < NP / 4; ++q) {
+            float a[4];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int n = 4 * q + i;
-            a[i] = (cval && n < p.N) ? p.A[((size_t)k * p.D + d) * p.N + n] * kLog2e : 0.0f;
+            for (int i = 0; i < 4; ++i) {
+                const int n = 4 * q + i;
+                a[i] = (cval && n < p.N) ? Ad[n] * kLog2e : 0.0f;
+            }
+            *reinterpret_cast<float4*>(sa2 + 4 * (q ^ sw)) = make_float4(a[0], a[1], a[2], a[3]);
         }
-        *reinterpret_cast<float4*>(sa2 + 4 * (q ^ sw)) = make_float4(a[0], a[1], a[2], a[3]);
-    }
-    float h[NP];
+    } else {
 #pragma unroll
-    for (int n = 0; n < NP; ++n) h[n] = 0.0f;
+        for (int i = 0; i < NG; ++i) {
+            const int n = g * NG + i;
+            A2r[i] = (cval && n < p.N) ? Ad[n] * kLog2e : 0.0f;
+        }
+    }
+    float h[NG];
+#pragma unroll
+    for (int i = 0; i < NG; ++i) h[i] = 0.0f;
     constexpr size_t sfl = (size_t)DT * NP;  // floats of one chunk's state (aggP uses the first DT)
     const size_t slot = (size_t)tile * p.n_chunks + chunk;
 
     const T* ru = raw + c * RS;
     const T* rd = raw + (DT + c) * RS;
-    const float* rb = fbc;
-    const float* rc = fbc + NP * FS;
+    const float* rb = fbc + g * NG * FS;  // this lane's B rows
+    const float* rc = rb + NP * FS;
     float* fd = sdl + c * FS;
     const int nvalid = min(CL, p.L - l0);
     T* yrow = static_cast<T*>(p.y) + (row0 + c) * (size_t)p.L + l0;
-    float ssum = 0.0f;
+    float ssum = 0.0f;  // this lane's share of the sum of delta over the chunk
 #pragma unroll 1
     for (int part = 0; part < NS; ++part) {
         cp_async_wait_upto(NS - 1 - part);
         __syncthreads();
-        // delta = softplus(raw + bias) (Eq. 6) for this thread's channel over the
-        // sub-stage, once per element with every step independent, as fp32 rows
+        // delta = softplus(raw + bias) (Eq. 6) of this channel over the sub-stage,
+        // once per element (the G lanes take alternate 4-step groups) with every
+        // step independent, as fp32 rows
 #pragma unroll
-        for (int t0 = part * SUB; t0 < part * SUB + SUB; t0 += 4) {
+        for (int t0 = part * SUB + 4 * g; t0 < part * SUB + SUB; t0 += 4 * G) {
             float r4[4];
             load4(rd + t0, r4);
 #pragma unroll
@@ -914,12 +930,13 @@ __global__ void __launch_bounds__(CS::DT, CS::MINB) full_chunk_kernel(const Full
             }
             *reinterpret_cast<float4*>(fd + t0) = make_float4(r4[0], r4[1], r4[2], r4[3]);
         }
+        if constexpr (G > 1) __syncwarp();  // the other lane's delta groups
         if (PH2 && part == 0) {
             pdl_wait();  // the carried-in states of launch 2
             if (chunk > 0) {
-                const float4* src = reinterpret_cast<const float4*>(p.incH + (slot - 1) * sfl + (size_t)c * NP);
+                const float4* src = reinterpret_cast<const float4*>(p.incH + (slot - 1) * sfl + (size_t)c * NP + g * NG);
 #pragma unroll
-                for (int q = 0; q < NP / 4; ++q) {
+                for (int q = 0; q < NG / 4; ++q) {
                     const float4 v = __ldcg(src + q);
                     h[4 * q] = v.x;
                     h[4 * q + 1] = v.y;
@@ -940,14 +957,19 @@ __global__ void __launch_bounds__(CS::DT, CS::MINB) full_chunk_kernel(const Full
             }
             float ya[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-            for (int q = 0; q < NP / 4; ++q) {
+            for (int q = 0; q < NG / 4; ++q) {
                 float a2[4];
-                load4(sa2 + 4 * (q ^ sw), a2);
+                if constexpr (G == 1) {
+                    load4(sa2 + 4 * (q ^ sw), a2);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) a2[i] = A2r[4 * q + i];
+                }
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
-                    const int n = 4 * q + i;
+                    const int n = 4 * q + i;  // state index within this lane's share
                     // B, C reads and the exponentials as ordered (volatile) asm: left
-                    // free, the compiler hoists all 32 row reads of the block and runs
+                    // free, the compiler hoists all row reads of the block and runs
                     // out of registers
                     float b4[4], c4[4];
                     lds4_ordered(rb + n * FS + t0, b4);
@@ -960,78 +982,94 @@ __global__ void __launch_bounds__(CS::DT, CS::MINB) full_chunk_kernel(const Full
                 }
             }
             if constexpr (PH2) {
-                float u4[4], o[4];
-                load4(ru + t0, u4);  // read again rather than held across the state loop
+                if constexpr (G == 1) {
+                    float u4[4], o[4];
+                    load4(ru + t0, u4);  // read again rather than held across the state loop
 #pragma unroll
-                for (int j = 0; j < 4; ++j) o[j] = fmaf(dsk, u4[j], ya[j]);
-                if (cval) store_row<T, 4>(yrow + t0, o, nvalid - t0, p.vec);
+                    for (int j = 0; j < 4; ++j) o[j] = fmaf(dsk, u4[j], ya[j]);
+                    if (cval) store_row<T, 4>(yrow + t0, o, nvalid - t0, p.vec);
+                } else {
+                    // lane g keeps steps 2g, 2g + 1 and adds the other lane's share
+                    const float k0 = g ? ya[2] : ya[0], k1 = g ? ya[3] : ya[1];
+                    const float s0 = g ? ya[0] : ya[2], s1 = g ? ya[1] : ya[3];
+                    float u4[4], o[2];
+                    load4(ru + t0, u4);
+                    o[0] = fmaf(dsk, g ? u4[2] : u4[0], k0 + __shfl_xor_sync(0xffffffffu, s0, 1));
+                    o[1] = fmaf(dsk, g ? u4[3] : u4[1], k1 + __shfl_xor_sync(0xffffffffu, s1, 1));
+                    if (cval) store_row<T, 2>(yrow + t0 + 2 * g, o, nvalid - t0 - 2 * g, p.vec);
+                }
             }
         }
     }
     if constexpr (!PH2) {
-        p.aggP[slot * sfl + c] = ssum;
-        float4* dst = reinterpret_cast<float4*>(p.aggH + slot * sfl + (size_t)c * NP);
+        if constexpr (G > 1) ssum += __shfl_xor_sync(0xffffffffu, ssum, 1);  // both lanes: lane 0 + lane 1
+        if (g == 0) p.aggP[slot * sfl + c] = ssum;
+        float4* dst = reinterpret_cast<float4*>(p.aggH + slot * sfl + (size_t)c * NP + g * NG);
 #pragma unroll
-        for (int q = 0; q < NP / 4; ++q) dst[q] = make_float4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
+        for (int q = 0; q < NG / 4; ++q) dst[q] = make_float4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
     }
 }
 
-// Launch 2 of the chunked variant: one thread per (channel, state) folds the
-// chunk aggregates of its tile left to right.  The fold itself is a short FMA
-// chain; what costs is the latency of fetching the aggregates, so they are
-// read kCarryBatch chunks at a time with the next batch in flight while the
-// current one is folded (compile-time chunk stride: no per-load address math).
-constexpr int kCarryThreads = 128;  // 8 channels x 16 states
-constexpr int kCarryBatch = 16;
+// Launch 2 of the chunked variant: the inclusive state after every chunk,
+// inc_m = 2^(A_n log2 e S_m) inc_{m-1} + H_m from inc_{-1} = 0, for every
+// (channel, state) of a tile.  The chain is short in arithmetic but long in
+// latency, so it is cut in two levels: warp s of a CTA owns segment s (kSegLen
+// consecutive chunks) for 32 (channel, state) pairs, folds it from zero, the
+// eight segment results are combined in shared memory (a fixed order, so the
+// result is deterministic), and each warp refolds its segment from its
+// carry-in, writing inc_m.  Groups of kSegs segments follow one another.
+constexpr int kSegLen = 16;
+constexpr int kSegs = 8;
+constexpr int kCarryThreads = 32 * kSegs;  // 32 pairs (2 channels x 16 states) x kSegs segments
 
 template <int DT>
 __global__ void __launch_bounds__(kCarryThreads) full_carry_kernel(const FullParams p) {
-    constexpr int groups = DT / 8;
+    constexpr int groups = DT / 2;
     constexpr size_t sfl = (size_t)DT * 16;
+    __shared__ float segP[kSegs][32], segH[kSegs][32];
     pdl_launch_dependents();
-    const int tid = threadIdx.x;
+    const int lane = threadIdx.x & 31, seg = threadIdx.x >> 5;
     const int tile = blockIdx.x / groups;
-    const int c = (blockIdx.x % groups) * 8 + (tid >> 4), n = tid & 15;
+    const int c = (blockIdx.x % groups) * 2 + (lane >> 4), n = lane & 15;
     const int bk = tile / p.tiles_per_bk;
     const int d = (tile % p.tiles_per_bk) * DT + c;
     const int k = bk % p.K;
     const float A2 = (d < p.D && n < p.N) ? p.A[((size_t)k * p.D + d) * p.N + n] * kLog2e : 0.0f;
     const int M = p.n_chunks - 1;  // aggregates to fold: the last chunk's is never needed
     const size_t base = (size_t)tile * p.n_chunks * sfl;
-    const float* sp = p.aggP + base + c;
-    const float* hp = p.aggH + base + (size_t)c * 16 + n;
-    float* ip = p.incH + base + (size_t)c * 16 + n;
-    float S[2][kCarryBatch], H[2][kCarryBatch];
-    auto fetch = [&](int m0, float(&s)[kCarryBatch], float(&hh)[kCarryBatch]) {
-#pragma unroll
-        for (int q = 0; q < kCarryBatch; ++q) {
-            if (m0 + q < M) {
-                s[q] = __ldcg(sp + (size_t)q * sfl);
-                hh[q] = __ldcg(hp + (size_t)q * sfl);
-            }
-        }
-        sp += kCarryBatch * sfl;
-        hp += kCarryBatch * sfl;
-    };
-    auto fold = [&](int m0, const float(&s)[kCarryBatch], const float(&hh)[kCarryBatch], float& RH) {
-#pragma unroll
-        for (int q = 0; q < kCarryBatch; ++q) {
-            if (m0 + q < M) {
-                RH = fmaf(ex2(A2 * s[q]), RH, hh[q]);
-                ip[(size_t)q * sfl] = RH;
-            }
-        }
-        ip += kCarryBatch * sfl;
-    };
-    float RH = 0.0f;
     pdl_wait();  // the aggregates of launch 1
-    fetch(0, S[0], H[0]);
-    for (int m0 = 0; m0 < M; m0 += 2 * kCarryBatch) {
-        if (m0 + kCarryBatch < M) fetch(m0 + kCarryBatch, S[1], H[1]);
-        fold(m0, S[0], H[0], RH);
-        if (m0 + kCarryBatch >= M) break;
-        if (m0 + 2 * kCarryBatch < M) fetch(m0 + 2 * kCarryBatch, S[0], H[0]);
-        fold(m0 + kCarryBatch, S[1], H[1], RH);
+    float carry = 0.0f;  // inclusive state before the current group
+    for (int g0 = 0; g0 < M; g0 += kSegs * kSegLen) {
+        const int m0 = g0 + seg * kSegLen;
+        const float* sp = p.aggP + base + (size_t)m0 * sfl + c;
+        const float* hp = p.aggH + base + (size_t)m0 * sfl + (size_t)c * 16 + n;
+        float e[kSegLen], hv[kSegLen];
+#pragma unroll
+        for (int q = 0; q < kSegLen; ++q) {
+            const bool ok = m0 + q < M;
+            e[q] = ok ? __ldcg(sp + (size_t)q * sfl) : 0.0f;
+            hv[q] = ok ? __ldcg(hp + (size_t)q * sfl) : 0.0f;  // past M: identity (factor 1, H 0)
+        }
+        float P = 1.0f, Hl = 0.0f;
+#pragma unroll
+        for (int q = 0; q < kSegLen; ++q) {
+            e[q] = ex2(A2 * e[q]);
+            Hl = fmaf(e[q], Hl, hv[q]);
+            P *= e[q];
+        }
+        segP[seg][lane] = P;
+        segH[seg][lane] = Hl;
+        __syncthreads();
+        float RH = carry;
+        for (int s2 = 0; s2 < seg; ++s2) RH = fmaf(segP[s2][lane], RH, segH[s2][lane]);
+        float* ip = p.incH + base + (size_t)m0 * sfl + (size_t)c * 16 + n;
+#pragma unroll
+        for (int q = 0; q < kSegLen; ++q) {
+            RH = fmaf(e[q], RH, hv[q]);
+            if (m0 + q < M) ip[(size_t)q * sfl] = RH;
+        }
+        for (int s2 = 0; s2 < kSegs; ++s2) carry = fmaf(segP[s2][lane], carry, segH[s2][lane]);
+        __syncthreads();  // segP / segH are rewritten by the next group
     }
 }
 
@@ -1081,15 +1119,15 @@ KernelInfo chunk_info() {
             attr_err = cudaFuncSetAttribute(ff, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LY::bytes);
     });
     const bool ok = attr_err == cudaSuccess;
-    return {ok ? ff : nullptr, LY::bytes, 1, LY::DT, LY::DT, LY::CL, ok ? fa : nullptr};
+    return {ok ? ff : nullptr, LY::bytes, LY::G, LY::DT, LY::THREADS, LY::CL, ok ? fa : nullptr};
 }
 
 // Tile shapes per padded state count, in order of preference (fewest lanes
 // per channel first).  The zero-order-hold variant uses the first shape.
-int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 11; }
+int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 12; }
 constexpr int kLanesShape = 7;   // index of the lane-per-state variant (N <= 16 padded to 16)
-constexpr int kChunkShape = 8;   // first index of the three-launch chunked variant (shapes 8, 9, 10)
-bool is_chunk_shape(int np, int shape) { return np == 16 && shape >= kChunkShape && shape < kChunkShape + 3; }
+constexpr int kChunkShape = 8;   // first index of the three-launch chunked variant (shapes 8 to 11)
+bool is_chunk_shape(int np, int shape) { return np == 16 && shape >= kChunkShape && shape < kChunkShape + 4; }
 
 template <typename T, bool ZOH>
 KernelInfo pick_t(int np, int shape) {
@@ -1110,9 +1148,10 @@ KernelInfo pick_t(int np, int shape) {
         case 5: return info_for<T, 16, Shape<1, 64, 16, 3>, false>();
         case 6: return info_for<T, 16, Shape<1, 32, 16, 3>, false>();
         case 7: return lanes_info<T, false>();
-        case 8: return chunk_info<T, ChunkShape<64, 32, 2, 8>>();
-        case 9: return chunk_info<T, ChunkShape<128, 32, 2, 4>>();
-        case 10: return chunk_info<T, ChunkShape<64, 64, 4, 5>>();
+        case 8: return chunk_info<T, ChunkShape<1, 64, 32, 2, 8>>();
+        case 9: return chunk_info<T, ChunkShape<2, 64, 32, 2, 4>>();
+        case 10: return chunk_info<T, ChunkShape<1, 64, 64, 4, 5>>();
+        case 11: return chunk_info<T, ChunkShape<2, 64, 64, 4, 4>>();
         default: return info_for<T, 16, Shape<1, 128, 0, 3, 7>, ZOH>();
         }
     }
@@ -1326,7 +1365,7 @@ vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
         const unsigned grid_agg = (unsigned)(plan.n_seq * (plan.n_chunks - 1));
         cudaError_t e = cudaLaunchKernel(ki.agg, dim3(grid_agg), dim3(ki.threads), args, ki.smem, stream);
         if (e != cudaSuccess) return VMB_ERR_CUDA;
-        const unsigned grid_carry = (unsigned)(plan.n_seq * (ki.DT / 8));
+        const unsigned grid_carry = (unsigned)(plan.n_seq * (ki.DT / 2));
         const void* carry = ki.DT == 128 ? reinterpret_cast<const void*>(&full_carry_kernel<128>)
                                          : reinterpret_cast<const void*>(&full_carry_kernel<64>);
         if (launch_pdl(carry, grid_carry, kCarryThreads, 0, args, stream) != cudaSuccess) return VMB_ERR_CUDA;

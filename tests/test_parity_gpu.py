@@ -172,8 +172,8 @@ def test_lookback_wait_times_out_cleanly(mean):
     check(to_numpy(y), ref, "f32", "after timeout")
 
 
-@pytest.mark.parametrize("plan", ["0", "1", "2", "3", "4", "5", "6", "7", "8", "9", "10", "0,3", "3,5", "4,2", "5,4",
-                                  "6,7", "7,3", "7,6"])
+@pytest.mark.parametrize("plan", ["0", "1", "2", "3", "4", "5", "6", "7", "8", "9", "10", "11", "0,3", "3,5", "4,2",
+                                  "5,4", "6,7", "7,3", "7,6"])
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
 def test_every_tile_shape(plan, dt, monkeypatch):
     """Each tile shape of the full scan (and forced L-chunking) against the oracle."""
@@ -198,7 +198,7 @@ CHUNKED_CASES = [
 ]
 
 
-@pytest.mark.parametrize("plan", ["8", "9", "10"])
+@pytest.mark.parametrize("plan", ["8", "9", "10", "11"])
 @pytest.mark.parametrize("case", CHUNKED_CASES, ids=[f"B{s[0]}_D{s[1]}_N{s[2]}_{s[3]}x{s[4]}_{s[5]}"
                                                      for s in CHUNKED_CASES])
 def test_chunked_full_scan(plan, case, monkeypatch):
