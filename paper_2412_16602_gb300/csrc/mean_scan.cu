@@ -34,6 +34,8 @@ namespace vmb {
 namespace {
 
 constexpr int kThreads = 256;
+
+__host__ __device__ constexpr size_t a16(size_t v) { return (v + 15) / 16 * 16; }
 constexpr int kMC = 8;  // steps per micro-chunk of the local scan
 
 struct MeanParams {
@@ -50,6 +52,8 @@ struct MeanParams {
     int softplus_on, skip_mean;
     int n_chunks, chunk_len, n_seq;
     int suppress;
+    int bcvec;   // B / C rows 16-byte aligned: async-copied
+    int tabvec;  // A, delta_bias, Dskip 16-byte aligned: async-copied
     WsHeader* hdr;
     unsigned* flags;
     float* aggP;
@@ -57,57 +61,102 @@ struct MeanParams {
     float* incH;
 };
 
-template <int NP, int TC, bool ZOH>
+template <typename T, int NP, int TC, bool ZOH>
 struct MLayout {
     static constexpr int S = kThreads / TC;  // channel groups
     static constexpr int NMC = TC / kMC;
     static constexpr int CG = 256;           // channels whose A / bias / Dskip are staged at a time
-    // shared memory (floats)
-    static constexpr int red = 0;                               // [S][NP][TC] partial sums of Abar
-    static constexpr int redb = red + S * TC * NP;              // [S][NP][TC] partial sums of Bbar u (ZOH)
-    static constexpr int redu = redb + (ZOH ? S * TC * NP : 0); // [S][TC] sums of delta u
-    static constexpr int reds = redu + S * TC;                  // [S][TC] sums of Dskip u (skip mean)
-    static constexpr int abar = reds + S * TC;                  // [TC][NP]
-    static constexpr int bubar = abar + TC * NP;                // [TC][NP]
-    static constexpr int bf = bubar + TC * NP;                  // [TC][NP]
-    static constexpr int cf = bf + TC * NP;                     // [TC][NP]
-    static constexpr int mc = cf + TC * NP;                     // [4][NMC][NP]
-    static constexpr int ybar = mc + 4 * NMC * NP;              // [TC]
-    static constexpr int dsu = ybar + TC;                       // [TC]
-    static constexpr int hin = dsu + TC;                        // [NP]
-    static constexpr int a2 = (hin + NP + 3) / 4 * 4;           // [CG][NP] A * log2 e (raw A for ZOH)
-    static constexpr int bias = a2 + CG * NP;                   // [CG]
-    static constexpr int dsk = bias + CG;                       // [CG]
-    static constexpr size_t bytes = (size_t)(dsk + CG) * 4;
+    static constexpr int BCS = TC + 16 / (int)sizeof(T);  // raw B / C row stride (elements), rows 16-byte aligned
+    // shared memory, byte offsets
+    static constexpr size_t red = 0;                                            // f32 [S][NP][TC] partial sums of Abar
+    static constexpr size_t redb = red + (size_t)S * TC * NP * 4;               // f32 [S][NP][TC] of Bbar u (ZOH)
+    static constexpr size_t redu = redb + (ZOH ? (size_t)S * TC * NP * 4 : 0);  // f32 [S][TC] sums of delta u
+    static constexpr size_t reds = redu + (size_t)S * TC * 4;                   // f32 [S][TC] sums of Dskip u
+    static constexpr size_t abar = reds + (size_t)S * TC * 4;                   // f32 [TC][NP]
+    static constexpr size_t bubar = abar + (size_t)TC * NP * 4;                 // f32 [TC][NP]
+    static constexpr size_t mc = bubar + (size_t)TC * NP * 4;                   // f32 [4][NMC][NP]
+    static constexpr size_t ybar = mc + (size_t)4 * NMC * NP * 4;               // f32 [TC]
+    static constexpr size_t dsu = ybar + (size_t)TC * 4;                        // f32 [TC]
+    static constexpr size_t hin = dsu + (size_t)TC * 4;                         // f32 [NP]
+    static constexpr size_t bc = a16(hin + (size_t)NP * 4);                     // T [2][NP][BCS] B, C rows as stored
+    // channel tables of one group of CG channels: A [CG][NP] (scaled by log2 e
+    // in place unless ZOH), delta bias [CG], Dskip [CG]
+    static constexpr size_t tab0 = a16(bc + (size_t)2 * NP * BCS * sizeof(T));
+    static constexpr size_t tab_bytes = (size_t)CG * NP * 4 + 2 * (size_t)CG * 4;
+    static constexpr size_t bytes1 = tab0 + tab_bytes;
+    static constexpr size_t bytes2 = bytes1;
     static_assert(kThreads % TC == 0 && TC % 32 == 0, "a warp covers 32 consecutive steps");
     static_assert(NP * NMC <= kThreads, "local scan mapping");
-    static_assert(bytes <= 100 * 1024, "mean-scan tile must leave room for two CTAs per SM");
+    static_assert(bytes2 <= 110 * 1024, "mean-scan tile must leave room for two CTAs per SM");
 };
 
+// Stage group g0 of the channel tables (raw A rows, delta bias, Dskip) into
+// buffer `tb`: 16-byte async copies where rows are aligned, element loads
+// otherwise; channels past the group are zero.
 template <typename T, int NP, int TC, bool ZOH>
-__global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p) {
-    using LY = MLayout<NP, TC, ZOH>;
-    constexpr int S = LY::S, NMC = LY::NMC, CG = LY::CG;
-    extern __shared__ __align__(16) float sm[];
-    float* red = sm + LY::red;
-    float* redb = sm + LY::redb;
-    float* redu = sm + LY::redu;
-    float* reds = sm + LY::reds;
-    float* abar = sm + LY::abar;
-    float* bubar = sm + LY::bubar;
-    float* bfm = sm + LY::bf;
-    float* cfm = sm + LY::cf;
-    float* mcP = sm + LY::mc;
+__device__ __forceinline__ void stage_tables(const MeanParams& p, unsigned char* tb, int k, int g0, int gn) {
+    using LY = MLayout<T, NP, TC, ZOH>;
+    constexpr int CG = LY::CG;
+    float* ta = reinterpret_cast<float*>(tb);
+    float* tbias = ta + CG * NP;
+    float* tdsk = tbias + CG;
+    const int tid = threadIdx.x;
+    const float* Ag = p.A + ((size_t)k * p.D + g0) * p.N;
+    bool rows_done = false;
+    if constexpr (NP % 4 == 0) {
+        if (p.N == NP && p.tabvec) {
+            for (int i = tid; i < CG * NP / 4; i += kThreads) {
+                const int r = i / (NP / 4);
+                const bool ok = r < gn;
+                cp_async16(ta + 4 * i, ok ? Ag + 4 * i : p.A, ok ? 16 : 0);
+            }
+            rows_done = true;
+        }
+    }
+    if (!rows_done) {
+        for (int i = tid; i < CG * NP; i += kThreads) {
+            const int r = i / NP, n = i % NP;
+            ta[i] = (r < gn && n < p.N) ? __ldg(Ag + (size_t)r * p.N + n) : 0.0f;
+        }
+    }
+    const float* bg = p.bias + (size_t)k * p.D + g0;
+    const float* dg = p.Dskip + (size_t)k * p.D + g0;
+    if (p.tabvec && (((size_t)k * p.D + g0) & 3) == 0) {
+        for (int i = tid; i < 2 * CG / 4; i += kThreads) {
+            const int which = i / (CG / 4), r = 4 * (i % (CG / 4));
+            const int nb = max(0, min(4, gn - r)) * 4;
+            cp_async16((which ? tdsk : tbias) + r, nb ? (which ? dg : bg) + r : p.bias, nb);
+        }
+    } else {
+        for (int i = tid; i < CG; i += kThreads) {
+            tbias[i] = i < gn ? __ldg(bg + i) : 0.0f;
+            tdsk[i] = i < gn ? __ldg(dg + i) : 0.0f;
+        }
+    }
+}
+
+template <typename T, int NP, int TC, bool ZOH>
+__global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const MeanParams p) {
+    using LY = MLayout<T, NP, TC, ZOH>;
+    constexpr int S = LY::S, NMC = LY::NMC, CG = LY::CG, BCS = LY::BCS;
+    extern __shared__ __align__(16) unsigned char smb[];
+    float* red = reinterpret_cast<float*>(smb + LY::red);
+    float* redb = reinterpret_cast<float*>(smb + LY::redb);
+    float* redu = reinterpret_cast<float*>(smb + LY::redu);
+    float* reds = reinterpret_cast<float*>(smb + LY::reds);
+    float* abar = reinterpret_cast<float*>(smb + LY::abar);
+    float* bubar = reinterpret_cast<float*>(smb + LY::bubar);
+    float* mcP = reinterpret_cast<float*>(smb + LY::mc);
     float* mcH = mcP + NMC * NP;
     float* exP = mcH + NMC * NP;
     float* exH = exP + NMC * NP;
-    float* s_ybar = sm + LY::ybar;
-    float* s_dsu = sm + LY::dsu;
-    float* s_hin = sm + LY::hin;
-    float* s_a2 = sm + LY::a2;
-    float* s_bias = sm + LY::bias;
-    float* s_dsk = sm + LY::dsk;
+    float* s_ybar = reinterpret_cast<float*>(smb + LY::ybar);
+    float* s_dsu = reinterpret_cast<float*>(smb + LY::dsu);
+    float* s_hin = reinterpret_cast<float*>(smb + LY::hin);
+    T* sB = reinterpret_cast<T*>(smb + LY::bc);
+    T* sC = sB + NP * BCS;
     __shared__ unsigned s_misc[2];
+    __shared__ unsigned s_scr[2 * kThreads / 32 + 2];
 
     const int tid = threadIdx.x;
     const bool chunked = p.n_chunks > 1;
@@ -142,16 +191,34 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
     const size_t bcrow0 = (size_t)seq * N;  // first row of Bs/Cs
     const T* u = static_cast<const T*>(p.u);
     const T* dlr = static_cast<const T*>(p.dl);
-    const float* Ak = p.A + (size_t)k * D * N;
 
-    // B and C of the chunk, transposed to [t][n]
-    for (int i = tid; i < NP * TC; i += kThreads) {
-        const int n = i / TC, t = i % TC;
-        const bool ok = n < N && t < nvalid;
-        const size_t gi = (bcrow0 + n) * (size_t)L + l0 + t;
-        bfm[t * NP + n] = ok ? io<T>::ld(static_cast<const T*>(p.Bs) + gi) : 0.0f;
-        cfm[t * NP + n] = ok ? io<T>::ld(static_cast<const T*>(p.Cs) + gi) : 0.0f;
+    // ---------------------------------------------------------------- prologue
+    // B and C of the chunk as stored ([n][t] rows, zero past the problem) and the
+    // first group's channel tables go in flight as async copies; the first
+    // delta / u values of phase A are requested before anything waits.
+    {
+        const T* Bs = static_cast<const T*>(p.Bs);
+        const T* Cs = static_cast<const T*>(p.Cs);
+        if (p.bcvec) {
+            constexpr int VE = 16 / (int)sizeof(T), CPR = TC / VE;
+            for (int i = tid; i < 2 * NP * CPR; i += kThreads) {
+                const int which = i / (NP * CPR), r = (i / CPR) % NP, ch = i % CPR;
+                const bool ok = r < N && ch * VE < nvalid;
+                const T* src = (which ? Cs : Bs) + (bcrow0 + r) * (size_t)L + l0 + ch * VE;
+                cp_async16((which ? sC : sB) + r * BCS + ch * VE, ok ? src : Bs, ok ? 16 : 0);
+            }
+        } else {
+            for (int i = tid; i < 2 * NP * TC; i += kThreads) {
+                const int which = i / (NP * TC), r = (i / TC) % NP, t = i % TC;
+                T v = T(0.0f);
+                if (r < N && t < nvalid) v = (which ? Cs : Bs)[(bcrow0 + r) * (size_t)L + l0 + t];
+                (which ? sC : sB)[r * BCS + t] = v;
+            }
+        }
     }
+    const int ngroups = (D + CG - 1) / CG;
+    stage_tables<T, NP, TC, ZOH>(p, smb + LY::tab0, k, 0, min(CG, D));
+    cp_async_commit();
 
     // ---------------------------------------------------------------- phase A
     const int rt = tid % TC;  // step of this thread
@@ -164,28 +231,32 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
         accb[n] = 0.0f;
     }
     float sdu = 0.0f, sdsu = 0.0f;
-    // Channel groups of CG: stage the group's A (times log2 e), bias and Dskip in
-    // shared memory, then every thread reduces its channels of the group with the
-    // delta and u of the next kPF channels already in flight.
+    // Channel groups of CG: the group's A, bias and Dskip are in shared memory
+    // (async copies, the first group's issued with the prologue), A is scaled by
+    // log2 e in place once it lands, then every thread reduces its channels of
+    // the group with the delta and u of the next kPF channels already in flight.
     constexpr int kPF = 8;
     const size_t col = (size_t)l0 + (tv ? rt : 0);
     const T* dcol = dlr + urow0 * (size_t)L + col;
     const T* ucol = u + urow0 * (size_t)L + col;
     // u is read again by the broadcast pass: keep it in L2; delta streams through
     const uint64_t keep = l2_evict_last(), stream = l2_evict_first();
-    for (int g0 = 0; g0 < D; g0 += CG) {
-        const int gn = min(CG, D - g0);
-        __syncthreads();  // previous group's tables are no longer read
-        for (int i = tid; i < CG * NP; i += kThreads) {
-            const int r = i / NP, n = i % NP;
-            const float av = (r < gn && n < N) ? Ak[(size_t)(g0 + r) * N + n] : 0.0f;
-            s_a2[i] = ZOH ? av : av * kLog2e;
+    float* s_a2 = reinterpret_cast<float*>(smb + LY::tab0);
+    const float* s_bias = s_a2 + CG * NP;
+    const float* s_dsk = s_bias + CG;
+    for (int gi = 0; gi < ngroups; ++gi) {
+        const int g0 = gi * CG, gn = min(CG, D - g0);
+        if (gi > 0) {
+            __syncthreads();  // the previous group's tables are no longer read
+            stage_tables<T, NP, TC, ZOH>(p, smb + LY::tab0, k, g0, gn);
+            cp_async_commit();
         }
-        for (int i = tid; i < CG; i += kThreads) {
-            s_bias[i] = i < gn ? p.bias[(size_t)k * D + g0 + i] : 0.0f;
-            s_dsk[i] = i < gn ? p.Dskip[(size_t)k * D + g0 + i] : 0.0f;
+        cp_async_wait<0>();
+        __syncthreads();  // this group's tables have landed
+        if constexpr (!ZOH) {
+            for (int i = tid; i < CG * NP; i += kThreads) s_a2[i] *= kLog2e;
+            __syncthreads();
         }
-        __syncthreads();
         if (!tv) continue;
         float vd[kPF], vu[kPF];
 #pragma unroll
@@ -261,18 +332,18 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
         const int n = i / TC, t = i % TC;
         float sa = 0.0f, sb = 0.0f, su = 0.0f;
 #pragma unroll
-        for (int s = 0; s < S; ++s) {
-            sa += red[(s * NP + n) * TC + t];
-            if constexpr (ZOH) sb += redb[(s * NP + n) * TC + t];
-            su += redu[s * TC + t];
+        for (int s2 = 0; s2 < S; ++s2) {
+            sa += red[(s2 * NP + n) * TC + t];
+            if constexpr (ZOH) sb += redb[(s2 * NP + n) * TC + t];
+            su += redu[s2 * TC + t];
         }
         abar[t * NP + n] = sa * invD;
-        bubar[t * NP + n] = bfm[t * NP + n] * (ZOH ? sb : su) * invD;
+        bubar[t * NP + n] = io<T>::cvt(sB[n * BCS + t]) * (ZOH ? sb : su) * invD;
     }
     for (int t = tid; t < TC; t += kThreads) {
         float sd = 0.0f;
 #pragma unroll
-        for (int s = 0; s < S; ++s) sd += reds[s * TC + t];
+        for (int s2 = 0; s2 < S; ++s2) sd += reds[s2 * TC + t];
         s_dsu[t] = sd * invD;
     }
     __syncthreads();
@@ -322,14 +393,11 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
             st_release(&p.flags[slot], flag_word(gen, chunk == 0 ? kFlagInclusive : kFlagAggregate));
         float RH = 0.0f;
         if (chunk > 0) {
-            // Decoupled look-back with a left fold after the inclusive state found
-            // (bit-identical carry whichever predecessor the walk stops at).
-            if (tid < 32) {
-                const int f = lookback_find(p.flags + (size_t)seq * p.n_chunks, chunk, gen, p.hdr, (unsigned)seq);
-                if (tid == 0) s_misc[0] = (unsigned)f;
-            }
-            __syncthreads();
-            const int found = (int)s_misc[0];
+            // Decoupled look-back (the whole block polls 256 predecessors per round)
+            // with a left fold after the inclusive state found: the carry is
+            // bit-identical whichever predecessor the walk stops at.
+            const int found = lookback_find_block<kThreads>(p.flags + (size_t)seq * p.n_chunks, chunk, gen, p.hdr,
+                                                            (unsigned)seq, s_scr);
             if (found >= 0) {
                 // Fold the aggregates after the inclusive state left to right.  They are
                 // staged into shared memory (the partial-sum area, free by now) in
@@ -374,40 +442,40 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
         for (int j = 0; j < kMC; ++j) {
             const int t = m * kMC + j;
             h = fmaf(abar[t * NP + n], h, bubar[t * NP + n]);
-            abar[t * NP + n] = cfm[t * NP + n] * h;
+            abar[t * NP + n] = io<T>::cvt(sC[n * BCS + t]) * h;
         }
     }
     __syncthreads();
     for (int t = tid; t < TC; t += kThreads) {
-        float s = 0.0f;
+        float s2 = 0.0f;
 #pragma unroll
-        for (int n = 0; n < NP; ++n) s += abar[t * NP + n];
-        s_ybar[t] = s;
-        if (p.ybar && t < nvalid) p.ybar[(size_t)seq * L + l0 + t] = s;
+        for (int n = 0; n < NP; ++n) s2 += abar[t * NP + n];
+        s_ybar[t] = s2;
+        if (p.ybar && t < nvalid) p.ybar[(size_t)seq * L + l0 + t] = s2;
     }
     __syncthreads();
 
     // ---------------------------------------------------------------- phase C
     if (tv) {
         T* y = static_cast<T*>(p.y);
-        const size_t col = (size_t)l0 + rt;
+        const size_t colc = (size_t)l0 + rt;
         const float yb = s_ybar[rt];
         const float dsu = s_dsu[rt];
-        constexpr int kPF = 8;
-        const uint64_t stream = l2_evict_first();
-        for (int d0 = sg; d0 < D; d0 += kPF * S) {
-            float uv[kPF];
+        constexpr int kPC = 8;  // u reads in flight per thread
+        const uint64_t ev = l2_evict_first();
+        for (int d0 = sg; d0 < D; d0 += kPC * S) {
+            float uv[kPC];
 #pragma unroll
-            for (int q = 0; q < kPF; ++q) {
+            for (int q = 0; q < kPC; ++q) {
                 const int d = d0 + q * S;
-                uv[q] = (d < D && !p.skip_mean) ? ld_hint(u + (urow0 + d) * (size_t)L + col, stream) : 0.0f;
+                uv[q] = (d < D && !p.skip_mean) ? ld_hint(u + (urow0 + d) * (size_t)L + colc, ev) : 0.0f;
             }
 #pragma unroll
-            for (int q = 0; q < kPF; ++q) {
+            for (int q = 0; q < kPC; ++q) {
                 const int d = d0 + q * S;
                 if (d < D) {
-                    const float skip = p.skip_mean ? dsu : __ldg(p.Dskip + (size_t)k * D + d) * uv[q];  // Dskip: 1 KB per 256 channels, L1-resident
-                    st_hint(y + (urow0 + d) * (size_t)L + col, yb + skip, stream);
+                    const float skip = p.skip_mean ? dsu : __ldg(p.Dskip + (size_t)k * D + d) * uv[q];  // Dskip: L1-resident
+                    st_hint(y + (urow0 + d) * (size_t)L + colc, yb + skip, ev);
                 }
             }
         }
@@ -423,20 +491,21 @@ __global__ void __launch_bounds__(kThreads) mean_scan_kernel(const MeanParams p)
 
 struct KInfo {
     const void* fn;
-    size_t smem;
+    size_t smem;   // D <= 256: one buffer of channel tables
+    size_t smem2;  // D > 256: two
 };
 
 template <typename T, int NP, int TC, bool ZOH>
 KInfo minfo() {
-    using LY = MLayout<NP, TC, ZOH>;
+    using LY = MLayout<T, NP, TC, ZOH>;
     const void* fn = reinterpret_cast<const void*>(&mean_scan_kernel<T, NP, TC, ZOH>);
     static std::once_flag once;
     static cudaError_t err = cudaSuccess;
     std::call_once(once, [&] {
-        err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LY::bytes);
+        err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LY::bytes2);
     });
-    if (err != cudaSuccess) return {nullptr, 0};
-    return {fn, LY::bytes};
+    if (err != cudaSuccess) return {nullptr, 0, 0};
+    return {fn, LY::bytes1, LY::bytes2};
 }
 
 template <typename T, int NP, bool ZOH>
@@ -482,7 +551,8 @@ vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan) {
         KInfo ki = mpick(a.dtype, np, cand, zoh);
         if (!ki.fn) return VMB_ERR_CUDA;
         int per_sm = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ki.fn, kThreads, ki.smem) != cudaSuccess)
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ki.fn, kThreads, a.D > 256 ? ki.smem2 : ki.smem) !=
+            cudaSuccess)
             return VMB_ERR_CUDA;
         const long long resident = (long long)(per_sm < 1 ? 1 : per_sm) * device_sm_count();
         if (forced || seqs * ((a.L + cand - 1) / cand) >= 2 * resident || cand == 32) {
@@ -526,6 +596,10 @@ vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     p.chunk_len = plan.chunk_len;
     p.n_seq = plan.n_seq;
     p.suppress = (a.flags & VMB_FLAG_TEST_SUPPRESS_PUBLISH) ? 1 : 0;
+    const size_t es = a.dtype == VMB_BF16 ? 2 : 4;
+    const auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
+    p.bcvec = ((size_t)a.L * es % 16 == 0) && al16(a.Bs) && al16(a.Cs);
+    p.tabvec = al16(a.A) && al16(a.bias) && al16(a.Dskip);
     const WsLayout w = ws_layout(plan);
     unsigned char* ws = static_cast<unsigned char*>(a.ws);
     p.hdr = reinterpret_cast<WsHeader*>(ws);
@@ -535,7 +609,7 @@ vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     p.incH = reinterpret_cast<float*>(ws + w.incH_off);
     const unsigned grid = (unsigned)(plan.n_seq * plan.n_chunks);
     void* args[] = {&p};
-    cudaError_t e = cudaLaunchKernel(ki.fn, dim3(grid), dim3(kThreads), args, ki.smem, stream);
+    cudaError_t e = cudaLaunchKernel(ki.fn, dim3(grid), dim3(kThreads), args, a.D > 256 ? ki.smem2 : ki.smem, stream);
     return e == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
 }
 

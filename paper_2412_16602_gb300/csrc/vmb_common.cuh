@@ -157,6 +157,80 @@ __device__ __forceinline__ int lookback_find(const unsigned* flags, int chunk, u
     }
 }
 
+// Block-wide look-back: every thread of a CTA of NT threads calls it, thread i
+// polls predecessor hi - i, so one round covers NT predecessors instead of 32.
+// Same contract as lookback_find (returns the nearest predecessor whose
+// inclusive state is published with every chunk after it at least aggregated,
+// or -1 when the wait ran out or another CTA reported an error).  s_scr holds
+// 2 NT / 32 + 2 words of shared memory.
+template <int NT>
+__device__ __forceinline__ int lookback_find_block(const unsigned* flags, int chunk, unsigned gen, WsHeader* hdr,
+                                                   unsigned seq, unsigned* s_scr) {
+    constexpr int NW = NT / 32;
+    constexpr int kRetry = -2;
+    const unsigned tag = gen & 0x3FFFFFFFu;
+    const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+    int hi = chunk - 1;
+    const uint64_t t0 = globaltimer_ns();
+    unsigned ns = 32;
+    for (unsigned it = 0;; ++it) {
+        const int j = hi - tid;
+        unsigned kind = 0;
+        if (j >= 0) {
+            const unsigned f = ld_acquire(&flags[j]);
+            kind = ((f >> 2) == tag) ? (f & 3u) : 0u;
+        }
+        const unsigned inc = __ballot_sync(0xffffffffu, kind == kFlagInclusive);
+        const unsigned valid = __ballot_sync(0xffffffffu, kind != 0 || j < 0);
+        if (lane == 0) {
+            s_scr[w] = inc;
+            s_scr[NW + w] = valid;
+        }
+        __syncthreads();
+        if (tid == 0) {
+            int res = kRetry, nhi = hi;
+            bool decided = false;
+            for (int ww = 0; ww < NW && !decided; ++ww) {
+                const unsigned iv = s_scr[ww], vv = s_scr[NW + ww];
+                if (iv) {
+                    const int l = __ffs(iv) - 1;
+                    const unsigned need = l == 0 ? 0u : ((1u << l) - 1u);
+                    if ((vv & need) == need) res = hi - (ww * 32 + l);
+                    decided = true;
+                } else if (vv != 0xffffffffu) {
+                    decided = true;  // a predecessor has published nothing yet
+                }
+            }
+            if (!decided && hi >= NT) {
+                nhi = hi - NT;  // the whole window is aggregated: look further back
+                res = kRetry - 1;
+            }
+            if (res == kRetry && (it & 15u) == 0) {
+                if (ld_relaxed(&hdr->err)) {
+                    res = -1;
+                } else if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                    if (atomicOr(&hdr->err, kErrTimeout) == 0) {
+                        hdr->err_seq = seq;
+                        hdr->err_chunk = (unsigned)chunk;
+                    }
+                    res = -1;
+                }
+            }
+            s_scr[2 * NW] = (unsigned)res;
+            s_scr[2 * NW + 1] = (unsigned)nhi;
+        }
+        __syncthreads();
+        const int res = (int)s_scr[2 * NW];
+        hi = (int)s_scr[2 * NW + 1];
+        __syncthreads();  // s_scr is rewritten by the next round
+        if (res >= -1) return res;
+        if (res == kRetry) {
+            __nanosleep(ns);
+            if (ns < 1024) ns <<= 1;
+        }
+    }
+}
+
 // Called by thread 0 of every CTA of a look-back launch once the CTA is done
 // with the workspace: the last CTA resets the ticket and completion counters
 // and advances the generation, leaving the workspace ready for the next launch.

@@ -126,8 +126,12 @@ def test_empty_problem_is_a_noop():
     assert vmb.vmb_cross_scan(x).shape == (0, 4, 4, 25)
 
 
-def test_workspace_reuse_over_many_calls():
-    """The look-back workspace stays consistent over repeated chunked calls."""
+@pytest.mark.parametrize("plan", ["", "5,6"])
+def test_workspace_reuse_over_many_calls(plan, monkeypatch):
+    """The workspace stays consistent over repeated chunked calls (the default
+    chunked variant and a forced look-back plan), with bit-identical results."""
+    if plan:
+        monkeypatch.setenv("VMB_FULL_PLAN", plan)
     wl = workloads.small_case(B=1, D=16, N=16, H=40, W=40, seed=10)
     inp = workloads.make_inputs(wl)
     g = to_device(inp, DEV)
@@ -144,9 +148,11 @@ def test_workspace_reuse_over_many_calls():
 
 
 @pytest.mark.parametrize("mean", [False, True])
-def test_lookback_wait_times_out_cleanly(mean):
+def test_lookback_wait_times_out_cleanly(mean, monkeypatch):
     """A chunk that never publishes makes its successors' bounded waits run out:
     the call reports VMB_ERR_TIMEOUT and the context and workspace stay usable."""
+    if not mean:
+        monkeypatch.setenv("VMB_FULL_PLAN", "5,6")  # a look-back plan (the default here is the chunked variant)
     wl = workloads.small_case(B=1, D=16, N=16, H=48, W=48, seed=11)
     inp = workloads.make_inputs(wl)
     g = to_device(inp, DEV)
