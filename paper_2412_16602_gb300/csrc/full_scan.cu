@@ -152,6 +152,7 @@ __device__ __forceinline__ void load_tile(const FullParams& p, T* dst, size_t ro
                                           int l0) {
     constexpr int VE = 16 / sizeof(T);  // elements per 16-byte chunk
     constexpr int CPR = kTS / VE;       // chunks per stage row
+    static_assert(kTS % VE == 0, "a stage row is a whole number of 16-byte chunks");
     const T* u = static_cast<const T*>(p.u);
     const T* dl = static_cast<const T*>(p.dl);
     const T* Bs = static_cast<const T*>(p.Bs);
@@ -833,6 +834,16 @@ __device__ __forceinline__ float ex2_ordered(float x) {
     asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
+__device__ __forceinline__ float fma_ordered(float a, float b, float c) {
+    float y;
+    asm volatile("fma.rn.f32 %0, %1, %2, %3;" : "=f"(y) : "f"(a), "f"(b), "f"(c));
+    return y;
+}
+__device__ __forceinline__ float mul_ordered(float a, float b) {
+    float y;
+    asm volatile("mul.rn.f32 %0, %1, %2;" : "=f"(y) : "f"(a), "f"(b));
+    return y;
+}
 
 __device__ __forceinline__ void cp_async_wait_upto(int n) {
     switch (n) {
@@ -1010,6 +1021,224 @@ __global__ void __launch_bounds__(ChunkLayout<T, CS>::THREADS, CS::MINB) full_ch
     }
 }
 
+// ---------------------------------------------------- streaming variant
+// For many channel rows (no L-chunking): the compute structure of the chunked
+// kernel over a cp.async ring of TS-step stages.  G lanes per channel (1 or 2)
+// own 16 / G states each; per stage the channel's delta row is turned into fp32
+// softplus values one stage ahead (the G lanes take alternate 4-step groups of
+// their own channel, so no barrier beyond the stage's), B and C are read as fp32
+// [n][t] rows four steps per 128-bit broadcast load (bf16 converted
+// cooperatively one stage ahead), A * log2 e sits in swizzled shared memory or
+// in registers, and the state loop is outermost within a 4-step block.  One
+// barrier per stage.
+template <int G_, int DT_, int TS_, int MINB_, int V_ = 0>
+struct StreamShape {
+    // V: 0 = A in shared memory, ordered B/C reads and exponentials;
+    //    1 = A in registers, ordered reads, exponentials and FMAs; 2 = A in registers, free order
+    static constexpr int G = G_, DT = DT_, TS = TS_, MINB = MINB_, V = V_;
+};
+
+template <typename T, class SS>
+struct StreamLayout {
+    // TS = 0: one 16-byte chunk per row and stage (4 fp32 or 8 bf16 steps)
+    static constexpr int G = SS::G, DT = SS::DT, TS = SS::TS ? SS::TS : 16 / (int)sizeof(T), NP = 16, NSTG = 3;
+    static constexpr int THREADS = G * DT, NG = NP / G;
+    static constexpr bool F32 = sizeof(T) == 4;
+    static constexpr int PAD = 16 / (int)sizeof(T);
+    static constexpr int RS = TS + PAD;                 // raw row stride (elements), 16-byte aligned rows
+    static constexpr int SLOT = (2 * DT + 2 * NP) * RS;  // u, delta, B, C rows of one stage
+    static constexpr int FS = TS + 4;                    // fp32 row stride
+    static constexpr size_t raw_bytes = a16((size_t)NSTG * SLOT * sizeof(T));
+    // bf16: fp32 delta rows [2][DT][FS] and fp32 B, C rows [2][2 NP][FS] (two
+    // slots: the stage being computed and the next); fp32 uses the raw rows
+    static constexpr size_t fdl_off = raw_bytes;
+    static constexpr size_t fbc_off = fdl_off + (F32 ? 0 : (size_t)2 * DT * FS * 4);
+    static constexpr size_t a2_off = fbc_off + (F32 ? 0 : (size_t)2 * 2 * NP * FS * 4);
+    static constexpr int V = SS::V;
+    static constexpr size_t bytes = a2_off + (V == 0 ? (size_t)DT * NP * 4 : 0);
+    static_assert(TS % (4 * G) == 0 && TS * sizeof(T) % 16 == 0 && DT % 32 == 0 && (G == 1 || G == 2),
+                  "stream tile shape");
+    static_assert(V != 0 || G == 1, "shared-memory A rows are one lane per channel");
+    static_assert(!F32 || RS == FS, "fp32 rows are rewritten in place");
+};
+
+template <typename T, class SS>
+__global__ void __launch_bounds__(StreamLayout<T, SS>::THREADS, SS::MINB) full_stream_kernel(const FullParams p) {
+    using LY = StreamLayout<T, SS>;
+    constexpr int G = LY::G, NG = LY::NG, DT = LY::DT, TS = LY::TS, NP = 16, NSTG = LY::NSTG, RS = LY::RS,
+                  SLOT = LY::SLOT, FS = LY::FS, THREADS = LY::THREADS;
+    extern __shared__ __align__(16) unsigned char smem[];
+    T* raw = reinterpret_cast<T*>(smem);
+
+    const int c = threadIdx.x / G, g = threadIdx.x % G;
+    const int tile = blockIdx.x;
+    const int bk = tile / p.tiles_per_bk;
+    const int d0 = (tile % p.tiles_per_bk) * DT;
+    const int k = bk % p.K;
+    const int d = d0 + c;
+    const bool cval = d < p.D;
+    const int nrows = min(DT, p.D - d0);
+    const size_t row0 = (size_t)bk * p.D + d0;
+    const size_t bcrow0 = (size_t)bk * p.N;
+    const int L = p.L;
+    const int nst = (L + TS - 1) / TS;
+#pragma unroll
+    for (int q = 0; q < NSTG - 1; ++q) {
+        if (q < nst) load_tile<T, NP, DT, TS, RS, THREADS, true>(p, raw + q * SLOT, row0, bcrow0, nrows, q * TS);
+        cp_async_commit();
+    }
+    const float bias = cval ? p.bias[(size_t)k * p.D + d] : 0.0f;
+    const float dsk = cval ? p.Dskip[(size_t)k * p.D + d] : 0.0f;
+    const float* Ad = p.A + ((size_t)k * p.D + d) * p.N;
+    constexpr int V = LY::V;
+    float A2r[V == 0 ? 1 : NG];  // V > 0: this lane's A * log2 e
+    float* sa2 = reinterpret_cast<float*>(smem + LY::a2_off) + c * NP;  // V = 0: this channel's row (own row only)
+    const int sw = (c >> 1) & 3;
+    if constexpr (V == 0) {
+#pragma unroll
+        for (int q = 0; q < NP / 4; ++q) {
+            float a[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int n = 4 * q + i;
+                a[i] = (cval && n < p.N) ? Ad[n] * kLog2e : 0.0f;
+            }
+            *reinterpret_cast<float4*>(sa2 + 4 * (q ^ sw)) = make_float4(a[0], a[1], a[2], a[3]);
+        }
+    } else {
+#pragma unroll
+        for (int i = 0; i < NG; ++i) {
+            const int n = g * NG + i;
+            A2r[i] = (cval && n < p.N) ? Ad[n] * kLog2e : 0.0f;
+        }
+    }
+    float h[NG];
+#pragma unroll
+    for (int i = 0; i < NG; ++i) h[i] = 0.0f;
+    T* yrow = static_cast<T*>(p.y) + (row0 + c) * (size_t)L;
+
+    // fp32 delta row of stage st (this channel) and fp32 B / C rows
+    auto fdl_of = [&](int st) -> float* {
+        if constexpr (LY::F32) return reinterpret_cast<float*>(raw + (st % NSTG) * SLOT + (DT + c) * RS);
+        else return reinterpret_cast<float*>(smem + LY::fdl_off) + ((st & 1) * DT + c) * FS;
+    };
+    auto fbc_of = [&](int st) -> const float* {
+        if constexpr (LY::F32) return reinterpret_cast<const float*>(raw + (st % NSTG) * SLOT + 2 * DT * RS);
+        else return reinterpret_cast<const float*>(smem + LY::fbc_off) + (st & 1) * 2 * NP * FS;
+    };
+    // delta = softplus(raw + bias) (Eq. 6) of this channel over stage st, in fp32
+    // (the G lanes take alternate 4-step groups); bf16 storage also converts the
+    // stage's B and C rows (cooperatively)
+    auto prepare = [&](int st) {
+        const T* rd = raw + (st % NSTG) * SLOT + (DT + c) * RS;
+        float* fd = fdl_of(st);
+#pragma unroll
+        for (int t0 = 4 * g; t0 < TS; t0 += 4 * G) {
+            float r4[4];
+            load4(rd + t0, r4);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float v = r4[j] + bias;
+                r4[j] = p.softplus_on ? softplus(v) : v;
+            }
+            *reinterpret_cast<float4*>(fd + t0) = make_float4(r4[0], r4[1], r4[2], r4[3]);
+        }
+        if constexpr (!LY::F32) {
+            const T* rbc = raw + (st % NSTG) * SLOT + 2 * DT * RS;
+            float* fbc = reinterpret_cast<float*>(smem + LY::fbc_off) + (st & 1) * 2 * NP * FS;
+            for (int i = threadIdx.x; i < 2 * NP * TS / 4; i += THREADS) {
+                const int r = i / (TS / 4), t0 = 4 * (i % (TS / 4));
+                float v4[4];
+                load4(rbc + r * RS + t0, v4);
+                *reinterpret_cast<float4*>(fbc + r * FS + t0) = make_float4(v4[0], v4[1], v4[2], v4[3]);
+            }
+        }
+    };
+    cp_async_wait<NSTG - 2>();
+    __syncthreads();
+    prepare(0);
+    for (int s = 0; s < nst; ++s) {
+        const int l0 = s * TS;
+        const int nvalid = min(TS, L - l0);
+        cp_async_wait<NSTG - 3>();  // stages <= s+1 have landed
+        __syncthreads();            // ... for every thread; stage s's fp32 rows are prepared
+        if (s + NSTG - 1 < nst)
+            load_tile<T, NP, DT, TS, RS, THREADS, true>(p, raw + ((s + NSTG - 1) % NSTG) * SLOT, row0, bcrow0,
+                                                        nrows, l0 + (NSTG - 1) * TS);
+        cp_async_commit();
+        if (s + 1 < nst) prepare(s + 1);
+        const T* ru = raw + (s % NSTG) * SLOT + c * RS;
+        const float* fd = fdl_of(s);
+        constexpr int BS = LY::F32 ? RS : FS;  // fp32 B / C row stride
+        const float* rb = fbc_of(s) + g * NG * BS;  // this lane's B rows
+        const float* rc = rb + NP * BS;
+#pragma unroll 1
+        for (int t0 = 0; t0 < TS; t0 += 4) {
+            float dl4[4], du4[4];
+            {
+                float u4[4];
+                load4(ru + t0, u4);
+                load4(fd + t0, dl4);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) du4[j] = dl4[j] * u4[j];
+            }
+            float ya[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+            for (int q = 0; q < NG / 4; ++q) {
+                float a2[4];
+                if constexpr (V == 0) {
+                    load4(sa2 + 4 * (q ^ sw), a2);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) a2[i] = A2r[4 * q + i];
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int n = 4 * q + i;
+                    float b4[4], c4[4];
+                    if constexpr (V == 2) {
+                        load4(rb + n * BS + t0, b4);
+                        load4(rc + n * BS + t0, c4);
+                    } else {
+                        lds4_ordered(rb + n * BS + t0, b4);
+                        lds4_ordered(rc + n * BS + t0, c4);
+                    }
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        if constexpr (V == 0) {
+                            h[n] = fmaf(ex2_ordered(dl4[j] * a2[i]), h[n], du4[j] * b4[j]);
+                            ya[j] = fmaf(c4[j], h[n], ya[j]);
+                        } else if constexpr (V == 1) {
+                            h[n] = fma_ordered(ex2_ordered(mul_ordered(dl4[j], a2[i])), h[n], mul_ordered(du4[j], b4[j]));
+                            ya[j] = fma_ordered(c4[j], h[n], ya[j]);
+                        } else {
+                            h[n] = fmaf(ex2(dl4[j] * a2[i]), h[n], du4[j] * b4[j]);
+                            ya[j] = fmaf(c4[j], h[n], ya[j]);
+                        }
+                    }
+                }
+            }
+            float u4[4];
+            load4(ru + t0, u4);  // read again rather than held across the state loop
+            if constexpr (G == 1) {
+                float o[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) o[j] = fmaf(dsk, u4[j], ya[j]);
+                if (cval) store_row<T, 4>(yrow + l0 + t0, o, nvalid - t0, p.vec);
+            } else {
+                // lane g keeps steps 2g, 2g + 1 and adds the other lane's share
+                const float k0 = g ? ya[2] : ya[0], k1 = g ? ya[3] : ya[1];
+                const float s0 = g ? ya[0] : ya[2], s1 = g ? ya[1] : ya[3];
+                float o[2];
+                o[0] = fmaf(dsk, g ? u4[2] : u4[0], k0 + __shfl_xor_sync(0xffffffffu, s0, 1));
+                o[1] = fmaf(dsk, g ? u4[3] : u4[1], k1 + __shfl_xor_sync(0xffffffffu, s1, 1));
+                if (cval) store_row<T, 2>(yrow + l0 + t0 + 2 * g, o, nvalid - t0 - 2 * g, p.vec);
+            }
+        }
+    }
+    cp_async_wait<0>();
+}
+
 // Launch 2 of the chunked variant: the inclusive state after every chunk,
 // inc_m = 2^(A_n log2 e S_m) inc_{m-1} + H_m from inc_{-1} = 0, for every
 // (channel, state) of a tile.  The chain is short in arithmetic but long in
@@ -1122,12 +1351,26 @@ KernelInfo chunk_info() {
     return {ok ? ff : nullptr, LY::bytes, LY::G, LY::DT, LY::THREADS, LY::CL, ok ? fa : nullptr};
 }
 
+template <typename T, class SS>
+KernelInfo stream_info() {
+    using LY = StreamLayout<T, SS>;
+    const void* fn = reinterpret_cast<const void*>(&full_stream_kernel<T, SS>);
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [&] {
+        attr_err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LY::bytes);
+    });
+    return {attr_err == cudaSuccess ? fn : nullptr, LY::bytes, LY::G, LY::DT, LY::THREADS, LY::TS};
+}
+
 // Tile shapes per padded state count, in order of preference (fewest lanes
 // per channel first).  The zero-order-hold variant uses the first shape.
-int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 12; }
+int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 16; }
 constexpr int kLanesShape = 7;   // index of the lane-per-state variant (N <= 16 padded to 16)
 constexpr int kChunkShape = 8;   // first index of the three-launch chunked variant (shapes 8 to 11)
 bool is_chunk_shape(int np, int shape) { return np == 16 && shape >= kChunkShape && shape < kChunkShape + 4; }
+constexpr int kStreamShape = 12;  // first index of the streaming one-lane variant (shapes 12 to 15)
+bool is_stream_shape(int np, int shape) { return np == 16 && shape >= kStreamShape && shape < kStreamShape + 4; }
 
 template <typename T, bool ZOH>
 KernelInfo pick_t(int np, int shape) {
@@ -1152,6 +1395,10 @@ KernelInfo pick_t(int np, int shape) {
         case 9: return chunk_info<T, ChunkShape<2, 64, 32, 2, 4>>();
         case 10: return chunk_info<T, ChunkShape<1, 64, 64, 4, 5>>();
         case 11: return chunk_info<T, ChunkShape<2, 64, 64, 4, 4>>();
+        case 12: return stream_info<T, StreamShape<1, 128, 8, 4, 0>>();
+        case 13: return stream_info<T, StreamShape<1, 128, 8, 4, 1>>();
+        case 14: return stream_info<T, StreamShape<1, 128, 8, 4, 2>>();
+        case 15: return stream_info<T, StreamShape<1, 64, 8, 8, 0>>();
         default: return info_for<T, 16, Shape<1, 128, 0, 3, 7>, ZOH>();
         }
     }
@@ -1209,8 +1456,9 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
         *resident = (long long)(per_sm < 1 ? 1 : per_sm) * sms;
         return VMB_OK;
     };
-    // Rules measured on GB300 over the benchmark workloads: plenty of rows ->
-    // one lane per channel; a fair number -> two lanes; too few -> cut L into
+    // Rules measured on GB300 over the benchmark workloads: 16 states, at least
+    // 256 channel rows per SM and L >= 128 -> the streaming kernel; otherwise plenty of
+    // rows -> one lane per channel; a fair number -> two lanes; too few -> cut L into
     // chunks: 64-step chunks of the three-launch variant while they fit in two
     // waves, else look-back chunks with one lane per channel when they stay
     // long (>= 256 steps) and the widest split otherwise (>= 128 steps).
@@ -1229,6 +1477,11 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
             const long long want = (res + tiles - 1) / tiles, mx = (a.L + 255) / 256;
             n_chunks = (int)(want < mx ? want : mx);
         }
+    } else if (np == 16 && rows >= 256LL * sms && a.L >= 128) {
+        // many rows: the streaming one-lane kernel, one pass over L (on very
+        // short sequences its stage prologue does not pay off)
+        shape = kStreamShape;
+        if ((st = info(shape, &ki, &res)) != VMB_OK) return st;
     } else {
         const ShapeRoles r = roles(np);
         if ((st = info(r.wide, &ki, &res)) != VMB_OK) return st;
@@ -1290,6 +1543,7 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
         }
     }
     if (is_chunk_shape(np, shape)) n_chunks = (a.L + ki.ts - 1) / ki.ts;  // chunks of exactly ts steps
+    if (is_stream_shape(np, shape)) n_chunks = 1;                       // one pass over L
     if (n_chunks < 1) n_chunks = 1;
     ScanPlan p{};
     p.np = np;
