@@ -160,29 +160,33 @@ __device__ __forceinline__ void load_tile(const FullParams& p, T* dst, size_t ro
     const int L = p.L;
     T* dB = dst + 2 * DT * RS;
     if (p.vec) {
-        constexpr int nU = DT * CPR, nB = NP * CPR;
-        constexpr int total = 2 * nU + (WITH_B ? (WITH_C ? 2 : 1) * nB : 0);
-        for (int i = threadIdx.x; i < total; i += kThreads) {
-            const T* src;
-            T* d;
-            bool ok;
-            if (i < 2 * nU) {
-                const int j = i < nU ? i : i - nU;
-                const int r = j / CPR, ch = j % CPR;
-                const T* base = i < nU ? u : dl;
-                ok = r < nrows && l0 + ch * VE < L;
-                src = ok ? base + ((row0 + r) * (size_t)L + l0 + ch * VE) : base;
-                d = dst + (i < nU ? 0 : DT * RS) + r * RS + ch * VE;
-            } else {
-                const int i2 = i - 2 * nU;
-                const int j = i2 < nB ? i2 : i2 - nB;
-                const int r = j / CPR, ch = j % CPR;
-                const T* base = i2 < nB ? Bs : Cs;
-                ok = r < p.N && l0 + ch * VE < L;
-                src = ok ? base + ((bcrow0 + r) * (size_t)L + l0 + ch * VE) : base;
-                d = dB + (i2 < nB ? 0 : NP * RS) + r * RS + ch * VE;
+        // thread i copies 16-byte column i % CPR of rows i / CPR + k * RPP
+        constexpr int RPP = kThreads / CPR;  // rows covered per pass of the CTA
+        static_assert(kThreads % CPR == 0, "tile loader mapping");
+        const int ch = threadIdx.x % CPR, r0 = threadIdx.x / CPR;
+        const int col = l0 + ch * VE;
+        const bool colok = col < L;
+#pragma unroll
+        for (int it = 0; it < (DT + RPP - 1) / RPP; ++it) {
+            const int r = r0 + it * RPP;
+            if (DT % RPP == 0 || r < DT) {
+                const bool ok = colok && r < nrows;
+                const size_t off = (row0 + r) * (size_t)L + col;
+                cp_async16(dst + r * RS + ch * VE, ok ? u + off : u, ok ? 16 : 0);
+                cp_async16(dst + (DT + r) * RS + ch * VE, ok ? dl + off : dl, ok ? 16 : 0);
             }
-            cp_async16(d, src, ok ? 16 : 0);
+        }
+        if constexpr (WITH_B) {
+#pragma unroll
+            for (int it = 0; it < (NP + RPP - 1) / RPP; ++it) {
+                const int r = r0 + it * RPP;
+                if (r < NP) {
+                    const bool ok = colok && r < p.N;
+                    const size_t off = (bcrow0 + r) * (size_t)L + col;
+                    cp_async16(dB + r * RS + ch * VE, ok ? Bs + off : Bs, ok ? 16 : 0);
+                    if constexpr (WITH_C) cp_async16(dB + (NP + r) * RS + ch * VE, ok ? Cs + off : Cs, ok ? 16 : 0);
+                }
+            }
         }
     } else {
         constexpr int nU = DT * kTS, nB = NP * kTS;
