@@ -222,6 +222,21 @@ class Step:
             ("cross_merge_full", lib.vmb_cross_merge, (P(outs["yf"]), P(outs["of"]), B, D, H, W, dt, s)),
             ("cross_merge_mean", lib.vmb_cross_merge, (P(outs["ym"]), P(outs["om"]), B, D, H, W, dt, s)),
         ]
+        # the channel-mean path with the broadcast fused into the merge (timed on
+        # its own, next to the unfused mean scan + cross-merge of the step)
+        self.fused = ("mean_scan_merge", lib.vmb_mean_scan_merge_fwd,
+                      (P(outs["xs"]), P(g["draw"]), P(g["A"]), P(g["Bs"]), P(g["Cs"]), P(g["Dskip"]), P(g["bias"]),
+                       P(g["x"]), P(outs["ofused"]), P(outs["ybar"]), B, D, N, H, W, fl, dt, P(wsm), wsm.numel(), s))
+        # kernels each call launches (the chunked full scan launches three)
+        self.launches = sum(int(lib.vmb_scan_kernel_count(path, B, K, D, N, H, W, dt)) if path >= 0 else 1
+                            for path in (-1, 0, 1, -1, -1))
+        self.fused_launches = int(lib.vmb_scan_kernel_count(1, B, K, D, N, H, W, dt)) + 1
+
+    def run_fused(self):
+        name, fn, args = self.fused
+        st = fn(*args)
+        if st != 0:
+            raise RuntimeError(f"{name}: {self.vmb.status_string(st)}")
 
     def run(self, events=None):
         for i, (name, fn, args) in enumerate(self.calls):
@@ -256,6 +271,8 @@ def run_ours(args, wl, rank, world, local_rank):
         "om": torch.empty((B, D, H, W), dtype=tdt, device=dev),
         "ws_full": torch.zeros(vmb.vmb_scan_workspace_bytes(0, B, 4, D, N, H, W, tdt), dtype=torch.uint8, device=dev),
         "ws_mean": torch.zeros(vmb.vmb_scan_workspace_bytes(1, B, 4, D, N, H, W, tdt), dtype=torch.uint8, device=dev),
+        "ofused": torch.empty((B, D, H, W), dtype=tdt, device=dev),
+        "ybar": torch.empty((B, 4, L), dtype=torch.float32, device=dev),
     }
     stream = torch.cuda.current_stream()
     step = Step(vmb, wl, g, outs, stream.cuda_stream)
@@ -287,6 +304,21 @@ def run_ours(args, wl, rank, world, local_rank):
         torch.distributed.barrier()
     if vmb.vmb_read_status(outs["ws_full"]) != 0 or vmb.vmb_read_status(outs["ws_mean"]) != 0:
         raise RuntimeError("device error word set during the timed steps")
+    # the fused channel-mean path, timed alone with the same L2 flush per call
+    fev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    for _ in range(args.warmup):
+        prelude()
+        step.run_fused()
+    torch.cuda.synchronize()
+    for i in range(args.steps):
+        prelude()
+        fev[i][0].record()
+        step.run_fused()
+        fev[i][1].record()
+    torch.cuda.synchronize()
+    if vmb.vmb_read_status(outs["ws_mean"]) != 0:
+        raise RuntimeError("device error word set in the fused mean path")
+    fused_ms = [e[0].elapsed_time(e[1]) for e in fev]
     per_kernel = {k: [] for k in KERNELS}
     step_ms = []
     for e in evs:
@@ -323,7 +355,8 @@ def run_ours(args, wl, rank, world, local_rank):
     e2e_ms = e0.elapsed_time(e1)
 
     res = {"total_ms": total_ms, "step_ms": step_ms, "per_kernel": per_kernel, "e2e_ms": e2e_ms,
-           "h2d": h2d, "d2h": d2h, "clocks": clk.summary()}
+           "h2d": h2d, "d2h": d2h, "clocks": clk.summary(), "fused_ms": fused_ms,
+           "launches_per_step": step.launches, "fused_launches": step.fused_launches}
     res["total_ms"], res["e2e_ms"] = max_over_ranks([total_ms, e2e_ms], world, dev)
     return res, inp
 
@@ -385,6 +418,7 @@ def main():
     for k in KERNELS:
         avg = statistics.mean(res["per_kernel"][k])
         per[k] = {"us": avg * 1e3, "gbs": kb[k] / (avg / 1e3) / 1e9, "frac_of_peak": kb[k] / (avg / 1e3) / 1e9 / peak}
+    fused_us = 1e3 * statistics.mean(res["fused_ms"])
     dominant = max(KERNELS, key=lambda k: statistics.mean(res["per_kernel"][k]))
     dom_ms = statistics.mean(res["per_kernel"][dominant])
     achieved = kb[dominant] / (dom_ms / 1e3) / 1e9
@@ -408,7 +442,15 @@ def main():
                      "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)" if peak_src == "measured"
                      else "fallback 6.8 TB/s", "unit": "GB/s", "frac": achieved / peak,
                      "algorithmic_bytes_per_launch": kb[dominant], "traffic": traffic},
-        "gpu_launches": len(KERNELS) * args.steps,
+        # the fused channel-mean path (broadcast inside the merge), timed separately
+        "mean_path_fused": {
+            "us": fused_us, "gbs": wl.fused_mean_bytes() / (fused_us / 1e6) / 1e9,
+            "frac_of_peak": wl.fused_mean_bytes() / (fused_us / 1e6) / 1e9 / peak,
+            "algorithmic_bytes": wl.fused_mean_bytes(),
+            "unfused_us": per["mean_scan"]["us"] + per["cross_merge_mean"]["us"],
+            "speedup_over_unfused": (per["mean_scan"]["us"] + per["cross_merge_mean"]["us"]) / fused_us,
+            "speedup_over_full_path": (per["full_scan"]["us"] + per["cross_merge_full"]["us"]) / fused_us},
+        "gpu_launches": res["launches_per_step"] * args.steps,
         "clocks": res["clocks"],
         "e2e": {"value": job_throughput(step_bytes, world, res["e2e_ms"] / args.e2e_steps), "unit": "GB/s",
                 "ms_per_step": res["e2e_ms"] / args.e2e_steps,

@@ -112,6 +112,17 @@ size_t vmb_scan_workspace_bytes(int path, int B, int K, int D, int N, int H, int
                                 vmb_dtype dtype);
 
 /*
+ * vmb_scan_kernel_count - number of kernels one vmb_selective_scan_fwd
+ * (VMB_PATH_FULL) or vmb_mean_scan_fwd (VMB_PATH_MEAN) call launches for this
+ * problem on the current device: 1, or 3 for the L-chunked full scan that
+ * resolves the chunk carry in launches of its own.  0 for an empty problem or
+ * invalid arguments.  (vmb_mean_scan_merge_fwd launches the mean scan's
+ * kernels plus one merge kernel.)  Bookkeeping for timing tools; the paper
+ * has no counterpart.
+ */
+int vmb_scan_kernel_count(int path, int B, int K, int D, int N, int H, int W, vmb_dtype dtype);
+
+/*
  * vmb_selective_scan_fwd - full-channel selective scan over K directions
  * (App. A: selection Eq. 6, discretisation Eq. 4, recurrence Eq. 3), with the
  * discretisation fused into the scan:
@@ -149,6 +160,32 @@ vmb_status vmb_mean_scan_fwd(const void* u, const void* delta, const float* A, c
                              float* ybar, int B, int K, int D, int N, int H, int W, unsigned flags,
                              vmb_dtype dtype, void* workspace, size_t workspace_bytes,
                              cudaStream_t stream);
+
+/*
+ * vmb_mean_scan_merge_fwd - the channel-mean path of an SS2D block (Sec. 2.2,
+ * Eq. 9, then the App. A cross-merge) with the broadcast T^-1 fused into the
+ * merge, so the per-channel output y [B, 4, D, L] is never written:
+ *   every direction's u at the position it merges into is the map itself,
+ *   u_k[b,d,p_k(h,w)] = x[b,d,h,w], hence
+ *   out[b,d,h,w] = (y0 + y2) + (y1 + y3),
+ *   y_k = ybar_k[b, p_k] + Dskip[k*D+d] x[b,d,h,w]  (p_k as in vmb_cross_merge;
+ *         VMB_FLAG_SKIP_MEAN: y_k = ybar_k[b, p_k] + the mean skip term of k)
+ *   u (= vmb_cross_scan(x)), delta [B, 4, D, L], Bs, Cs [B, 4, N, L] (dtype);
+ *   A [4*D, N], Dskip [4*D], delta_bias [4*D] (fp32);
+ *   x, out [B, D, H, W] (dtype), out must not alias x;
+ *   ybar [B, 4, L] fp32, required: receives ybar_k(t) (plus the broadcast mean
+ *   skip term under VMB_FLAG_SKIP_MEAN) and is read back by the merge.
+ *   workspace: as vmb_mean_scan_fwd with K = 4 (VMB_PATH_MEAN).
+ * The same fp32 operations in the same order as vmb_cross_merge applied to
+ * vmb_mean_scan_fwd's y, so fp32 results are bit-identical to that unfused
+ * pair; bf16 storage rounds once, at the end (the unfused pair rounds y
+ * first).  Not in the paper as such: its kernels keep the steps apart.
+ */
+vmb_status vmb_mean_scan_merge_fwd(const void* u, const void* delta, const float* A, const void* Bs,
+                                   const void* Cs, const float* Dskip, const float* delta_bias,
+                                   const void* x, void* out, float* ybar, int B, int D, int N, int H,
+                                   int W, unsigned flags, vmb_dtype dtype, void* workspace,
+                                   size_t workspace_bytes, cudaStream_t stream);
 
 /*
  * vmb_selective_scan_fwd_noalloc - vmb_selective_scan_fwd for callers that

@@ -469,4 +469,142 @@ vmb_status launch_cross_merge(const void* ys, void* out, int B, int D, int H, in
                           : launch_csm<float>(true, ys, out, B, D, H, W, stream);
 }
 
+// ------------------------------------------- channel-mean path: broadcast + merge
+// The channel-mean scan's output is y_k[b,d,l] = ybar_k[b,l] + Dskip[kD+d] u_k[b,d,l]
+// (Eq. 9 broadcast), and every direction's u at the position it merges into is
+// the map itself: u_k[b,d,p_k(h,w)] = x[b,d,h,w].  So the merged map is
+//   out[b,d,h,w] = (y0 + y2) + (y1 + y3),  y_k = ybar_k[b, p_k] + Dskip[kD+d] x[b,d,h,w]
+// (y_k = ybar_k[b, p_k] when the skip term is already folded into ybar), read
+// from x and the four ybar rows of (b, .) without y ever being written.  The
+// fp32 operations and their order are those of the broadcast and of the
+// cross-merge, so fp32 results are bit-identical to the unfused path; bf16
+// rounds once, at the end.  A thread owns kMP consecutive positions and keeps
+// their four ybar values in registers across the CTA's channels.
+namespace {
+constexpr int kMMThreads = 128;
+constexpr int kMP = 2;  // positions per thread
+constexpr int kMMMaxDC = 64;
+
+struct MeanMergeParams {
+    const void* x;
+    void* out;
+    const float* ybar;   // [B, 4, L]
+    const float* Dskip;  // [4 D]
+    int B, D, H, W;
+    int per_channel;  // 0: skip already in ybar
+    int vec;          // kMP positions of a row vector-accessible (aligned rows, L % kMP == 0)
+    int dc;           // channels per CTA
+};
+
+template <typename T>
+__global__ void __launch_bounds__(kMMThreads) mean_merge_kernel(const MeanMergeParams p) {
+    __shared__ float sd[4][kMMMaxDC];
+    const int H = p.H, W = p.W, L = H * W;
+    const int b = blockIdx.y;
+    const int dbeg = blockIdx.z * p.dc, dn = min(p.dc, p.D - dbeg);
+    for (int i = threadIdx.x; i < 4 * kMMMaxDC; i += kMMThreads) {
+        const int kd = i / kMMMaxDC, j = i % kMMMaxDC;
+        sd[kd][j] = (p.per_channel && j < dn) ? __ldg(p.Dskip + (size_t)kd * p.D + dbeg + j) : 0.0f;
+    }
+    const int pos0 = (blockIdx.x * kMMThreads + threadIdx.x) * kMP;
+    const float* yb = p.ybar + (size_t)b * 4 * L;
+    float y0[kMP], y1[kMP], y2[kMP], y3[kMP];
+#pragma unroll
+    for (int j = 0; j < kMP; ++j) {
+        const int pos = pos0 + j;
+        if (pos < L) {
+            const int h = pos / W, w = pos - h * W, p1 = w * H + h;
+            y0[j] = __ldg(yb + pos);
+            y2[j] = __ldg(yb + 2 * (size_t)L + (L - 1 - pos));
+            y1[j] = __ldg(yb + (size_t)L + p1);
+            y3[j] = __ldg(yb + 3 * (size_t)L + (L - 1 - p1));
+        } else {
+            y0[j] = y1[j] = y2[j] = y3[j] = 0.0f;
+        }
+    }
+    __syncthreads();
+    if (pos0 >= L) return;
+    const bool full = p.vec && pos0 + kMP <= L;
+    const T* x = static_cast<const T*>(p.x) + ((size_t)b * p.D + dbeg) * L + pos0;
+    T* out = static_cast<T*>(p.out) + ((size_t)b * p.D + dbeg) * L + pos0;
+    const uint64_t ev = l2_evict_first();
+    for (int dd = 0; dd < dn; ++dd, x += L, out += L) {
+        float xv[kMP], o[kMP];
+        if (full) {
+            if constexpr (sizeof(T) == 4) {
+                const float2 q = *reinterpret_cast<const float2*>(x);
+                xv[0] = q.x;
+                xv[1] = q.y;
+            } else {
+                const unsigned q = *reinterpret_cast<const unsigned*>(x);
+                xv[0] = __uint_as_float(q << 16);
+                xv[1] = __uint_as_float(q & 0xffff0000u);
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < kMP; ++j) xv[j] = pos0 + j < L ? io<T>::cvt(x[j]) : 0.0f;
+        }
+        const float s0 = sd[0][dd], s1 = sd[1][dd], s2 = sd[2][dd], s3 = sd[3][dd];
+#pragma unroll
+        for (int j = 0; j < kMP; ++j) {
+            const float a = fmaf(s0, xv[j], y0[j]) + fmaf(s2, xv[j], y2[j]);
+            const float c = fmaf(s1, xv[j], y1[j]) + fmaf(s3, xv[j], y3[j]);
+            o[j] = a + c;
+        }
+        if (full) {
+            if constexpr (sizeof(T) == 4) {
+                asm volatile("st.global.L2::cache_hint.v2.f32 [%0], {%1, %2}, %3;" ::"l"(out), "f"(o[0]), "f"(o[1]),
+                             "l"(ev)
+                             : "memory");
+            } else {
+                const unsigned q = __bfloat16_as_ushort(io<T>::to(o[0])) |
+                                   ((unsigned)__bfloat16_as_ushort(io<T>::to(o[1])) << 16);
+                *reinterpret_cast<unsigned*>(out) = q;
+            }
+        } else {
+#pragma unroll
+            for (int j = 0; j < kMP; ++j)
+                if (pos0 + j < L) out[j] = io<T>::to(o[j]);
+        }
+    }
+}
+
+template <typename T>
+vmb_status launch_mean_merge_t(const void* x, const float* ybar, const float* Dskip, void* out, int B, int D, int H,
+                               int W, bool per_channel, cudaStream_t stream) {
+    const long long L = (long long)H * W;
+    const unsigned nblk = (unsigned)((L + kMMThreads * kMP - 1) / (kMMThreads * kMP));
+    // channels per CTA: enough CTAs for a few waves, each amortising its ybar
+    // reads over as many channels as that leaves
+    const long long per_ch = (long long)nblk * B;
+    long long dc = per_ch * D / (8LL * device_sm_count());
+    dc = dc < 8 ? 8 : dc > kMMMaxDC ? kMMMaxDC : dc;
+    if (dc > D) dc = D;
+    const auto al = [](const void* q, size_t a) { return (reinterpret_cast<uintptr_t>(q) % a) == 0; };
+    MeanMergeParams p{};
+    p.x = x;
+    p.out = out;
+    p.ybar = ybar;
+    p.Dskip = Dskip;
+    p.B = B;
+    p.D = D;
+    p.H = H;
+    p.W = W;
+    p.per_channel = per_channel ? 1 : 0;
+    p.vec = (L % kMP == 0) && al(x, kMP * sizeof(T)) && al(out, kMP * sizeof(T));
+    p.dc = (int)dc;
+    const dim3 grid(nblk, (unsigned)B, (unsigned)((D + dc - 1) / dc));
+    if (grid.y > 65535u || grid.z > 65535u) return VMB_ERR_UNSUPPORTED;
+    mean_merge_kernel<T><<<grid, kMMThreads, 0, stream>>>(p);
+    return cudaGetLastError() == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+}
+}  // namespace
+
+vmb_status launch_mean_merge(const void* x, const float* ybar, const float* Dskip, void* out, int B, int D, int H,
+                             int W, bool per_channel_skip, vmb_dtype dt, cudaStream_t stream) {
+    return dt == VMB_BF16
+               ? launch_mean_merge_t<__nv_bfloat16>(x, ybar, Dskip, out, B, D, H, W, per_channel_skip, stream)
+               : launch_mean_merge_t<float>(x, ybar, Dskip, out, B, D, H, W, per_channel_skip, stream);
+}
+
 }  // namespace vmb

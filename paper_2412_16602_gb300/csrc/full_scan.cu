@@ -1583,6 +1583,10 @@ static cudaError_t launch_pdl(const void* fn, unsigned grid, int threads, size_t
     return cudaLaunchKernelExC(&cfg, fn, args);
 }
 
+int full_plan_launches(const ScanPlan& plan) {
+    return (is_chunk_shape(plan.np, plan.split) && plan.n_chunks > 1) ? 3 : 1;
+}
+
 vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream) {
     KernelInfo ki = pick(a.dtype, plan.np, plan.split, (a.flags & VMB_FLAG_B_ZOH) != 0);
     if (!ki.fn) return VMB_ERR_CUDA;

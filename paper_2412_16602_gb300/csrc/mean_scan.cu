@@ -54,6 +54,7 @@ struct MeanParams {
     int suppress;
     int bcvec;   // B / C rows 16-byte aligned: async-copied
     int tabvec;  // A, delta_bias, Dskip 16-byte aligned: async-copied
+    int no_bcast;  // fused with the cross-merge: no y; ybar (+ the broadcast skip term) only
     WsHeader* hdr;
     unsigned* flags;
     float* aggP;
@@ -244,6 +245,17 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
     float* s_a2 = reinterpret_cast<float*>(smb + LY::tab0);
     const float* s_bias = s_a2 + CG * NP;
     const float* s_dsk = s_bias + CG;
+    float vd[kPF], vu[kPF];
+    {
+        // the first group's first channels, requested before the tables are waited on
+        const int gn = min(CG, D);
+#pragma unroll
+        for (int q = 0; q < kPF; ++q) {
+            const int d = sg + q * S;
+            vd[q] = (tv && d < gn) ? ld_hint(dcol + (size_t)d * L, stream) : 0.0f;
+            vu[q] = (tv && d < gn) ? ld_hint(ucol + (size_t)d * L, keep) : 0.0f;
+        }
+    }
     for (int gi = 0; gi < ngroups; ++gi) {
         const int g0 = gi * CG, gn = min(CG, D - g0);
         if (gi > 0) {
@@ -258,12 +270,13 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
             __syncthreads();
         }
         if (!tv) continue;
-        float vd[kPF], vu[kPF];
+        if (gi > 0) {
 #pragma unroll
-        for (int q = 0; q < kPF; ++q) {
-            const int d = sg + q * S;
-            vd[q] = d < gn ? ld_hint(dcol + (size_t)(g0 + d) * L, stream) : 0.0f;
-            vu[q] = d < gn ? ld_hint(ucol + (size_t)(g0 + d) * L, keep) : 0.0f;
+            for (int q = 0; q < kPF; ++q) {
+                const int d = sg + q * S;
+                vd[q] = d < gn ? ld_hint(dcol + (size_t)(g0 + d) * L, stream) : 0.0f;
+                vu[q] = d < gn ? ld_hint(ucol + (size_t)(g0 + d) * L, keep) : 0.0f;
+            }
         }
         for (int d0 = sg; d0 < gn; d0 += kPF * S) {
             float nd[kPF], nu[kPF];
@@ -451,18 +464,23 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
 #pragma unroll
         for (int n = 0; n < NP; ++n) s2 += abar[t * NP + n];
         s_ybar[t] = s2;
-        if (p.ybar && t < nvalid) p.ybar[(size_t)seq * L + l0 + t] = s2;
+        // fused with the merge, ybar carries the broadcast skip term (the same
+        // fp32 add the broadcast below would do)
+        if (p.ybar && t < nvalid) p.ybar[(size_t)seq * L + l0 + t] = (p.no_bcast && p.skip_mean) ? s2 + s_dsu[t] : s2;
     }
     __syncthreads();
 
     // ---------------------------------------------------------------- phase C
-    if (tv) {
+    if (tv && !p.no_bcast) {
         T* y = static_cast<T*>(p.y);
         const size_t colc = (size_t)l0 + rt;
         const float yb = s_ybar[rt];
         const float dsu = s_dsu[rt];
-        constexpr int kPC = 8;  // u reads in flight per thread
+        // u reads in flight per thread: with short chunks (many channels per
+        // thread) all of a thread's channels of a 192-channel map in one round
+        constexpr int kPC = TC == 32 ? 24 : 8;
         const uint64_t ev = l2_evict_first();
+        const bool dsk_smem = ngroups == 1;  // Dskip of every channel is still staged
         for (int d0 = sg; d0 < D; d0 += kPC * S) {
             float uv[kPC];
 #pragma unroll
@@ -474,8 +492,10 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
             for (int q = 0; q < kPC; ++q) {
                 const int d = d0 + q * S;
                 if (d < D) {
-                    const float skip = p.skip_mean ? dsu : __ldg(p.Dskip + (size_t)k * D + d) * uv[q];  // Dskip: L1-resident
-                    st_hint(y + (urow0 + d) * (size_t)L + colc, yb + skip, ev);
+                    const float dk = dsk_smem ? s_dsk[d] : __ldg(p.Dskip + (size_t)k * D + d);
+                    // y = ybar + Dskip u as one FMA (the fused merge does the same)
+                    const float yv = p.skip_mean ? yb + dsu : fmaf(dk, uv[q], yb);
+                    st_hint(y + (urow0 + d) * (size_t)L + colc, yv, ev);
                 }
             }
         }
@@ -599,6 +619,7 @@ vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     const size_t es = a.dtype == VMB_BF16 ? 2 : 4;
     const auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
     p.bcvec = ((size_t)a.L * es % 16 == 0) && al16(a.Bs) && al16(a.Cs);
+    p.no_bcast = a.no_bcast ? 1 : 0;
     p.tabvec = al16(a.A) && al16(a.bias) && al16(a.Dskip);
     const WsLayout w = ws_layout(plan);
     unsigned char* ws = static_cast<unsigned char*>(a.ws);

@@ -76,10 +76,12 @@ vmb_status check_scan(const ScanArgs& a, bool mean, bool* empty) {
     if (a.N > 16) return VMB_ERR_UNSUPPORTED;
     long long grid_rows = 0;
     if (!count(&grid_rows, {a.B, a.K, a.D}) || grid_rows > INT_MAX / 2) return VMB_ERR_UNSUPPORTED;
-    if (!a.u || !a.delta || !a.A || !a.Bs || !a.Cs || !a.Dskip || !a.bias || !a.y) return VMB_ERR_INVALID_ARG;
+    if (!a.u || !a.delta || !a.A || !a.Bs || !a.Cs || !a.Dskip || !a.bias || (!a.y && !a.no_bcast))
+        return VMB_ERR_INVALID_ARG;
+    if (a.no_bcast && !a.ybar) return VMB_ERR_INVALID_ARG;
     const size_t es = esize(a.dtype);
     if (!aligned(a.u, es) || !aligned(a.delta, es) || !aligned(a.Bs, es) || !aligned(a.Cs, es) ||
-        !aligned(a.y, es) || !aligned(a.A, 4) || !aligned(a.Dskip, 4) || !aligned(a.bias, 4) ||
+        (a.y && !aligned(a.y, es)) || !aligned(a.A, 4) || !aligned(a.Dskip, 4) || !aligned(a.bias, 4) ||
         (a.ybar && !aligned(a.ybar, 4)))
         return VMB_ERR_MISALIGNED;
     return VMB_OK;
@@ -142,6 +144,27 @@ size_t vmb_scan_workspace_bytes(int path, int B, int K, int D, int N, int H, int
     return plan.ws_bytes;
 }
 
+int vmb_scan_kernel_count(int path, int B, int K, int D, int N, int H, int W, vmb_dtype dtype) {
+    if (path != VMB_PATH_FULL && path != VMB_PATH_MEAN) return 0;
+    if (H < 0 || W < 0 || (long long)H * W > INT_MAX) return 0;
+    ScanArgs a{};
+    a.B = B;
+    a.K = K;
+    a.D = D;
+    a.N = N;
+    a.L = H * W;
+    a.dtype = dtype;
+    static const float dummy[4] = {0, 0, 0, 0};
+    a.u = a.delta = a.Bs = a.Cs = dummy;
+    a.A = a.Dskip = a.bias = dummy;
+    a.y = const_cast<float*>(dummy);
+    bool empty = false;
+    if (check_scan(a, path == VMB_PATH_MEAN, &empty) != VMB_OK || empty) return 0;
+    ScanPlan plan{};
+    if (path == VMB_PATH_MEAN) return plan_mean(a, &plan) == VMB_OK ? 1 : 0;
+    return plan_full(a, &plan) == VMB_OK ? full_plan_launches(plan) : 0;
+}
+
 vmb_status vmb_selective_scan_fwd(const void* u, const void* delta, const float* A, const void* Bs, const void* Cs,
                                   const float* Dskip, const float* delta_bias, void* y, int B, int K, int D, int N,
                                   int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,
@@ -160,6 +183,22 @@ vmb_status vmb_mean_scan_fwd(const void* u, const void* delta, const float* A, c
     if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
     ScanArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, y, ybar, B, K, D, N, H * W, flags, dtype, workspace, workspace_bytes};
     return run_scan(a, true, stream);
+}
+
+vmb_status vmb_mean_scan_merge_fwd(const void* u, const void* delta, const float* A, const void* Bs, const void* Cs,
+                                   const float* Dskip, const float* delta_bias, const void* x, void* out, float* ybar,
+                                   int B, int D, int N, int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,
+                                   size_t workspace_bytes, cudaStream_t stream) {
+    bool empty = false;
+    vmb_status s = check_csm(x, out, B, D, H, W, dtype, &empty);
+    if (s != VMB_OK || empty) return s;
+    if (x == out) return VMB_ERR_INVALID_ARG;
+    ScanArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, nullptr, ybar, B, 4, D, N, H * W, flags, dtype,
+               workspace, workspace_bytes};
+    a.no_bcast = true;
+    s = run_scan(a, true, stream);
+    if (s != VMB_OK) return s;
+    return launch_mean_merge(x, ybar, Dskip, out, B, D, H, W, (flags & VMB_FLAG_SKIP_MEAN) == 0, dtype, stream);
 }
 
 vmb_status vmb_read_status(void* workspace, cudaStream_t stream) {

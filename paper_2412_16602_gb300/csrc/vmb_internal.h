@@ -26,6 +26,7 @@ struct ScanArgs {
     vmb_dtype dtype;
     void* ws;
     size_t ws_bytes;
+    bool no_bcast = false;  // mean path fused with the cross-merge: ybar only, no y
 };
 
 // Execution plan of an L-chunked scan: how the (sequence, chunk) grid is cut
@@ -67,10 +68,13 @@ int device_sm_count();
 vmb_status plan_full(const ScanArgs& a, ScanPlan* plan);
 vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan);
 vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream);
+int full_plan_launches(const ScanPlan& plan);  // kernels launch_full starts for this plan
 vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream);
 vmb_status launch_cross_scan(const void* x, void* xs, int B, int D, int H, int W, vmb_dtype dt,
                              cudaStream_t stream);
 vmb_status launch_cross_merge(const void* ys, void* out, int B, int D, int H, int W, vmb_dtype dt,
                               cudaStream_t stream);
+vmb_status launch_mean_merge(const void* x, const float* ybar, const float* Dskip, void* out, int B, int D, int H,
+                             int W, bool per_channel_skip, vmb_dtype dt, cudaStream_t stream);
 
 }  // namespace vmb

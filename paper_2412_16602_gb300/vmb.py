@@ -37,8 +37,9 @@ VMB_FLAG_TEST_SUPPRESS_PUBLISH = 0x40000000
 VMB_PATH_FULL = 0
 VMB_PATH_MEAN = 1
 
-EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb_selective_scan_fwd",
-           "vmb_mean_scan_fwd", "vmb_read_status", "vmb_status_string", "vmb_version"]
+EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb_scan_kernel_count",
+           "vmb_selective_scan_fwd",
+           "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_read_status", "vmb_status_string", "vmb_version"]
 
 
 class VmbError(RuntimeError):
@@ -56,14 +57,17 @@ def _load() -> ctypes.CDLL:
     lib.vmb_cross_merge.argtypes = [vp, vp, i, i, i, i, i, vp]
     lib.vmb_scan_workspace_bytes.argtypes = [i, i, i, i, i, i, i, i]
     lib.vmb_scan_workspace_bytes.restype = sz
+    lib.vmb_scan_kernel_count.argtypes = [i, i, i, i, i, i, i, i]
+    lib.vmb_scan_kernel_count.restype = i
     lib.vmb_selective_scan_fwd.argtypes = [vp] * 8 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_fwd.argtypes = [vp] * 9 + [i] * 6 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_merge_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
     lib.vmb_read_status.argtypes = [vp, vp]
     lib.vmb_status_string.argtypes = [i]
     lib.vmb_status_string.restype = ctypes.c_char_p
     lib.vmb_version.argtypes = []
     for name in ["vmb_cross_scan", "vmb_cross_merge", "vmb_selective_scan_fwd", "vmb_mean_scan_fwd",
-                 "vmb_read_status", "vmb_version"]:
+                 "vmb_mean_scan_merge_fwd", "vmb_read_status", "vmb_version"]:
         getattr(lib, name).restype = i
     return lib
 
@@ -155,6 +159,11 @@ def vmb_scan_workspace_bytes(path: int, B: int, K: int, D: int, N: int, H: int, 
     return int(lib.vmb_scan_workspace_bytes(path, B, K, D, N, H, W, _dtype_code(dtype)))
 
 
+def vmb_scan_kernel_count(path: int, B: int, K: int, D: int, N: int, H: int, W: int,
+                          dtype: torch.dtype = torch.float32) -> int:
+    return int(lib.vmb_scan_kernel_count(path, B, K, D, N, H, W, _dtype_code(dtype)))
+
+
 class Workspace:
     """A zero-initialised device workspace that grows on demand (one per device).
 
@@ -243,6 +252,36 @@ def vmb_mean_scan_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, H: int, W: int, *,
                                  _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
                                  _stream(stream)), "vmb_mean_scan_fwd")
     return y, ybar
+
+
+def vmb_mean_scan_merge_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, x, H: int, W: int, *,
+                            out=None, ybar=None, flags: int = VMB_FLAG_SOFTPLUS, workspace=None, stream=None):
+    """Channel-mean path with the broadcast fused into the cross-merge:
+    returns (out [B, D, H, W], ybar [B, 4, L] fp32)."""
+    B, K, D, N, L = _scan_shapes(u, delta, A, Bs, Cs, Dskip, delta_bias, H, W)
+    if K != 4:
+        raise ValueError("the fused merge needs the four SS2D directions (K = 4)")
+    _dev(x, "x")
+    if tuple(x.shape) != (B, D, H, W) or x.dtype != u.dtype:
+        raise ValueError("x must be [B, D, H, W] in the storage dtype of u")
+    if out is None:
+        out = torch.empty_like(x)
+    _dev(out, "out")
+    if out.shape != x.shape or out.dtype != x.dtype:
+        raise ValueError("out must match x")
+    if ybar is None:
+        ybar = torch.empty((B, 4, L), dtype=torch.float32, device=u.device)
+    _dev(ybar, "ybar")
+    if ybar.shape != (B, 4, L) or ybar.dtype != torch.float32:
+        raise ValueError("ybar must be float32 [B, 4, L]")
+    ws_bytes = vmb_scan_workspace_bytes(VMB_PATH_MEAN, B, 4, D, N, H, W, u.dtype)
+    if workspace is None:
+        workspace = _default_ws.get(ws_bytes, u.device)
+    _check(lib.vmb_mean_scan_merge_fwd(_ptr(u), _ptr(delta), _ptr(A), _ptr(Bs), _ptr(Cs), _ptr(Dskip),
+                                       _ptr(delta_bias), _ptr(x), _ptr(out), _ptr(ybar), B, D, N, H, W, flags,
+                                       _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
+                                       _stream(stream)), "vmb_mean_scan_merge_fwd")
+    return out, ybar
 
 
 def vmb_read_status(workspace=None, device=None, stream=None) -> int:

@@ -20,8 +20,11 @@ def lib():
     lib.vmb_cross_merge.argtypes = [vp, vp, i, i, i, i, i, vp]
     lib.vmb_scan_workspace_bytes.argtypes = [i] * 8
     lib.vmb_scan_workspace_bytes.restype = sz
+    lib.vmb_scan_kernel_count.argtypes = [i] * 8
+    lib.vmb_scan_kernel_count.restype = i
     lib.vmb_selective_scan_fwd.argtypes = [vp] * 8 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_fwd.argtypes = [vp] * 9 + [i] * 6 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_merge_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
     lib.vmb_status_string.argtypes = [i]
     lib.vmb_status_string.restype = ctypes.c_char_p
     lib.vmb_read_status.argtypes = [vp, vp]
@@ -102,6 +105,30 @@ def test_workspace_query_invalid_and_empty(lib):
     assert lib.vmb_scan_workspace_bytes(1, 0, 4, 8, 16, 4, 4, 0) == 256
 
 
+def test_kernel_count_invalid_and_empty(lib):
+    assert lib.vmb_scan_kernel_count(7, 1, 4, 8, 16, 4, 4, 0) == 0
+    assert lib.vmb_scan_kernel_count(0, 1, 4, 8, 17, 4, 4, 0) == 0
+    assert lib.vmb_scan_kernel_count(1, 0, 4, 8, 16, 4, 4, 0) == 0
+
+
 def test_read_status_rejects_null(lib):
     assert lib.vmb_read_status(0, 0) == 1
     assert lib.vmb_read_status(FAKE + 8, 0) == 2
+
+
+def merge_call(lib, *, ptrs=None, B=1, D=8, N=16, H=4, W=4, flags=1, dtype=0, ws=0x100000, ws_bytes=1 << 20):
+    p = [FAKE] * 7 + [FAKE, FAKE + 0x1000, FAKE + 0x2000] if ptrs is None else ptrs
+    return lib.vmb_mean_scan_merge_fwd(*p, B, D, N, H, W, flags, dtype, ws, ws_bytes, S)
+
+
+def test_mean_scan_merge_validation(lib):
+    base = [FAKE] * 7 + [FAKE, FAKE + 0x1000, FAKE + 0x2000]
+    assert merge_call(lib, B=-1) == 1
+    assert merge_call(lib, ptrs=base[:7] + [0] + base[8:]) == 1                # null x
+    assert merge_call(lib, ptrs=base[:8] + [FAKE] + base[9:]) == 1             # out aliases x
+    assert merge_call(lib, ptrs=base[:9] + [0]) == 1                           # ybar is required
+    assert merge_call(lib, ptrs=base[:7] + [FAKE + 2] + base[8:]) == 2         # misaligned fp32 map
+    assert merge_call(lib, N=17) == 3
+    assert merge_call(lib, flags=0x100) == 1
+    assert merge_call(lib, ws=0) == 4
+    assert merge_call(lib, ptrs=[0] * 10, B=0, ws=0) == 0                      # empty problem

@@ -71,6 +71,18 @@ class Workload:
         one map of B*D*L elements on one side, four on the other."""
         return self.esize * 5 * self.B * self.D * self.L
 
+    def fused_mean_bytes(self) -> int:
+        """Algorithmic bytes of the channel-mean path with the broadcast fused
+        into the cross-merge: u and delta read once, Bs and Cs read once, the
+        map x read and the merged map written once, ybar (fp32, [B, K, L])
+        written and read back once, plus the per-channel parameters."""
+        s = self.esize
+        bkdl = self.B * self.K * self.D * self.L
+        bknl = self.B * self.K * self.N * self.L
+        bdl = self.B * self.D * self.L
+        params = self.K * self.D * (self.N + 2) * 4
+        return s * (2 * bkdl + 2 * bknl + 2 * bdl) + 2 * 4 * self.B * self.K * self.L + params
+
     def replace(self, **kw) -> "Workload":
         d = dict(self.__dict__)
         d.update(kw)
