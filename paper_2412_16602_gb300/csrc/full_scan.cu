@@ -833,6 +833,11 @@ __device__ __forceinline__ void lds4_ordered(const float* p, float (&v)[4]) {
     const unsigned a = (unsigned)__cvta_generic_to_shared(p);
     asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]) : "r"(a));
 }
+// The same from a 32-bit shared-window address (a base computed once plus a
+// constant offset folds into the load's immediate).
+__device__ __forceinline__ void lds4_ordered_u32(unsigned a, float (&v)[4]) {
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]) : "r"(a));
+}
 __device__ __forceinline__ float ex2_ordered(float x) {
     float y;
     asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -970,6 +975,7 @@ __global__ void __launch_bounds__(ChunkLayout<T, CS>::THREADS, CS::MINB) full_ch
 #pragma unroll
                 for (int j = 0; j < 4; ++j) du4[j] = dl4[j] * u4[j];
             }
+            const unsigned sb = (unsigned)__cvta_generic_to_shared(rb + t0);  // this lane's B rows at t0
             float ya[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
             for (int q = 0; q < NG / 4; ++q) {
@@ -987,8 +993,8 @@ __global__ void __launch_bounds__(ChunkLayout<T, CS>::THREADS, CS::MINB) full_ch
                     // free, the compiler hoists all row reads of the block and runs
                     // out of registers
                     float b4[4], c4[4];
-                    lds4_ordered(rb + n * FS + t0, b4);
-                    if constexpr (PH2) lds4_ordered(rc + n * FS + t0, c4);
+                    lds4_ordered_u32(sb + n * FS * 4, b4);
+                    if constexpr (PH2) lds4_ordered_u32(sb + (NP + n) * FS * 4, c4);
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         h[n] = fmaf(ex2_ordered(dl4[j] * a2[i]), h[n], du4[j] * b4[j]);
@@ -1186,6 +1192,7 @@ __global__ void __launch_bounds__(StreamLayout<T, SS>::THREADS, SS::MINB) full_s
 #pragma unroll
                 for (int j = 0; j < 4; ++j) du4[j] = dl4[j] * u4[j];
             }
+            const unsigned sb = (unsigned)__cvta_generic_to_shared(rb + t0);  // this lane's B rows at t0
             float ya[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
             for (int q = 0; q < NG / 4; ++q) {
@@ -1204,8 +1211,9 @@ __global__ void __launch_bounds__(StreamLayout<T, SS>::THREADS, SS::MINB) full_s
                         load4(rb + n * BS + t0, b4);
                         load4(rc + n * BS + t0, c4);
                     } else {
-                        lds4_ordered(rb + n * BS + t0, b4);
-                        lds4_ordered(rc + n * BS + t0, c4);
+                        // B row n and C row n of this 4-step block: fixed offsets from sb
+                        lds4_ordered_u32(sb + n * BS * 4, b4);
+                        lds4_ordered_u32(sb + (NP + n) * BS * 4, c4);
                     }
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
@@ -1400,9 +1408,9 @@ KernelInfo pick_t(int np, int shape) {
         case 10: return chunk_info<T, ChunkShape<1, 64, 64, 4, 5>>();
         case 11: return chunk_info<T, ChunkShape<2, 64, 64, 4, 4>>();
         case 12: return stream_info<T, StreamShape<1, 128, 8, 4, 0>>();
-        case 13: return stream_info<T, StreamShape<1, 128, 8, 4, 1>>();
+        case 13: return stream_info<T, StreamShape<1, 64, 8, 8, 0>>();
         case 14: return stream_info<T, StreamShape<1, 128, 8, 4, 2>>();
-        case 15: return stream_info<T, StreamShape<1, 64, 8, 8, 0>>();
+        case 15: return stream_info<T, StreamShape<2, 64, 8, 6, 2>>();
         default: return info_for<T, 16, Shape<1, 128, 0, 3, 7>, ZOH>();
         }
     }
