@@ -245,17 +245,50 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
     float* s_a2 = reinterpret_cast<float*>(smb + LY::tab0);
     const float* s_bias = s_a2 + CG * NP;
     const float* s_dsk = s_bias + CG;
+    // Offsets within the (b, k) slab are 32-bit (D * L < 2^31, checked by the
+    // planner); a thread's consecutive channels are SL elements apart.
+    const int SL = S * L;
     float vd[kPF], vu[kPF];
     {
         // the first group's first channels, requested before the tables are waited on
         const int gn = min(CG, D);
+        int o = sg * L;
 #pragma unroll
-        for (int q = 0; q < kPF; ++q) {
+        for (int q = 0; q < kPF; ++q, o += SL) {
             const int d = sg + q * S;
-            vd[q] = (tv && d < gn) ? ld_hint(dcol + (size_t)d * L, stream) : 0.0f;
-            vu[q] = (tv && d < gn) ? ld_hint(ucol + (size_t)d * L, keep) : 0.0f;
+            vd[q] = (tv && d < gn) ? ld_hint(dcol + o, stream) : 0.0f;
+            vu[q] = (tv && d < gn) ? ld_hint(ucol + o, keep) : 0.0f;
         }
     }
+    // one channel's contribution: softplus, the N exponentials of Abar, delta u
+    auto reduce_one = [&](float vdq, float vuq, int d) {
+        const float v = vdq + s_bias[d];
+        const float dv = p.softplus_on ? softplus(v) : v;
+        const float* a2 = s_a2 + d * NP;  // broadcast reads: every lane has the same d
+        if constexpr (ZOH) {
+#pragma unroll
+            for (int n = 0; n < NP; ++n) {
+                const float an = a2[n];
+                const float em1 = expm1f(dv * an);
+                acc[n] += 1.0f + em1;
+                accb[n] = fmaf(an != 0.0f ? em1 / an : dv, vuq, accb[n]);
+            }
+        } else if constexpr (NP % 4 == 0) {
+#pragma unroll
+            for (int n = 0; n < NP; n += 4) {
+                const float4 qa = *reinterpret_cast<const float4*>(a2 + n);
+                acc[n] += ex2(dv * qa.x);
+                acc[n + 1] += ex2(dv * qa.y);
+                acc[n + 2] += ex2(dv * qa.z);
+                acc[n + 3] += ex2(dv * qa.w);
+            }
+        } else {
+#pragma unroll
+            for (int n = 0; n < NP; ++n) acc[n] += ex2(dv * a2[n]);
+        }
+        sdu = fmaf(dv, vuq, sdu);
+        if (p.skip_mean) sdsu = fmaf(s_dsk[d], vuq, sdsu);
+    };
     for (int gi = 0; gi < ngroups; ++gi) {
         const int g0 = gi * CG, gn = min(CG, D - g0);
         if (gi > 0) {
@@ -271,52 +304,42 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
         }
         if (!tv) continue;
         if (gi > 0) {
+            int o = (g0 + sg) * L;
 #pragma unroll
-            for (int q = 0; q < kPF; ++q) {
+            for (int q = 0; q < kPF; ++q, o += SL) {
                 const int d = sg + q * S;
-                vd[q] = d < gn ? ld_hint(dcol + (size_t)(g0 + d) * L, stream) : 0.0f;
-                vu[q] = d < gn ? ld_hint(ucol + (size_t)(g0 + d) * L, keep) : 0.0f;
+                vd[q] = d < gn ? ld_hint(dcol + o, stream) : 0.0f;
+                vu[q] = d < gn ? ld_hint(ucol + o, keep) : 0.0f;
             }
         }
         for (int d0 = sg; d0 < gn; d0 += kPF * S) {
             float nd[kPF], nu[kPF];
+            int o = (g0 + d0 + kPF * S) * L;  // the next batch's first channel
+            if (d0 + (2 * kPF - 1) * S < gn) {
+                // the next batch is entirely in range: no per-channel checks
 #pragma unroll
-            for (int q = 0; q < kPF; ++q) {
-                const int d = d0 + (q + kPF) * S;
-                nd[q] = d < gn ? ld_hint(dcol + (size_t)(g0 + d) * L, stream) : 0.0f;
-                nu[q] = d < gn ? ld_hint(ucol + (size_t)(g0 + d) * L, keep) : 0.0f;
-            }
-#pragma unroll
-            for (int q = 0; q < kPF; ++q) {
-                const int d = d0 + q * S;
-                if (d >= gn) break;
-                const float v = vd[q] + s_bias[d];
-                const float uv = vu[q];
-                const float dv = p.softplus_on ? softplus(v) : v;
-                const float* a2 = s_a2 + d * NP;  // broadcast reads: every lane has the same d
-                if constexpr (ZOH) {
-#pragma unroll
-                    for (int n = 0; n < NP; ++n) {
-                        const float an = a2[n];
-                        const float em1 = expm1f(dv * an);
-                        acc[n] += 1.0f + em1;
-                        accb[n] = fmaf(an != 0.0f ? em1 / an : dv, uv, accb[n]);
-                    }
-                } else if constexpr (NP % 4 == 0) {
-#pragma unroll
-                    for (int n = 0; n < NP; n += 4) {
-                        const float4 qa = *reinterpret_cast<const float4*>(a2 + n);
-                        acc[n] += ex2(dv * qa.x);
-                        acc[n + 1] += ex2(dv * qa.y);
-                        acc[n + 2] += ex2(dv * qa.z);
-                        acc[n + 3] += ex2(dv * qa.w);
-                    }
-                } else {
-#pragma unroll
-                    for (int n = 0; n < NP; ++n) acc[n] += ex2(dv * a2[n]);
+                for (int q = 0; q < kPF; ++q, o += SL) {
+                    nd[q] = ld_hint(dcol + o, stream);
+                    nu[q] = ld_hint(ucol + o, keep);
                 }
-                sdu = fmaf(dv, uv, sdu);
-                if (p.skip_mean) sdsu = fmaf(s_dsk[d], uv, sdsu);
+            } else {
+#pragma unroll
+                for (int q = 0; q < kPF; ++q, o += SL) {
+                    const int d = d0 + (q + kPF) * S;
+                    nd[q] = d < gn ? ld_hint(dcol + o, stream) : 0.0f;
+                    nu[q] = d < gn ? ld_hint(ucol + o, keep) : 0.0f;
+                }
+            }
+            if (d0 + (kPF - 1) * S < gn) {
+#pragma unroll
+                for (int q = 0; q < kPF; ++q) reduce_one(vd[q], vu[q], d0 + q * S);
+            } else {
+#pragma unroll
+                for (int q = 0; q < kPF; ++q) {
+                    const int d = d0 + q * S;
+                    if (d >= gn) break;
+                    reduce_one(vd[q], vu[q], d);
+                }
             }
 #pragma unroll
             for (int q = 0; q < kPF; ++q) {
@@ -472,30 +495,36 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
 
     // ---------------------------------------------------------------- phase C
     if (tv && !p.no_bcast) {
-        T* y = static_cast<T*>(p.y);
-        const size_t colc = (size_t)l0 + rt;
+        T* yc = static_cast<T*>(p.y) + urow0 * (size_t)L + l0 + rt;
+        const T* uc = u + urow0 * (size_t)L + l0 + rt;
         const float yb = s_ybar[rt];
-        const float dsu = s_dsu[rt];
-        // u reads in flight per thread: with short chunks (many channels per
-        // thread) all of a thread's channels of a 192-channel map in one round
-        constexpr int kPC = TC == 32 ? 24 : 8;
         const uint64_t ev = l2_evict_first();
-        const bool dsk_smem = ngroups == 1;  // Dskip of every channel is still staged
-        for (int d0 = sg; d0 < D; d0 += kPC * S) {
-            float uv[kPC];
+        if (p.skip_mean) {
+            // y = ybar + the mean skip term: one value for every channel
+            const float yv = yb + s_dsu[rt];
+            int o = sg * L;
+            for (int d = sg; d < D; d += S, o += SL) st_hint(yc + o, yv, ev);
+        } else {
+            // y = ybar + Dskip u as one FMA (the fused merge does the same); with
+            // short chunks (many channels per thread) all of a thread's channels
+            // of a 192-channel map are in flight in one round
+            constexpr int kPC = TC == 32 ? 24 : 8;
+            const bool dsk_smem = ngroups == 1;  // Dskip of every channel is still staged
+            const float* dsk_g = p.Dskip + (size_t)k * D;
+            for (int d0 = sg; d0 < D; d0 += kPC * S) {
+                float uv[kPC];
+                const bool full = d0 + (kPC - 1) * S < D;
+                int o = d0 * L;
 #pragma unroll
-            for (int q = 0; q < kPC; ++q) {
-                const int d = d0 + q * S;
-                uv[q] = (d < D && !p.skip_mean) ? ld_hint(u + (urow0 + d) * (size_t)L + colc, ev) : 0.0f;
-            }
+                for (int q = 0; q < kPC; ++q, o += SL)
+                    uv[q] = (full || d0 + q * S < D) ? ld_hint(uc + o, ev) : 0.0f;
+                o = d0 * L;
 #pragma unroll
-            for (int q = 0; q < kPC; ++q) {
-                const int d = d0 + q * S;
-                if (d < D) {
-                    const float dk = dsk_smem ? s_dsk[d] : __ldg(p.Dskip + (size_t)k * D + d);
-                    // y = ybar + Dskip u as one FMA (the fused merge does the same)
-                    const float yv = p.skip_mean ? yb + dsu : fmaf(dk, uv[q], yb);
-                    st_hint(y + (urow0 + d) * (size_t)L + colc, yv, ev);
+                for (int q = 0; q < kPC; ++q, o += SL) {
+                    const int d = d0 + q * S;
+                    if (!full && d >= D) break;
+                    const float dk = dsk_smem ? s_dsk[d] : __ldg(dsk_g + d);
+                    st_hint(yc + o, fmaf(dk, uv[q], yb), ev);
                 }
             }
         }
@@ -557,6 +586,7 @@ KInfo mpick(vmb_dtype dt, int np, int tc, bool zoh) {
 
 vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan) {
     if (a.N < 1 || a.N > 16) return VMB_ERR_UNSUPPORTED;
+    if ((long long)a.D * a.L >= (1LL << 31)) return VMB_ERR_UNSUPPORTED;  // 32-bit offsets within a (b, k) slab
     int np = 1;
     while (np < a.N) np <<= 1;
     const bool zoh = (a.flags & VMB_FLAG_B_ZOH) != 0;
