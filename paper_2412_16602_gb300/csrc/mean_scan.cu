@@ -55,6 +55,7 @@ struct MeanParams {
     int bcvec;   // B / C rows 16-byte aligned: async-copied
     int tabvec;  // A, delta_bias, Dskip 16-byte aligned: async-copied
     int no_bcast;  // fused with the cross-merge: no y; ybar (+ the broadcast skip term) only
+    int cvec;      // u / y rows allow 4-step vector access (L % 4 == 0, 4-element aligned)
     WsHeader* hdr;
     unsigned* flags;
     float* aggP;
@@ -76,7 +77,7 @@ struct MLayout {
     static constexpr size_t abar = reds + (size_t)S * TC * 4;                   // f32 [TC][NP]
     static constexpr size_t bubar = abar + (size_t)TC * NP * 4;                 // f32 [TC][NP]
     static constexpr size_t mc = bubar + (size_t)TC * NP * 4;                   // f32 [4][NMC][NP]
-    static constexpr size_t ybar = mc + (size_t)4 * NMC * NP * 4;               // f32 [TC]
+    static constexpr size_t ybar = a16(mc + (size_t)4 * NMC * NP * 4);          // f32 [TC], 16-byte aligned
     static constexpr size_t dsu = ybar + (size_t)TC * 4;                        // f32 [TC]
     static constexpr size_t hin = dsu + (size_t)TC * 4;                         // f32 [NP]
     static constexpr size_t bc = a16(hin + (size_t)NP * 4);                     // T [2][NP][BCS] B, C rows as stored
@@ -134,6 +135,33 @@ __device__ __forceinline__ void stage_tables(const MeanParams& p, unsigned char*
             tdsk[i] = i < gn ? __ldg(dg + i) : 0.0f;
         }
     }
+}
+
+// Four consecutive elements with an L2 eviction policy (16 bytes fp32, 8 bytes bf16).
+__device__ __forceinline__ void ld4_hint(const float* q, uint64_t pol, float (&v)[4]) {
+    asm volatile("ld.global.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], %5;"
+                 : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3])
+                 : "l"(q), "l"(pol));
+}
+__device__ __forceinline__ void ld4_hint(const __nv_bfloat16* q, uint64_t pol, float (&v)[4]) {
+    unsigned a, b;
+    asm volatile("ld.global.L2::cache_hint.v2.b32 {%0, %1}, [%2], %3;" : "=r"(a), "=r"(b) : "l"(q), "l"(pol));
+    v[0] = __uint_as_float(a << 16);
+    v[1] = __uint_as_float(a & 0xffff0000u);
+    v[2] = __uint_as_float(b << 16);
+    v[3] = __uint_as_float(b & 0xffff0000u);
+}
+__device__ __forceinline__ void st4_hint(float* q, const float (&v)[4], uint64_t pol) {
+    asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(q), "f"(v[0]), "f"(v[1]),
+                 "f"(v[2]), "f"(v[3]), "l"(pol)
+                 : "memory");
+}
+__device__ __forceinline__ void st4_hint(__nv_bfloat16* q, const float (&v)[4], uint64_t pol) {
+    const unsigned a = __bfloat16_as_ushort(__float2bfloat16_rn(v[0])) |
+                       ((unsigned)__bfloat16_as_ushort(__float2bfloat16_rn(v[1])) << 16);
+    const unsigned b = __bfloat16_as_ushort(__float2bfloat16_rn(v[2])) |
+                       ((unsigned)__bfloat16_as_ushort(__float2bfloat16_rn(v[3])) << 16);
+    asm volatile("st.global.L2::cache_hint.v2.b32 [%0], {%1, %2}, %3;" ::"l"(q), "r"(a), "r"(b), "l"(pol) : "memory");
 }
 
 template <typename T, int NP, int TC, bool ZOH>
@@ -494,7 +522,67 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
     __syncthreads();
 
     // ---------------------------------------------------------------- phase C
-    if (tv && !p.no_bcast) {
+    if (!p.no_bcast && p.cvec) {
+        // thread (quad, channel group): four consecutive steps of every DG-th
+        // channel, 128-bit (bf16: 64-bit) loads and stores
+        constexpr int Q = TC / 4, DG = kThreads / Q;
+        const int t4 = 4 * (tid % Q), dg = tid / Q;
+        if (t4 < nvalid) {
+            const bool qfull = t4 + 4 <= nvalid;
+            T* yc = static_cast<T*>(p.y) + urow0 * (size_t)L + l0 + t4;
+            const T* uc = u + urow0 * (size_t)L + l0 + t4;
+            const float4 yq = *reinterpret_cast<const float4*>(s_ybar + t4);
+            const float yb[4] = {yq.x, yq.y, yq.z, yq.w};
+            const uint64_t ev = l2_evict_first();
+            const int SLg = DG * L;
+            if (p.skip_mean) {
+                float yv[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) yv[j] = yb[j] + s_dsu[t4 + j];
+                int o = dg * L;
+                for (int d = dg; d < D; d += DG, o += SLg) {
+                    if (qfull) {
+                        st4_hint(yc + o, yv, ev);
+                    } else {
+                        for (int j = 0; j < nvalid - t4; ++j) st_hint(yc + o + j, yv[j], ev);
+                    }
+                }
+            } else {
+                constexpr int kPC = 8;
+                const bool dsk_smem = ngroups == 1;
+                const float* dsk_g = p.Dskip + (size_t)k * D;
+                for (int d0 = dg; d0 < D; d0 += kPC * DG) {
+                    float uv[kPC][4];
+                    int o = d0 * L;
+#pragma unroll
+                    for (int q = 0; q < kPC; ++q, o += SLg) {
+                        const int d = d0 + q * DG;
+                        if (d < D && qfull) {
+                            ld4_hint(uc + o, ev, uv[q]);
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) uv[q][j] = (d < D && t4 + j < nvalid) ? ld_hint(uc + o + j, ev) : 0.0f;
+                        }
+                    }
+                    o = d0 * L;
+#pragma unroll
+                    for (int q = 0; q < kPC; ++q, o += SLg) {
+                        const int d = d0 + q * DG;
+                        if (d >= D) break;
+                        const float dk = dsk_smem ? s_dsk[d] : __ldg(dsk_g + d);
+                        float yv[4];
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) yv[j] = fmaf(dk, uv[q][j], yb[j]);  // as the fused merge does
+                        if (qfull) {
+                            st4_hint(yc + o, yv, ev);
+                        } else {
+                            for (int j = 0; j < nvalid - t4; ++j) st_hint(yc + o + j, yv[j], ev);
+                        }
+                    }
+                }
+            }
+        }
+    } else if (tv && !p.no_bcast) {
         T* yc = static_cast<T*>(p.y) + urow0 * (size_t)L + l0 + rt;
         const T* uc = u + urow0 * (size_t)L + l0 + rt;
         const float yb = s_ybar[rt];
@@ -649,6 +737,8 @@ vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     const size_t es = a.dtype == VMB_BF16 ? 2 : 4;
     const auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
     p.bcvec = ((size_t)a.L * es % 16 == 0) && al16(a.Bs) && al16(a.Cs);
+    const auto al4e = [&](const void* q) { return (reinterpret_cast<uintptr_t>(q) % (4 * es)) == 0; };
+    p.cvec = (a.L % 4 == 0) && al4e(a.u) && (a.y == nullptr || al4e(a.y));
     p.no_bcast = a.no_bcast ? 1 : 0;
     p.tabvec = al16(a.A) && al16(a.bias) && al16(a.Dskip);
     const WsLayout w = ws_layout(plan);
