@@ -305,10 +305,24 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
 #pragma unroll
             for (int n = 0; n < NP; n += 4) {
                 const float4 qa = *reinterpret_cast<const float4*>(a2 + n);
-                acc[n] += ex2(dv * qa.x);
-                acc[n + 1] += ex2(dv * qa.y);
-                acc[n + 2] += ex2(dv * qa.z);
-                acc[n + 3] += ex2(dv * qa.w);
+                if constexpr (TC >= 64) {
+                    // packed f32x2 products and sums: half the issue slots (measured
+                    // 4-5% faster on the large maps that take these chunk lengths)
+                    const float2 dv2 = make_float2(dv, dv);
+                    const float2 t01 = __fmul2_rn(dv2, make_float2(qa.x, qa.y));
+                    const float2 t23 = __fmul2_rn(dv2, make_float2(qa.z, qa.w));
+                    const float2 a01 = __fadd2_rn(make_float2(acc[n], acc[n + 1]), make_float2(ex2(t01.x), ex2(t01.y)));
+                    const float2 a23 = __fadd2_rn(make_float2(acc[n + 2], acc[n + 3]), make_float2(ex2(t23.x), ex2(t23.y)));
+                    acc[n] = a01.x;
+                    acc[n + 1] = a01.y;
+                    acc[n + 2] = a23.x;
+                    acc[n + 3] = a23.y;
+                } else {
+                    acc[n] += ex2(dv * qa.x);
+                    acc[n + 1] += ex2(dv * qa.y);
+                    acc[n + 2] += ex2(dv * qa.z);
+                    acc[n + 3] += ex2(dv * qa.w);
+                }
             }
         } else {
 #pragma unroll
