@@ -290,20 +290,33 @@ def run_ours(args, wl, rank, world, local_rank):
     if vmb.vmb_read_status(outs["ws_full"]) != 0 or vmb.vmb_read_status(outs["ws_mean"]) != 0:
         raise RuntimeError("device error word set during warm-up")
 
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(KERNELS) + 1)] for _ in range(args.steps)]
+    # the timed steps: one event pair per step, nothing between the kernels
+    sev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
     with ClockSampler(local_rank) as clk:
         for i in range(args.steps):
             prelude()
-            evs[i][0].record()
-            step.run(evs[i])
+            sev[i][0].record()
+            step.run()
+            sev[i][1].record()
         torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     if vmb.vmb_read_status(outs["ws_full"]) != 0 or vmb.vmb_read_status(outs["ws_mean"]) != 0:
         raise RuntimeError("device error word set during the timed steps")
+    # the per-kernel breakdown: the same steps again with an event after every
+    # call (each event costs the stream a few microseconds, so these durations
+    # add up to more than the step time above)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(KERNELS) + 1)] for _ in range(args.steps)]
+    for i in range(args.steps):
+        prelude()
+        evs[i][0].record()
+        step.run(evs[i])
+    torch.cuda.synchronize()
+    if vmb.vmb_read_status(outs["ws_full"]) != 0 or vmb.vmb_read_status(outs["ws_mean"]) != 0:
+        raise RuntimeError("device error word set during the breakdown steps")
     # the fused channel-mean path, timed alone with the same L2 flush per call
     fev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
     for _ in range(args.warmup):
@@ -320,9 +333,8 @@ def run_ours(args, wl, rank, world, local_rank):
         raise RuntimeError("device error word set in the fused mean path")
     fused_ms = [e[0].elapsed_time(e[1]) for e in fev]
     per_kernel = {k: [] for k in KERNELS}
-    step_ms = []
+    step_ms = [e[0].elapsed_time(e[1]) for e in sev]
     for e in evs:
-        step_ms.append(e[0].elapsed_time(e[-1]))
         for j, k in enumerate(KERNELS):
             per_kernel[k].append(e[j].elapsed_time(e[j + 1]))
     total_ms = float(sum(step_ms))

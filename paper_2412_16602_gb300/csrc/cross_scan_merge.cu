@@ -56,6 +56,8 @@ union Vec {
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads) cross_scan_kernel(const CsmParams p) {
+    pdl_wait();
+    pdl_launch_dependents();
     extern __shared__ __align__(16) unsigned char smem_raw[];
     T* sp = reinterpret_cast<T*>(smem_raw);  // [ppc][H][W+1]
     constexpr int VE = 16 / sizeof(T);
@@ -134,6 +136,8 @@ __global__ void __launch_bounds__(kThreads) cross_scan_kernel(const CsmParams p)
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads) cross_merge_kernel(const CsmParams p) {
+    pdl_wait();
+    pdl_launch_dependents();
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int L = p.L, W = p.W, H = p.H, HP = p.H + 1;
     const long long p0 = (long long)blockIdx.x * p.ppc;
@@ -225,6 +229,8 @@ struct BandParams {
 
 template <typename T>
 __global__ void __launch_bounds__(kBandThreads) cross_scan_band_kernel(const BandParams p) {
+    pdl_wait();
+    pdl_launch_dependents();
     extern __shared__ __align__(16) unsigned char smem_raw[];
     T* tile = reinterpret_cast<T*>(smem_raw);  // [kRB][W+1]
     constexpr int VE = 16 / sizeof(T);
@@ -292,6 +298,8 @@ __global__ void __launch_bounds__(kBandThreads) cross_scan_band_kernel(const Ban
 
 template <typename T>
 __global__ void __launch_bounds__(kBandThreads) cross_merge_band_kernel(const BandParams p) {
+    pdl_wait();
+    pdl_launch_dependents();
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int W = p.W, H = p.H, L = p.L, WP = p.W + 1;
     T* s1 = reinterpret_cast<T*>(smem_raw);  // [kRB][W+1]: ys1 at pixel (h0 + j, w)
@@ -363,6 +371,8 @@ __global__ void __launch_bounds__(kBandThreads) cross_merge_band_kernel(const Ba
 // Planes too large for shared memory: one thread per element, plain gathers.
 template <typename T>
 __global__ void cross_scan_direct(const T* x, T* xs, int D, int H, int W, long long total) {
+    pdl_wait();
+    pdl_launch_dependents();
     const long long L = (long long)H * W;
     for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total; e += (long long)gridDim.x * blockDim.x) {
         const long long l = e % L, row = e / L;  // row = (b*4 + kd)*D + d
@@ -376,6 +386,8 @@ __global__ void cross_scan_direct(const T* x, T* xs, int D, int H, int W, long l
 
 template <typename T>
 __global__ void cross_merge_direct(const T* ys, T* out, int D, int H, int W, long long total) {
+    pdl_wait();
+    pdl_launch_dependents();
     const long long L = (long long)H * W;
     for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < total; e += (long long)gridDim.x * blockDim.x) {
         const long long pos = e % L, pl = e / L, d = pl % D, b = pl / D;
@@ -399,11 +411,12 @@ vmb_status launch_csm(bool merge, const void* in, void* outp, int B, int D, int 
     if (!small_enough) {
         const long long total = merge ? planes * L : planes * 4 * L;
         const int grid = (int)std::min<long long>((total + kThreads - 1) / kThreads, 152ll * 32);
-        if (merge)
-            cross_merge_direct<T><<<grid, kThreads, 0, stream>>>(static_cast<const T*>(in), static_cast<T*>(outp), D, H, W, total);
-        else
-            cross_scan_direct<T><<<grid, kThreads, 0, stream>>>(static_cast<const T*>(in), static_cast<T*>(outp), D, H, W, total);
-        return cudaGetLastError() == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+        const void* fn = merge ? reinterpret_cast<const void*>(&cross_merge_direct<T>)
+                               : reinterpret_cast<const void*>(&cross_scan_direct<T>);
+        const T* src = static_cast<const T*>(in);
+        T* dst = static_cast<T*>(outp);
+        void* args[] = {&src, &dst, &D, &H, &W, const_cast<long long*>(&total)};
+        return launch_kernel(fn, dim3(grid), dim3(kThreads), 0, args, stream) == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
     }
     if (L >= kBandMinL && (size_t)2 * kRB * (W + 1) * es <= kMaxSmem && planes * ((H + kRB - 1) / kRB) < (1ll << 31)) {
         BandParams bp{};
@@ -425,8 +438,8 @@ vmb_status launch_csm(bool merge, const void* in, void* outp, int B, int D, int 
             return VMB_ERR_CUDA;
         void* args[] = {&bp};
         const unsigned nblk = (unsigned)(planes * bp.nbands);
-        return cudaLaunchKernel(fn, dim3(nblk), dim3(kBandThreads), args, smem, stream) == cudaSuccess ? VMB_OK
-                                                                                                        : VMB_ERR_CUDA;
+        return launch_kernel(fn, dim3(nblk), dim3(kBandThreads), smem, args, stream) == cudaSuccess ? VMB_OK
+                                                                                                     : VMB_ERR_CUDA;
     }
     // about 8K elements per CTA, bounded by shared memory
     int ppc = (int)std::max<long long>(1, 8192 / L);
@@ -454,7 +467,7 @@ vmb_status launch_csm(bool merge, const void* in, void* outp, int B, int D, int 
         return VMB_ERR_CUDA;
     const unsigned grid = (unsigned)((planes + ppc - 1) / ppc);
     void* args[] = {&p};
-    return cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, stream) == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+    return launch_kernel(fn, dim3(grid), dim3(kThreads), smem, args, stream) == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
 }
 
 }  // namespace
@@ -498,6 +511,8 @@ struct MeanMergeParams {
 
 template <typename T>
 __global__ void __launch_bounds__(kMMThreads) mean_merge_kernel(const MeanMergeParams p) {
+    pdl_wait();
+    pdl_launch_dependents();
     __shared__ float sd[4][kMMMaxDC];
     const int H = p.H, W = p.W, L = H * W;
     const int b = blockIdx.y;
@@ -595,8 +610,11 @@ vmb_status launch_mean_merge_t(const void* x, const float* ybar, const float* Ds
     p.dc = (int)dc;
     const dim3 grid(nblk, (unsigned)B, (unsigned)((D + dc - 1) / dc));
     if (grid.y > 65535u || grid.z > 65535u) return VMB_ERR_UNSUPPORTED;
-    mean_merge_kernel<T><<<grid, kMMThreads, 0, stream>>>(p);
-    return cudaGetLastError() == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+    void* args[] = {&p};
+    return launch_kernel(reinterpret_cast<const void*>(&mean_merge_kernel<T>), grid, dim3(kMMThreads), 0, args, stream) ==
+                   cudaSuccess
+               ? VMB_OK
+               : VMB_ERR_CUDA;
 }
 }  // namespace
 

@@ -221,6 +221,8 @@ __device__ __forceinline__ void load_stage(const FullParams& p, T* dst, size_t r
 template <typename T, int NP, class SH, bool ZOH>
 __global__ void __launch_bounds__(Layout<T, NP, SH>::THREADS, Layout<T, NP, SH>::MINB)
     full_scan_kernel(const FullParams p) {
+    pdl_wait();
+    pdl_launch_dependents();
     using LY = Layout<T, NP, SH>;
     constexpr int kThreads = LY::THREADS, kTS = LY::TS, RS = LY::RS, SLOT = LY::SLOT, DT = LY::DT;
     constexpr int G = LY::G, NSTG = LY::NSTG;
@@ -507,6 +509,8 @@ __device__ __forceinline__ void reduce_level(float (&v)[16], bool up) {
 
 template <typename T, bool ZOH>
 __global__ void __launch_bounds__(256) full_scan_lanes_kernel(const FullParams p) {
+    pdl_wait();
+    pdl_launch_dependents();
     using LY = Layout<T, 16, LanesShape>;
     constexpr int kTS = LY::TS, RS = LY::RS, SLOT = LY::SLOT, DT = LY::DT, NSTG = LY::NSTG;
     extern __shared__ __align__(16) unsigned char smem[];
@@ -748,11 +752,6 @@ struct ChunkLayout {
     static_assert(sizeof(T) == 2 || RS == FS, "fp32 delta rows are rewritten in place");
 };
 
-// Programmatic dependent launch (sm_90+): let the next kernel of the stream be
-// scheduled now / wait until the previous kernel's writes are visible.  Both
-// are no-ops for a kernel launched without the programmatic attribute.
-__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
-__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 // Load of sub-stage `part` (steps part*SUB .. part*SUB+SUB-1) of the u and
 // delta rows of the chunk tile: thread i always copies 16-byte column i % CPR
@@ -872,6 +871,11 @@ __global__ void __launch_bounds__(ChunkLayout<T, CS>::THREADS, CS::MINB) full_ch
     T* raw = reinterpret_cast<T*>(smem);
     float* sdl = reinterpret_cast<float*>(smem + LY::dl_off);
 
+    // launch 1 (and a single-chunk launch) reads its inputs only after the
+    // previous kernel has completed; launch 3 loads its tile before it waits
+    // for the carry of launch 2 (the inputs were complete before launch 1 passed
+    // its own wait, and launches 1 and 2 signal only after theirs)
+    if (!PH2 || p.n_chunks == 1) pdl_wait();
     pdl_launch_dependents();
     const int c = threadIdx.x / G, g = threadIdx.x % G;  // channel within the tile, lane of the channel
     const int tile = blockIdx.x % p.n_tiles;
@@ -1074,6 +1078,8 @@ struct StreamLayout {
 
 template <typename T, class SS>
 __global__ void __launch_bounds__(StreamLayout<T, SS>::THREADS, SS::MINB) full_stream_kernel(const FullParams p) {
+    pdl_wait();
+    pdl_launch_dependents();
     using LY = StreamLayout<T, SS>;
     constexpr int G = LY::G, NG = LY::NG, DT = LY::DT, TS = LY::TS, NP = 16, NSTG = LY::NSTG, RS = LY::RS,
                   SLOT = LY::SLOT, FS = LY::FS, THREADS = LY::THREADS;
@@ -1268,6 +1274,8 @@ __global__ void __launch_bounds__(kCarryThreads) full_carry_kernel(const FullPar
     constexpr int groups = DT / 2;
     constexpr size_t sfl = (size_t)DT * 16;
     __shared__ float segP[kSegs][32], segH[kSegs][32];
+    // launch 3 may start now: before its own wait it reads only the step inputs
+    // (complete since launch 1 passed its wait), as this kernel reads A here
     pdl_launch_dependents();
     const int lane = threadIdx.x & 31, seg = threadIdx.x >> 5;
     const int tile = blockIdx.x / groups;
@@ -1573,24 +1581,6 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     return VMB_OK;
 }
 
-// Launch that may begin while the previous kernel of the stream is still
-// running (programmatic stream serialization); the kernel orders its reads of
-// that kernel's results with griddepcontrol.wait.
-static cudaError_t launch_pdl(const void* fn, unsigned grid, int threads, size_t smem, void** args,
-                              cudaStream_t stream) {
-    cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3((unsigned)threads);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelExC(&cfg, fn, args);
-}
-
 int full_plan_launches(const ScanPlan& plan) {
     return (is_chunk_shape(plan.np, plan.split) && plan.n_chunks > 1) ? 3 : 1;
 }
@@ -1633,17 +1623,19 @@ vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
         // launches 1 and 2 of the chunked variant: aggregates, then the carry fold
         if (!ki.agg) return VMB_ERR_CUDA;
         const unsigned grid_agg = (unsigned)(plan.n_seq * (plan.n_chunks - 1));
-        cudaError_t e = cudaLaunchKernel(ki.agg, dim3(grid_agg), dim3(ki.threads), args, ki.smem, stream);
-        if (e != cudaSuccess) return VMB_ERR_CUDA;
+        if (launch_kernel(ki.agg, dim3(grid_agg), dim3(ki.threads), ki.smem, args, stream) != cudaSuccess)
+            return VMB_ERR_CUDA;
         const unsigned grid_carry = (unsigned)(plan.n_seq * (ki.DT / 2));
         const void* carry = ki.DT == 128 ? reinterpret_cast<const void*>(&full_carry_kernel<128>)
                                          : reinterpret_cast<const void*>(&full_carry_kernel<64>);
-        if (launch_pdl(carry, grid_carry, kCarryThreads, 0, args, stream) != cudaSuccess) return VMB_ERR_CUDA;
+        if (launch_kernel(carry, dim3(grid_carry), dim3(kCarryThreads), 0, args, stream) != cudaSuccess)
+            return VMB_ERR_CUDA;
         // launch 3 loads its tile and applies the softplus before it waits for the carry
-        return launch_pdl(ki.fn, grid, ki.threads, ki.smem, args, stream) == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+        return launch_kernel(ki.fn, dim3(grid), dim3(ki.threads), ki.smem, args, stream) == cudaSuccess ? VMB_OK
+                                                                                                       : VMB_ERR_CUDA;
     }
-    cudaError_t e = cudaLaunchKernel(ki.fn, dim3(grid), dim3(ki.threads), args, ki.smem, stream);
-    return e == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+    return launch_kernel(ki.fn, dim3(grid), dim3(ki.threads), ki.smem, args, stream) == cudaSuccess ? VMB_OK
+                                                                                                   : VMB_ERR_CUDA;
 }
 
 }  // namespace vmb

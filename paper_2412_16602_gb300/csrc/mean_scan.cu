@@ -187,6 +187,8 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
     __shared__ unsigned s_misc[2];
     __shared__ unsigned s_scr[2 * kThreads / 32 + 2];
 
+    pdl_wait();
+    pdl_launch_dependents();
     const int tid = threadIdx.x;
     const bool chunked = p.n_chunks > 1;
     int seq, chunk;
@@ -764,7 +766,7 @@ vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     p.incH = reinterpret_cast<float*>(ws + w.incH_off);
     const unsigned grid = (unsigned)(plan.n_seq * plan.n_chunks);
     void* args[] = {&p};
-    cudaError_t e = cudaLaunchKernel(ki.fn, dim3(grid), dim3(kThreads), args, a.D > 256 ? ki.smem2 : ki.smem, stream);
+    cudaError_t e = launch_kernel(ki.fn, dim3(grid), dim3(kThreads), a.D > 256 ? ki.smem2 : ki.smem, args, stream);
     return e == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
 }
 

@@ -62,6 +62,37 @@ __device__ __forceinline__ float softplus(float v) {
     return fmaxf(v, 0.0f) + 2.0f * z * p;
 }
 
+// ------------------------------------------- programmatic dependent launch
+
+// Every kernel of libvmb is launched with programmatic stream serialization,
+// so that its CTAs can be scheduled while the previous kernel of the stream
+// drains.  Each kernel therefore executes pdl_wait() (griddepcontrol.wait:
+// the previous kernel has completed and its writes are visible) before it
+// touches global memory, and only then pdl_launch_dependents(), which lets
+// the next kernel be scheduled.  Because no kernel signals its dependents
+// before its own wait has returned, a kernel that is already running may
+// read data written two or more launches earlier before its own wait (the
+// third launch of the chunked full scan does so).  Both instructions are
+// no-ops in a kernel launched without the attribute.
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Host side: launch `fn` with the programmatic attribute set.
+inline cudaError_t launch_kernel(const void* fn, dim3 grid, dim3 block, size_t smem, void** args,
+                                 cudaStream_t stream) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelExC(&cfg, fn, args);
+}
+
 // ------------------------------------------------------ memory-model helpers
 
 __device__ __forceinline__ unsigned ld_acquire(const unsigned* p) {
