@@ -80,6 +80,12 @@ class Oracle:
         lib.oracle_mean_scan.restype = i
         lib.oracle_softplus.argtypes = [P, P, lg]
         lib.oracle_softplus.restype = None
+        lib.oracle_discretise.argtypes = [P] * 7 + [lg] * 5 + [i, i]
+        lib.oracle_discretise.restype = None
+        lib.oracle_discretise_mean.argtypes = [P] * 7 + [lg] * 5 + [i, i]
+        lib.oracle_discretise_mean.restype = None
+        lib.oracle_scan_only.argtypes = [P] * 4 + [lg] * 5
+        lib.oracle_scan_only.restype = None
         self.lib = lib
         self.path = lib_path
 
@@ -144,6 +150,49 @@ class Oracle:
             raise RuntimeError("oracle_mean_scan failed")
         return y, ybar
 
+    def _disc_args(self, u, delta, A, Bs, bias):
+        u, delta, A, Bs, bias = (_f64(a) for a in (u, delta, A, Bs, bias))
+        B, K, D, L = u.shape
+        N = Bs.shape[2]
+        if delta.shape != u.shape or Bs.shape != (B, K, N, L) or A.shape != (K * D, N) or bias.shape != (K * D,):
+            raise ValueError("shape mismatch")
+        return (u, delta, A, Bs, bias), (B, K, D, N, L)
+
+    def discretise(self, u, delta, A, Bs, bias, *, softplus_on=True, b_mode=B_EULER):
+        """Eqs. 4, 6 outside the scan (Sec. 4 kernel setting): (dA, dBu), each [B, K, D, N, L]."""
+        arrs, (B, K, D, N, L) = self._disc_args(u, delta, A, Bs, bias)
+        dA = np.empty((B, K, D, N, L), dtype=np.float64)
+        dBu = np.empty_like(dA)
+        self.lib.oracle_discretise(*(_ptr(a) for a in arrs), _ptr(dA), _ptr(dBu), B, K, D, N, L,
+                                   int(bool(softplus_on)), int(b_mode))
+        return dA, dBu
+
+    def discretise_mean(self, u, delta, A, Bs, bias, *, softplus_on=True, b_mode=B_EULER):
+        """Eq. 9's T on the discretised operands: (dAm, dBum), each [B, K, N, L]."""
+        arrs, (B, K, D, N, L) = self._disc_args(u, delta, A, Bs, bias)
+        dAm = np.empty((B, K, N, L), dtype=np.float64)
+        dBum = np.empty_like(dAm)
+        self.lib.oracle_discretise_mean(*(_ptr(a) for a in arrs), _ptr(dAm), _ptr(dBum), B, K, D, N, L,
+                                        int(bool(softplus_on)), int(b_mode))
+        return dAm, dBum
+
+    def scan_only(self, dA, dBu, Cs) -> np.ndarray:
+        """The scan alone (Eq. 3 without the skip) on discretised operands.
+
+        dA, dBu [B, K, Dm, N, L] (or [B, K, N, L] for one channel), Cs [B, K, N, L]
+        -> y [B, K, Dm, L] (or [B, K, L])."""
+        dA, dBu, Cs = _f64(dA), _f64(dBu), _f64(Cs)
+        squeeze = dA.ndim == 4
+        if squeeze:
+            dA, dBu = dA[:, :, None], dBu[:, :, None]
+        B, K, Dm, N, L = dA.shape
+        if dBu.shape != dA.shape or Cs.shape != (B, K, N, L):
+            raise ValueError("shape mismatch")
+        dA, dBu = np.ascontiguousarray(dA), np.ascontiguousarray(dBu)
+        y = np.empty((B, K, Dm, L), dtype=np.float64)
+        self.lib.oracle_scan_only(_ptr(dA), _ptr(dBu), _ptr(Cs), _ptr(y), B, K, Dm, N, L)
+        return y[:, :, 0] if squeeze else y
+
     def ss2d_full(self, inp, **kw):
         """Cross-scan, full scan, cross-merge on one `workloads.Inputs` set."""
         wl = inp.wl
@@ -190,6 +239,18 @@ def selective_scan(*a, **kw):
 
 def mean_scan(*a, **kw):
     return get().mean_scan(*a, **kw)
+
+
+def discretise(*a, **kw):
+    return get().discretise(*a, **kw)
+
+
+def discretise_mean(*a, **kw):
+    return get().discretise_mean(*a, **kw)
+
+
+def scan_only(*a, **kw):
+    return get().scan_only(*a, **kw)
 
 
 def ss2d_full(inp, **kw):

@@ -14,6 +14,9 @@
  *   recurrence ..................... App. A, Eq. 3 (h_t = Abar h_{t-1} + Bbar u_t, y_t = C h_t + D u_t)
  *   channel mean (VMeanba) ......... Sec. 2.2, Eq. 9 (y = T^-1(Mamba(T(Abar, Bbar u, C))),
  *                                     T = mean over the inner channel axis, T^-1 = broadcast)
+ *   scan-only kernel setting ....... Sec. 4, "Kernel Implementation" (discretisation done
+ *                                     before the scan; the scan reads materialised Abar,
+ *                                     Bbar u with D channels, or one channel after T)
  *
  * Readings of points the paper leaves open (each is listed in the design notes):
  *   - scan directions: 0 row-major, 1 column-major, 2 = reverse of 0, 3 = reverse of 1;
@@ -247,6 +250,81 @@ int oracle_mean_scan(const double* u, const double* delta, const double* A, cons
     problem p = {u, delta, A, Bs, Cs, Dskip, bias, y, ybar, B, K, D, N, L, softplus_on, b_mode,
                  skip_mode};
     return run(&p, 1, nthreads);
+}
+
+/* ------------------------------------- the paper's scan-only kernel setting */
+
+/* Sec. 4 ("Kernel Implementation"): the paper's own kernel runs the scan alone,
+ * with the discretisation done before it.  These three functions split the
+ * path the same way.
+ *
+ * Discretisation (Eq. 6 softplus, Eq. 4) of every (b, k, d, n, l):
+ *   dA[b][k][d][n][l] = exp(delta A[c][n]),  dBu[b][k][d][n][l] = Bbar u. */
+void oracle_discretise(const double* u, const double* delta, const double* A, const double* Bs,
+                       const double* bias, double* dA, double* dBu, long B, long K, long D, long N,
+                       long L, int softplus_on, int b_mode) {
+    for (long b = 0; b < B; ++b)
+        for (long k = 0; k < K; ++k)
+            for (long d = 0; d < D; ++d) {
+                long c = k * D + d, row = (b * K + k) * D + d;
+                for (long n = 0; n < N; ++n)
+                    for (long l = 0; l < L; ++l) {
+                        double v = delta[row * L + l] + bias[c];
+                        double dlt = softplus_on ? softplus(v) : v;
+                        double a = A[c * N + n];
+                        dA[(row * N + n) * L + l] = exp(dlt * a);
+                        dBu[(row * N + n) * L + l] =
+                            discretise_b(dlt, a, Bs[((b * K + k) * N + n) * L + l], b_mode) * u[row * L + l];
+                    }
+            }
+}
+
+/* Eq. 9's T applied to the discretised operands: their means over the D
+ * channels of each (b, k), dAm, dBum [B][K][N][L] (the operands of the scan
+ * kernel with the channel axis reduced to one). */
+void oracle_discretise_mean(const double* u, const double* delta, const double* A, const double* Bs,
+                            const double* bias, double* dAm, double* dBum, long B, long K, long D, long N,
+                            long L, int softplus_on, int b_mode) {
+    for (long b = 0; b < B; ++b)
+        for (long k = 0; k < K; ++k)
+            for (long n = 0; n < N; ++n)
+                for (long l = 0; l < L; ++l) {
+                    double sa = 0.0, sb = 0.0;
+                    for (long d = 0; d < D; ++d) {
+                        long c = k * D + d, row = (b * K + k) * D + d;
+                        double v = delta[row * L + l] + bias[c];
+                        double dlt = softplus_on ? softplus(v) : v;
+                        double a = A[c * N + n];
+                        sa += exp(dlt * a);
+                        sb += discretise_b(dlt, a, Bs[((b * K + k) * N + n) * L + l], b_mode) * u[row * L + l];
+                    }
+                    dAm[((b * K + k) * N + n) * L + l] = sa / (double)D;
+                    dBum[((b * K + k) * N + n) * L + l] = sb / (double)D;
+                }
+}
+
+/* The scan alone (Eq. 3 without the skip term) on discretised operands of Dm
+ * channels per (b, k): h[n] = dA h[n] + dBu from h = 0 and
+ *   y[b][k][d][l] = sum_n C[b][k][n][l] h[n]  (C has no channel axis). */
+void oracle_scan_only(const double* dA, const double* dBu, const double* Cs, double* y, long B, long K,
+                      long Dm, long N, long L) {
+    double* h = (double*)malloc(sizeof(double) * (size_t)(N > 0 ? N : 1));
+    if (!h) return;
+    for (long b = 0; b < B; ++b)
+        for (long k = 0; k < K; ++k)
+            for (long d = 0; d < Dm; ++d) {
+                long row = (b * K + k) * Dm + d;
+                for (long n = 0; n < N; ++n) h[n] = 0.0;
+                for (long l = 0; l < L; ++l) {
+                    double acc = 0.0;
+                    for (long n = 0; n < N; ++n) {
+                        h[n] = dA[(row * N + n) * L + l] * h[n] + dBu[(row * N + n) * L + l];
+                        acc += Cs[((b * K + k) * N + n) * L + l] * h[n];
+                    }
+                    y[row * L + l] = acc;
+                }
+            }
+    free(h);
 }
 
 /* Eq. 6 softplus, exposed so that tests can pin it against known values. */

@@ -372,4 +372,83 @@ def pin_mean_skip_mean_mode(orc):
            what="skip mean")
 
 
+# -------------------------------------- scan-only setting (discretise, then scan)
+
+
+def pin_discretise_hand_worked(orc):
+    """raw + bias = 0 gives delta = softplus(0) = ln 2; with A = -1 that is
+    dA = e^{-ln 2} = 1/2 exactly, and with B = u = 1 the Euler dBu = ln 2; the
+    zero-order hold gives (e^{-ln 2} - 1) / (-1) = 1/2."""
+    u = np.ones((1, 1, 1, 2))
+    draw = np.array([[[[0.5, -0.25]]]])
+    bias = np.array([-0.5])
+    draw[0, 0, 0, 1] = 0.5  # both steps at raw + bias = 0
+    A = np.array([[-1.0]])
+    Bs = np.ones((1, 1, 1, 2))
+    dA, dBu = orc.discretise(u, draw, A, Bs, bias)
+    _close(dA, np.full((1, 1, 1, 1, 2), 0.5), what="dA")
+    _close(dBu, np.full((1, 1, 1, 1, 2), LN2), what="dBu euler")
+    _, dBz = orc.discretise(u, draw, A, Bs, bias, b_mode=1)
+    _close(dBz, np.full((1, 1, 1, 1, 2), 0.5), what="dBu zoh")
+
+
+def pin_scan_only_closed_forms(orc):
+    """Scan alone: at L = 1, y_0 = sum_n C_n dBu_n; with constant dA_n = a_n and
+    dBu = C = 1, y_t = sum_n (1 - a_n^{t+1}) / (1 - a_n) (geometric sums)."""
+    rng = np.random.default_rng(30)
+    dA = rng.uniform(0.1, 0.9, size=(2, 1, 3, 4, 1))
+    dBu = rng.standard_normal(dA.shape)
+    Cs = rng.standard_normal((2, 1, 4, 1))
+    y = orc.scan_only(dA, dBu, Cs)
+    _close(y[..., 0], np.einsum("bkdn,bkn->bkd", dBu[..., 0], Cs[..., 0]), what="L=1")
+    a = np.array([0.3, 0.7, 0.95])
+    L = 12
+    dA = np.broadcast_to(a[None, None, None, :, None], (1, 1, 1, 3, L)).copy()
+    y = orc.scan_only(dA, np.ones_like(dA), np.ones((1, 1, 3, L)))
+    t = np.arange(L)
+    exp = sum((1 - an ** (t + 1)) / (1 - an) for an in a)
+    _close(y[0, 0, 0], exp, what="geometric")
+
+
+def pin_scan_only_composes_to_full(orc):
+    """Discretising first and scanning the materialised operands, plus the skip
+    term, reproduces the brute-force unrolling of the full path (both B-bar forms)."""
+    rng = np.random.default_rng(31)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, B=2, K=2, D=3, N=4, L=9)
+    K, D = 2, 3
+    skip = Dskip.reshape(K, D)[None, :, :, None] * u
+    for b_mode in (0, 1):
+        dA, dBu = orc.discretise(u, draw, A, Bs, bias, b_mode=b_mode)
+        y = orc.scan_only(dA, dBu, Cs) + skip
+        _close(y, brute_force_full(u, draw, A, Bs, Cs, Dskip, bias, b_mode=b_mode), rtol=1e-11,
+               atol=1e-12, what=f"compose b_mode={b_mode}")
+
+
+def pin_scan_only_mean_composes_to_ybar(orc):
+    """The scan alone on the channel means of the discretised operands (one
+    channel) is the brute-force ybar of the averaged system (both B-bar forms)."""
+    rng = np.random.default_rng(32)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, B=2, K=2, D=5, N=3, L=8, draw_scale=1.5)
+    for b_mode in (0, 1):
+        dAm, dBum = orc.discretise_mean(u, draw, A, Bs, bias, b_mode=b_mode)
+        _close(orc.scan_only(dAm, dBum, Cs), brute_force_mean(u, draw, A, Bs, Cs, Dskip, bias, b_mode=b_mode),
+               rtol=1e-11, atol=1e-12, what=f"mean compose b_mode={b_mode}")
+
+
+def pin_discretise_mean_identical_channels(orc):
+    """With every channel of a direction identical, the channel means of the
+    discretised operands equal any one channel's operands."""
+    rng = np.random.default_rng(33)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, B=1, K=2, D=4, N=3, L=6)
+    K, D = 2, 4
+    u[:] = u[:, :, :1]
+    draw[:] = draw[:, :, :1]
+    A = np.repeat(A.reshape(K, D, -1)[:, :1], D, axis=1).reshape(K * D, -1)
+    bias = np.repeat(bias.reshape(K, D)[:, :1], D, axis=1).reshape(-1)
+    dA, dBu = orc.discretise(u, draw, A, Bs, bias)
+    dAm, dBum = orc.discretise_mean(u, draw, A, Bs, bias)
+    _close(dAm, dA[:, :, 2], rtol=1e-13, atol=1e-15, what="dA mean")
+    _close(dBum, dBu[:, :, 2], rtol=1e-13, atol=1e-15, what="dBu mean")
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

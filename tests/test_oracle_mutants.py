@@ -33,6 +33,17 @@ MUTANTS = {
     "mean_output_before_update": ("h[n] = abar[n] * h[n] + bubar[n];\n            ybar += Ck[n * L + t] * h[n];",
                                   "ybar += Ck[n * L + t] * h[n];\n            h[n] = abar[n] * h[n] + bubar[n];"),
     "mean_bu_without_u": ("p->b_mode) * u[d * L + t];", "p->b_mode);"),
+    "disc_abar_sign": ("dA[(row * N + n) * L + l] = exp(dlt * a);", "dA[(row * N + n) * L + l] = exp(-dlt * a);"),
+    "disc_bu_wrong_b_row": ("dBu[(row * N + n) * L + l] =\n                            discretise_b(dlt, a, Bs[((b * K + k) * N + n) * L + l]",
+                            "dBu[(row * N + n) * L + l] =\n                            discretise_b(dlt, a, Bs[((b * K + k) * N + 0) * L + l]"),
+    "disc_mean_sum_not_mean": ("dAm[((b * K + k) * N + n) * L + l] = sa / (double)D;",
+                               "dAm[((b * K + k) * N + n) * L + l] = sa;"),
+    "disc_mean_bias_wrong_channel": ("double v = delta[row * L + l] + bias[c];\n                        double dlt = softplus_on ? softplus(v) : v;\n                        double a = A[c * N + n];\n                        sa",
+                                     "double v = delta[row * L + l] + bias[k];\n                        double dlt = softplus_on ? softplus(v) : v;\n                        double a = A[c * N + n];\n                        sa"),
+    "scan_only_drops_decay": ("h[n] = dA[(row * N + n) * L + l] * h[n] + dBu[(row * N + n) * L + l];",
+                              "h[n] = h[n] + dBu[(row * N + n) * L + l];"),
+    "scan_only_output_before_update": ("h[n] = dA[(row * N + n) * L + l] * h[n] + dBu[(row * N + n) * L + l];\n                        acc += Cs[((b * K + k) * N + n) * L + l] * h[n];",
+                                       "acc += Cs[((b * K + k) * N + n) * L + l] * h[n];\n                        h[n] = dA[(row * N + n) * L + l] * h[n] + dBu[(row * N + n) * L + l];"),
 }
 
 
