@@ -52,6 +52,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-paper-style", action="store_true",
+                    help="skip the timing of the paper's split (discretise, then scan alone)")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch size (smaller captures for profiling)")
@@ -247,6 +249,55 @@ class Step:
                 events[i + 1].record()
 
 
+def time_paper_style(vmb, B, K, D, N, H, W, dev, prelude, steps, warmup):
+    """The paper's kernel split (Sec. 4): discretisation into materialised fp32
+    operands, then the scan alone, for the full channel axis and for the
+    channel means; each call timed alone after an L2 flush (synthetic inputs)."""
+    import torch
+    L = H * W
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(7)
+    u = torch.randn(B, K, D, L, device=dev, generator=gen)
+    draw = 0.5 * torch.randn(B, K, D, L, device=dev, generator=gen)
+    Bs = torch.randn(B, K, N, L, device=dev, generator=gen)
+    Cs = torch.randn(B, K, N, L, device=dev, generator=gen)
+    A = -torch.arange(1, N + 1, device=dev, dtype=torch.float32).repeat(K * D, 1).contiguous()
+    bias = torch.full((K * D,), -3.0, device=dev)
+    dA = torch.empty(B, K, D, N, L, device=dev)
+    dBu = torch.empty_like(dA)
+    dAm = torch.empty(B, K, N, L, device=dev)
+    dBum = torch.empty_like(dAm)
+    y = torch.empty(B, K, D, L, device=dev)
+    yb = torch.empty(B, K, L, device=dev)
+    calls = {
+        "discretise": lambda: vmb.vmb_discretise_fwd(u, draw, A, Bs, bias, H, W, dA=dA, dBu=dBu),
+        "scan_only_full": lambda: vmb.vmb_scan_only_fwd(dA, dBu, Cs, H, W, y=y),
+        "discretise_mean": lambda: vmb.vmb_discretise_mean_fwd(u, draw, A, Bs, bias, H, W, dAm=dAm, dBum=dBum),
+        "scan_only_mean": lambda: vmb.vmb_scan_only_fwd(dAm, dBum, Cs, H, W, y=yb),
+    }
+    ops, res = B * K * D * N * L, {}
+    byt = {"discretise": 4 * (2 * ops + 2 * B * K * D * L + B * K * N * L),
+           "scan_only_full": 4 * (2 * ops + B * K * N * L + B * K * D * L),
+           "discretise_mean": 4 * (2 * B * K * D * L + 3 * B * K * N * L),
+           "scan_only_mean": 4 * (3 * B * K * N * L + B * K * L)}
+    for name, fn in calls.items():
+        for _ in range(warmup):
+            prelude()
+            fn()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for e0, e1 in evs:
+            prelude()
+            e0.record()
+            fn()
+            e1.record()
+        torch.cuda.synchronize()
+        us = 1e3 * statistics.median(e0.elapsed_time(e1) for e0, e1 in evs)
+        res[name] = {"us": us, "algorithmic_bytes": byt[name], "gbs": byt[name] / (us / 1e6) / 1e9}
+    res["shape"] = {"B": B, "K": K, "D": D, "N": N, "L": L}
+    res["scan_only_speedup_mean_over_full"] = res["scan_only_full"]["us"] / res["scan_only_mean"]["us"]
+    return res
+
+
 def run_ours(args, wl, rank, world, local_rank):
     import torch
     import paper_2412_16602_gb300 as vmb
@@ -366,11 +417,39 @@ def run_ours(args, wl, rank, world, local_rank):
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
 
+    # the materialised operands of the bench workload: 2 x B*4*D*N*L fp32
+    small_enough = 8 * wl.B * 4 * wl.D * wl.N * wl.L <= (32 << 30)
+    paper = None if args.no_paper_style else {
+        "bench_workload": (time_paper_style(vmb, wl.B, 4, wl.D, wl.N, wl.H, wl.W, dev, prelude, args.steps,
+                                            args.warmup) if small_enough else None),
+        # Table 1 / Table 2 "Base" row of the paper: inner dimension 512, L = 3136,
+        # batch 128, d_state 1 (the byte counts of Table 2 fix batch x N = 128)
+        "paper_table_base_512x3136": time_paper_style(vmb, 128, 4, 128, 1, 56, 56, dev, prelude,
+                                                      min(args.steps, 10), args.warmup),
+    }
     res = {"total_ms": total_ms, "step_ms": step_ms, "per_kernel": per_kernel, "e2e_ms": e2e_ms,
+           "paper_style": paper,
            "h2d": h2d, "d2h": d2h, "clocks": clk.summary(), "fused_ms": fused_ms,
            "launches_per_step": step.launches, "fused_launches": step.fused_launches}
     res["total_ms"], res["e2e_ms"] = max_over_ranks([total_ms, e2e_ms], world, dev)
     return res, inp
+
+
+# The paper's own scan-only kernel times on one RTX A6000 (Table 1, "Base"
+# rows; VMeanba about 0.02 ms in every row), for context next to the split
+# measured here.  Different hardware: not a target.
+PAPER_A6000_BASE_512x3136 = {"scan_only_full_ms": 5.86, "scan_only_mean_ms": 0.02, "speedup": 293}
+
+
+def paper_style_summary(ps, peak):
+    if ps is None:
+        return None
+    out = {}
+    for key, r in ps.items():
+        out[key] = {k: (dict(v, frac_of_peak=v["gbs"] / peak) if isinstance(v, dict) and "gbs" in v else v)
+                    for k, v in r.items()}
+    out["paper_a6000_base_512x3136"] = PAPER_A6000_BASE_512x3136
+    return out
 
 
 def main():
@@ -463,6 +542,7 @@ def main():
             "speedup_over_unfused": (per["mean_scan"]["us"] + per["cross_merge_mean"]["us"]) / fused_us,
             "speedup_over_full_path": (per["full_scan"]["us"] + per["cross_merge_full"]["us"]) / fused_us},
         "gpu_launches": res["launches_per_step"] * args.steps,
+        "paper_style": paper_style_summary(res["paper_style"], peak),
         "clocks": res["clocks"],
         "e2e": {"value": job_throughput(step_bytes, world, res["e2e_ms"] / args.e2e_steps), "unit": "GB/s",
                 "ms_per_step": res["e2e_ms"] / args.e2e_steps,

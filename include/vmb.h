@@ -154,6 +154,8 @@ vmb_status vmb_selective_scan_fwd(const void* u, const void* delta, const float*
  * Same arguments as vmb_selective_scan_fwd, plus
  *   ybar [B, K, L] fp32 device pointer, or NULL: optional copy of ybar.
  * The recurrence runs once per (b, k) instead of once per (b, k, d).
+ * Returns VMB_ERR_UNSUPPORTED when D * L >= 2^31 (the kernel addresses one
+ * (b, k) slab with 32-bit offsets).
  */
 vmb_status vmb_mean_scan_fwd(const void* u, const void* delta, const float* A, const void* Bs,
                              const void* Cs, const float* Dskip, const float* delta_bias, void* y,
@@ -212,6 +214,46 @@ vmb_status vmb_selective_scan_fwd_noalloc(const void* u, const void* delta, cons
                                           const float* delta_bias, void* y, int B, int K, int D,
                                           int N, int H, int W, unsigned flags, vmb_dtype dtype,
                                           cudaStream_t stream);
+
+/*
+ * The paper's own kernel setting (Sec. 4, "Kernel Implementation"): the
+ * discretisation runs outside the scan kernel, which reads the materialised
+ * operands Abar and Bbar u.  These three calls reproduce that split, for
+ * measuring it next to the fused scans above; they are not needed to compute
+ * the SS2D output.  Operands are fp32; their sizes grow with N (a B=1 VMamba-T
+ * stage-1 map with N = 16 materialises 2 x 154 MB).
+ *
+ * vmb_discretise_fwd - Eqs. 4 and 6 for every (b, k, d, n, l):
+ *   delta = softplus(delta_raw + delta_bias[c]) (or raw + bias without
+ *   VMB_FLAG_SOFTPLUS), dA[b,k,d,n,l] = exp(delta A[c,n]),
+ *   dBu[b,k,d,n,l] = delta B[b,k,n,l] u[b,k,d,l] (Euler) or
+ *   (exp(delta A) - 1) / A B u under VMB_FLAG_B_ZOH.
+ *   u, delta [B,K,D,L], Bs [B,K,N,L] in dtype; A [K*D,N], delta_bias [K*D] fp32;
+ *   dA, dBu [B,K,D,N,L] fp32 out.  flags: VMB_FLAG_SOFTPLUS | VMB_FLAG_B_ZOH.
+ *   N in 1..16 (VMB_ERR_UNSUPPORTED above).
+ *
+ * vmb_discretise_mean_fwd - Eq. 9's T applied to the discretised operands:
+ *   dAm[b,k,n,l] = mean_d exp(delta_d A[c_d,n]),
+ *   dBum[b,k,n,l] = mean_d Bbar[b,k,d,n,l] u[b,k,d,l], fp32 [B,K,N,L] out (the
+ *   [B,K,1,N,L] operands of the scan kernel).  Same inputs and flags as above.
+ *
+ * vmb_scan_only_fwd - Eq. 3 without the skip term on materialised operands of
+ *   Dm channels per (b, k) (Dm = D for the full path, 1 after the mean):
+ *   h[n] = dA h[n] + dBu from h = 0, y[b,k,d,l] = sum_n Cs[b,k,n,l] h[n].
+ *   dA, dBu [B,K,Dm,N,L] fp32, Cs [B,K,N,L] in dtype, y [B,K,Dm,L] fp32 out.
+ *   Deterministic; no workspace.  N in 1..16.
+ */
+vmb_status vmb_discretise_fwd(const void* u, const void* delta, const float* A, const void* Bs,
+                              const float* delta_bias, float* dA, float* dBu, int B, int K, int D,
+                              int N, int H, int W, unsigned flags, vmb_dtype dtype,
+                              cudaStream_t stream);
+vmb_status vmb_discretise_mean_fwd(const void* u, const void* delta, const float* A, const void* Bs,
+                                   const float* delta_bias, float* dAm, float* dBum, int B, int K,
+                                   int D, int N, int H, int W, unsigned flags, vmb_dtype dtype,
+                                   cudaStream_t stream);
+vmb_status vmb_scan_only_fwd(const float* dA, const float* dBu, const void* Cs, float* y, int B,
+                             int K, int Dm, int N, int H, int W, vmb_dtype dtype,
+                             cudaStream_t stream);
 
 /*
  * vmb_read_status - synchronise `stream`, then return and clear the device

@@ -87,6 +87,29 @@ vmb_status check_scan(const ScanArgs& a, bool mean, bool* empty) {
     return VMB_OK;
 }
 
+// Checks of the discretisation calls; sets a.L.
+vmb_status check_disc(DiscArgs& a, int H, int W, bool mean, bool* empty) {
+    if (!dtype_ok(a.dtype) || a.B < 0 || a.K < 0 || a.D < 0 || a.N < 0 || H < 0 || W < 0) return VMB_ERR_INVALID_ARG;
+    if (a.flags & ~(VMB_FLAG_SOFTPLUS | VMB_FLAG_B_ZOH)) return VMB_ERR_INVALID_ARG;
+    long long n = 0, nop = 0;
+    if (!count(&n, {a.B, a.K, a.D, H, W}) || !count(&nop, {a.B, a.K, mean ? 1 : a.D, a.N > 0 ? a.N : 1, H, W}))
+        return VMB_ERR_INVALID_ARG;
+    *empty = n == 0;
+    if (*empty) return VMB_OK;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    a.L = H * W;
+    if (a.N < 1) return VMB_ERR_INVALID_ARG;
+    if (a.N > 16) return VMB_ERR_UNSUPPORTED;
+    long long rows = 0;
+    if (!count(&rows, {a.B, a.K, a.D}) || rows > INT_MAX / 2) return VMB_ERR_UNSUPPORTED;
+    if (!a.u || !a.delta || !a.A || !a.Bs || !a.bias || !a.dA || !a.dBu) return VMB_ERR_INVALID_ARG;
+    const size_t es = esize(a.dtype);
+    if (!aligned(a.u, es) || !aligned(a.delta, es) || !aligned(a.Bs, es) || !aligned(a.A, 4) || !aligned(a.bias, 4) ||
+        !aligned(a.dA, 4) || !aligned(a.dBu, 4))
+        return VMB_ERR_MISALIGNED;
+    return VMB_OK;
+}
+
 vmb_status run_scan(ScanArgs& a, bool mean, cudaStream_t stream) {
     bool empty = false;
     vmb_status s = check_scan(a, mean, &empty);
@@ -199,6 +222,41 @@ vmb_status vmb_mean_scan_merge_fwd(const void* u, const void* delta, const float
     s = run_scan(a, true, stream);
     if (s != VMB_OK) return s;
     return launch_mean_merge(x, ybar, Dskip, out, B, D, H, W, (flags & VMB_FLAG_SKIP_MEAN) == 0, dtype, stream);
+}
+
+vmb_status vmb_discretise_fwd(const void* u, const void* delta, const float* A, const void* Bs,
+                              const float* delta_bias, float* dA, float* dBu, int B, int K, int D, int N, int H,
+                              int W, unsigned flags, vmb_dtype dtype, cudaStream_t stream) {
+    DiscArgs a{u, delta, A, Bs, delta_bias, dA, dBu, B, K, D, N, 0, flags, dtype};
+    bool empty = false;
+    vmb_status s = check_disc(a, H, W, false, &empty);
+    if (s != VMB_OK || empty) return s;
+    return launch_discretise(a, false, stream);
+}
+
+vmb_status vmb_discretise_mean_fwd(const void* u, const void* delta, const float* A, const void* Bs,
+                                   const float* delta_bias, float* dAm, float* dBum, int B, int K, int D, int N,
+                                   int H, int W, unsigned flags, vmb_dtype dtype, cudaStream_t stream) {
+    DiscArgs a{u, delta, A, Bs, delta_bias, dAm, dBum, B, K, D, N, 0, flags, dtype};
+    bool empty = false;
+    vmb_status s = check_disc(a, H, W, true, &empty);
+    if (s != VMB_OK || empty) return s;
+    return launch_discretise(a, true, stream);
+}
+
+vmb_status vmb_scan_only_fwd(const float* dA, const float* dBu, const void* Cs, float* y, int B, int K, int Dm,
+                             int N, int H, int W, vmb_dtype dtype, cudaStream_t stream) {
+    if (!dtype_ok(dtype) || B < 0 || K < 0 || Dm < 0 || N < 0 || H < 0 || W < 0) return VMB_ERR_INVALID_ARG;
+    long long n = 0, nop = 0;
+    if (!count(&n, {B, K, Dm, H, W}) || !count(&nop, {B, K, Dm, N > 0 ? N : 1, H, W})) return VMB_ERR_INVALID_ARG;
+    if (n == 0) return VMB_OK;
+    if ((long long)H * W > INT_MAX - 1024) return VMB_ERR_UNSUPPORTED;  // segment offsets stay in int
+    if (N < 1) return VMB_ERR_INVALID_ARG;
+    if (N > 16) return VMB_ERR_UNSUPPORTED;
+    if (!dA || !dBu || !Cs || !y) return VMB_ERR_INVALID_ARG;
+    if (!aligned(dA, 4) || !aligned(dBu, 4) || !aligned(y, 4) || !aligned(Cs, esize(dtype))) return VMB_ERR_MISALIGNED;
+    OnlyArgs a{dA, dBu, Cs, y, B, K, Dm, N, H * W, dtype};
+    return launch_scan_only(a, stream);
 }
 
 vmb_status vmb_read_status(void* workspace, cudaStream_t stream) {

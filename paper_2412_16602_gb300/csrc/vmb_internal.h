@@ -63,6 +63,29 @@ inline WsLayout ws_layout(const ScanPlan& p) {
     return w;
 }
 
+// The paper's scan-only setting (Sec. 4): discretisation into materialised
+// fp32 operands, then the scan alone.
+struct DiscArgs {
+    const void* u;
+    const void* delta;
+    const float* A;
+    const void* Bs;
+    const float* bias;
+    float* dA;   // [B][K][D][N][L], or [B][K][N][L] for the channel means
+    float* dBu;  // same shape as dA
+    int B, K, D, N, L;
+    unsigned flags;
+    vmb_dtype dtype;
+};
+struct OnlyArgs {
+    const float* dA;   // [B][K][Dm][N][L]
+    const float* dBu;  // [B][K][Dm][N][L]
+    const void* Cs;    // [B][K][N][L], dtype
+    float* y;          // [B][K][Dm][L]
+    int B, K, Dm, N, L;
+    vmb_dtype dtype;
+};
+
 int device_sm_count();
 
 vmb_status plan_full(const ScanArgs& a, ScanPlan* plan);
@@ -74,6 +97,8 @@ vmb_status launch_cross_scan(const void* x, void* xs, int B, int D, int H, int W
                              cudaStream_t stream);
 vmb_status launch_cross_merge(const void* ys, void* out, int B, int D, int H, int W, vmb_dtype dt,
                               cudaStream_t stream);
+vmb_status launch_discretise(const DiscArgs& a, bool mean, cudaStream_t stream);
+vmb_status launch_scan_only(const OnlyArgs& a, cudaStream_t stream);
 vmb_status launch_mean_merge(const void* x, const float* ybar, const float* Dskip, void* out, int B, int D, int H,
                              int W, bool per_channel_skip, vmb_dtype dt, cudaStream_t stream);
 

@@ -39,7 +39,8 @@ VMB_PATH_MEAN = 1
 
 EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb_scan_kernel_count",
            "vmb_selective_scan_fwd",
-           "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_read_status", "vmb_status_string", "vmb_version"]
+           "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_discretise_fwd", "vmb_discretise_mean_fwd",
+           "vmb_scan_only_fwd", "vmb_read_status", "vmb_status_string", "vmb_version"]
 
 
 class VmbError(RuntimeError):
@@ -62,12 +63,16 @@ def _load() -> ctypes.CDLL:
     lib.vmb_selective_scan_fwd.argtypes = [vp] * 8 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_fwd.argtypes = [vp] * 9 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_merge_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
+    lib.vmb_discretise_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
+    lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
+    lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
     lib.vmb_read_status.argtypes = [vp, vp]
     lib.vmb_status_string.argtypes = [i]
     lib.vmb_status_string.restype = ctypes.c_char_p
     lib.vmb_version.argtypes = []
     for name in ["vmb_cross_scan", "vmb_cross_merge", "vmb_selective_scan_fwd", "vmb_mean_scan_fwd",
-                 "vmb_mean_scan_merge_fwd", "vmb_read_status", "vmb_version"]:
+                 "vmb_mean_scan_merge_fwd", "vmb_discretise_fwd", "vmb_discretise_mean_fwd", "vmb_scan_only_fwd",
+                 "vmb_read_status", "vmb_version"]:
         getattr(lib, name).restype = i
     return lib
 
@@ -282,6 +287,81 @@ def vmb_mean_scan_merge_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, x, H: int, W
                                        _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
                                        _stream(stream)), "vmb_mean_scan_merge_fwd")
     return out, ybar
+
+
+# ------------------------------------------- the paper's scan-only kernel setting
+
+
+def _disc_shapes(u, delta, A, Bs, delta_bias, H, W):
+    for t, n in [(u, "u"), (delta, "delta"), (A, "A"), (Bs, "Bs"), (delta_bias, "delta_bias")]:
+        _dev(t, n)
+    B, K, D, L = u.shape
+    N = Bs.shape[2]
+    if L != H * W or delta.shape != u.shape or Bs.shape != (B, K, N, L):
+        raise ValueError("u, delta [B,K,D,H*W] and Bs [B,K,N,H*W] expected")
+    if len({u.dtype, delta.dtype, Bs.dtype}) != 1:
+        raise ValueError("u, delta, Bs must share one dtype")
+    if A.shape != (K * D, N) or delta_bias.shape != (K * D,) or A.dtype != torch.float32 \
+            or delta_bias.dtype != torch.float32:
+        raise ValueError("A [K*D, N], delta_bias [K*D] float32 expected")
+    return B, K, D, N, L
+
+
+def vmb_discretise_fwd(u, delta, A, Bs, delta_bias, H: int, W: int, *, dA=None, dBu=None,
+                       flags: int = VMB_FLAG_SOFTPLUS, stream=None):
+    """Eqs. 4, 6 outside the scan: (dA, dBu), each float32 [B, K, D, N, H*W]."""
+    B, K, D, N, L = _disc_shapes(u, delta, A, Bs, delta_bias, H, W)
+    shape = (B, K, D, N, L)
+    dA = torch.empty(shape, dtype=torch.float32, device=u.device) if dA is None else dA
+    dBu = torch.empty(shape, dtype=torch.float32, device=u.device) if dBu is None else dBu
+    for t, n in [(dA, "dA"), (dBu, "dBu")]:
+        _dev(t, n)
+        if t.shape != shape or t.dtype != torch.float32:
+            raise ValueError(f"{n} must be float32 {shape}")
+    _check(lib.vmb_discretise_fwd(_ptr(u), _ptr(delta), _ptr(A), _ptr(Bs), _ptr(delta_bias), _ptr(dA), _ptr(dBu),
+                                  B, K, D, N, H, W, flags, _dtype_code(u.dtype), _stream(stream)),
+           "vmb_discretise_fwd")
+    return dA, dBu
+
+
+def vmb_discretise_mean_fwd(u, delta, A, Bs, delta_bias, H: int, W: int, *, dAm=None, dBum=None,
+                            flags: int = VMB_FLAG_SOFTPLUS, stream=None):
+    """Channel means of the discretised operands (Eq. 9's T): (dAm, dBum), float32 [B, K, N, H*W]."""
+    B, K, D, N, L = _disc_shapes(u, delta, A, Bs, delta_bias, H, W)
+    shape = (B, K, N, L)
+    dAm = torch.empty(shape, dtype=torch.float32, device=u.device) if dAm is None else dAm
+    dBum = torch.empty(shape, dtype=torch.float32, device=u.device) if dBum is None else dBum
+    for t, n in [(dAm, "dAm"), (dBum, "dBum")]:
+        _dev(t, n)
+        if t.shape != shape or t.dtype != torch.float32:
+            raise ValueError(f"{n} must be float32 {shape}")
+    _check(lib.vmb_discretise_mean_fwd(_ptr(u), _ptr(delta), _ptr(A), _ptr(Bs), _ptr(delta_bias), _ptr(dAm),
+                                       _ptr(dBum), B, K, D, N, H, W, flags, _dtype_code(u.dtype), _stream(stream)),
+           "vmb_discretise_mean_fwd")
+    return dAm, dBum
+
+
+def vmb_scan_only_fwd(dA, dBu, Cs, H: int, W: int, *, y=None, stream=None):
+    """The scan alone (Eq. 3 without the skip): dA, dBu float32 [B, K, Dm, N, L] (or
+    [B, K, N, L] for one channel), Cs [B, K, N, L] -> y float32 [B, K, Dm, L] (or [B, K, L])."""
+    for t, n in [(dA, "dA"), (dBu, "dBu"), (Cs, "Cs")]:
+        _dev(t, n)
+    one = dA.dim() == 4
+    B, K = dA.shape[:2]
+    Dm = 1 if one else dA.shape[2]
+    N, L = dA.shape[-2:]
+    if L != H * W or dBu.shape != dA.shape or Cs.shape != (B, K, N, L):
+        raise ValueError("dA, dBu [B,K,Dm,N,H*W] and Cs [B,K,N,H*W] expected")
+    if dA.dtype != torch.float32 or dBu.dtype != torch.float32:
+        raise ValueError("dA, dBu must be float32")
+    shape = (B, K, L) if one else (B, K, Dm, L)
+    y = torch.empty(shape, dtype=torch.float32, device=dA.device) if y is None else y
+    _dev(y, "y")
+    if tuple(y.shape) != shape or y.dtype != torch.float32:
+        raise ValueError(f"y must be float32 {shape}")
+    _check(lib.vmb_scan_only_fwd(_ptr(dA), _ptr(dBu), _ptr(Cs), _ptr(y), B, K, Dm, N, H, W, _dtype_code(Cs.dtype),
+                                 _stream(stream)), "vmb_scan_only_fwd")
+    return y
 
 
 def vmb_read_status(workspace=None, device=None, stream=None) -> int:

@@ -25,6 +25,9 @@ def lib():
     lib.vmb_selective_scan_fwd.argtypes = [vp] * 8 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_fwd.argtypes = [vp] * 9 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_merge_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
+    lib.vmb_discretise_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
+    lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
+    lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
     lib.vmb_status_string.argtypes = [i]
     lib.vmb_status_string.restype = ctypes.c_char_p
     lib.vmb_read_status.argtypes = [vp, vp]
@@ -132,3 +135,34 @@ def test_mean_scan_merge_validation(lib):
     assert merge_call(lib, flags=0x100) == 1
     assert merge_call(lib, ws=0) == 4
     assert merge_call(lib, ptrs=[0] * 10, B=0, ws=0) == 0                      # empty problem
+
+
+def disc_call(fn, *, ptrs=None, B=1, K=4, D=8, N=16, H=4, W=4, flags=1, dtype=0):
+    p = [FAKE] * 7 if ptrs is None else ptrs
+    return fn(*p, B, K, D, N, H, W, flags, dtype, S)
+
+
+@pytest.mark.parametrize("mean", [False, True])
+def test_discretise_validation(lib, mean):
+    fn = lib.vmb_discretise_mean_fwd if mean else lib.vmb_discretise_fwd
+    assert disc_call(fn, B=-1) == 1
+    assert disc_call(fn, N=0) == 1
+    assert disc_call(fn, N=17) == 3
+    assert disc_call(fn, flags=0x4) == 1                                 # skip-mode flag: not a discretisation flag
+    assert disc_call(fn, dtype=3) == 1
+    assert disc_call(fn, ptrs=[FAKE] * 6 + [0]) == 1                     # null output
+    assert disc_call(fn, ptrs=[FAKE] * 5 + [FAKE + 2, FAKE]) == 2        # misaligned fp32 output
+    assert disc_call(fn, ptrs=[FAKE + 2] + [FAKE] * 6, dtype=1) != 2     # bf16 input: 2-byte aligned is fine
+    assert disc_call(fn, ptrs=[0] * 7, W=0) == 0                         # empty problem
+
+
+def test_scan_only_validation(lib):
+    f = lib.vmb_scan_only_fwd
+    assert f(FAKE, FAKE, FAKE, FAKE, -1, 4, 8, 16, 4, 4, 0, S) == 1
+    assert f(FAKE, FAKE, FAKE, FAKE, 1, 4, 8, 0, 4, 4, 0, S) == 1
+    assert f(FAKE, FAKE, FAKE, FAKE, 1, 4, 8, 17, 4, 4, 0, S) == 3
+    assert f(FAKE, FAKE, FAKE, 0, 1, 4, 8, 16, 4, 4, 0, S) == 1          # null y
+    assert f(FAKE, FAKE + 2, FAKE, FAKE, 1, 4, 8, 16, 4, 4, 0, S) == 2   # misaligned dBu
+    assert f(FAKE, FAKE, FAKE + 1, FAKE, 1, 4, 8, 16, 4, 4, 1, S) == 2   # misaligned bf16 C
+    assert f(FAKE, FAKE, FAKE, FAKE, 1, 4, 8, 16, 4, 4, 9, S) == 1       # bad dtype
+    assert f(0, 0, 0, 0, 1, 4, 0, 16, 4, 4, 0, S) == 0                   # empty problem
