@@ -86,6 +86,8 @@ class Oracle:
         lib.oracle_discretise_mean.restype = None
         lib.oracle_scan_only.argtypes = [P] * 4 + [lg] * 5
         lib.oracle_scan_only.restype = None
+        lib.oracle_mean_scan_grouped.argtypes = [P] * 9 + [lg] * 6 + [i, i, i]
+        lib.oracle_mean_scan_grouped.restype = i
         self.lib = lib
         self.path = lib_path
 
@@ -148,6 +150,19 @@ class Oracle:
                                        nthreads or default_threads())
         if rc:
             raise RuntimeError("oracle_mean_scan failed")
+        return y, ybar
+
+    def mean_scan_grouped(self, u, delta, A, Bs, Cs, Dskip, bias, groups: int, *, softplus_on=True,
+                          b_mode=B_EULER, skip_mode=SKIP_PER_CHANNEL):
+        """Grouped basis (reduced channel dimension d = groups): the mean of Eq. 9 over each of
+        `groups` consecutive channel groups; returns (y [B, K, D, L], ybar [B, K, groups, L])."""
+        arrs, (B, K, D, N, L) = self._scan_args(u, delta, A, Bs, Cs, Dskip, bias)
+        y = np.empty((B, K, D, L), dtype=np.float64)
+        ybar = np.empty((B, K, groups, L), dtype=np.float64)
+        rc = self.lib.oracle_mean_scan_grouped(*(_ptr(a) for a in arrs), _ptr(y), _ptr(ybar), B, K, D, N, L,
+                                               int(groups), int(bool(softplus_on)), int(b_mode), int(skip_mode))
+        if rc:
+            raise ValueError("groups must divide D")
         return y, ybar
 
     def _disc_args(self, u, delta, A, Bs, bias):
@@ -239,6 +254,10 @@ def selective_scan(*a, **kw):
 
 def mean_scan(*a, **kw):
     return get().mean_scan(*a, **kw)
+
+
+def mean_scan_grouped(*a, **kw):
+    return get().mean_scan_grouped(*a, **kw)
 
 
 def discretise(*a, **kw):

@@ -14,6 +14,8 @@
  *   recurrence ..................... App. A, Eq. 3 (h_t = Abar h_{t-1} + Bbar u_t, y_t = C h_t + D u_t)
  *   channel mean (VMeanba) ......... Sec. 2.2, Eq. 9 (y = T^-1(Mamba(T(Abar, Bbar u, C))),
  *                                     T = mean over the inner channel axis, T^-1 = broadcast)
+ *   grouped basis (d > 1) .......... Sec. 2.1 I_basis, Eq. 8 (reduced channel dimension d; the
+ *                                     mean over each of d channel groups)
  *   scan-only kernel setting ....... Sec. 4, "Kernel Implementation" (discretisation done
  *                                     before the scan; the scan reads materialised Abar,
  *                                     Bbar u with D channels, or one channel after T)
@@ -250,6 +252,61 @@ int oracle_mean_scan(const double* u, const double* delta, const double* A, cons
     problem p = {u, delta, A, Bs, Cs, Dskip, bias, y, ybar, B, K, D, N, L, softplus_on, b_mode,
                  skip_mode};
     return run(&p, 1, nthreads);
+}
+
+/* --------------------------------------- grouped basis (d > 1 reduced channels) */
+
+/* Sec. 2.1 / App. B: I_basis has a reduced channel dimension d (Eq. 8 counts
+ * 9BLd FLOPs for it); VMeanba is d = 1.  With d = G > 1 the D channels of a
+ * direction are split into G consecutive groups of D/G channels and T is the
+ * mean over each group: one recurrence per (b, k, g), broadcast back to the
+ * group's channels.  ybar is [B][K][G][L]; skip_mode as in the mean scan, over
+ * the group. */
+int oracle_mean_scan_grouped(const double* u, const double* delta, const double* A, const double* Bs,
+                             const double* Cs, const double* Dskip, const double* bias, double* y,
+                             double* ybar, long B, long K, long D, long N, long L, long G, int softplus_on,
+                             int b_mode, int skip_mode) {
+    if (G < 1 || D % G != 0) return 1;
+    long Dg = D / G;
+    double* h = (double*)malloc(sizeof(double) * 3 * (size_t)(N > 0 ? N : 1));
+    if (!h) return 1;
+    double *abar = h + N, *bubar = h + 2 * N;
+    for (long b = 0; b < B; ++b)
+        for (long k = 0; k < K; ++k) {
+            const double* Bk = Bs + (b * K + k) * N * L;
+            const double* Ck = Cs + (b * K + k) * N * L;
+            for (long g = 0; g < G; ++g) {
+                long d0 = g * Dg;
+                for (long n = 0; n < N; ++n) h[n] = 0.0;
+                for (long t = 0; t < L; ++t) {
+                    double du_sum = 0.0;
+                    for (long n = 0; n < N; ++n) { abar[n] = 0.0; bubar[n] = 0.0; }
+                    for (long d = d0; d < d0 + Dg; ++d) {
+                        long c = k * D + d, row = (b * K + k) * D + d;
+                        double v = delta[row * L + t] + bias[c];
+                        double dlt = softplus_on ? softplus(v) : v;
+                        for (long n = 0; n < N; ++n) {
+                            abar[n] += exp(dlt * A[c * N + n]);
+                            bubar[n] += discretise_b(dlt, A[c * N + n], Bk[n * L + t], b_mode) * u[row * L + t];
+                        }
+                        du_sum += Dskip[c] * u[row * L + t];
+                    }
+                    double yb = 0.0;
+                    for (long n = 0; n < N; ++n) {
+                        h[n] = abar[n] / (double)Dg * h[n] + bubar[n] / (double)Dg;
+                        yb += Ck[n * L + t] * h[n];
+                    }
+                    ybar[((b * K + k) * G + g) * L + t] = yb;
+                    for (long d = d0; d < d0 + Dg; ++d) {
+                        long c = k * D + d, row = (b * K + k) * D + d;
+                        y[row * L + t] = yb + (skip_mode == ORACLE_SKIP_MEAN ? du_sum / (double)Dg
+                                                                           : Dskip[c] * u[row * L + t]);
+                    }
+                }
+            }
+        }
+    free(h);
+    return 0;
 }
 
 /* ------------------------------------- the paper's scan-only kernel setting */

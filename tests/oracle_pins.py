@@ -372,6 +372,39 @@ def pin_mean_skip_mean_mode(orc):
            what="skip mean")
 
 
+# ------------------------------------------------- grouped basis (d > 1 groups)
+
+
+def pin_grouped_reduces_to_mean_and_full(orc):
+    """One group is the channel mean of Eq. 9; D groups of one channel each leave
+    the scan unchanged (the mean of one channel is itself)."""
+    rng = np.random.default_rng(40)
+    args = _rand_problem(rng, B=2, K=2, D=6, N=3, L=9, draw_scale=1.5)
+    y1, yb1 = orc.mean_scan_grouped(*args, 1)
+    ym, ybm = orc.mean_scan(*args)
+    _close(y1, ym, rtol=1e-12, atol=1e-13, what="G=1 y")
+    _close(yb1[:, :, 0], ybm, rtol=1e-12, atol=1e-13, what="G=1 ybar")
+    yD, _ = orc.mean_scan_grouped(*args, 6)
+    _close(yD, orc.selective_scan(*args), rtol=1e-11, atol=1e-12, what="G=D")
+
+
+def pin_grouped_brute_force(orc):
+    """Each group's ybar is the brute-force unrolling of the averaged system of
+    that group's channels alone; y = ybar of the channel's group + D_c u."""
+    rng = np.random.default_rng(41)
+    u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, B=1, K=2, D=6, N=3, L=7, draw_scale=1.5)
+    K, D, G = 2, 6, 3
+    Dg = D // G
+    y, yb = orc.mean_scan_grouped(u, draw, A, Bs, Cs, Dskip, bias, G)
+    for g in range(G):
+        sl = slice(g * Dg, (g + 1) * Dg)
+        sub = (u[:, :, sl], draw[:, :, sl], A.reshape(K, D, -1)[:, sl].reshape(K * Dg, -1), Bs, Cs,
+               Dskip.reshape(K, D)[:, sl].reshape(-1), bias.reshape(K, D)[:, sl].reshape(-1))
+        _close(yb[:, :, g], brute_force_mean(*sub), rtol=1e-11, atol=1e-12, what=f"group {g} ybar")
+        skip = Dskip.reshape(K, D)[None, :, sl, None] * u[:, :, sl]
+        _close(y[:, :, sl], yb[:, :, g][:, :, None, :] + skip, rtol=1e-12, atol=1e-13, what=f"group {g} y")
+
+
 # -------------------------------------- scan-only setting (discretise, then scan)
 
 

@@ -40,6 +40,9 @@ MUTANTS = {
                                "dAm[((b * K + k) * N + n) * L + l] = sa;"),
     "disc_mean_bias_wrong_channel": ("double v = delta[row * L + l] + bias[c];\n                        double dlt = softplus_on ? softplus(v) : v;\n                        double a = A[c * N + n];\n                        sa",
                                      "double v = delta[row * L + l] + bias[k];\n                        double dlt = softplus_on ? softplus(v) : v;\n                        double a = A[c * N + n];\n                        sa"),
+    "grouped_divides_by_D": ("h[n] = abar[n] / (double)Dg * h[n] + bubar[n] / (double)Dg;",
+                             "h[n] = abar[n] / (double)D * h[n] + bubar[n] / (double)Dg;"),
+    "grouped_first_group_only": ("long d0 = g * Dg;", "long d0 = 0;"),
     "scan_only_drops_decay": ("h[n] = dA[(row * N + n) * L + l] * h[n] + dBu[(row * N + n) * L + l];",
                               "h[n] = h[n] + dBu[(row * N + n) * L + l];"),
     "scan_only_output_before_update": ("h[n] = dA[(row * N + n) * L + l] * h[n] + dBu[(row * N + n) * L + l];\n                        acc += Cs[((b * K + k) * N + n) * L + l] * h[n];",
