@@ -417,6 +417,31 @@ def run_ours(args, wl, rank, world, local_rank):
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
 
+    # the grouped basis (d channel groups, each its own mean and recurrence) on the step's inputs
+    grouped = {}
+    for G in (4, 16):
+        if wl.D % G:
+            continue
+        wsg = torch.zeros(vmb.vmb_scan_workspace_bytes(1, wl.B, 4 * G, wl.D // G, wl.N, wl.H, wl.W, tdt),
+                          dtype=torch.uint8, device=dev)
+        yg = torch.empty_like(outs["ym"])
+
+        def fn():
+            vmb.vmb_mean_scan_grouped_fwd(outs["xs"], g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"],
+                                          wl.H, wl.W, G, y=yg, workspace=wsg, stream=stream)
+        for _ in range(args.warmup):
+            prelude()
+            fn()
+        gev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        for e0, e1 in gev:
+            prelude()
+            e0.record()
+            fn()
+            e1.record()
+        torch.cuda.synchronize()
+        if vmb.vmb_read_status(wsg) != 0:
+            raise RuntimeError("device error word set in the grouped mean scan")
+        grouped[G] = 1e3 * statistics.mean(e0.elapsed_time(e1) for e0, e1 in gev)
     # the materialised operands of the bench workload: 2 x B*4*D*N*L fp32
     small_enough = 8 * wl.B * 4 * wl.D * wl.N * wl.L <= (32 << 30)
     paper = None if args.no_paper_style else {
@@ -428,7 +453,7 @@ def run_ours(args, wl, rank, world, local_rank):
                                                       min(args.steps, 10), args.warmup),
     }
     res = {"total_ms": total_ms, "step_ms": step_ms, "per_kernel": per_kernel, "e2e_ms": e2e_ms,
-           "paper_style": paper,
+           "paper_style": paper, "grouped_us": grouped,
            "h2d": h2d, "d2h": d2h, "clocks": clk.summary(), "fused_ms": fused_ms,
            "launches_per_step": step.launches, "fused_launches": step.fused_launches}
     res["total_ms"], res["e2e_ms"] = max_over_ranks([total_ms, e2e_ms], world, dev)
@@ -543,6 +568,11 @@ def main():
             "speedup_over_full_path": (per["full_scan"]["us"] + per["cross_merge_full"]["us"]) / fused_us},
         "gpu_launches": res["launches_per_step"] * args.steps,
         "paper_style": paper_style_summary(res["paper_style"], peak),
+        # grouped basis: d channel groups per direction, each its own channel mean
+        # and recurrence (same algorithmic bytes as the mean scan)
+        "mean_grouped": {str(G): {"groups": G, "us": us, "gbs": kb["mean_scan"] / (us / 1e6) / 1e9,
+                                  "frac_of_peak": kb["mean_scan"] / (us / 1e6) / 1e9 / peak}
+                         for G, us in res["grouped_us"].items()},
         "clocks": res["clocks"],
         "e2e": {"value": job_throughput(step_bytes, world, res["e2e_ms"] / args.e2e_steps), "unit": "GB/s",
                 "ms_per_step": res["e2e_ms"] / args.e2e_steps,

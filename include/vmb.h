@@ -164,6 +164,28 @@ vmb_status vmb_mean_scan_fwd(const void* u, const void* delta, const float* A, c
                              cudaStream_t stream);
 
 /*
+ * vmb_mean_scan_grouped_fwd - grouped basis: the reduced input set I_basis of
+ * Sec. 2.1 with a reduced channel dimension d = groups instead of VMeanba's
+ * d = 1 (Eq. 8 counts 9BLd FLOPs for it).  The D channels of each direction
+ * are split into `groups` consecutive groups of D/groups channels; T is the
+ * mean over each group and T^-1 broadcasts each group's ybar to its channels:
+ *   ybar[b,k,g,t] as in vmb_mean_scan_fwd over channels g*D/G .. (g+1)*D/G - 1,
+ *   y[b,k,d,t] = ybar[b,k,d/(D/G),t] + Dskip[c] u[b,k,d,t] (VMB_FLAG_SKIP_MEAN:
+ *   the mean of Dskip u over the group).
+ * Same arguments as vmb_mean_scan_fwd plus `groups` (>= 1, divides D;
+ * VMB_ERR_INVALID_ARG otherwise); ybar, if not NULL, is [B, K, groups, L]
+ * fp32.  groups = 1 is vmb_mean_scan_fwd; groups = D gives the full scan's y.
+ * workspace: >= vmb_scan_workspace_bytes(VMB_PATH_MEAN, B, K*groups,
+ * D/groups, N, H, W, dtype) bytes (the grouped problem runs as K*groups
+ * directions of D/groups channels).
+ */
+vmb_status vmb_mean_scan_grouped_fwd(const void* u, const void* delta, const float* A, const void* Bs,
+                                     const void* Cs, const float* Dskip, const float* delta_bias,
+                                     void* y, float* ybar, int B, int K, int D, int N, int H, int W,
+                                     int groups, unsigned flags, vmb_dtype dtype, void* workspace,
+                                     size_t workspace_bytes, cudaStream_t stream);
+
+/*
  * vmb_mean_scan_merge_fwd - the channel-mean path of an SS2D block (Sec. 2.2,
  * Eq. 9, then the App. A cross-merge) with the broadcast T^-1 fused into the
  * merge, so the per-channel output y [B, 4, D, L] is never written:

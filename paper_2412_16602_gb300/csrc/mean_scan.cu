@@ -56,6 +56,7 @@ struct MeanParams {
     int tabvec;  // A, delta_bias, Dskip 16-byte aligned: async-copied
     int no_bcast;  // fused with the cross-merge: no y; ybar (+ the broadcast skip term) only
     int cvec;      // u / y rows allow 4-step vector access (L % 4 == 0, 4-element aligned)
+    int bc_group;  // sequences per B / C row block: 1, or G for the grouped basis (K, D are K*G, D/G)
     WsHeader* hdr;
     unsigned* flags;
     float* aggP;
@@ -219,7 +220,7 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
     const int l0 = chunk * p.chunk_len;
     const int nvalid = min(TC, L - l0);
     const size_t urow0 = (size_t)seq * D;   // first row of u/delta/y for (b, k)
-    const size_t bcrow0 = (size_t)seq * N;  // first row of Bs/Cs
+    const size_t bcrow0 = (size_t)(seq / p.bc_group) * N;  // first row of Bs/Cs
     const T* u = static_cast<const T*>(p.u);
     const T* dlr = static_cast<const T*>(p.dl);
 
@@ -756,6 +757,7 @@ vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     const auto al4e = [&](const void* q) { return (reinterpret_cast<uintptr_t>(q) % (4 * es)) == 0; };
     p.cvec = (a.L % 4 == 0) && al4e(a.u) && (a.y == nullptr || al4e(a.y));
     p.no_bcast = a.no_bcast ? 1 : 0;
+    p.bc_group = a.bc_group;
     p.tabvec = al16(a.A) && al16(a.bias) && al16(a.Dskip);
     const WsLayout w = ws_layout(plan);
     unsigned char* ws = static_cast<unsigned char*>(a.ws);

@@ -208,6 +208,24 @@ vmb_status vmb_mean_scan_fwd(const void* u, const void* delta, const float* A, c
     return run_scan(a, true, stream);
 }
 
+vmb_status vmb_mean_scan_grouped_fwd(const void* u, const void* delta, const float* A, const void* Bs, const void* Cs,
+                                     const float* Dskip, const float* delta_bias, void* y, float* ybar, int B, int K,
+                                     int D, int N, int H, int W, int groups, unsigned flags, vmb_dtype dtype,
+                                     void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+    if (H < 0 || W < 0 || groups < 1) return VMB_ERR_INVALID_ARG;
+    if (D % groups != 0) return VMB_ERR_INVALID_ARG;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    long long kg = 0;
+    if (!count(&kg, {K, groups}) || kg > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    // the (b, k, g) sequences are the (b, k') sequences of a problem with K*G
+    // directions of D/G channels: u, delta, y rows, A, bias, Dskip and ybar
+    // are laid out identically; only B / C rows are shared by G sequences
+    ScanArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, y, ybar, B, (int)kg, D / groups, N, H * W, flags, dtype,
+               workspace, workspace_bytes};
+    a.bc_group = groups;
+    return run_scan(a, true, stream);
+}
+
 vmb_status vmb_mean_scan_merge_fwd(const void* u, const void* delta, const float* A, const void* Bs, const void* Cs,
                                    const float* Dskip, const float* delta_bias, const void* x, void* out, float* ybar,
                                    int B, int D, int N, int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,

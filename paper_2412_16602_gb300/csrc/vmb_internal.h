@@ -27,6 +27,7 @@ struct ScanArgs {
     void* ws;
     size_t ws_bytes;
     bool no_bcast = false;  // mean path fused with the cross-merge: ybar only, no y
+    int bc_group = 1;       // grouped basis: K and D above are K*G and D/G; B / C rows per G sequences
 };
 
 // Execution plan of an L-chunked scan: how the (sequence, chunk) grid is cut

@@ -39,7 +39,8 @@ VMB_PATH_MEAN = 1
 
 EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb_scan_kernel_count",
            "vmb_selective_scan_fwd",
-           "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_discretise_fwd", "vmb_discretise_mean_fwd",
+           "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd",
+           "vmb_discretise_fwd", "vmb_discretise_mean_fwd",
            "vmb_scan_only_fwd", "vmb_read_status", "vmb_status_string", "vmb_version"]
 
 
@@ -63,6 +64,7 @@ def _load() -> ctypes.CDLL:
     lib.vmb_selective_scan_fwd.argtypes = [vp] * 8 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_fwd.argtypes = [vp] * 9 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_merge_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_grouped_fwd.argtypes = [vp] * 9 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_discretise_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
@@ -71,7 +73,8 @@ def _load() -> ctypes.CDLL:
     lib.vmb_status_string.restype = ctypes.c_char_p
     lib.vmb_version.argtypes = []
     for name in ["vmb_cross_scan", "vmb_cross_merge", "vmb_selective_scan_fwd", "vmb_mean_scan_fwd",
-                 "vmb_mean_scan_merge_fwd", "vmb_discretise_fwd", "vmb_discretise_mean_fwd", "vmb_scan_only_fwd",
+                 "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_discretise_fwd",
+                 "vmb_discretise_mean_fwd", "vmb_scan_only_fwd",
                  "vmb_read_status", "vmb_version"]:
         getattr(lib, name).restype = i
     return lib
@@ -256,6 +259,35 @@ def vmb_mean_scan_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, H: int, W: int, *,
                                  _ptr(delta_bias), _ptr(y), _ptr(ybar), B, K, D, N, H, W, flags,
                                  _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
                                  _stream(stream)), "vmb_mean_scan_fwd")
+    return y, ybar
+
+
+def vmb_mean_scan_grouped_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, H: int, W: int, groups: int, *,
+                              y=None, ybar=None, want_ybar: bool = False, flags: int = VMB_FLAG_SOFTPLUS,
+                              workspace=None, stream=None):
+    """Grouped basis (reduced channel dimension d = groups): the channel mean of Eq. 9 over each
+    of `groups` channel groups; returns (y [B, K, D, L], ybar [B, K, groups, L] fp32 or None)."""
+    B, K, D, N, L = _scan_shapes(u, delta, A, Bs, Cs, Dskip, delta_bias, H, W)
+    if groups < 1 or D % groups:
+        raise ValueError("groups must be >= 1 and divide D")
+    if y is None:
+        y = torch.empty_like(u)
+    _dev(y, "y")
+    if y.shape != u.shape or y.dtype != u.dtype:
+        raise ValueError("y must match u")
+    if ybar is None and want_ybar:
+        ybar = torch.empty((B, K, groups, L), dtype=torch.float32, device=u.device)
+    if ybar is not None:
+        _dev(ybar, "ybar")
+        if ybar.shape != (B, K, groups, L) or ybar.dtype != torch.float32:
+            raise ValueError("ybar must be float32 [B, K, groups, L]")
+    ws_bytes = vmb_scan_workspace_bytes(VMB_PATH_MEAN, B, K * groups, D // groups, N, H, W, u.dtype)
+    if workspace is None:
+        workspace = _default_ws.get(ws_bytes, u.device)
+    _check(lib.vmb_mean_scan_grouped_fwd(_ptr(u), _ptr(delta), _ptr(A), _ptr(Bs), _ptr(Cs), _ptr(Dskip),
+                                         _ptr(delta_bias), _ptr(y), _ptr(ybar), B, K, D, N, H, W, groups, flags,
+                                         _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
+                                         _stream(stream)), "vmb_mean_scan_grouped_fwd")
     return y, ybar
 
 

@@ -25,6 +25,7 @@ def lib():
     lib.vmb_selective_scan_fwd.argtypes = [vp] * 8 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_fwd.argtypes = [vp] * 9 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_merge_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_grouped_fwd.argtypes = [vp] * 9 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_discretise_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
@@ -166,3 +167,16 @@ def test_scan_only_validation(lib):
     assert f(FAKE, FAKE, FAKE + 1, FAKE, 1, 4, 8, 16, 4, 4, 1, S) == 2   # misaligned bf16 C
     assert f(FAKE, FAKE, FAKE, FAKE, 1, 4, 8, 16, 4, 4, 9, S) == 1       # bad dtype
     assert f(0, 0, 0, 0, 1, 4, 0, 16, 4, 4, 0, S) == 0                   # empty problem
+
+
+def test_grouped_validation(lib):
+    f = lib.vmb_mean_scan_grouped_fwd
+
+    def call(groups, D=8, ptrs=None, ws=0x100000):
+        p = [FAKE] * 9 if ptrs is None else ptrs
+        return f(*p, 1, 4, D, 16, 4, 4, groups, 1, 0, ws, 1 << 20, S)
+    assert call(0) == 1                  # no groups
+    assert call(3) == 1                  # does not divide D
+    assert call(2, ptrs=[FAKE] * 7 + [0, FAKE]) == 1   # null y
+    assert call(2, ws=0) == 4
+    assert call(4, D=0, ptrs=[0] * 9, ws=0) == 0        # empty problem
