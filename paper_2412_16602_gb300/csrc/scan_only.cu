@@ -152,13 +152,16 @@ __global__ void __launch_bounds__(kDiscThreads) discretise_mean_kernel(const Dis
 }
 
 // ----------------------------------------------------------------- scan alone
-// A CTA owns CC whole channels.  Each channel's L steps are cut into S
-// segments; lane (s, n) scans state n over segment s twice: first from zero,
-// giving the segment's decay product P and end state H, then, after the
-// segments' carries have been folded in order (h_in[s+1] = P[s] h_in[s] +
-// H[s], h_in[0] = 0), from its carry, producing the output.  The NP lanes of
-// one (channel, segment) are adjacent, and y = sum_n C_n h_n is reduced over
-// them every 8 steps by a transposed butterfly.
+// A CTA owns one channel.  Its L steps are cut into S segments; lane (s, n)
+// scans state n over segment s twice: first from zero, giving the segment's
+// decay product P and end state H, then from its carry, producing the output.
+// The carries are an exclusive scan over the segments of the affine maps
+// h -> P h + H (composition (P1, H1) then (P2, H2) = (P2 P1, P2 H1 + H2)), done
+// in shared memory in log2(S) rounds (Hillis-Steele: a fixed order, so the
+// result is reproducible).  A channel's operands (N L floats each) are small
+// enough, and few enough CTAs are resident, that the second pass reads them
+// from L2.  The NP lanes of one segment are adjacent, and y = sum_n C_n h_n is
+// reduced over them every 8 steps by a transposed butterfly.
 struct OnlyParams {
     const float* dA;
     const float* dBu;
@@ -170,10 +173,10 @@ struct OnlyParams {
     int vec;      // rows 32-byte aligned at every 8-step block
 };
 
-template <int NP, int S>
+template <int NP>
 struct OnlyShape {
-    static constexpr int CC = (S * NP >= 256) ? 1 : 256 / (S * NP);
-    static constexpr int THREADS = CC * S * NP;
+    static constexpr int S = NP >= 4 ? 64 : 256 / NP;  // segments per channel
+    static constexpr int THREADS = S * NP;             // 1024, 512 or 256
 };
 
 template <typename T>
@@ -242,23 +245,20 @@ __device__ __forceinline__ void reduce8(float (&v)[8], int r) {
     }
 }
 
-template <typename T, int NP, int S>
-__global__ void __launch_bounds__(OnlyShape<NP, S>::THREADS) scan_only_kernel(const OnlyParams p) {
+template <typename T, int NP>
+__global__ void __launch_bounds__(OnlyShape<NP>::THREADS) scan_only_kernel(const OnlyParams p) {
     pdl_wait();
     pdl_launch_dependents();
-    using SH = OnlyShape<NP, S>;
-    constexpr int CC = SH::CC;
-    __shared__ float sP[CC][S][NP], sH[CC][S][NP];
+    constexpr int S = OnlyShape<NP>::S;
+    __shared__ float sP[S][NP], sH[S][NP];
     const int n = threadIdx.x % NP;
-    const int s = (threadIdx.x / NP) % S;
-    const int cc = threadIdx.x / (NP * S);
-    const long long ch = (long long)blockIdx.x * CC + cc;
-    const bool cv = ch < p.channels;
-    const bool nv = cv && n < p.N;
-    const long long bk = cv ? ch / p.Dm : 0;
+    const int s = threadIdx.x / NP;
+    const long long ch = blockIdx.x;
+    const bool nv = n < p.N;
+    const long long bk = ch / p.Dm;
     const int t0 = min(p.L, s * p.seg_len), t1 = min(p.L, t0 + p.seg_len);
-    const float* ra = p.dA + ((size_t)(cv ? ch : 0) * p.N + (nv ? n : 0)) * p.L;
-    const float* rb = p.dBu + ((size_t)(cv ? ch : 0) * p.N + (nv ? n : 0)) * p.L;
+    const float* ra = p.dA + ((size_t)ch * p.N + (nv ? n : 0)) * p.L;
+    const float* rb = p.dBu + ((size_t)ch * p.N + (nv ? n : 0)) * p.L;
     const T* rc = static_cast<const T*>(p.Cs) + ((size_t)bk * p.N + (nv ? n : 0)) * p.L;
     const bool vec = p.vec != 0;
     // pass 1: the segment from a zero state
@@ -275,20 +275,28 @@ __global__ void __launch_bounds__(OnlyShape<NP, S>::THREADS) scan_only_kernel(co
             }
         }
     }
-    sP[cc][s][n] = P;
-    sH[cc][s][n] = H;
+    sP[s][n] = P;
+    sH[s][n] = H;
     __syncthreads();
-    if (s == 0) {  // the carries of the segments, folded in order
-        float h = 0.0f;
-        for (int q = 0; q < S; ++q) {
-            const float pq = sP[cc][q][n], hq = sH[cc][q][n];
-            sH[cc][q][n] = h;  // carry into segment q
-            h = fmaf(pq, h, hq);
+    // inclusive scan over the segments (earlier segment applied first)
+#pragma unroll 1
+    for (int off = 1; off < S; off <<= 1) {
+        float pp = 1.0f, hh = 0.0f;
+        if (s >= off) {
+            pp = sP[s - off][n];
+            hh = sH[s - off][n];
         }
+        __syncthreads();
+        if (s >= off) {
+            H = fmaf(P, hh, H);
+            P *= pp;
+            sP[s][n] = P;
+            sH[s][n] = H;
+        }
+        __syncthreads();
     }
-    __syncthreads();
-    float h = nv ? sH[cc][s][n] : 0.0f;
-    float* yr = p.y + (size_t)(cv ? ch : 0) * p.L;
+    float h = (nv && s > 0) ? sH[s - 1][n] : 0.0f;  // carry into this segment
+    float* yr = p.y + (size_t)ch * p.L;
     const int r = n;
     constexpr int PER = NP >= 8 ? 1 : 8 / NP;  // outputs per lane per block
     const int base = NP >= 16 ? (r >> 1) : (NP >= 8 ? r : r * PER);
@@ -313,7 +321,7 @@ __global__ void __launch_bounds__(OnlyShape<NP, S>::THREADS) scan_only_kernel(co
             v[j] = c[j] * h;
         }
         reduce8<NP>(v, r);
-        if (cv && t < t1 && (NP < 16 || (r & 1) == 0)) {
+        if (t < t1 && (NP < 16 || (r & 1) == 0)) {
 #pragma unroll
             for (int j = 0; j < PER; ++j)
                 if (t + base + j < t1) yr[t + base + j] = v[j];
@@ -321,27 +329,18 @@ __global__ void __launch_bounds__(OnlyShape<NP, S>::THREADS) scan_only_kernel(co
     }
 }
 
-template <typename T, int NP>
-const void* only_fn(int S) {
-    return S == 64 ? reinterpret_cast<const void*>(&scan_only_kernel<T, NP, 64>)
-                   : reinterpret_cast<const void*>(&scan_only_kernel<T, NP, 16>);
-}
-
 template <typename T>
-const void* only_fn_np(int np, int S) {
+const void* only_fn(int np) {
     switch (np) {
-    case 1: return only_fn<T, 1>(S);
-    case 2: return only_fn<T, 2>(S);
-    case 4: return only_fn<T, 4>(S);
-    case 8: return only_fn<T, 8>(S);
-    default: return only_fn<T, 16>(S);
+    case 1: return reinterpret_cast<const void*>(&scan_only_kernel<T, 1>);
+    case 2: return reinterpret_cast<const void*>(&scan_only_kernel<T, 2>);
+    case 4: return reinterpret_cast<const void*>(&scan_only_kernel<T, 4>);
+    case 8: return reinterpret_cast<const void*>(&scan_only_kernel<T, 8>);
+    default: return reinterpret_cast<const void*>(&scan_only_kernel<T, 16>);
     }
 }
 
-int only_threads(int np, int S) {
-    const int cc = (S * np >= 256) ? 1 : 256 / (S * np);
-    return cc * S * np;
-}
+int only_segments(int np) { return np >= 4 ? 64 : 256 / np; }
 
 }  // namespace
 
@@ -395,21 +394,17 @@ vmb_status launch_scan_only(const OnlyArgs& a, cudaStream_t stream) {
     p.N = a.N;
     p.L = a.L;
     const int np = a.N <= 1 ? 1 : a.N <= 2 ? 2 : a.N <= 4 ? 4 : a.N <= 8 ? 8 : 16;
-    // 16 segments per channel when that fills the GPU about twice over, else
-    // 64 (shorter segments for problems with few channels)
-    const long long lanes16 = p.channels * np * 16;
-    const int S = lanes16 >= 2ll * device_sm_count() * 256 ? 16 : 64;
+    const int S = only_segments(np);
     p.seg_len = (int)(((long long)a.L + S - 1) / S);
     p.seg_len = (p.seg_len + 7) / 8 * 8;
     const size_t es = a.dtype == VMB_BF16 ? 2 : 4;
     const auto al = [](const void* q, size_t b) { return (reinterpret_cast<uintptr_t>(q) % b) == 0; };
     // every 8-step block starts 32 bytes into an fp32 row (16 into a bf16 one)
     p.vec = (a.L % 8 == 0) && al(a.dA, 32) && al(a.dBu, 32) && al(a.Cs, 8 * es) ? 1 : 0;
-    const int threads = only_threads(np, S);
-    const int cc = threads / (S * np);
-    const long long grid = (p.channels + cc - 1) / cc;
+    const int threads = S * np;
+    const long long grid = p.channels;
     if (grid > INT32_MAX) return VMB_ERR_UNSUPPORTED;
-    const void* fn = a.dtype == VMB_BF16 ? only_fn_np<__nv_bfloat16>(np, S) : only_fn_np<float>(np, S);
+    const void* fn = a.dtype == VMB_BF16 ? only_fn<__nv_bfloat16>(np) : only_fn<float>(np);
     void* args[] = {&p};
     return launch_kernel(fn, dim3((unsigned)grid), dim3(threads), 0, args, stream) == cudaSuccess ? VMB_OK
                                                                                                    : VMB_ERR_CUDA;

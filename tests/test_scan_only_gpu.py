@@ -100,11 +100,11 @@ def scan_only_case(B, K, Dm, N, H, W, dt, seed, one=False):
 
 ONLY_SHAPES = [
     # (B, K, Dm, N, H, W, dtype, one channel)
-    (1, 4, 8, 16, 5, 7, "f32", False),     # few channels: 64 segments, L = 35
-    (1, 4, 96, 16, 56, 56, "f32", False),  # 384 channels: 16 segments, L = 3136
+    (1, 4, 8, 16, 5, 7, "f32", False),     # L = 35 over 64 segments: most of them empty
+    (1, 4, 96, 16, 56, 56, "f32", False),  # 384 channels, L = 3136
     (2, 4, 1, 16, 56, 56, "f32", True),    # the channel-mean operands [B, K, N, L]
     (2, 3, 7, 5, 9, 11, "f32", False),     # padded states, L = 99
-    (1, 2, 33, 1, 8, 8, "f32", False),     # N = 1 (16 channels per CTA), ragged channel count
+    (1, 2, 33, 1, 8, 8, "f32", False),     # N = 1 (256 segments per channel), odd channel count
     (2, 2, 5, 2, 6, 10, "bf16", False),    # N = 2, bf16 C
     (1, 2, 9, 4, 16, 16, "bf16", False),   # N = 4, vector loads
     (1, 1, 3, 8, 1, 3, "f32", False),      # L = 3 < one block
