@@ -1521,14 +1521,19 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
             KernelInfo km{};
             long long rm = 0;
             if ((st = info(r.mid, &km, &rm)) != VMB_OK) return st;
-            KernelInfo kc{};
-            long long rc = 0;
+            KernelInfo kc{}, k9{};
+            long long rc = 0, r9 = 0;
             long long chunk_ctas = 0;
             if (np == 16) {
-                // few rows: the three-launch chunked variant while its grid of
-                // 64-step chunks fits in two waves (beyond that its aggregate
-                // traffic outweighs the look-back's second pass)
+                // few rows: the three-launch chunked variant while a grid of
+                // 64-step, one-lane chunks would fit in two waves (beyond that
+                // its aggregate traffic outweighs the look-back's second pass).
+                // It then runs as two lanes per channel over 32-step chunks,
+                // which measured fastest on GB300 with the launches chained
+                // (stage-1 maps at batch 1 to 3: 5 to 6% shorter steps than
+                // the 64-step chunks)
                 if ((st = info(kChunkShape + 2, &kc, &rc)) != VMB_OK) return st;
+                if ((st = info(kChunkShape + 1, &k9, &r9)) != VMB_OK) return st;
                 chunk_ctas = a.B * a.K * (long long)((a.D + kc.DT - 1) / kc.DT) * ((a.L + kc.ts - 1) / kc.ts);
             }
             if (rows * km.G * 2 >= rm * km.threads) {
@@ -1536,9 +1541,9 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
                 ki = km;
                 res = rm;
             } else if (np == 16 && chunk_ctas <= 2 * rc) {
-                shape = kChunkShape + 2;
-                ki = kc;
-                res = rc;
+                shape = kChunkShape + 1;
+                ki = k9;
+                res = r9;
             } else {
                 KernelInfo kn{};
                 long long rn = 0;
