@@ -695,8 +695,12 @@ vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan) {
     int np = 1;
     while (np < a.N) np <<= 1;
     const bool zoh = (a.flags & VMB_FLAG_B_ZOH) != 0;
-    // Longest chunk whose grid still gives every SM a few CTAs
-    // (one CTA per (b, k, chunk)); VMB_MEAN_TC forces a chunk length (tuning).
+    // Longest chunk whose grid still fills the GPU (one CTA per (b, k, chunk)):
+    // two waves of CTAs when a sequence has many channels (each CTA stages its
+    // channels' tables and reduces D channels per step), 0.8 of a wave when it
+    // has at most 256 (there a longer chunk amortises the fixed work of a CTA;
+    // measured on GB300 over batch 1 to 4 stage-1 maps, the batch-32 stages and
+    // grouped-basis views).  VMB_MEAN_TC forces a chunk length (tuning).
     const long long seqs = (long long)a.B * a.K;
     int tc = 32;
     const char* e = getenv("VMB_MEAN_TC");
@@ -710,7 +714,9 @@ vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan) {
             cudaSuccess)
             return VMB_ERR_CUDA;
         const long long resident = (long long)(per_sm < 1 ? 1 : per_sm) * device_sm_count();
-        if (forced || seqs * ((a.L + cand - 1) / cand) >= 2 * resident || cand == 32) {
+        const long long ctas = seqs * ((a.L + cand - 1) / cand);
+        const bool fills = a.D <= 256 ? 5 * ctas >= 4 * resident : ctas >= 2 * resident;
+        if (forced || fills || cand == 32) {
             tc = cand;
             break;
         }
