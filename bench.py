@@ -54,6 +54,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-paper-style", action="store_true",
                     help="skip the timing of the paper's split (discretise, then scan alone)")
+    ap.add_argument("--no-grouped", action="store_true", help="skip the timing of the grouped basis")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch size (smaller captures for profiling)")
@@ -419,7 +420,7 @@ def run_ours(args, wl, rank, world, local_rank):
 
     # the grouped basis (d channel groups, each its own mean and recurrence) on the step's inputs
     grouped = {}
-    for G in (4, 16):
+    for G in ((4, 16) if not args.no_grouped else ()):
         if wl.D % G:
             continue
         wsg = torch.zeros(vmb.vmb_scan_workspace_bytes(1, wl.B, 4 * G, wl.D // G, wl.N, wl.H, wl.W, tdt),
