@@ -505,6 +505,28 @@ def run_ours(args, wl, rank, world, local_rank):
 PAPER_A6000_BASE_512x3136 = {"scan_only_full_ms": 5.86, "scan_only_mean_ms": 0.02, "speedup": 293}
 
 
+# ALU ceilings of the state updates (b, k, d, n, l) on one GB300 (152 SMs,
+# 2.07 GHz; ex2 at 32 results/clk/SM and FP32 at 128 lanes/clk/SM, both
+# measured; 4 warp-instruction issues/clk/SM).  Full scan: one ex2 and four
+# FP32 operations per update (delta*A, delta*u*B, the state FMA, the output
+# FMA), five warp instructions per 32 updates: issue-bound at 8.05e12/s.
+# Channel-mean scan: one ex2 and two FP32 operations per (d, n) term of the
+# reduction: ex2-bound at 1.01e13/s.
+ALU_UPDATES_PER_S = {"full_scan": 4 * 152 * 2.07e9 * 32 / 5, "mean_scan": 32 * 152 * 2.07e9}
+ALU_BASIS = {"full_scan": "5 warp instructions per 32 state updates, 4 issues/clk/SM, 152 SMs, 2.07 GHz",
+             "mean_scan": "one ex2 per (d, n) term, 32 ex2/clk/SM, 152 SMs, 2.07 GHz"}
+
+
+def alu_view(kernel, wl, ms):
+    """The dominant kernel against the ALU ceiling of its state updates."""
+    if kernel not in ALU_UPDATES_PER_S:
+        return None
+    achieved = wl.B * 4 * wl.D * wl.N * wl.L / (ms / 1e3)
+    peak = ALU_UPDATES_PER_S[kernel]
+    return {"bound": "alu", "unit": "state updates/s", "achieved": achieved, "peak": peak, "frac": achieved / peak,
+            "basis": ALU_BASIS[kernel]}
+
+
 def paper_style_summary(ps, peak):
     if ps is None:
         return None
@@ -596,7 +618,8 @@ def main():
         "roofline": {"kernel": dominant, "bound": "hbm", "achieved": achieved, "peak": peak,
                      "peak_source": f"{peak_src} hbm_gbs (MEASURED_PEAKS.json)" if peak_src == "measured"
                      else "fallback 6.8 TB/s", "unit": "GB/s", "frac": achieved / peak,
-                     "algorithmic_bytes_per_launch": kb[dominant], "traffic": traffic},
+                     "algorithmic_bytes_per_launch": kb[dominant], "traffic": traffic,
+                     "alu_view": alu_view(dominant, wl, dom_ms)},
         # the fused channel-mean path (broadcast inside the merge), timed separately
         "mean_path_fused": {
             "us": fused_us, "gbs": wl.fused_mean_bytes() / (fused_us / 1e6) / 1e9,
