@@ -1479,9 +1479,10 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     // Rules measured on GB300 over the benchmark workloads: 16 states, at least
     // 256 channel rows per SM and L >= 128 -> the streaming kernel; otherwise plenty of
     // rows -> one lane per channel; a fair number -> two lanes; too few -> cut L into
-    // chunks: 64-step chunks of the three-launch variant while they fit in two
-    // waves, else look-back chunks with one lane per channel when they stay
-    // long (>= 256 steps) and the widest split otherwise (>= 128 steps).
+    // chunks: the three-launch variant (two lanes per channel, 32-step chunks)
+    // while a grid of 64-step one-lane chunks would fit in two waves, else
+    // look-back chunks with one lane per channel when they stay long (>= 256
+    // steps) and the widest split otherwise (>= 128 steps).
     int shape = 0, n_chunks = 1, forced_chunks = 0, env_shape = 0;
     KernelInfo ki{};
     long long res = 0;
