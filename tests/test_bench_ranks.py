@@ -50,3 +50,21 @@ def test_job_throughput_counts_every_rank():
     assert bench.job_throughput(10**9, 1, 1000.0) == pytest.approx(1.0)
     assert bench.job_throughput(10**9, 4, 1000.0) == pytest.approx(4.0)
     assert bench.max_over_ranks([3.0, 4.0], 1) == [3.0, 4.0]
+
+
+def test_alu_view_and_paper_summary():
+    import bench
+    import workloads
+    wl = workloads.WORKLOADS[bench.DEFAULT_WORKLOAD]
+    updates = wl.B * 4 * wl.D * wl.N * wl.L
+    v = bench.alu_view("full_scan", wl, 1.0)               # one millisecond
+    assert v["bound"] == "alu" and v["achieved"] == pytest.approx(updates * 1e3)
+    assert v["peak"] == pytest.approx(4 * 152 * 2.07e9 * 32 / 5)
+    assert v["frac"] == pytest.approx(v["achieved"] / v["peak"])
+    assert bench.alu_view("mean_scan", wl, 1.0)["peak"] == pytest.approx(32 * 152 * 2.07e9)
+    assert bench.alu_view("cross_scan", wl, 1.0) is None
+    ps = {"w": {"scan_only_full": {"us": 10.0, "gbs": 678.48}, "shape": {"B": 1}}}
+    out = bench.paper_style_summary(ps, 6784.8)
+    assert out["w"]["scan_only_full"]["frac_of_peak"] == pytest.approx(0.1)
+    assert out["paper_a6000_base_512x3136"]["scan_only_full_ms"] == 5.86
+    assert bench.paper_style_summary(None, 6784.8) is None
