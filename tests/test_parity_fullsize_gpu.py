@@ -75,3 +75,87 @@ def test_fullsize_sampled(name):
     for d in rng.choice(D, size=2, replace=False):
         merged = oracle.cross_merge(y_ref[:, :, d:d + 1], wl.H, wl.W)[0, 0]
         check(to_numpy(om[b, d]), merged, dt, f"{name} mean merged b={b} d={d}")
+
+
+# ------------------------------------------------------------- the next-item calls
+# At the sizes bench.py times them: the fused channel-mean path and the grouped
+# basis on the benchmark workload, the paper-style split on the benchmark
+# workload and on the paper's Table 1/2 "Base" shape.
+
+
+def test_fullsize_fused_and_grouped():
+    wl = workloads.WORKLOADS[workloads.STAGE1_B1]
+    inp = workloads.make_inputs(wl)
+    g = to_device(inp, DEV)
+    xs = vmb.vmb_cross_scan(g["x"])
+    out, ybar = vmb.vmb_mean_scan_merge_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], g["x"],
+                                            wl.H, wl.W)
+    grouped = {G: vmb.vmb_mean_scan_grouped_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"],
+                                                wl.H, wl.W, G, want_ybar=True) for G in (4, 16)}
+    assert vmb.vmb_read_status() == vmb.VMB_OK
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(77)
+    D, K, dt = wl.D, 4, wl.dtype
+    u_ref = oracle.cross_scan(inp.x[0:1])
+    y_ref, yb_ref = oracle.mean_scan(u_ref, inp.draw[0:1], inp.A, inp.Bs[0:1], inp.Cs[0:1], inp.Dskip, inp.bias)
+    check(to_numpy(ybar[0]), yb_ref[0], "f32", "fused ybar")
+    for d in rng.choice(D, size=3, replace=False):
+        merged = oracle.cross_merge(y_ref[:, :, d:d + 1], wl.H, wl.W)[0, 0]
+        check(to_numpy(out[0, d]), merged, dt, f"fused merged d={d}")
+    for G, (yg, ybg) in grouped.items():
+        Dg = D // G
+        for _ in range(2):
+            k, gi = int(rng.integers(K)), int(rng.integers(G))
+            sl = slice(gi * Dg, (gi + 1) * Dg)
+            A, Dsk, bias = _param_slice(inp, k, np.arange(gi * Dg, (gi + 1) * Dg))
+            y_s, yb_s = oracle.mean_scan(u_ref[:, k:k + 1, sl], inp.draw[0:1, k:k + 1, sl], A, inp.Bs[0:1, k:k + 1],
+                                         inp.Cs[0:1, k:k + 1], Dsk, bias)
+            check(to_numpy(ybg[0, k, gi]), yb_s[0, 0], "f32", f"grouped G={G} ybar k={k} g={gi}")
+            dd = rng.choice(Dg, size=4, replace=False)
+            check(to_numpy(yg[0, k, sl][dd]), y_s[0, 0][dd], dt, f"grouped G={G} rows k={k} g={gi}")
+
+
+def _paper_inputs(B, K, D, N, H, W):
+    """Seeded device inputs of the paper-style timing (the recipe bench.py uses)."""
+    L = H * W
+    gen = torch.Generator(device=DEV)
+    gen.manual_seed(7)
+    u = torch.randn(B, K, D, L, device=DEV, generator=gen)
+    draw = 0.5 * torch.randn(B, K, D, L, device=DEV, generator=gen)
+    Bs = torch.randn(B, K, N, L, device=DEV, generator=gen)
+    Cs = torch.randn(B, K, N, L, device=DEV, generator=gen)
+    A = -torch.arange(1, N + 1, device=DEV, dtype=torch.float32).repeat(K * D, 1).contiguous()
+    bias = torch.full((K * D,), -3.0, device=DEV)
+    return u, draw, Bs, Cs, A, bias
+
+
+@pytest.mark.parametrize("shape", [(1, 4, 192, 16, 56, 56), (128, 4, 128, 1, 56, 56)],
+                         ids=["stage1_b1_d192_n16", "paper_base_inner512_b128_n1"])
+def test_fullsize_paper_split(shape):
+    B, K, D, N, H, W = shape
+    u, draw, Bs, Cs, A, bias = _paper_inputs(B, K, D, N, H, W)
+    dA, dBu = vmb.vmb_discretise_fwd(u, draw, A, Bs, bias, H, W)
+    y = vmb.vmb_scan_only_fwd(dA, dBu, Cs, H, W)
+    dAm, dBum = vmb.vmb_discretise_mean_fwd(u, draw, A, Bs, bias, H, W)
+    ym = vmb.vmb_scan_only_fwd(dAm, dBum, Cs, H, W)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(88)
+    h = lambda t: t.cpu().numpy().astype(np.float64)  # noqa: E731
+    for _ in range(3):
+        b, k, d = int(rng.integers(B)), int(rng.integers(K)), int(rng.integers(D))
+        c = k * D + d
+        rA, rB = oracle.discretise(h(u[b:b + 1, k:k + 1, d:d + 1]), h(draw[b:b + 1, k:k + 1, d:d + 1]),
+                                   h(A[c:c + 1]), h(Bs[b:b + 1, k:k + 1]), h(bias[c:c + 1]))
+        check(to_numpy(dA[b, k, d]), rA[0, 0, 0], "f32", f"dA b={b} k={k} d={d}")
+        check(to_numpy(dBu[b, k, d]), rB[0, 0, 0], "f32", f"dBu b={b} k={k} d={d}")
+        ry = oracle.scan_only(h(dA[b:b + 1, k:k + 1, d:d + 1]), h(dBu[b:b + 1, k:k + 1, d:d + 1]),
+                              h(Cs[b:b + 1, k:k + 1]))
+        check(to_numpy(y[b, k, d]), ry[0, 0, 0], "f32", f"scan only b={b} k={k} d={d}")
+    b, k = int(rng.integers(B)), int(rng.integers(K))
+    cs = slice(k * D, (k + 1) * D)
+    rAm, rBm = oracle.discretise_mean(h(u[b:b + 1, k:k + 1]), h(draw[b:b + 1, k:k + 1]), h(A[cs]),
+                                      h(Bs[b:b + 1, k:k + 1]), h(bias[cs]))
+    check(to_numpy(dAm[b, k]), rAm[0, 0], "f32", f"dA mean b={b} k={k}")
+    check(to_numpy(dBum[b, k]), rBm[0, 0], "f32", f"dBu mean b={b} k={k}")
+    rym = oracle.scan_only(h(dAm[b:b + 1, k:k + 1]), h(dBum[b:b + 1, k:k + 1]), h(Cs[b:b + 1, k:k + 1]))
+    check(to_numpy(ym[b, k]), rym[0, 0], "f32", f"scan only on the means b={b} k={k}")
