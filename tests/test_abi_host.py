@@ -180,3 +180,11 @@ def test_grouped_validation(lib):
     assert call(2, ptrs=[FAKE] * 7 + [0, FAKE]) == 1   # null y
     assert call(2, ws=0) == 4
     assert call(4, D=0, ptrs=[0] * 9, ws=0) == 0        # empty problem
+
+
+def test_mean_scan_rejects_slabs_beyond_32bit_offsets(lib):
+    # D * L >= 2^31: a (b, k) slab no longer fits the mean kernel's 32-bit offsets
+    D, H, W = 65536, 182, 182
+    assert scan_call(lib, lib.vmb_mean_scan_fwd, D=D, H=H, W=W, mean=True) == 3
+    assert lib.vmb_scan_workspace_bytes(1, 1, 4, D, 16, H, W, 0) == 0
+    assert scan_call(lib, lib.vmb_mean_scan_fwd, D=D // 2, H=H, W=W, ws=0, mean=True) == 4  # below the limit
