@@ -88,6 +88,8 @@ class Oracle:
         lib.oracle_scan_only.restype = None
         lib.oracle_mean_scan_grouped.argtypes = [P] * 9 + [lg] * 6 + [i, i, i]
         lib.oracle_mean_scan_grouped.restype = i
+        lib.oracle_selection.argtypes = [P] * 8 + [lg] * 6
+        lib.oracle_selection.restype = None
         self.lib = lib
         self.path = lib_path
 
@@ -164,6 +166,21 @@ class Oracle:
         if rc:
             raise ValueError("groups must divide D")
         return y, ybar
+
+    def selection(self, u, WB, WC, Wz, Wup):
+        """Eq. 6 selection functions: u [B, K, D, L], WB and WC [K, N, D], Wz [K, R, D],
+        Wup [K, D, R] -> (delta_raw [B, K, D, L], Bs [B, K, N, L], Cs [B, K, N, L])."""
+        u, WB, WC, Wz, Wup = (_f64(a) for a in (u, WB, WC, Wz, Wup))
+        B, K, D, L = u.shape
+        N, R = WB.shape[1], Wz.shape[1]
+        if WB.shape != (K, N, D) or WC.shape != (K, N, D) or Wz.shape != (K, R, D) or Wup.shape != (K, D, R):
+            raise ValueError("weight shape mismatch")
+        dr = np.empty((B, K, D, L), dtype=np.float64)
+        Bs = np.empty((B, K, N, L), dtype=np.float64)
+        Cs = np.empty_like(Bs)
+        self.lib.oracle_selection(_ptr(u), _ptr(WB), _ptr(WC), _ptr(Wz), _ptr(Wup), _ptr(Bs), _ptr(Cs), _ptr(dr),
+                                  B, K, D, N, R, L)
+        return dr, Bs, Cs
 
     def _disc_args(self, u, delta, A, Bs, bias):
         u, delta, A, Bs, bias = (_f64(a) for a in (u, delta, A, Bs, bias))
@@ -254,6 +271,10 @@ def selective_scan(*a, **kw):
 
 def mean_scan(*a, **kw):
     return get().mean_scan(*a, **kw)
+
+
+def selection(*a, **kw):
+    return get().selection(*a, **kw)
 
 
 def mean_scan_grouped(*a, **kw):

@@ -14,6 +14,7 @@
  *   recurrence ..................... App. A, Eq. 3 (h_t = Abar h_{t-1} + Bbar u_t, y_t = C h_t + D u_t)
  *   channel mean (VMeanba) ......... Sec. 2.2, Eq. 9 (y = T^-1(Mamba(T(Abar, Bbar u, C))),
  *                                     T = mean over the inner channel axis, T^-1 = broadcast)
+ *   selection functions ............ App. A, Eq. 6 (B, C, Delta as linear maps of the input)
  *   grouped basis (d > 1) .......... Sec. 2.1 I_basis, Eq. 8 (reduced channel dimension d; the
  *                                     mean over each of d channel groups)
  *   scan-only kernel setting ....... Sec. 4, "Kernel Implementation" (discretisation done
@@ -382,6 +383,51 @@ void oracle_scan_only(const double* dA, const double* dBu, const double* Cs, dou
                 }
             }
     free(h);
+}
+
+/* ------------------------------------------- the selection functions (Eq. 6) */
+
+/* Eq. 6 makes B, C and Delta functions of the input: s_B = Linear_N(u),
+ * s_C = Linear_N(u), s_Delta = Broadcast_D(Linear_1(u)), each a linear map over
+ * the D channels of one step of one direction (weights per direction k).  The
+ * Delta branch is written as a rank-R map, Linear_D(Linear_R(u)): with R = 1
+ * and unit second-stage weights it is the printed Broadcast_D(Linear_1(u)).
+ * The scan itself applies Delta = softplus(Parameter + delta_raw).
+ *   Bs[b][k][n][l]        = sum_d WB[k][n][d] u[b][k][d][l]
+ *   Cs[b][k][n][l]        = sum_d WC[k][n][d] u[b][k][d][l]
+ *   z[r]                  = sum_d Wz[k][r][d] u[b][k][d][l]
+ *   delta_raw[b][k][d][l] = sum_r Wup[k][d][r] z[r] */
+void oracle_selection(const double* u, const double* WB, const double* WC, const double* Wz,
+                      const double* Wup, double* Bs, double* Cs, double* delta_raw, long B, long K,
+                      long D, long N, long R, long L) {
+    double* z = (double*)malloc(sizeof(double) * (size_t)(R > 0 ? R : 1));
+    if (!z) return;
+    for (long b = 0; b < B; ++b)
+        for (long k = 0; k < K; ++k) {
+            const double* uk = u + (b * K + k) * D * L;
+            for (long l = 0; l < L; ++l) {
+                for (long n = 0; n < N; ++n) {
+                    double sb = 0.0, sc = 0.0;
+                    for (long d = 0; d < D; ++d) {
+                        sb += WB[(k * N + n) * D + d] * uk[d * L + l];
+                        sc += WC[(k * N + n) * D + d] * uk[d * L + l];
+                    }
+                    Bs[((b * K + k) * N + n) * L + l] = sb;
+                    Cs[((b * K + k) * N + n) * L + l] = sc;
+                }
+                for (long r = 0; r < R; ++r) {
+                    double sz = 0.0;
+                    for (long d = 0; d < D; ++d) sz += Wz[(k * R + r) * D + d] * uk[d * L + l];
+                    z[r] = sz;
+                }
+                for (long d = 0; d < D; ++d) {
+                    double sd = 0.0;
+                    for (long r = 0; r < R; ++r) sd += Wup[(k * D + d) * R + r] * z[r];
+                    delta_raw[((b * K + k) * D + d) * L + l] = sd;
+                }
+            }
+        }
+    free(z);
 }
 
 /* Eq. 6 softplus, exposed so that tests can pin it against known values. */

@@ -372,6 +372,56 @@ def pin_mean_skip_mean_mode(orc):
            what="skip mean")
 
 
+# ------------------------------------------------------ selection (Eq. 6)
+
+
+def _selection_weights(rng, K=2, D=5, N=3, R=2):
+    return (rng.standard_normal((K, N, D)), rng.standard_normal((K, N, D)), rng.standard_normal((K, R, D)),
+            rng.standard_normal((K, D, R)))
+
+
+def pin_selection_one_hot(orc):
+    """A one-hot input (channel d0 of direction k0 at step l0) reads out one
+    column of every weight: Bs = WB[k0][:, d0], Cs = WC[k0][:, d0],
+    delta_raw[d] = sum_r Wup[k0][d][r] Wz[k0][r][d0]; every other step and
+    direction is zero."""
+    rng = np.random.default_rng(50)
+    WB, WC, Wz, Wup = _selection_weights(rng)
+    K, N, D = WB.shape
+    u = np.zeros((2, K, D, 6))
+    b0, k0, d0, l0 = 1, 1, 3, 4
+    u[b0, k0, d0, l0] = 1.0
+    dr, Bs, Cs = orc.selection(u, WB, WC, Wz, Wup)
+    eB = np.zeros_like(Bs)
+    eB[b0, k0, :, l0] = WB[k0][:, d0]
+    eC = np.zeros_like(Cs)
+    eC[b0, k0, :, l0] = WC[k0][:, d0]
+    eD = np.zeros_like(dr)
+    for d in range(D):
+        eD[b0, k0, d, l0] = sum(Wup[k0][d][r] * Wz[k0][r][d0] for r in range(Wz.shape[1]))
+    _close(Bs, eB, what="one-hot B")
+    _close(Cs, eC, what="one-hot C")
+    _close(dr, eD, what="one-hot delta")
+
+
+def pin_selection_printed_form_and_linearity(orc):
+    """R = 1 with unit second-stage weights is the printed Broadcast_D(Linear_1(u)):
+    every channel of a step carries the same value.  The maps are linear in u."""
+    rng = np.random.default_rng(51)
+    WB, WC, Wz, Wup = _selection_weights(rng, R=1)
+    K, N, D = WB.shape
+    u = rng.standard_normal((2, K, D, 7))
+    dr, _, _ = orc.selection(u, WB, WC, Wz, np.ones_like(Wup))
+    _close(dr, np.broadcast_to(dr[:, :, :1], dr.shape), what="broadcast over D")
+    WB, WC, Wz, Wup = _selection_weights(rng, R=3)
+    u2 = rng.standard_normal(u.shape)
+    a = orc.selection(u, WB, WC, Wz, Wup)
+    b = orc.selection(u2, WB, WC, Wz, Wup)
+    c = orc.selection(2.0 * u - 0.5 * u2, WB, WC, Wz, Wup)
+    for x, y, z, nm in zip(a, b, c, ("delta", "B", "C")):
+        _close(z, 2.0 * x - 0.5 * y, rtol=1e-12, atol=1e-12, what=f"linear {nm}")
+
+
 # ------------------------------------------------- grouped basis (d > 1 groups)
 
 

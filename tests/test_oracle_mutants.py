@@ -43,6 +43,13 @@ MUTANTS = {
     "grouped_divides_by_D": ("h[n] = abar[n] / (double)Dg * h[n] + bubar[n] / (double)Dg;",
                              "h[n] = abar[n] / (double)D * h[n] + bubar[n] / (double)Dg;"),
     "grouped_first_group_only": ("long d0 = g * Dg;", "long d0 = 0;"),
+    "selection_transposed_B": ("sb += WB[(k * N + n) * D + d] * uk[d * L + l];",
+                               "sb += WB[(k * D + d) * N + n] * uk[d * L + l];"),
+    "selection_C_from_B": ("sc += WC[(k * N + n) * D + d] * uk[d * L + l];",
+                           "sc += WB[(k * N + n) * D + d] * uk[d * L + l];"),
+    "selection_up_transposed": ("sd += Wup[(k * D + d) * R + r] * z[r];", "sd += Wup[(k * R + r) * D + d] * z[r];"),
+    "selection_first_direction_weights": ("sz += Wz[(k * R + r) * D + d] * uk[d * L + l];",
+                                          "sz += Wz[r * D + d] * uk[d * L + l];"),
     "scan_only_drops_decay": ("h[n] = dA[(row * N + n) * L + l] * h[n] + dBu[(row * N + n) * L + l];",
                               "h[n] = h[n] + dBu[(row * N + n) * L + l];"),
     "scan_only_output_before_update": ("h[n] = dA[(row * N + n) * L + l] * h[n] + dBu[(row * N + n) * L + l];\n                        acc += Cs[((b * K + k) * N + n) * L + l] * h[n];",
