@@ -23,6 +23,7 @@ import argparse
 import ctypes
 import hashlib
 import json
+import math
 import os
 import statistics
 import subprocess
@@ -56,6 +57,7 @@ def parse():
     ap.add_argument("--no-paper-style", action="store_true",
                     help="skip the timing of the paper's split (discretise, then scan alone)")
     ap.add_argument("--no-grouped", action="store_true", help="skip the timing of the grouped basis")
+    ap.add_argument("--no-selection", action="store_true", help="skip the timing of the Eq. 6 selection functions")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch size (smaller captures for profiling)")
@@ -481,6 +483,30 @@ def run_ours(args, wl, rank, world, local_rank):
         if vmb.vmb_read_status(wsg) != 0:
             raise RuntimeError("device error word set in the grouped mean scan")
         grouped[G] = 1e3 * statistics.mean(e0.elapsed_time(e1) for e0, e1 in gev)
+    # the selection functions of Eq. 6 (B, C, raw Delta from the cross-scanned
+    # input; rank-6 Delta projection as in VMamba-T) on the step's input
+    sel_us = None
+    if not args.no_selection:
+        gsel = torch.Generator(device=dev)
+        gsel.manual_seed(11)
+        R = 6
+        sw = [torch.randn(s, device=dev, generator=gsel) / math.sqrt(wl.D)
+              for s in ((4, wl.N, wl.D), (4, wl.N, wl.D), (4, R, wl.D), (4, wl.D, R))]
+        sdr, sB, sC = torch.empty_like(outs["xs"]), torch.empty_like(g["Bs"]), torch.empty_like(g["Cs"])
+
+        def sel():
+            vmb.vmb_selection_fwd(outs["xs"], *sw, wl.H, wl.W, delta_raw=sdr, Bs=sB, Cs=sC, stream=stream)
+        for _ in range(args.warmup):
+            prelude()
+            sel()
+        sev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        for e0, e1 in sev2:
+            prelude()
+            e0.record()
+            sel()
+            e1.record()
+        torch.cuda.synchronize()
+        sel_us = 1e3 * statistics.mean(e0.elapsed_time(e1) for e0, e1 in sev2)
     # the materialised operands of the bench workload: 2 x B*4*D*N*L fp32
     small_enough = 8 * wl.B * 4 * wl.D * wl.N * wl.L <= (32 << 30)
     paper = None if args.no_paper_style else {
@@ -492,7 +518,7 @@ def run_ours(args, wl, rank, world, local_rank):
                                                       min(args.steps, 10), args.warmup),
     }
     res = {"total_ms": total_ms, "step_ms": step_ms, "per_kernel": per_kernel, "e2e_ms": e2e_ms,
-           "paper_style": paper, "grouped_us": grouped,
+           "paper_style": paper, "grouped_us": grouped, "selection_us": sel_us,
            "h2d": h2d, "d2h": d2h, "clocks": clk.summary(), "fused_ms": fused_ms,
            "launches_per_step": step.launches, "fused_launches": step.fused_launches}
     res["total_ms"], res["e2e_ms"] = max_over_ranks([total_ms, e2e_ms], world, dev)
@@ -525,6 +551,17 @@ def alu_view(kernel, wl, ms):
     peak = ALU_UPDATES_PER_S[kernel]
     return {"bound": "alu", "unit": "state updates/s", "achieved": achieved, "peak": peak, "frac": achieved / peak,
             "basis": ALU_BASIS[kernel]}
+
+
+def selection_summary(us, wl, peak, R=6):
+    """Eq. 6 selection on the step's input: reads u, writes B, C and the raw Delta."""
+    if us is None:
+        return None
+    s = 2 if wl.dtype == "bf16" else 4
+    bytes_ = s * (2 * wl.B * 4 * wl.D * wl.L + 2 * wl.B * 4 * wl.N * wl.L) + 4 * 4 * (2 * wl.N + 2 * R) * wl.D
+    gbs = bytes_ / (us / 1e6) / 1e9
+    return {"us": us, "algorithmic_bytes": bytes_, "gbs": gbs, "frac_of_peak": gbs / peak, "rank": R,
+            "kernel": "CUDA-core FMA (no tensor cores yet)"}
 
 
 def paper_style_summary(ps, peak):
@@ -632,6 +669,7 @@ def main():
         "paper_style": paper_style_summary(res["paper_style"], peak),
         # grouped basis: d channel groups per direction, each its own channel mean
         # and recurrence (same algorithmic bytes as the mean scan)
+        "selection": selection_summary(res["selection_us"], wl, peak),
         "mean_grouped": {str(G): {"groups": G, "us": us, "gbs": kb["mean_scan"] / (us / 1e6) / 1e9,
                                   "frac_of_peak": kb["mean_scan"] / (us / 1e6) / 1e9 / peak}
                          for G, us in res["grouped_us"].items()},

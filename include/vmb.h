@@ -285,6 +285,24 @@ vmb_status vmb_scan_only_fwd(const float* dA, const float* dBu, const void* Cs, 
                              cudaStream_t stream);
 
 /*
+ * vmb_selection_fwd - the selection functions of Eq. 6 (App. A): B, C and the
+ * raw Delta of every step as linear maps of the scan input over the D channels
+ * of that step and direction, with per-direction weights:
+ *   Bs[b,k,n,l] = sum_d WB[k,n,d] u[b,k,d,l]      s_B = Linear_N(u)
+ *   Cs[b,k,n,l] = sum_d WC[k,n,d] u[b,k,d,l]      s_C = Linear_N(u)
+ *   z_r = sum_d Wz[k,r,d] u[b,k,d,l],  delta_raw[b,k,d,l] = sum_r Wup[k,d,r] z_r
+ * The Delta branch is a rank-R map; R = 1 with Wup = 1 is the printed
+ * s_Delta = Broadcast_D(Linear_1(u)).  The scans then apply
+ * Delta = softplus(delta_raw + delta_bias) (VMB_FLAG_SOFTPLUS).
+ *   u [B,K,D,L] (dtype); WB, WC [K,N,D], Wz [K,R,D], Wup [K,D,R] fp32;
+ *   Bs, Cs [B,K,N,L], delta_raw [B,K,D,L] (dtype) out.  N and R in 1..16
+ *   (VMB_ERR_UNSUPPORTED above).  Accumulation in fp32 (channels in order).
+ */
+vmb_status vmb_selection_fwd(const void* u, const float* WB, const float* WC, const float* Wz,
+                             const float* Wup, void* Bs, void* Cs, void* delta_raw, int B, int K,
+                             int D, int N, int R, int H, int W, vmb_dtype dtype, cudaStream_t stream);
+
+/*
  * vmb_read_status - synchronise `stream`, then return and clear the device
  * error word of `workspace` (VMB_OK, VMB_ERR_TIMEOUT or VMB_ERR_BOUNDS).  A
  * device-side error leaves the outputs of that call undefined but the CUDA

@@ -277,6 +277,27 @@ vmb_status vmb_scan_only_fwd(const float* dA, const float* dBu, const void* Cs, 
     return launch_scan_only(a, stream);
 }
 
+vmb_status vmb_selection_fwd(const void* u, const float* WB, const float* WC, const float* Wz, const float* Wup,
+                             void* Bs, void* Cs, void* delta_raw, int B, int K, int D, int N, int R, int H, int W,
+                             vmb_dtype dtype, cudaStream_t stream) {
+    if (!dtype_ok(dtype) || B < 0 || K < 0 || D < 0 || N < 0 || R < 0 || H < 0 || W < 0) return VMB_ERR_INVALID_ARG;
+    long long n = 0, nbc = 0;
+    if (!count(&n, {B, K, D, H, W}) || !count(&nbc, {B, K, N > 0 ? N : 1, H, W})) return VMB_ERR_INVALID_ARG;
+    if (n == 0) return VMB_OK;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    if (N < 1 || R < 1) return VMB_ERR_INVALID_ARG;
+    if (N > 16 || R > 16) return VMB_ERR_UNSUPPORTED;
+    long long rows = 0;
+    if (!count(&rows, {B, K, D}) || rows > INT_MAX / 2) return VMB_ERR_UNSUPPORTED;
+    if (!u || !WB || !WC || !Wz || !Wup || !Bs || !Cs || !delta_raw) return VMB_ERR_INVALID_ARG;
+    const size_t es = esize(dtype);
+    if (!aligned(u, es) || !aligned(Bs, es) || !aligned(Cs, es) || !aligned(delta_raw, es) || !aligned(WB, 4) ||
+        !aligned(WC, 4) || !aligned(Wz, 4) || !aligned(Wup, 4))
+        return VMB_ERR_MISALIGNED;
+    SelArgs a{u, WB, WC, Wz, Wup, Bs, Cs, delta_raw, B, K, D, N, R, H * W, dtype};
+    return launch_selection(a, stream);
+}
+
 vmb_status vmb_read_status(void* workspace, cudaStream_t stream) {
     if (!workspace) return VMB_ERR_INVALID_ARG;
     if (!aligned(workspace, 256)) return VMB_ERR_MISALIGNED;

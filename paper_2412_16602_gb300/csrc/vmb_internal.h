@@ -87,6 +87,20 @@ struct OnlyArgs {
     vmb_dtype dtype;
 };
 
+// The selection functions of Eq. 6 (B, C and the raw Delta from the input).
+struct SelArgs {
+    const void* u;     // [B][K][D][L], dtype
+    const float* WB;   // [K][N][D]
+    const float* WC;   // [K][N][D]
+    const float* Wz;   // [K][R][D]
+    const float* Wup;  // [K][D][R]
+    void* Bs;          // [B][K][N][L], dtype
+    void* Cs;          // [B][K][N][L], dtype
+    void* delta_raw;   // [B][K][D][L], dtype
+    int B, K, D, N, R, L;
+    vmb_dtype dtype;
+};
+
 int device_sm_count();
 
 vmb_status plan_full(const ScanArgs& a, ScanPlan* plan);
@@ -99,6 +113,7 @@ vmb_status launch_cross_scan(const void* x, void* xs, int B, int D, int H, int W
 vmb_status launch_cross_merge(const void* ys, void* out, int B, int D, int H, int W, vmb_dtype dt,
                               cudaStream_t stream);
 vmb_status launch_discretise(const DiscArgs& a, bool mean, cudaStream_t stream);
+vmb_status launch_selection(const SelArgs& a, cudaStream_t stream);
 vmb_status launch_scan_only(const OnlyArgs& a, cudaStream_t stream);
 vmb_status launch_mean_merge(const void* x, const float* ybar, const float* Dskip, void* out, int B, int D, int H,
                              int W, bool per_channel_skip, vmb_dtype dt, cudaStream_t stream);

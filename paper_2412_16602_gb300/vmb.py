@@ -41,7 +41,7 @@ EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb
            "vmb_selective_scan_fwd",
            "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd",
            "vmb_discretise_fwd", "vmb_discretise_mean_fwd",
-           "vmb_scan_only_fwd", "vmb_read_status", "vmb_status_string", "vmb_version"]
+           "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_read_status", "vmb_status_string", "vmb_version"]
 
 
 class VmbError(RuntimeError):
@@ -68,13 +68,14 @@ def _load() -> ctypes.CDLL:
     lib.vmb_discretise_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
+    lib.vmb_selection_fwd.argtypes = [vp] * 8 + [i] * 7 + [i, vp]
     lib.vmb_read_status.argtypes = [vp, vp]
     lib.vmb_status_string.argtypes = [i]
     lib.vmb_status_string.restype = ctypes.c_char_p
     lib.vmb_version.argtypes = []
     for name in ["vmb_cross_scan", "vmb_cross_merge", "vmb_selective_scan_fwd", "vmb_mean_scan_fwd",
                  "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_discretise_fwd",
-                 "vmb_discretise_mean_fwd", "vmb_scan_only_fwd",
+                 "vmb_discretise_mean_fwd", "vmb_scan_only_fwd", "vmb_selection_fwd",
                  "vmb_read_status", "vmb_version"]:
         getattr(lib, name).restype = i
     return lib
@@ -394,6 +395,31 @@ def vmb_scan_only_fwd(dA, dBu, Cs, H: int, W: int, *, y=None, stream=None):
     _check(lib.vmb_scan_only_fwd(_ptr(dA), _ptr(dBu), _ptr(Cs), _ptr(y), B, K, Dm, N, H, W, _dtype_code(Cs.dtype),
                                  _stream(stream)), "vmb_scan_only_fwd")
     return y
+
+
+def vmb_selection_fwd(u, WB, WC, Wz, Wup, H: int, W: int, *, delta_raw=None, Bs=None, Cs=None, stream=None):
+    """Eq. 6 selection functions: u [B, K, D, H*W] -> (delta_raw [B, K, D, L], Bs, Cs [B, K, N, L]),
+    all in u's dtype; WB, WC [K, N, D], Wz [K, R, D], Wup [K, D, R] float32."""
+    for t, n in [(u, "u"), (WB, "WB"), (WC, "WC"), (Wz, "Wz"), (Wup, "Wup")]:
+        _dev(t, n)
+    B, K, D, L = u.shape
+    N, R = WB.shape[1], Wz.shape[1]
+    if L != H * W or tuple(WB.shape) != (K, N, D) or tuple(WC.shape) != (K, N, D) or \
+            tuple(Wz.shape) != (K, R, D) or tuple(Wup.shape) != (K, D, R):
+        raise ValueError("u [B,K,D,H*W], WB/WC [K,N,D], Wz [K,R,D], Wup [K,D,R] expected")
+    if any(w.dtype != torch.float32 for w in (WB, WC, Wz, Wup)):
+        raise ValueError("weights must be float32")
+    delta_raw = torch.empty_like(u) if delta_raw is None else delta_raw
+    Bs = torch.empty((B, K, N, L), dtype=u.dtype, device=u.device) if Bs is None else Bs
+    Cs = torch.empty((B, K, N, L), dtype=u.dtype, device=u.device) if Cs is None else Cs
+    for t, n, shp in [(delta_raw, "delta_raw", (B, K, D, L)), (Bs, "Bs", (B, K, N, L)), (Cs, "Cs", (B, K, N, L))]:
+        _dev(t, n)
+        if tuple(t.shape) != shp or t.dtype != u.dtype:
+            raise ValueError(f"{n} must be {u.dtype} {shp}")
+    _check(lib.vmb_selection_fwd(_ptr(u), _ptr(WB), _ptr(WC), _ptr(Wz), _ptr(Wup), _ptr(Bs), _ptr(Cs),
+                                 _ptr(delta_raw), B, K, D, N, R, H, W, _dtype_code(u.dtype), _stream(stream)),
+           "vmb_selection_fwd")
+    return delta_raw, Bs, Cs
 
 
 def vmb_read_status(workspace=None, device=None, stream=None) -> int:

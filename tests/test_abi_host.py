@@ -29,6 +29,7 @@ def lib():
     lib.vmb_discretise_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
+    lib.vmb_selection_fwd.argtypes = [vp] * 8 + [i] * 7 + [i, vp]
     lib.vmb_status_string.argtypes = [i]
     lib.vmb_status_string.restype = ctypes.c_char_p
     lib.vmb_read_status.argtypes = [vp, vp]
@@ -188,3 +189,21 @@ def test_mean_scan_rejects_slabs_beyond_32bit_offsets(lib):
     assert scan_call(lib, lib.vmb_mean_scan_fwd, D=D, H=H, W=W, mean=True) == 3
     assert lib.vmb_scan_workspace_bytes(1, 1, 4, D, 16, H, W, 0) == 0
     assert scan_call(lib, lib.vmb_mean_scan_fwd, D=D // 2, H=H, W=W, ws=0, mean=True) == 4  # below the limit
+
+
+def test_selection_validation(lib):
+    f = lib.vmb_selection_fwd
+
+    def call(ptrs=None, B=1, K=4, D=8, N=16, R=6, H=4, W=4, dtype=0):
+        p = [FAKE] * 8 if ptrs is None else ptrs
+        return f(*p, B, K, D, N, R, H, W, dtype, S)
+    assert call(B=-1) == 1
+    assert call(N=0) == 1
+    assert call(R=0) == 1
+    assert call(N=17) == 3
+    assert call(R=17) == 3
+    assert call(dtype=4) == 1
+    assert call(ptrs=[FAKE] * 7 + [0]) == 1                 # null delta_raw
+    assert call(ptrs=[FAKE + 2] + [FAKE] * 7) == 2          # misaligned fp32 input
+    assert call(ptrs=[FAKE, FAKE + 2] + [FAKE] * 6) == 2    # misaligned weights
+    assert call(ptrs=[0] * 8, D=0) == 0                     # empty problem
