@@ -26,7 +26,16 @@ def tiny_outputs():
     inp = workloads.make_inputs(TINY)
     u, yf, outf = oracle.ss2d_full(inp)
     _, ym, ybar, outm = oracle.ss2d_mean(inp)
-    return {"u": u, "y_full": yf, "out_full": outf, "y_mean": ym, "ybar": ybar, "out_mean": outm}
+    dA, dBu = oracle.discretise(u, inp.draw, inp.A, inp.Bs, inp.bias)
+    dAm, dBum = oracle.discretise_mean(u, inp.draw, inp.A, inp.Bs, inp.bias)
+    _, ybar_g = oracle.mean_scan_grouped(u, inp.draw, inp.A, inp.Bs, inp.Cs, inp.Dskip, inp.bias, 3)
+    rng = np.random.default_rng(5)  # selection weights: K = 4, D = 3, N = 2, R = 2
+    ws = [rng.standard_normal(s) for s in ((4, 2, 3), (4, 2, 3), (4, 2, 3), (4, 3, 2))]
+    sel_dr, sel_B, _ = oracle.selection(u, *ws)
+    return {"u": u, "y_full": yf, "out_full": outf, "y_mean": ym, "ybar": ybar, "out_mean": outm,
+            "dA": dA, "dBu": dBu, "scan_only": oracle.scan_only(dA, dBu, inp.Cs),
+            "scan_only_mean": oracle.scan_only(dAm, dBum, inp.Cs), "ybar_grouped3": ybar_g,
+            "selection_delta": sel_dr, "selection_B": sel_B}
 
 
 def main():

@@ -14,6 +14,7 @@ def _load(name):
     return np.array([float(v) for v in lines[2:]]).reshape(shape)
 
 
-@pytest.mark.parametrize("name", ["u", "y_full", "out_full", "y_mean", "ybar", "out_mean"])
+@pytest.mark.parametrize("name", ["u", "y_full", "out_full", "y_mean", "ybar", "out_mean", "dA", "dBu", "scan_only",
+                                  "scan_only_mean", "ybar_grouped3", "selection_delta", "selection_B"])
 def test_oracle_matches_fixture(name):
     np.testing.assert_allclose(tiny_outputs()[name], _load(name), rtol=1e-13, atol=1e-15)
