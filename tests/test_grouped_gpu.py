@@ -43,7 +43,7 @@ def run(inp, groups, flags=vmb.VMB_FLAG_SOFTPLUS):
 def test_grouped_parity(case):
     B, D, N, H, W, dt, G = case
     wl = workloads.small_case(B=B, D=D, N=N, H=H, W=W, dtype=dt, seed=500 + D + G)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     _, xs, y, yb = run(inp, G)
     u = oracle.cross_scan(inp.x)
     y_ref, yb_ref = oracle.mean_scan_grouped(u, inp.draw, inp.A, inp.Bs, inp.Cs, inp.Dskip, inp.bias, G)
@@ -58,7 +58,7 @@ def test_grouped_parity(case):
                                    vmb.VMB_FLAG_SOFTPLUS | vmb.VMB_FLAG_B_ZOH], ids=["skip_mean", "zoh"])
 def test_grouped_flags(flags):
     wl = workloads.small_case(B=1, D=20, N=16, H=10, W=12, seed=520)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     _, _, y, yb = run(inp, 4, flags=flags)
     u = oracle.cross_scan(inp.x)
     kw = dict(skip_mode=1 if flags & vmb.VMB_FLAG_SKIP_MEAN else 0, b_mode=1 if flags & vmb.VMB_FLAG_B_ZOH else 0)
@@ -69,7 +69,7 @@ def test_grouped_flags(flags):
 
 def test_one_group_is_the_mean_scan_bit_for_bit():
     wl = workloads.small_case(B=2, D=32, N=16, H=14, W=14, seed=530)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     g, xs, y, yb = run(inp, 1)
     ym, ybm = vmb.vmb_mean_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W,
                                     want_ybar=True)
@@ -80,7 +80,7 @@ def test_one_group_is_the_mean_scan_bit_for_bit():
 
 def test_grouped_rejects_non_divisor():
     wl = workloads.small_case(B=1, D=10, N=4, H=4, W=4, seed=531)
-    g = to_device(workloads.make_inputs(wl), DEV)
+    g = to_device(workloads.make_inputs(wl, params="random"), DEV)
     xs = vmb.vmb_cross_scan(g["x"])
     with pytest.raises(ValueError):
         vmb.vmb_mean_scan_grouped_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], 4, 4, 3)

@@ -48,7 +48,7 @@ def _run(inp, flags=vmb.VMB_FLAG_SOFTPLUS):
 def test_fused_mean_merge_matches_oracle(shape):
     B, D, N, H, W, dt = shape
     wl = workloads.small_case(B=B, D=D, N=N, H=H, W=W, dtype=dt, seed=700 + D + N)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     out, ybar, om, yb_plain = _run(inp)
     _, _, ybar_ref, out_ref = oracle.ss2d_mean(inp)
     check(to_numpy(out), out_ref, dt, "fused mean out")
@@ -62,7 +62,7 @@ def test_fused_mean_merge_matches_oracle(shape):
 
 def test_fused_mean_merge_skip_mean_mode():
     wl = workloads.small_case(B=2, D=40, N=16, H=12, W=10, seed=731)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     flags = vmb.VMB_FLAG_SOFTPLUS | vmb.VMB_FLAG_SKIP_MEAN
     out, _, om, _ = _run(inp, flags=flags)
     _, _, _, out_ref = oracle.ss2d_mean(inp, skip_mode=oracle.SKIP_MEAN)
@@ -72,7 +72,7 @@ def test_fused_mean_merge_skip_mean_mode():
 
 def test_fused_mean_merge_zoh():
     wl = workloads.small_case(B=1, D=24, N=8, H=9, W=9, seed=732)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     flags = vmb.VMB_FLAG_SOFTPLUS | vmb.VMB_FLAG_B_ZOH
     out, _, om, _ = _run(inp, flags=flags)
     _, _, _, out_ref = oracle.ss2d_mean(inp, b_mode=1)
@@ -83,7 +83,7 @@ def test_fused_mean_merge_zoh():
 def test_fused_mean_merge_misaligned_map():
     """x and out one element off a 16-byte boundary: the element-wise merge path."""
     wl = workloads.small_case(B=1, D=16, N=16, H=8, W=8, seed=733)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     g = to_device(inp, DEV)
     xbuf = torch.empty(g["x"].numel() + 1, device=DEV)
     x = xbuf[1:].view_as(g["x"])

@@ -33,10 +33,30 @@ def _param_slice(inp, k, d_idx):
     return inp.A[c], inp.Dskip[c], inp.bias[c]
 
 
-@pytest.mark.parametrize("name", sorted(workloads.WORKLOADS))
-def test_fullsize_sampled(name):
+# Every benchmark workload with the benchmark's parameters, and the largest
+# ones again with random per-channel A and skip weights (every channel and
+# state its own value), which catches a kernel that reads the parameters of
+# the wrong channel, channel tile or state.
+FULLSIZE_CASES = [(name, "paper") for name in sorted(workloads.WORKLOADS)] + [
+    ("batch128_d256_n16_56x56_sigma0.05_f32", "random"),
+    ("seg512_stage1_b8_d192_n16_128x128_bf16", "random"),
+    ("vmamba_t_224_b32_stage1_d192_56x56_f32", "random"),
+    ("vmamba_t_224_b32_stage4_d1536_7x7_f32", "random"),
+]
+TAIL = 256  # the last steps of a row are checked on their own as well (the last L-chunk)
+
+
+def _planes(rng, B, D):
+    """(b, d) planes to sample: the last batch element with the last channel
+    (last channel tile), the first channel of the second 128-channel tile, and
+    a random plane."""
+    return [(B - 1, D - 1), (int(rng.integers(B)), min(D - 1, 128)), (int(rng.integers(B)), int(rng.integers(D)))]
+
+
+@pytest.mark.parametrize("name,params", FULLSIZE_CASES, ids=[f"{n}-{p}" for n, p in FULLSIZE_CASES])
+def test_fullsize_sampled(name, params):
     wl = workloads.WORKLOADS[name]
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params=params)
     g = to_device(inp, DEV)
     xs = vmb.vmb_cross_scan(g["x"])
     yf = vmb.vmb_selective_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W)
@@ -46,12 +66,12 @@ def test_fullsize_sampled(name):
     om = vmb.vmb_cross_merge(ym, wl.H, wl.W)
     assert vmb.vmb_read_status() == vmb.VMB_OK
     torch.cuda.synchronize()
-    rng = np.random.default_rng(zlib.crc32(name.encode()))
+    rng = np.random.default_rng(zlib.crc32(f"{name}/{params}".encode()))
     B, D = wl.B, wl.D
     dt = wl.dtype
+    tail = min(TAIL, wl.L)
     # ---- sampled planes: cross-scan bit-exact, full rows of all four directions, merged plane
-    for _ in range(3):
-        b, d = int(rng.integers(B)), int(rng.integers(D))
+    for b, d in _planes(rng, B, D):
         u_ref = oracle.cross_scan(inp.x[b:b + 1, d:d + 1])                        # [1, 4, 1, L]
         assert np.array_equal(to_numpy(xs[b, :, d]), u_ref[0, :, 0]), "cross-scan must be bit-exact"
         rows = []
@@ -60,21 +80,26 @@ def test_fullsize_sampled(name):
             y = oracle.selective_scan(u_ref[:, k:k + 1], inp.draw[b:b + 1, k:k + 1, d:d + 1], A,
                                       inp.Bs[b:b + 1, k:k + 1], inp.Cs[b:b + 1, k:k + 1], Dsk, bias)
             rows.append(y[0, 0, 0])
-            check(to_numpy(yf[b, k, d]), y[0, 0, 0], dt, f"{name} full row b={b} k={k} d={d}")
+            got = to_numpy(yf[b, k, d])
+            check(got, y[0, 0, 0], dt, f"{name} full row b={b} k={k} d={d}")
+            check(got[-tail:], y[0, 0, 0, -tail:], dt, f"{name} full row tail b={b} k={k} d={d}")
         merged = oracle.cross_merge(np.stack(rows)[None, :, None, :], wl.H, wl.W)[0, 0]
         check(to_numpy(of[b, d]), merged, dt, f"{name} full merged b={b} d={d}")
-    # ---- the channel-mean path for one batch element: all four directions, all channels
-    b = int(rng.integers(B))
-    u_ref = oracle.cross_scan(inp.x[b:b + 1])                                      # [1, 4, D, L]
-    y_ref, yb_ref = oracle.mean_scan(u_ref, inp.draw[b:b + 1], inp.A, inp.Bs[b:b + 1], inp.Cs[b:b + 1],
-                                     inp.Dskip, inp.bias)
-    check(to_numpy(ybar[b]), yb_ref[0], "f32" if dt == "f32" else "bf16", f"{name} ybar b={b}")
-    for k in range(4):
-        dd = rng.choice(D, size=min(D, 16), replace=False)
-        check(to_numpy(ym[b, k][dd]), y_ref[0, k][dd], dt, f"{name} mean rows b={b} k={k}")
-    for d in rng.choice(D, size=2, replace=False):
-        merged = oracle.cross_merge(y_ref[:, :, d:d + 1], wl.H, wl.W)[0, 0]
-        check(to_numpy(om[b, d]), merged, dt, f"{name} mean merged b={b} d={d}")
+    # ---- the channel-mean path for the last and a random batch element: all
+    # four directions, all channels (the mean needs every channel of a (b, k))
+    for b in sorted({B - 1, int(rng.integers(B))}):
+        u_ref = oracle.cross_scan(inp.x[b:b + 1])                                  # [1, 4, D, L]
+        y_ref, yb_ref = oracle.mean_scan(u_ref, inp.draw[b:b + 1], inp.A, inp.Bs[b:b + 1], inp.Cs[b:b + 1],
+                                         inp.Dskip, inp.bias)
+        ybt = "f32" if dt == "f32" else "bf16"
+        check(to_numpy(ybar[b]), yb_ref[0], ybt, f"{name} ybar b={b}")
+        check(to_numpy(ybar[b, :, -tail:]), yb_ref[0, :, -tail:], ybt, f"{name} ybar tail b={b}")
+        for k in range(4):
+            dd = np.unique(np.concatenate([[D - 1], rng.choice(D, size=min(D, 16), replace=False)]))
+            check(to_numpy(ym[b, k][dd]), y_ref[0, k][dd], dt, f"{name} mean rows b={b} k={k}")
+        for d in sorted({D - 1, int(rng.integers(D))}):
+            merged = oracle.cross_merge(y_ref[:, :, d:d + 1], wl.H, wl.W)[0, 0]
+            check(to_numpy(om[b, d]), merged, dt, f"{name} mean merged b={b} d={d}")
 
 
 # ------------------------------------------------------------- the next-item calls
@@ -85,7 +110,7 @@ def test_fullsize_sampled(name):
 
 def test_fullsize_fused_and_grouped():
     wl = workloads.WORKLOADS[workloads.STAGE1_B1]
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     g = to_device(inp, DEV)
     xs = vmb.vmb_cross_scan(g["x"])
     out, ybar = vmb.vmb_mean_scan_merge_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], g["x"],
@@ -115,8 +140,9 @@ def test_fullsize_fused_and_grouped():
             check(to_numpy(yg[0, k, sl][dd]), y_s[0, 0][dd], dt, f"grouped G={G} rows k={k} g={gi}")
 
 
-def _paper_inputs(B, K, D, N, H, W):
-    """Seeded device inputs of the paper-style timing (the recipe bench.py uses)."""
+def _paper_inputs(B, K, D, N, H, W, params="paper"):
+    """Seeded device inputs of the paper-style timing (the recipe bench.py uses;
+    params="random" draws A[c, n] = -U[0.5, 3] for every channel and state)."""
     L = H * W
     gen = torch.Generator(device=DEV)
     gen.manual_seed(7)
@@ -125,15 +151,18 @@ def _paper_inputs(B, K, D, N, H, W):
     Bs = torch.randn(B, K, N, L, device=DEV, generator=gen)
     Cs = torch.randn(B, K, N, L, device=DEV, generator=gen)
     A = -torch.arange(1, N + 1, device=DEV, dtype=torch.float32).repeat(K * D, 1).contiguous()
+    if params == "random":
+        A = -(0.5 + 2.5 * torch.rand(K * D, N, device=DEV, generator=gen))
     bias = torch.full((K * D,), -3.0, device=DEV)
     return u, draw, Bs, Cs, A, bias
 
 
+@pytest.mark.parametrize("params", ["paper", "random"])
 @pytest.mark.parametrize("shape", [(1, 4, 192, 16, 56, 56), (128, 4, 128, 1, 56, 56)],
                          ids=["stage1_b1_d192_n16", "paper_base_inner512_b128_n1"])
-def test_fullsize_paper_split(shape):
+def test_fullsize_paper_split(shape, params):
     B, K, D, N, H, W = shape
-    u, draw, Bs, Cs, A, bias = _paper_inputs(B, K, D, N, H, W)
+    u, draw, Bs, Cs, A, bias = _paper_inputs(B, K, D, N, H, W, params)
     dA, dBu = vmb.vmb_discretise_fwd(u, draw, A, Bs, bias, H, W)
     y = vmb.vmb_scan_only_fwd(dA, dBu, Cs, H, W)
     dAm, dBum = vmb.vmb_discretise_mean_fwd(u, draw, A, Bs, bias, H, W)

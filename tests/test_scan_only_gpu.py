@@ -27,7 +27,7 @@ DEV = torch.device("cuda", 0)
 
 def inputs(B, D, N, H, W, dt, seed):
     wl = workloads.small_case(B=B, D=D, N=N, H=H, W=W, dtype=dt, seed=seed)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     u = oracle.cross_scan(inp.x)
     tdt = torch.bfloat16 if dt == "bf16" else torch.float32
 

@@ -64,7 +64,7 @@ def test_selection_parity(case):
 def test_selection_feeds_the_scan():
     """u -> selection (Delta raw, B, C) -> full scan, against the oracle chain."""
     wl = workloads.small_case(B=1, D=32, N=16, H=10, W=12, seed=610)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     g = to_device(inp, DEV)
     xs = vmb.vmb_cross_scan(g["x"])
     rng = np.random.default_rng(611)

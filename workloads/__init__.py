@@ -137,8 +137,11 @@ class Inputs:
                     A=self.A, Dskip=self.Dskip, bias=self.bias)
 
 
+PARAMS = ("paper", "random")
+
+
 def make_inputs(wl: Workload, seed: int | None = None, *, sigma: float | None = None,
-                channel_identical: bool = False) -> Inputs:
+                channel_identical: bool = False, params: str = "paper") -> Inputs:
     """Draw one seeded input set for workload `wl`.
 
     Draw order (fixed): s, e, draw, Bs, Cs, dt.
@@ -146,14 +149,23 @@ def make_inputs(wl: Workload, seed: int | None = None, *, sigma: float | None = 
       draw       ~ N(0, 0.5^2)
       Bs, Cs     ~ N(0, 1)
       dt_c       = exp(U[ln 1e-3, ln 1e-1]),  bias_c = the value whose softplus is dt_c
-      A[c, n]    = -(n + 1)    (an input like any other; kernels do not rely on it)
-      Dskip      = 1
+    Per-channel parameters, by `params`:
+      "paper"  (the benchmark recipe): A[c, n] = -(n + 1), Dskip_c = 1
+      "random" (parity tests): A[c, n] = -U[0.5, 3] drawn independently for
+               every (c, n), Dskip_c = U[0.5, 1.5] per channel, from a second
+               generator seeded with (seed, 2), so that the draws above are
+               the same under both settings.  Every channel then has its own
+               A row and skip weight, and a kernel that reads the parameters
+               of the wrong channel or state gives a different result.
     bf16 workloads round x, draw, Bs, Cs to bf16 (ties to even) after drawing.
 
     channel_identical=True makes every channel of a direction identical
-    (sigma = 0, draw/bias shared over d): the case in which the channel mean
-    loses nothing.
+    (sigma = 0, draw/bias shared over d, and under "random" the A rows and
+    skip weights shared over d): the case in which the channel mean loses
+    nothing.
     """
+    if params not in PARAMS:
+        raise ValueError(f"params must be one of {PARAMS}, not {params!r}")
     seed = wl.seed if seed is None else seed
     sigma = wl.sigma if sigma is None else sigma
     B, K, D, N, H, W, L = wl.B, wl.K, wl.D, wl.N, wl.H, wl.W, wl.L
@@ -176,8 +188,16 @@ def make_inputs(wl: Workload, seed: int | None = None, *, sigma: float | None = 
     if channel_identical:
         draw[:] = draw[:, :, :1, :]
         bias = np.repeat(bias.reshape(K, D)[:, :1], D, axis=1).reshape(K * D).astype(f32)
-    A = np.tile(-(np.arange(N, dtype=f32) + 1.0), (K * D, 1)).astype(f32)
-    Dskip = np.ones(K * D, dtype=f32)
+    if params == "random":
+        prng = np.random.default_rng([seed, 2])
+        A = (-prng.uniform(0.5, 3.0, size=(K * D, N))).astype(f32)
+        Dskip = prng.uniform(0.5, 1.5, size=K * D).astype(f32)
+        if channel_identical:
+            A = np.repeat(A.reshape(K, D, N)[:, :1], D, axis=1).reshape(K * D, N).astype(f32)
+            Dskip = np.repeat(Dskip.reshape(K, D)[:, :1], D, axis=1).reshape(K * D).astype(f32)
+    else:
+        A = np.tile(-(np.arange(N, dtype=f32) + 1.0), (K * D, 1)).astype(f32)
+        Dskip = np.ones(K * D, dtype=f32)
     if wl.dtype == "bf16":
         x = round_to_bf16(x)
         draw = round_to_bf16(draw)
