@@ -21,9 +21,6 @@
 // carry-in state; the second pass recomputes the chunk from that state and
 // writes y.  Chunk order follows a ticket counter, so a CTA only waits on
 // CTAs that started before it; every wait is bounded.
-#include <stdlib.h>
-#include <string.h>
-
 #include <mutex>
 #include <type_traits>
 
@@ -1435,15 +1432,10 @@ int pad_states(int N) {
     return np;
 }
 
-// Optional tuning override "shape[,chunks]" from the environment
-// (VMB_FULL_PLAN), used to sweep tile shapes; unset in normal use.
-bool env_plan(int* shape, int* chunks) {
-    const char* e = getenv("VMB_FULL_PLAN");
-    if (!e || !*e) return false;
-    *shape = atoi(e);
-    const char* comma = strchr(e, ',');
-    *chunks = comma ? atoi(comma + 1) : 0;
-    return true;
+// Test-only override of the tile shape and chunk count (vmb_testing.h).
+bool forced_plan(int* shape, int* chunks) {
+    *shape = forced_full_shape(chunks);
+    return *shape >= 0;
 }
 
 }  // namespace
@@ -1483,12 +1475,12 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     // while a grid of 64-step one-lane chunks would fit in two waves, else
     // look-back chunks with one lane per channel when they stay long (>= 256
     // steps) and the widest split otherwise (>= 128 steps).
-    int shape = 0, n_chunks = 1, forced_chunks = 0, env_shape = 0;
+    int shape = 0, n_chunks = 1, forced_chunks = 0, forced_shape = 0;
     KernelInfo ki{};
     long long res = 0;
     vmb_status st;
-    if (!zoh && env_plan(&env_shape, &forced_chunks)) {
-        shape = env_shape % shape_count(np);
+    if (!zoh && forced_plan(&forced_shape, &forced_chunks)) {
+        shape = forced_shape % shape_count(np);
         if ((st = info(shape, &ki, &res)) != VMB_OK) return st;
         n_chunks = forced_chunks > 1 ? forced_chunks : 1;
     } else if (zoh) {

@@ -23,8 +23,6 @@
 // The recurrence and the C.h work run once per (b, k) instead of once per
 // (b, k, d); the exponentials of Abar stay per (b, k, d, n) because the mean
 // is taken after them.
-#include <stdlib.h>
-
 #include <mutex>
 
 #include "vmb_common.cuh"
@@ -700,11 +698,10 @@ vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan) {
     // channels' tables and reduces D channels per step), 0.8 of a wave when it
     // has at most 256 (there a longer chunk amortises the fixed work of a CTA;
     // measured on GB300 over batch 1 to 4 stage-1 maps, the batch-32 stages and
-    // grouped-basis views).  VMB_MEAN_TC forces a chunk length (tuning).
+    // grouped-basis views).  The tests can force a chunk length (vmb_testing.h).
     const long long seqs = (long long)a.B * a.K;
     int tc = 32;
-    const char* e = getenv("VMB_MEAN_TC");
-    const int forced = e ? atoi(e) : 0;
+    const int forced = forced_mean_chunk();
     for (int cand : {128, 64, 32}) {
         if (forced && cand != forced) continue;
         KInfo ki = mpick(a.dtype, np, cand, zoh);

@@ -56,7 +56,7 @@ SHAPES = [
 def test_ss2d_parity(shape):
     B, D, N, H, W, dt = shape
     wl = workloads.small_case(B=B, D=D, N=N, H=H, W=W, dtype=dt, seed=100 + D + N)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     out = gpu_step(inp)
     u_ref, yf_ref, of_ref = oracle.ss2d_full(inp)
     _, ym_ref, ybar_ref, om_ref = oracle.ss2d_mean(inp)
@@ -72,7 +72,7 @@ def test_ss2d_parity(shape):
 @pytest.mark.parametrize("flags", [0, vmb.VMB_FLAG_SOFTPLUS | vmb.VMB_FLAG_B_ZOH, vmb.VMB_FLAG_B_ZOH])
 def test_flag_variants(flags):
     wl = workloads.small_case(B=1, D=50, N=16, H=10, W=12, seed=5)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     if not flags & vmb.VMB_FLAG_SOFTPLUS:
         inp.bias[:] = np.abs(inp.bias)          # keep delta = raw + bias positive without softplus
         inp.draw[:] = np.abs(inp.draw) * 0.05
@@ -86,7 +86,7 @@ def test_flag_variants(flags):
 
 def test_skip_mean_mode():
     wl = workloads.small_case(B=2, D=30, N=4, H=6, W=8, seed=6)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     out = gpu_step(inp, mean_flags=vmb.VMB_FLAG_SOFTPLUS | vmb.VMB_FLAG_SKIP_MEAN)
     _, ym_ref, _, _ = oracle.ss2d_mean(inp, skip_mode=oracle.SKIP_MEAN)
     check(to_numpy(out["ym"]), ym_ref, "f32", "mean y (skip mean)")
@@ -104,7 +104,7 @@ def test_merge_exact_on_integers():
 def test_misaligned_views_take_element_path():
     """Tensors starting 4 bytes into an allocation are valid (element-wise path)."""
     wl = workloads.small_case(B=1, D=20, N=16, H=8, W=8, seed=8)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     g = to_device(inp, DEV)
 
     def shifted(t):
@@ -127,13 +127,13 @@ def test_empty_problem_is_a_noop():
 
 
 @pytest.mark.parametrize("plan", ["", "5,6"])
-def test_workspace_reuse_over_many_calls(plan, monkeypatch):
+def test_workspace_reuse_over_many_calls(plan, force_plan):
     """The workspace stays consistent over repeated chunked calls (the default
     chunked variant and a forced look-back plan), with bit-identical results."""
     if plan:
-        monkeypatch.setenv("VMB_FULL_PLAN", plan)
+        force_plan.full(plan)
     wl = workloads.small_case(B=1, D=16, N=16, H=40, W=40, seed=10)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     g = to_device(inp, DEV)
     xs = vmb.vmb_cross_scan(g["x"])
     ref = None
@@ -148,13 +148,13 @@ def test_workspace_reuse_over_many_calls(plan, monkeypatch):
 
 
 @pytest.mark.parametrize("mean", [False, True])
-def test_lookback_wait_times_out_cleanly(mean, monkeypatch):
+def test_lookback_wait_times_out_cleanly(mean, force_plan):
     """A chunk that never publishes makes its successors' bounded waits run out:
     the call reports VMB_ERR_TIMEOUT and the context and workspace stay usable."""
     if not mean:
-        monkeypatch.setenv("VMB_FULL_PLAN", "5,6")  # a look-back plan (the default here is the chunked variant)
+        force_plan.full("5,6")  # a look-back plan (the default here is the chunked variant)
     wl = workloads.small_case(B=1, D=16, N=16, H=48, W=48, seed=11)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     g = to_device(inp, DEV)
     xs = vmb.vmb_cross_scan(g["x"])
     ws = torch.zeros(vmb.vmb_scan_workspace_bytes(1 if mean else 0, 1, 4, 16, 16, 48, 48) + 256,
@@ -181,11 +181,11 @@ def test_lookback_wait_times_out_cleanly(mean, monkeypatch):
 @pytest.mark.parametrize("plan", ["0", "1", "2", "3", "4", "5", "6", "7", "8", "9", "10", "11", "12", "13", "14", "15",
                                   "0,3", "3,5", "4,2", "5,4", "6,7", "7,3", "7,6"])
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
-def test_every_tile_shape(plan, dt, monkeypatch):
+def test_every_tile_shape(plan, dt, force_plan):
     """Each tile shape of the full scan (and forced L-chunking) against the oracle."""
-    monkeypatch.setenv("VMB_FULL_PLAN", plan)
+    force_plan.full(plan)
     wl = workloads.small_case(B=1, D=72, N=16, H=24, W=28, dtype=dt, seed=21)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     g = to_device(inp, DEV)
     xs = vmb.vmb_cross_scan(g["x"])
     y = vmb.vmb_selective_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W)
@@ -207,12 +207,12 @@ CHUNKED_CASES = [
 @pytest.mark.parametrize("plan", ["8", "9", "10", "11"])
 @pytest.mark.parametrize("case", CHUNKED_CASES, ids=[f"B{s[0]}_D{s[1]}_N{s[2]}_{s[3]}x{s[4]}_{s[5]}"
                                                      for s in CHUNKED_CASES])
-def test_chunked_full_scan(plan, case, monkeypatch):
+def test_chunked_full_scan(plan, case, force_plan):
     """The three-launch chunked full scan (aggregates, carry fold, rerun) against the oracle."""
-    monkeypatch.setenv("VMB_FULL_PLAN", plan)
+    force_plan.full(plan)
     B, D, N, H, W, dt = case
     wl = workloads.small_case(B=B, D=D, N=N, H=H, W=W, dtype=dt, seed=31 + D)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     g = to_device(inp, DEV)
     xs = vmb.vmb_cross_scan(g["x"])
     y = vmb.vmb_selective_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W)
@@ -225,11 +225,11 @@ def test_chunked_full_scan(plan, case, monkeypatch):
 
 @pytest.mark.parametrize("tc", ["32", "64", "128"])
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
-def test_every_mean_chunk_length(tc, dt, monkeypatch):
+def test_every_mean_chunk_length(tc, dt, force_plan):
     """Each chunk length of the channel-mean scan against the oracle (ragged last chunk)."""
-    monkeypatch.setenv("VMB_MEAN_TC", tc)
+    force_plan.mean(tc)
     wl = workloads.small_case(B=2, D=70, N=16, H=19, W=21, dtype=dt, seed=22)
-    inp = workloads.make_inputs(wl)
+    inp = workloads.make_inputs(wl, params="random")
     g = to_device(inp, DEV)
     xs = vmb.vmb_cross_scan(g["x"])
     y, yb = vmb.vmb_mean_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W,
@@ -238,3 +238,46 @@ def test_every_mean_chunk_length(tc, dt, monkeypatch):
     _, ref, ybar_ref, _ = oracle.ss2d_mean(inp)
     check(to_numpy(y), ref, dt, f"mean y tc {tc}")
     check(to_numpy(yb), ybar_ref, dt, f"mean ybar tc {tc}")
+
+
+_ZOH_FIRST = r"""
+import sys
+sys.path.insert(0, sys.argv[1])
+import torch
+import oracle, workloads
+import paper_2412_16602_gb300 as vmb
+from tests.parity import check, to_device, to_numpy
+
+dev = torch.device("cuda", 0)
+wl = workloads.small_case(B=1, D=8, N=16, H=32, W=32, seed=61)
+inp = workloads.make_inputs(wl, params="random")
+g = to_device(inp, dev)
+xs = vmb.vmb_cross_scan(g["x"])
+args = (xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W)
+flags = vmb.VMB_FLAG_SOFTPLUS | vmb.VMB_FLAG_B_ZOH
+wsf = torch.zeros(vmb.vmb_scan_workspace_bytes(0, 1, 4, 8, 16, 32, 32), dtype=torch.uint8, device=dev)
+wsm = torch.zeros(vmb.vmb_scan_workspace_bytes(1, 1, 4, 8, 16, 32, 32), dtype=torch.uint8, device=dev)
+yf = vmb.vmb_selective_scan_fwd(*args, flags=flags, workspace=wsf)
+ym, _ = vmb.vmb_mean_scan_fwd(*args, flags=flags, workspace=wsm)
+assert vmb.vmb_read_status(wsf) == 0 and vmb.vmb_read_status(wsm) == 0
+_, rf, _ = oracle.ss2d_full(inp, b_mode=1)
+_, rm, _, _ = oracle.ss2d_mean(inp, b_mode=1)
+check(to_numpy(yf), rf, "f32", "zoh full y")
+check(to_numpy(ym), rm, "f32", "zoh mean y")
+print("zoh-first ok")
+"""
+
+
+def test_zoh_first_call_with_exactly_sized_workspace():
+    """In a fresh process (no workspace grown by earlier calls), the first scans
+    use the zero-order-hold form on a workspace of exactly the size the query
+    returns: on this few-row, L = 1024 map the ZOH plan is chunked while the
+    Euler plan is not, so the query must cover both forms."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, "-c", _ZOH_FIRST, root], cwd=root, capture_output=True, text=True,
+                       timeout=600)
+    assert r.returncode == 0, r.stdout + r.stderr
+    assert "zoh-first ok" in r.stdout
