@@ -11,8 +11,11 @@
  *
  * Conventions shared by every call
  *   - All tensor pointers are caller-owned DEVICE memory, dense row-major.
- *     The library allocates nothing and keeps no global state; scratch memory
- *     (the look-back workspace of the scans) is passed in by the caller.
+ *     The library allocates nothing, and scratch memory (the look-back
+ *     workspace of the scans) is passed in by the caller.  The one exception
+ *     is vmb_selective_scan_fwd_noalloc, for callers that cannot allocate:
+ *     its scratch is a fixed array built into the library (one per device),
+ *     and it keeps a host-side table of that array's device addresses.
  *   - Every call only validates its arguments and enqueues kernels on
  *     `stream`; it never synchronises (except vmb_read_status) and never
  *     throws or aborts.  Validation errors return before any launch, with no
@@ -107,9 +110,10 @@ vmb_status vmb_cross_merge(const void* ys, void* out, int B, int D, int H, int W
 /*
  * vmb_scan_workspace_bytes - bytes of zero-initialised device workspace that
  * vmb_selective_scan_fwd (path VMB_PATH_FULL) or vmb_mean_scan_fwd
- * (VMB_PATH_MEAN) needs for this problem on the current device.  Always >= 256
- * (the status header).  The workspace holds the status word and the
- * chunk-carry exchange of the L-chunked scans.
+ * (VMB_PATH_MEAN) needs for this problem on the current device, under any
+ * flags (the larger of the plans of the two Bbar forms, which differ in tile
+ * shape and chunking).  Always >= 256 (the status header).  The workspace
+ * holds the status word and the chunk-carry exchange of the L-chunked scans.
  *
  * The workspace must be zero-filled once before its first use (cudaMemset or
  * a zeros tensor); afterwards every call leaves it ready for the next one.
@@ -228,15 +232,19 @@ vmb_status vmb_mean_scan_merge_fwd(const void* u, const void* delta, const float
  *   workspace: the chunk-exchange scratch is a 16 MiB array built into the
  *   library, which every GPU that loads libvmb holds until the process exits.
  *   The call allocates nothing.
- *   Returns VMB_ERR_WORKSPACE when the problem's plan needs more than 16 MiB of
- *   scratch (vmb_scan_workspace_bytes(VMB_PATH_FULL, ...) > 16 MiB).
+ *   Every argument check runs first: a rejected call queues nothing.
+ *   Returns VMB_ERR_WORKSPACE when this call's plan (problem and flags) needs
+ *   more than 16 MiB of scratch; vmb_scan_workspace_bytes(VMB_PATH_FULL, ...)
+ *   <= 16 MiB guarantees that it does not.
  *   The first call made with a given device current looks up the array's
- *   device address on that device; make that first call before any stream
- *   capture.  Each call first clears the part of the array that must start at
- *   zero (an asynchronous memset on `stream`).  All calls share the one array
- *   per device, so calls that overlap in time on the GPU (other streams, other
- *   host threads) race and must be serialised by the caller.  Device-side wait
- *   timeouts have no readback for this entry point.
+ *   device address on that device and keeps it for the life of the process;
+ *   make that first call before any stream capture, and do not use this
+ *   entry point across a cudaDeviceReset of that device.  Each call first
+ *   clears the part of the array that must start at zero (an asynchronous
+ *   memset on `stream`).  All calls share the one array per device, so calls
+ *   that overlap in time on the GPU (other streams, other host threads) race
+ *   and must be serialised by the caller.  Device-side wait timeouts have no
+ *   readback for this entry point.
  */
 vmb_status vmb_selective_scan_fwd_noalloc(const void* u, const void* delta, const float* A,
                                           const void* Bs, const void* Cs, const float* Dskip,

@@ -30,7 +30,9 @@ std::mutex g_mu;
 void* g_scratch_ptr[kMaxDevices] = {nullptr};
 
 // Device address of g_scratch on the current device; looked up on the first
-// call made with that device current.
+// call made with that device current and kept for the life of the process
+// (the entry point must therefore not be used across a cudaDeviceReset of
+// that device, after which the cached address no longer names the array).
 vmb_status scratch_for_current_device(void** out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return VMB_ERR_CUDA;
@@ -57,31 +59,27 @@ extern "C" vmb_status vmb_selective_scan_fwd_noalloc(const void* u, const void* 
                                                      cudaStream_t stream) {
     if (H < 0 || W < 0) return VMB_ERR_INVALID_ARG;
     if ((long long)H * W > 0x7fffffffLL) return VMB_ERR_UNSUPPORTED;
-    // Shape and pointer checks, and the scratch size this problem needs, come
-    // from the public query so both entry points agree on the plan.
-    const size_t need = vmb_scan_workspace_bytes(VMB_PATH_FULL, B, K, D, N, H, W, dtype);
-    if (need == 0) {
-        // invalid shape: let the regular entry point name the error
-        return vmb_selective_scan_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, y, B, K, D, N, H, W, flags, dtype,
-                                      nullptr, 0, stream);
-    }
-    if (need > kScratchBytes) return VMB_ERR_WORKSPACE;  // problem needs more scratch than the static array
-    void* scratch = nullptr;
-    vmb_status s = scratch_for_current_device(&scratch);
-    if (s != VMB_OK) return s;
-    // The array keeps whatever the previous call left in it.  The status
-    // header and the chunk flags must start at zero; the published states are
-    // only read after their flag is set, so they need no clearing.
-    ScanArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, y, nullptr, B, K, D, N, H * W, flags, dtype, scratch,
-               kScratchBytes};
+    // Every argument check of vmb_selective_scan_fwd runs before anything is
+    // queued on the GPU, so that a rejected call has no side effects.
+    ScanArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, y, nullptr, B, K, D, N, H * W, flags, dtype, nullptr, 0};
+    bool empty = false;
+    vmb_status s = validate_scan(a, false, &empty);
+    if (s != VMB_OK || empty) return s;
     ScanPlan plan{};
-    bool empty = (long long)B * K * D * H * W == 0;
-    if (empty) return VMB_OK;
     s = plan_full(a, &plan);
     if (s != VMB_OK) return s;
+    if (plan.ws_bytes > kScratchBytes) return VMB_ERR_WORKSPACE;  // more scratch than the built-in array
+    void* scratch = nullptr;
+    s = scratch_for_current_device(&scratch);
+    if (s != VMB_OK) return s;
+    a.ws = scratch;
+    a.ws_bytes = kScratchBytes;
+    // The array keeps whatever the previous call left in it.  The status
+    // header and the chunk flags of this plan must start at zero; the
+    // published states are only read after their flag is set, so they need
+    // no clearing.
     const WsLayout w = ws_layout(plan);
     const size_t clear = plan.n_chunks > 1 ? w.aggP_off : 256;
     if (cudaMemsetAsync(scratch, 0, clear, stream) != cudaSuccess) return VMB_ERR_CUDA;
-    return vmb_selective_scan_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, y, B, K, D, N, H, W, flags, dtype,
-                                  scratch, kScratchBytes, stream);
+    return launch_full(a, plan, stream);
 }

@@ -2,12 +2,24 @@
 // argument validation, plan and workspace sizing, launch on the caller's stream.
 #include <limits.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "vmb_common.cuh"
 #include "vmb_internal.h"
+#include "vmb_testing.h"
 
 namespace vmb {
+
+namespace {
+std::atomic<int> g_force_shape{-1}, g_force_chunks{0}, g_force_tc{0};
+}  // namespace
+
+int forced_full_shape(int* chunks) {
+    *chunks = g_force_chunks.load(std::memory_order_relaxed);
+    return g_force_shape.load(std::memory_order_relaxed);
+}
+int forced_mean_chunk() { return g_force_tc.load(std::memory_order_relaxed); }
 
 int device_sm_count() {
     static std::mutex mu;
@@ -123,7 +135,39 @@ vmb_status run_scan(ScanArgs& a, bool mean, cudaStream_t stream) {
     return mean ? launch_mean(a, plan, stream) : launch_full(a, plan, stream);
 }
 
+// Workspace bytes of the plans for each of `flag_sets` (the largest).
+size_t plan_bytes(int path, const unsigned* flag_sets, int nsets, int B, int K, int D, int N, int H, int W,
+                  vmb_dtype dtype) {
+    if (path != VMB_PATH_FULL && path != VMB_PATH_MEAN) return 0;
+    if (H < 0 || W < 0 || (long long)H * W > INT_MAX) return 0;
+    ScanArgs a{};
+    a.B = B;
+    a.K = K;
+    a.D = D;
+    a.N = N;
+    a.L = H * W;
+    a.dtype = dtype;
+    // shape-only validation: stand-in non-null, aligned pointers
+    static const float dummy[4] = {0, 0, 0, 0};
+    a.u = a.delta = a.Bs = a.Cs = dummy;
+    a.A = a.Dskip = a.bias = dummy;
+    a.y = const_cast<float*>(dummy);
+    size_t need = 0;
+    for (int i = 0; i < nsets; ++i) {
+        a.flags = flag_sets[i];
+        bool empty = false;
+        if (check_scan(a, path == VMB_PATH_MEAN, &empty) != VMB_OK) return 0;
+        if (empty) return 256;
+        ScanPlan plan{};
+        if ((path == VMB_PATH_MEAN ? plan_mean(a, &plan) : plan_full(a, &plan)) != VMB_OK) return 0;
+        if (plan.ws_bytes > need) need = plan.ws_bytes;
+    }
+    return need;
+}
 }  // namespace
+
+vmb_status validate_scan(const ScanArgs& a, bool mean, bool* empty) { return check_scan(a, mean, empty); }
+
 }  // namespace vmb
 
 using namespace vmb;
@@ -145,26 +189,16 @@ vmb_status vmb_cross_merge(const void* ys, void* out, int B, int D, int H, int W
 }
 
 size_t vmb_scan_workspace_bytes(int path, int B, int K, int D, int N, int H, int W, vmb_dtype dtype) {
-    if (path != VMB_PATH_FULL && path != VMB_PATH_MEAN) return 0;
-    if (H < 0 || W < 0 || (long long)H * W > INT_MAX) return 0;
-    ScanArgs a{};
-    a.B = B;
-    a.K = K;
-    a.D = D;
-    a.N = N;
-    a.L = H * W;
-    a.dtype = dtype;
-    // shape-only validation: stand-in non-null, aligned pointers
-    static const float dummy[4] = {0, 0, 0, 0};
-    a.u = a.delta = a.Bs = a.Cs = dummy;
-    a.A = a.Dskip = a.bias = dummy;
-    a.y = const_cast<float*>(dummy);
-    bool empty = false;
-    if (check_scan(a, path == VMB_PATH_MEAN, &empty) != VMB_OK) return 0;
-    if (empty) return 256;
-    ScanPlan plan{};
-    if ((path == VMB_PATH_MEAN ? plan_mean(a, &plan) : plan_full(a, &plan)) != VMB_OK) return 0;
-    return plan.ws_bytes;
+    // The planners pick the tile shape and chunk count from the problem and
+    // the B-bar form (the zero-order-hold kernels have their own shapes), so
+    // the query covers both forms: one workspace serves every flag setting.
+    static const unsigned forms[2] = {0u, (unsigned)VMB_FLAG_B_ZOH};
+    return plan_bytes(path, forms, 2, B, K, D, N, H, W, dtype);
+}
+
+size_t vmb_testing_plan_workspace_bytes(int path, unsigned flags, int B, int K, int D, int N, int H, int W,
+                                        vmb_dtype dtype) {
+    return plan_bytes(path, &flags, 1, B, K, D, N, H, W, dtype);
 }
 
 int vmb_scan_kernel_count(int path, int B, int K, int D, int N, int H, int W, vmb_dtype dtype) {
@@ -327,5 +361,17 @@ const char* vmb_status_string(vmb_status s) {
 }
 
 int vmb_version(void) { return 100; }
+
+int vmb_testing_force_full_plan(int shape, int chunks) {
+    g_force_chunks.store(chunks, std::memory_order_relaxed);
+    g_force_shape.store(shape < 0 ? -1 : shape, std::memory_order_relaxed);
+    return 0;
+}
+
+int vmb_testing_force_mean_chunk(int tc) {
+    if (tc != 0 && tc != 32 && tc != 64 && tc != 128) return 1;
+    g_force_tc.store(tc, std::memory_order_relaxed);
+    return 0;
+}
 
 }  // extern "C"

@@ -103,6 +103,14 @@ struct SelArgs {
 
 int device_sm_count();
 
+// The argument checks of the scan entry points (shapes, flags, pointers,
+// alignment); *empty is set for a problem with no elements.
+vmb_status validate_scan(const ScanArgs& a, bool mean, bool* empty);
+
+// Test-only plan overrides (vmb_testing.h); -1 / 0 when unset.
+int forced_full_shape(int* chunks);
+int forced_mean_chunk();
+
 vmb_status plan_full(const ScanArgs& a, ScanPlan* plan);
 vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan);
 vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream);
