@@ -4,16 +4,20 @@
 One step = one SS2D pass over one synthetic batch, both paths:
     cross-scan x -> xs;  full scan xs -> y_full;  channel-mean scan xs -> y_mean;
     cross-merge y_full -> out_full;  cross-merge y_mean -> out_mean
-all through the C ABI of libvmb.  The default workload is the VMamba-T
-stage-1 scan at batch 1 (D=192, N=16, 56x56, fp32).
+all through the C ABI of libvmb.  The default workload is the largest
+single-GPU configuration: batch 128, D=256, N=16, 56x56 maps, fp32, channel
+noise 0.05 (5.1 GB of scan operands per call, far larger than L2, so the
+steps run back to back without an L2 flush; smaller workloads given with
+--workload flush L2 before every step).
 
 Prints ONE JSON line (rank 0).  `value` is the step's algorithmic HBM bytes
 (sum over its five kernels) per second of device time, with inputs resident
-in HBM and L2 flushed before every step; `e2e` is the same metric with the
-inputs copied from pinned host memory and both outputs copied back inside
-the timed region (every step; the copies of one step overlap the kernels of
-its neighbours).  `--impl reference` times the fp64 CPU oracle on the same
-workload instead.
+in HBM; `e2e` is the same metric with the inputs copied from pinned host
+memory and both outputs copied back inside the timed region (every step; the
+copies of one step overlap the kernels of its neighbours).  `configs` times
+every workload of the scan's configuration list (inputs drawn on the device
+with the same recipe), kernel by kernel.  `--impl reference` times the fp64
+CPU oracle on a one-batch-element slice of the workload instead.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
 """
@@ -39,7 +43,7 @@ import workloads  # noqa: E402
 
 METRIC = ("selective-scan HBM GB/s and (B·K·D·L)/s, full vs channel-mean, "
           "% of GB300 HBM peak")
-DEFAULT_WORKLOAD = workloads.STAGE1_B1
+DEFAULT_WORKLOAD = "batch128_d256_n16_56x56_sigma0.05_f32"
 FALLBACK_HBM_GBS = 6800.0
 KERNELS = ["cross_scan", "full_scan", "mean_scan", "cross_merge_full", "cross_merge_mean"]
 SOURCES = {"full_scan": "full_scan.cu", "mean_scan": "mean_scan.cu", "cross_scan": "cross_scan_merge.cu",
@@ -49,7 +53,7 @@ SOURCES = {"full_scan": "full_scan.cu", "mean_scan": "mean_scan.cu", "cross_scan
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
@@ -59,6 +63,9 @@ def parse():
     ap.add_argument("--no-grouped", action="store_true", help="skip the timing of the grouped basis")
     ap.add_argument("--no-selection", action="store_true", help="skip the timing of the Eq. 6 selection functions")
     ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--no-configs", action="store_true", help="skip the per-workload timing table")
+    ap.add_argument("--extra-steps", type=int, default=20,
+                    help="timed calls of each extra measurement (fused path, grouped, selection, paper split)")
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch size (smaller captures for profiling)")
     return ap.parse_args()
@@ -302,23 +309,15 @@ def time_paper_style(vmb, B, K, D, N, H, W, dev, prelude, steps, warmup):
     return res
 
 
-def run_ours(args, wl, rank, world, local_rank):
-    import torch
-    import paper_2412_16602_gb300 as vmb
+def needs_flush(wl, l2_bytes: int) -> bool:
+    """Flush L2 between steps unless one step's inputs are far larger than L2."""
+    return wl.scan_bytes() < 4 * l2_bytes
 
-    dev = torch.device("cuda", local_rank)
-    torch.cuda.set_device(dev)
-    inp = workloads.make_inputs(wl, seed=rank_seed(wl, rank))
-    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
-    host = {}
-    for k, v in inp.arrays().items():
-        t = torch.from_numpy(np.ascontiguousarray(v))
-        if k in ("x", "draw", "Bs", "Cs"):
-            t = t.to(tdt)
-        host[k] = t.pin_memory()
-    g = {k: v.to(dev) for k, v in host.items()}
+
+def make_outs(wl, dev, tdt, vmb):
+    import torch
     B, D, N, H, W, L = wl.B, wl.D, wl.N, wl.H, wl.W, wl.L
-    outs = {
+    return {
         "xs": torch.empty((B, 4, D, L), dtype=tdt, device=dev),
         "yf": torch.empty((B, 4, D, L), dtype=tdt, device=dev),
         "ym": torch.empty((B, 4, D, L), dtype=tdt, device=dev),
@@ -329,70 +328,154 @@ def run_ours(args, wl, rank, world, local_rank):
         "ofused": torch.empty((B, D, H, W), dtype=tdt, device=dev),
         "ybar": torch.empty((B, 4, L), dtype=torch.float32, device=dev),
     }
-    stream = torch.cuda.current_stream()
-    step = Step(vmb, wl, g, outs, stream.cuda_stream)
-    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
-    flush = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.float32, device=dev)
 
-    def prelude():
-        flush.fill_(1.0)           # evict the inputs from L2
-        torch.cuda._sleep(100000)  # let the host enqueue the whole step before the GPU reaches it
 
-    for _ in range(args.warmup):
-        prelude()
-        step.run()
-    torch.cuda.synchronize()
+def check_status(vmb, outs, where):
     if vmb.vmb_read_status(outs["ws_full"]) != 0 or vmb.vmb_read_status(outs["ws_mean"]) != 0:
-        raise RuntimeError("device error word set during warm-up")
+        raise RuntimeError(f"device error word set {where}")
 
-    # the timed steps: one event pair per step, nothing between the kernels
-    sev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
-    if world > 1:
-        torch.distributed.barrier()
-    torch.cuda.synchronize()
-    with ClockSampler(local_rank) as clk:
-        for i in range(args.steps):
-            prelude()
-            sev[i][0].record()
-            step.run()
-            sev[i][1].record()
-        torch.cuda.synchronize()
-    if world > 1:
-        torch.distributed.barrier()
-    if vmb.vmb_read_status(outs["ws_full"]) != 0 or vmb.vmb_read_status(outs["ws_mean"]) != 0:
-        raise RuntimeError("device error word set during the timed steps")
-    # the per-kernel breakdown: the same steps again with an event after every
-    # call (each event costs the stream a few microseconds, so these durations
-    # add up to more than the step time above)
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(KERNELS) + 1)] for _ in range(args.steps)]
-    for i in range(args.steps):
+
+def time_breakdown(step, n, prelude):
+    """n steps with an event after every call: per-kernel durations (ms lists)
+    and the fused channel-mean path timed alone (ms list)."""
+    import torch
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(KERNELS) + 1)] for _ in range(n)]
+    for i in range(n):
         prelude()
         evs[i][0].record()
         step.run(evs[i])
-    torch.cuda.synchronize()
-    if vmb.vmb_read_status(outs["ws_full"]) != 0 or vmb.vmb_read_status(outs["ws_mean"]) != 0:
-        raise RuntimeError("device error word set during the breakdown steps")
-    # the fused channel-mean path, timed alone with the same L2 flush per call
-    fev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
-    for _ in range(args.warmup):
-        prelude()
-        step.run_fused()
-    torch.cuda.synchronize()
-    for i in range(args.steps):
+    fev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(n)]
+    for i in range(n):
         prelude()
         fev[i][0].record()
         step.run_fused()
         fev[i][1].record()
     torch.cuda.synchronize()
-    if vmb.vmb_read_status(outs["ws_mean"]) != 0:
-        raise RuntimeError("device error word set in the fused mean path")
-    fused_ms = [e[0].elapsed_time(e[1]) for e in fev]
-    per_kernel = {k: [] for k in KERNELS}
-    step_ms = [e[0].elapsed_time(e[1]) for e in sev]
-    for e in evs:
-        for j, k in enumerate(KERNELS):
-            per_kernel[k].append(e[j].elapsed_time(e[j + 1]))
+    per_kernel = {k: [e[j].elapsed_time(e[j + 1]) for e in evs] for j, k in enumerate(KERNELS)}
+    return per_kernel, [e[0].elapsed_time(e[1]) for e in fev]
+
+
+def kernel_table(wl, per_kernel_ms, fused_ms, peak):
+    kb = kernel_bytes(wl)
+    per = {}
+    for k in KERNELS:
+        avg = statistics.mean(per_kernel_ms[k])
+        gbs = kb[k] / (avg / 1e3) / 1e9
+        per[k] = {"us": avg * 1e3, "gbs": gbs, "frac_of_peak": gbs / peak}
+    fused_us = 1e3 * statistics.mean(fused_ms)
+    fb = wl.fused_mean_bytes()
+    fused = {"us": fused_us, "gbs": fb / (fused_us / 1e6) / 1e9, "frac_of_peak": fb / (fused_us / 1e6) / 1e9 / peak,
+             "algorithmic_bytes": fb,
+             "unfused_us": per["mean_scan"]["us"] + per["cross_merge_mean"]["us"],
+             "speedup_over_unfused": (per["mean_scan"]["us"] + per["cross_merge_mean"]["us"]) / fused_us,
+             "speedup_over_full_path": (per["full_scan"]["us"] + per["cross_merge_full"]["us"]) / fused_us}
+    return per, fused
+
+
+def sweep_configs(vmb, dev, peak, prelude_flush, warmup):
+    """Every workload of the configuration list, kernel by kernel (inputs drawn on
+    the device with the workload recipe; about 50 ms of timed calls each)."""
+    import torch
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    stream = torch.cuda.current_stream()
+    table = {}
+    for name, wl in workloads.WORKLOADS.items():
+        tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+        g = workloads.make_device_inputs(wl, dev)
+        outs = make_outs(wl, dev, tdt, vmb)
+        step = Step(vmb, wl, g, outs, stream.cuda_stream)
+        flush = needs_flush(wl, l2)
+        prelude = prelude_flush if flush else (lambda: None)
+        for _ in range(warmup):
+            prelude()
+            step.run()
+            step.run_fused()
+        torch.cuda.synchronize()
+        est_s = sum(kernel_bytes(wl).values()) / 3e12
+        n = int(min(50, max(5, 0.05 / est_s)))
+        per_kernel, fused_ms = time_breakdown(step, n, prelude)
+        check_status(vmb, outs, f"in the {name} sweep")
+        per, fused = kernel_table(wl, per_kernel, fused_ms, peak)
+        table[name] = {"B": wl.B, "D": wl.D, "N": wl.N, "H": wl.H, "W": wl.W, "storage": wl.dtype,
+                       "sigma": wl.sigma, "calls": n, "l2": "flushed before every step" if flush else
+                       "not flushed (inputs far larger than L2)",
+                       "kernels": per, "mean_speedup_over_full": per["full_scan"]["us"] / per["mean_scan"]["us"],
+                       "mean_path_fused": fused, "gpu_launches_per_step": step.launches}
+        del g, outs, step
+        torch.cuda.empty_cache()
+    return table
+
+
+def run_ours(args, wl, rank, world, local_rank):
+    import torch
+    import paper_2412_16602_gb300 as vmb
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    # the workload recipe drawn on the device (seeded per rank); a pinned host
+    # copy feeds the end-to-end leg
+    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    g = workloads.make_device_inputs(wl, dev, seed=rank_seed(wl, rank))
+    host = {k: v.cpu().pin_memory() for k, v in g.items()}
+    outs = make_outs(wl, dev, tdt, vmb)
+    stream = torch.cuda.current_stream()
+    step = Step(vmb, wl, g, outs, stream.cuda_stream)
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    flush_buf = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.float32, device=dev)
+
+    def prelude_flush():
+        flush_buf.fill_(1.0)       # evict the inputs from L2
+        torch.cuda._sleep(100000)  # let the host enqueue the whole step before the GPU reaches it
+
+    flush = needs_flush(wl, l2)
+    prelude = prelude_flush if flush else (lambda: None)
+
+    for _ in range(args.warmup):
+        prelude()
+        step.run()
+    torch.cuda.synchronize()
+    check_status(vmb, outs, "during warm-up")
+
+    # the timed steps.  Inputs far larger than L2: the steps run back to back,
+    # an event before every step and one after the last (nothing else on the
+    # stream).  Smaller inputs: L2 is flushed before every step, outside the
+    # step's own pair of events.
+    if flush:
+        sev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    else:
+        sev = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local_rank) as clk:
+        if flush:
+            for i in range(args.steps):
+                prelude()
+                sev[i][0].record()
+                step.run()
+                sev[i][1].record()
+        else:
+            sev[0].record()
+            for i in range(args.steps):
+                step.run()
+                sev[i + 1].record()
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    check_status(vmb, outs, "during the timed steps")
+    if flush:
+        step_ms = [e0.elapsed_time(e1) for e0, e1 in sev]
+    else:
+        step_ms = [sev[i].elapsed_time(sev[i + 1]) for i in range(args.steps)]
     total_ms = float(sum(step_ms))
+
+    # per-kernel breakdown and the fused channel-mean path (separate steps with
+    # an event after every call; each event costs the stream a few microseconds)
+    for _ in range(2):
+        prelude()
+        step.run_fused()
+    per_kernel, fused_ms = time_breakdown(step, min(args.steps, 50), prelude)
+    check_status(vmb, outs, "during the breakdown steps")
 
     # ---- end-to-end leg: pinned host inputs -> device -> step -> host outputs.
     # Every step copies all its inputs from pinned host memory (packed in one
@@ -455,8 +538,23 @@ def run_ours(args, wl, rank, world, local_rank):
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1)
-    if vmb.vmb_read_status(outs["ws_full"]) != 0 or vmb.vmb_read_status(outs["ws_mean"]) != 0:
-        raise RuntimeError("device error word set during the end-to-end steps")
+    check_status(vmb, outs, "during the end-to-end steps")
+    del sets, h_in
+
+    nx = max(3, args.extra_steps)
+
+    def time_alone(fn):
+        for _ in range(args.warmup):
+            prelude()
+            fn()
+        ev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(nx)]
+        for a0, a1 in ev2:
+            prelude()
+            a0.record()
+            fn()
+            a1.record()
+        torch.cuda.synchronize()
+        return 1e3 * statistics.mean(a0.elapsed_time(a1) for a0, a1 in ev2)
 
     # the grouped basis (d channel groups, each its own mean and recurrence) on the step's inputs
     grouped = {}
@@ -465,24 +563,14 @@ def run_ours(args, wl, rank, world, local_rank):
             continue
         wsg = torch.zeros(vmb.vmb_scan_workspace_bytes(1, wl.B, 4 * G, wl.D // G, wl.N, wl.H, wl.W, tdt),
                           dtype=torch.uint8, device=dev)
-        yg = torch.empty_like(outs["ym"])
+        yg = outs["ym"]
 
         def fn():
             vmb.vmb_mean_scan_grouped_fwd(outs["xs"], g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"],
                                           wl.H, wl.W, G, y=yg, workspace=wsg, stream=stream)
-        for _ in range(args.warmup):
-            prelude()
-            fn()
-        gev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-        for e0, e1 in gev:
-            prelude()
-            e0.record()
-            fn()
-            e1.record()
-        torch.cuda.synchronize()
+        grouped[G] = time_alone(fn)
         if vmb.vmb_read_status(wsg) != 0:
             raise RuntimeError("device error word set in the grouped mean scan")
-        grouped[G] = 1e3 * statistics.mean(e0.elapsed_time(e1) for e0, e1 in gev)
     # the selection functions of Eq. 6 (B, C, raw Delta from the cross-scanned
     # input; rank-6 Delta projection as in VMamba-T) on the step's input
     sel_us = None
@@ -490,39 +578,47 @@ def run_ours(args, wl, rank, world, local_rank):
         gsel = torch.Generator(device=dev)
         gsel.manual_seed(11)
         R = 6
-        sw = [torch.randn(s, device=dev, generator=gsel) / math.sqrt(wl.D)
-              for s in ((4, wl.N, wl.D), (4, wl.N, wl.D), (4, R, wl.D), (4, wl.D, R))]
-        sdr, sB, sC = torch.empty_like(outs["xs"]), torch.empty_like(g["Bs"]), torch.empty_like(g["Cs"])
+        sw = [torch.randn(sz, device=dev, generator=gsel) / math.sqrt(wl.D)
+              for sz in ((4, wl.N, wl.D), (4, wl.N, wl.D), (4, R, wl.D), (4, wl.D, R))]
+        sdr, sB, sC = outs["yf"], torch.empty_like(g["Bs"]), torch.empty_like(g["Cs"])
 
         def sel():
             vmb.vmb_selection_fwd(outs["xs"], *sw, wl.H, wl.W, delta_raw=sdr, Bs=sB, Cs=sC, stream=stream)
-        for _ in range(args.warmup):
-            prelude()
-            sel()
-        sev2 = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-        for e0, e1 in sev2:
-            prelude()
-            e0.record()
-            sel()
-            e1.record()
-        torch.cuda.synchronize()
-        sel_us = 1e3 * statistics.mean(e0.elapsed_time(e1) for e0, e1 in sev2)
+        sel_us = time_alone(sel)
     # the materialised operands of the bench workload: 2 x B*4*D*N*L fp32
     small_enough = 8 * wl.B * 4 * wl.D * wl.N * wl.L <= (32 << 30)
     paper = None if args.no_paper_style else {
-        "bench_workload": (time_paper_style(vmb, wl.B, 4, wl.D, wl.N, wl.H, wl.W, dev, prelude, args.steps,
-                                            args.warmup) if small_enough else None),
+        "bench_workload": (time_paper_style(vmb, wl.B, 4, wl.D, wl.N, wl.H, wl.W, dev, prelude_flush, nx,
+                                            args.warmup) if small_enough else
+                           "not timed: the materialised operands exceed 32 GB"),
         # Table 1 / Table 2 "Base" row of the paper: inner dimension 512, L = 3136,
         # batch 128, d_state 1 (the byte counts of Table 2 fix batch x N = 128)
-        "paper_table_base_512x3136": time_paper_style(vmb, 128, 4, 128, 1, 56, 56, dev, prelude,
-                                                      min(args.steps, 10), args.warmup),
+        "paper_table_base_512x3136": time_paper_style(vmb, 128, 4, 128, 1, 56, 56, dev, prelude_flush,
+                                                      min(nx, 10), args.warmup),
     }
     res = {"total_ms": total_ms, "step_ms": step_ms, "per_kernel": per_kernel, "e2e_ms": e2e_ms,
            "paper_style": paper, "grouped_us": grouped, "selection_us": sel_us,
            "h2d": h2d, "d2h": d2h, "clocks": clk.summary(), "fused_ms": fused_ms,
-           "launches_per_step": step.launches, "fused_launches": step.fused_launches}
+           "launches_per_step": step.launches, "fused_launches": step.fused_launches,
+           "flushed": flush}
+    del g, outs, step, flush_buf
+    torch.cuda.empty_cache()
+    peak, _ = measured_peaks()
+    res["configs"] = None if args.no_configs else sweep_configs(vmb, dev, peak, prelude_flush_factory(dev),
+                                                                 min(args.warmup, 3))
     res["total_ms"], res["e2e_ms"] = max_over_ranks([total_ms, e2e_ms], world, dev)
-    return res, inp
+    return res, None
+
+
+def prelude_flush_factory(dev):
+    import torch
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    buf = torch.empty(max(2 * l2, 256 << 20) // 4, dtype=torch.float32, device=dev)
+
+    def prelude():
+        buf.fill_(1.0)
+        torch.cuda._sleep(100000)
+    return prelude
 
 
 # The paper's own scan-only kernel times on one RTX A6000 (Table 1, "Base"
@@ -569,6 +665,9 @@ def paper_style_summary(ps, peak):
         return None
     out = {}
     for key, r in ps.items():
+        if not isinstance(r, dict):
+            out[key] = r
+            continue
         out[key] = {k: (dict(v, frac_of_peak=v["gbs"] / peak) if isinstance(v, dict) and "gbs" in v else v)
                     for k, v in r.items()}
     out["paper_a6000_base_512x3136"] = PAPER_A6000_BASE_512x3136
@@ -586,30 +685,36 @@ def main():
     step_bytes = sum(kernel_bytes(wl).values())
     elems = wl.scan_elements()
     config = {"workload": wl.name, "B": wl.B, "K": 4, "D": wl.D, "N": wl.N, "H": wl.H, "W": wl.W, "L": wl.L,
-              "storage": wl.dtype, "sigma": wl.sigma, "l2": "flushed before every step (2x L2 write)",
+              "storage": wl.dtype, "sigma": wl.sigma,
               "step": "cross_scan + full_scan + mean_scan + 2 x cross_merge"}
+    # The oracle (fp64, host cores) runs on a bounded sample of the workload:
+    # one batch element (the same recipe with B = 1); its throughput is the
+    # sample's algorithmic bytes per second.
+    cpu_wl = wl.replace(B=1, name=f"{wl.name}[one batch element]") if wl.B > 1 else wl
+    cpu_bytes = sum(kernel_bytes(cpu_wl).values())
+    cpu_sample = (f"one batch element of {wl.name} (B = 1 of {wl.B}, same recipe) per oracle step, "
+                  "full + mean paths with the cross-scan and both merges")
 
     if args.impl == "reference":
         if rank != 0:
             return
-        inp = workloads.make_inputs(wl)
+        inp = workloads.make_inputs(cpu_wl)
         import oracle
-        for _ in range(min(args.warmup, 1)):
-            oracle_step(inp, oracle.default_threads())
-        times = []
         nth = oracle.default_threads()
+        for _ in range(min(args.warmup, 1)):
+            oracle_step(inp, nth)
+        times = []
         for _ in range(args.steps):
             t0 = time.perf_counter()
             oracle_step(inp, nth)
             times.append(time.perf_counter() - t0)
         ms = 1e3 * sum(times) / len(times)
-        v = step_bytes / (ms / 1e3) / 1e9
+        v = cpu_bytes / (ms / 1e3) / 1e9
         line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "GB/s", "n_gpus": args.gpus,
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config,
-                "elements_per_s": 2 * elems / (ms / 1e3),
-                "cpu_baseline": {"value": v, "unit": "GB/s", "cores": nth, "kind": "oracle",
-                                 "sample": f"whole {wl.name} step per timed step (full + mean paths)"},
+                "elements_per_s": 2 * cpu_wl.scan_elements() / (ms / 1e3),
+                "cpu_baseline": {"value": v, "unit": "GB/s", "cores": nth, "kind": "oracle", "sample": cpu_sample},
                 "e2e": {"value": v, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
         print(json.dumps(line))
         return
@@ -617,7 +722,7 @@ def main():
     if world > 1:
         import torch
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
-    res, inp = run_ours(args, wl, rank, world, local_rank)
+    res, _ = run_ours(args, wl, rank, world, local_rank)
     if rank != 0:
         if world > 1:
             import torch
@@ -626,6 +731,9 @@ def main():
 
     ms = res["total_ms"] / args.steps
     value = job_throughput(step_bytes, world, ms)
+    config["l2"] = ("flushed before every step (2x L2 write, outside the timed events)" if res["flushed"] else
+                    "not flushed: a step's inputs are far larger than L2; steps run back to back")
+    config["timed_region_s"] = res["total_ms"] / 1e3
     kb = kernel_bytes(wl)
     peak, peak_src = measured_peaks()
     per = {}
@@ -640,7 +748,8 @@ def main():
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "f32", "data": "synthetic (seeded; shared map + per-channel noise)",
+        "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic (seeded; shared map + per-channel noise, the workload recipe drawn on the device)",
         "config": config,
         "elements_per_s": world * 2 * elems / (ms / 1e3),
         "frac_of_peak": value / peak,
@@ -674,18 +783,21 @@ def main():
                                   "frac_of_peak": kb["mean_scan"] / (us / 1e6) / 1e9 / peak}
                          for G, us in res["grouped_us"].items()},
         "clocks": res["clocks"],
+        # every workload of the configuration list, kernel by kernel (inputs drawn
+        # on the device with the same recipe; the headline above is one of them)
+        "configs": res["configs"],
         "e2e": {"value": job_throughput(step_bytes, world, res["e2e_ms"] / args.e2e_steps), "unit": "GB/s",
                 "ms_per_step": res["e2e_ms"] / args.e2e_steps,
                 "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"],
                 "pipelined": "one packed H2D copy and two D2H copies per step, overlapping the neighbouring "
                              "steps' kernels (two buffer sets, copy streams ordered by events)"},
     }
-    if not args.no_cpu_baseline and world >= 1 and rank == 0:
-        times, nth = time_oracle(inp, target_s=10.0)
+    if not args.no_cpu_baseline and world == 1 and rank == 0:
+        times, nth = time_oracle(workloads.make_inputs(cpu_wl), target_s=10.0)
         cms = 1e3 * statistics.mean(times)
-        line["cpu_baseline"] = {"value": step_bytes / (cms / 1e3) / 1e9, "unit": "GB/s", "cores": nth,
+        line["cpu_baseline"] = {"value": cpu_bytes / (cms / 1e3) / 1e9, "unit": "GB/s", "cores": nth,
                                 "kind": "oracle", "ms_per_step": cms,
-                                "sample": f"{len(times)} whole {wl.name} steps (full + mean paths), ~10 s"}
+                                "sample": f"{len(times)} oracle steps, ~10 s: {cpu_sample}"}
     print(json.dumps(line))
     if world > 1:
         import torch

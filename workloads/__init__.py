@@ -209,3 +209,36 @@ def make_inputs(wl: Workload, seed: int | None = None, *, sigma: float | None = 
 def small_case(B=1, D=5, N=3, H=3, W=4, dtype="f32", sigma=0.1, seed=7) -> Workload:
     """A tiny ad-hoc workload for brute-force and edge-case tests."""
     return Workload(f"tiny_b{B}_d{D}_n{N}_{H}x{W}_{dtype}", B, D, N, H, W, dtype, sigma, seed)
+
+
+def make_device_inputs(wl: Workload, device, seed: int | None = None, params: str = "paper") -> dict:
+    """The recipe of make_inputs drawn on the GPU with torch's generator (same
+    distributions and shapes, different values): for timing runs over many and
+    large workloads, where only the sizes and the value ranges matter.  Parity
+    tests use make_inputs.  Returns torch tensors x, draw, Bs, Cs (storage
+    dtype) and A, Dskip, bias (fp32)."""
+    import torch
+
+    if params not in PARAMS:
+        raise ValueError(f"params must be one of {PARAMS}, not {params!r}")
+    seed = wl.seed if seed is None else seed
+    B, K, D, N, H, W, L = wl.B, wl.K, wl.D, wl.N, wl.H, wl.W, wl.L
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    f = dict(device=device, dtype=torch.float32, generator=gen)
+    x = torch.randn(B, 1, H, W, **f) + wl.sigma * torch.randn(B, D, H, W, **f)
+    draw = 0.5 * torch.randn(B, K, D, L, **f)
+    Bs = torch.randn(B, K, N, L, **f)
+    Cs = torch.randn(B, K, N, L, **f)
+    u01 = torch.rand(K * D, device=device, dtype=torch.float64, generator=gen)
+    dt = torch.exp(math.log(1e-3) + u01 * (math.log(1e-1) - math.log(1e-3)))
+    bias = (dt + torch.log(-torch.expm1(-dt))).float()
+    if params == "random":
+        A = -(0.5 + 2.5 * torch.rand(K * D, N, **f))
+        Dskip = 0.5 + torch.rand(K * D, **f)
+    else:
+        A = -(torch.arange(N, device=device, dtype=torch.float32) + 1.0).repeat(K * D, 1).contiguous()
+        Dskip = torch.ones(K * D, device=device, dtype=torch.float32)
+    sdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    return dict(x=x.contiguous().to(sdt), draw=draw.to(sdt), Bs=Bs.to(sdt), Cs=Cs.to(sdt), A=A, Dskip=Dskip,
+                bias=bias)
