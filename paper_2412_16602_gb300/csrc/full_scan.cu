@@ -1042,23 +1042,25 @@ __global__ void __launch_bounds__(ChunkLayout<T, CS>::THREADS, CS::MINB) full_ch
 // cooperatively one stage ahead), A * log2 e sits in swizzled shared memory or
 // in registers, and the state loop is outermost within a 4-step block.  One
 // barrier per stage.
-template <int G_, int DT_, int TS_, int MINB_, int V_ = 0>
+template <int G_, int DT_, int TS_, int MINB_, int V_ = 0, int NSTG_ = 3>
 struct StreamShape {
     // V: 0 = A in shared memory, ordered B/C reads and exponentials;
     //    1 = A in registers, ordered reads, exponentials and FMAs; 2 = A in registers, free order
-    static constexpr int G = G_, DT = DT_, TS = TS_, MINB = MINB_, V = V_;
+    static constexpr int G = G_, DT = DT_, TS = TS_, MINB = MINB_, V = V_, NSTG = NSTG_;
 };
 
 template <typename T, class SS>
 struct StreamLayout {
     // TS = 0: one 16-byte chunk per row and stage (4 fp32 or 8 bf16 steps)
-    static constexpr int G = SS::G, DT = SS::DT, TS = SS::TS ? SS::TS : 16 / (int)sizeof(T), NP = 16, NSTG = 3;
+    static constexpr int G = SS::G, DT = SS::DT, TS = SS::TS ? SS::TS : 16 / (int)sizeof(T), NP = 16, NSTG = SS::NSTG;
     static constexpr int THREADS = G * DT, NG = NP / G;
     static constexpr bool F32 = sizeof(T) == 4;
-    static constexpr int PAD = 16 / (int)sizeof(T);
-    static constexpr int RS = TS + PAD;                 // raw row stride (elements), 16-byte aligned rows
+    // raw row stride (elements): rows of one 16-byte chunk need no padding (a
+    // quarter warp's 128-bit reads of consecutive rows hit distinct banks);
+    // longer rows are padded by one chunk
+    static constexpr int RS = TS * (int)sizeof(T) == 16 ? TS : TS + 16 / (int)sizeof(T);
     static constexpr int SLOT = (2 * DT + 2 * NP) * RS;  // u, delta, B, C rows of one stage
-    static constexpr int FS = TS + 4;                    // fp32 row stride
+    static constexpr int FS = F32 ? RS : TS + 4;         // fp32 row stride
     static constexpr size_t raw_bytes = a16((size_t)NSTG * SLOT * sizeof(T));
     // bf16: fp32 delta rows [2][DT][FS] and fp32 B, C rows [2][2 NP][FS] (two
     // slots: the stage being computed and the next); fp32 uses the raw rows
@@ -1067,7 +1069,7 @@ struct StreamLayout {
     static constexpr size_t a2_off = fbc_off + (F32 ? 0 : (size_t)2 * 2 * NP * FS * 4);
     static constexpr int V = SS::V;
     static constexpr size_t bytes = a2_off + (V == 0 ? (size_t)DT * NP * 4 : 0);
-    static_assert(TS % (4 * G) == 0 && TS * sizeof(T) % 16 == 0 && DT % 32 == 0 && (G == 1 || G == 2),
+    static_assert(TS % (4 * G) == 0 && TS * sizeof(T) % 16 == 0 && DT % 32 == 0 && (G == 1 || G == 2) && NSTG >= 3,
                   "stream tile shape");
     static_assert(V != 0 || G == 1, "shared-memory A rows are one lane per channel");
     static_assert(!F32 || RS == FS, "fp32 rows are rewritten in place");
@@ -1254,6 +1256,189 @@ __global__ void __launch_bounds__(StreamLayout<T, SS>::THREADS, SS::MINB) full_s
     cp_async_wait<0>();
 }
 
+// ---------------------------------------------------- packed streaming variant
+// For many channel rows (no L-chunking), with the state update on the packed
+// f32x2 operations: G lanes per channel (1, 2 or 4) each own 16 / G states,
+// held as pairs (n, n+1).  Per step and pair: Abar = 2^(delta A log2 e) (one
+// packed product, two ex2), Bbar u = (delta u) B (one packed product),
+// h = Abar h + Bbar u and the output sum C.h (two packed FMAs), so a state
+// update costs two FMA-pipe instructions and one ex2 instead of four and one.
+// The stage's B and C rows are transposed once per stage into fp32 [t][B..C]
+// rows, so a lane reads the pairs of its states at step t as 128-bit
+// broadcast loads; delta = softplus(raw + bias) is computed one stage ahead
+// on the packed operations as well (the G lanes of a channel split the
+// stage's steps).  cp.async ring of 8-step stages, one barrier per stage.
+template <int G_, int DT_, int MINB_, int TS_ = 8, int NSTG_ = 3>
+struct PackedShape {
+    // TS = 0: one 16-byte chunk per row and stage (4 fp32 or 8 bf16 steps)
+    static constexpr int G = G_, DT = DT_, MINB = MINB_, TS = TS_, NSTG = NSTG_;
+};
+
+template <typename T, class PS>
+struct PackedLayout {
+    static constexpr int G = PS::G, DT = PS::DT, MINB = PS::MINB, NP = 16, NG = NP / G, NPR = NG / 2;
+    static constexpr int TS = PS::TS ? PS::TS : 16 / (int)sizeof(T), NSTG = PS::NSTG;
+    static constexpr int THREADS = G * DT;
+    static constexpr bool F32 = sizeof(T) == 4;
+    // raw row stride (elements): rows of one 16-byte chunk need no padding (a
+    // quarter warp's 128-bit reads of consecutive rows hit distinct banks);
+    // longer rows are padded by one chunk
+    static constexpr int RS = TS * (int)sizeof(T) == 16 ? TS : TS + 16 / (int)sizeof(T);
+    static constexpr int SLOT = (2 * DT + 2 * NP) * RS;  // u, delta, B, C rows of one stage
+    static constexpr int FS = F32 ? RS : TS + 4;         // fp32 delta row stride
+    static constexpr int BCW = 2 * NP;                   // floats per transposed step: B[0..15], C[0..15]
+    static constexpr size_t raw_bytes = a16((size_t)NSTG * SLOT * sizeof(T));
+    // bf16: fp32 delta rows [2][DT][FS]; fp32 rewrites the raw delta rows in place
+    static constexpr size_t fdl_off = raw_bytes;
+    static constexpr size_t bct_off = fdl_off + (F32 ? 0 : (size_t)2 * DT * FS * 4);  // fp32 [2][TS][BCW]
+    static constexpr size_t bytes = bct_off + (size_t)2 * TS * BCW * 4;
+    static_assert((G == 1 || G == 2 || G == 4) && DT % 32 == 0 && THREADS % 32 == 0 && TS % 4 == 0 &&
+                      (TS / G) % 2 == 0 && NSTG >= 3, "packed tile shape");
+    static_assert(!F32 || RS == FS, "fp32 delta rows are rewritten in place");
+};
+
+template <typename T, class PS>
+__global__ void __launch_bounds__(PackedLayout<T, PS>::THREADS, PS::MINB) full_packed_kernel(const FullParams p) {
+    pdl_wait();
+    pdl_launch_dependents();
+    using LY = PackedLayout<T, PS>;
+    constexpr int G = LY::G, NG = LY::NG, NPR = LY::NPR, DT = LY::DT, TS = LY::TS, NP = 16, NSTG = LY::NSTG,
+                  RS = LY::RS, SLOT = LY::SLOT, FS = LY::FS, BCW = LY::BCW, THREADS = LY::THREADS;
+    extern __shared__ __align__(16) unsigned char smem[];
+    T* raw = reinterpret_cast<T*>(smem);
+
+    const int c = threadIdx.x / G, g = threadIdx.x % G;
+    const int tile = blockIdx.x;
+    const int bk = tile / p.tiles_per_bk;
+    const int d0 = (tile % p.tiles_per_bk) * DT;
+    const int k = bk % p.K;
+    const int d = d0 + c;
+    const bool cval = d < p.D;
+    const int nrows = min(DT, p.D - d0);
+    const size_t row0 = (size_t)bk * p.D + d0;
+    const size_t bcrow0 = (size_t)bk * p.N;
+    const int L = p.L;
+    const int nst = (L + TS - 1) / TS;
+#pragma unroll
+    for (int q = 0; q < NSTG - 1; ++q) {
+        if (q < nst) load_tile<T, NP, DT, TS, RS, THREADS, true>(p, raw + q * SLOT, row0, bcrow0, nrows, q * TS);
+        cp_async_commit();
+    }
+    const float bias = cval ? p.bias[(size_t)k * p.D + d] : 0.0f;
+    const float dsk = cval ? p.Dskip[(size_t)k * p.D + d] : 0.0f;
+    const float* Ad = p.A + ((size_t)k * p.D + d) * p.N;
+    float2 A2[NPR], h[NPR];
+#pragma unroll
+    for (int i = 0; i < NPR; ++i) {
+        const int n = g * NG + 2 * i;
+        A2[i] = make_float2((cval && n < p.N) ? Ad[n] * kLog2e : 0.0f, (cval && n + 1 < p.N) ? Ad[n + 1] * kLog2e : 0.0f);
+        h[i] = make_float2(0.0f, 0.0f);
+    }
+    T* yrow = static_cast<T*>(p.y) + (row0 + c) * (size_t)L;
+
+    auto fdl_of = [&](int st) -> float* {
+        if constexpr (LY::F32) return reinterpret_cast<float*>(raw + (st % NSTG) * SLOT + (DT + c) * RS);
+        else return reinterpret_cast<float*>(smem + LY::fdl_off) + ((st & 1) * DT + c) * FS;
+    };
+    auto bct_of = [&](int st) -> float* { return reinterpret_cast<float*>(smem + LY::bct_off) + (st & 1) * TS * BCW; };
+    // stage st: delta = softplus(raw + bias) (Eq. 6) of this lane's share of its
+    // channel's steps, in fp32; the B and C rows transposed to fp32 [t][B..C]
+    auto prepare = [&](int st) {
+        constexpr int SPL = TS / G;  // steps per lane
+        const T* rd = raw + (st % NSTG) * SLOT + (DT + c) * RS + g * SPL;
+        float* fd = fdl_of(st) + g * SPL;
+#pragma unroll
+        for (int j = 0; j < SPL; j += 2) {
+            float2 v = make_float2(io<T>::cvt(rd[j]) + bias, io<T>::cvt(rd[j + 1]) + bias);
+            if (p.softplus_on) v = softplus2(v);
+            *reinterpret_cast<float2*>(fd + j) = v;
+        }
+        const T* rb = raw + (st % NSTG) * SLOT + 2 * DT * RS;  // B rows, then C rows, [2 NP][RS]
+        float* bo = bct_of(st);
+        for (int i = threadIdx.x; i < BCW * TS; i += THREADS) {
+            const int r = i % BCW, t = i / BCW;
+            bo[t * BCW + r] = io<T>::cvt(rb[r * RS + t]);
+        }
+    };
+    cp_async_wait<NSTG - 2>();
+    __syncthreads();
+    prepare(0);
+    for (int s = 0; s < nst; ++s) {
+        const int l0 = s * TS;
+        const int nvalid = min(TS, L - l0);
+        cp_async_wait<NSTG - 3>();  // stages <= s+1 have landed
+        __syncthreads();            // ... for every thread; stage s is prepared
+        if (s + NSTG - 1 < nst)
+            load_tile<T, NP, DT, TS, RS, THREADS, true>(p, raw + ((s + NSTG - 1) % NSTG) * SLOT, row0, bcrow0, nrows,
+                                                        l0 + (NSTG - 1) * TS);
+        cp_async_commit();
+        if (s + 1 < nst) prepare(s + 1);
+        const T* ru = raw + (s % NSTG) * SLOT + c * RS;
+        const float* fd = fdl_of(s);
+        const float* bct = bct_of(s) + g * NG;  // this lane's B states of step 0 (C at + NP)
+#pragma unroll 1
+        for (int t0 = 0; t0 < TS; t0 += 4) {
+            float u4[4], d4[4];
+            load4(ru + t0, u4);
+            load4(fd + t0, d4);
+            float yp[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float2 dd = make_float2(d4[j], d4[j]);
+                const float du = d4[j] * u4[j];
+                const float2 uu = make_float2(du, du);
+                const float* bt = bct + (t0 + j) * BCW;
+                float2 ya = make_float2(0.0f, 0.0f);
+#pragma unroll
+                for (int q = 0; q < NG / 4; ++q) {
+                    const float4 b = *reinterpret_cast<const float4*>(bt + 4 * q);
+                    const float4 cc = *reinterpret_cast<const float4*>(bt + NP + 4 * q);
+                    {
+                        const float2 x = __fmul2_rn(dd, A2[2 * q]);
+                        const float2 a = make_float2(ex2(x.x), ex2(x.y));
+                        h[2 * q] = __ffma2_rn(a, h[2 * q], __fmul2_rn(uu, make_float2(b.x, b.y)));
+                        ya = __ffma2_rn(make_float2(cc.x, cc.y), h[2 * q], ya);
+                    }
+                    {
+                        const float2 x = __fmul2_rn(dd, A2[2 * q + 1]);
+                        const float2 a = make_float2(ex2(x.x), ex2(x.y));
+                        h[2 * q + 1] = __ffma2_rn(a, h[2 * q + 1], __fmul2_rn(uu, make_float2(b.z, b.w)));
+                        ya = __ffma2_rn(make_float2(cc.z, cc.w), h[2 * q + 1], ya);
+                    }
+                }
+                yp[j] = ya.x + ya.y;
+            }
+            // y = sum over the channel's lanes + D u, stored straight from registers
+            if constexpr (G == 1) {
+                float o[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) o[j] = fmaf(dsk, u4[j], yp[j]);
+                if (cval) store_row<T, 4>(yrow + l0 + t0, o, nvalid - t0, p.vec);
+            } else if constexpr (G == 2) {
+                // lane g keeps steps 2g and 2g+1
+                const float k0 = g ? yp[2] : yp[0], k1 = g ? yp[3] : yp[1];
+                const float s0 = g ? yp[0] : yp[2], s1 = g ? yp[1] : yp[3];
+                float o[2];
+                o[0] = fmaf(dsk, g ? u4[2] : u4[0], k0 + __shfl_xor_sync(0xffffffffu, s0, 1));
+                o[1] = fmaf(dsk, g ? u4[3] : u4[1], k1 + __shfl_xor_sync(0xffffffffu, s1, 1));
+                if (cval) store_row<T, 2>(yrow + l0 + t0 + 2 * g, o, nvalid - t0 - 2 * g, p.vec);
+            } else {
+                const bool hi = g & 2;
+                float k0 = hi ? yp[2] : yp[0], k1 = hi ? yp[3] : yp[1];
+                const float s0 = hi ? yp[0] : yp[2], s1 = hi ? yp[1] : yp[3];
+                k0 += __shfl_xor_sync(0xffffffffu, s0, 2);
+                k1 += __shfl_xor_sync(0xffffffffu, s1, 2);
+                const bool odd = g & 1;
+                const float kk = odd ? k1 : k0, ss = odd ? k0 : k1;
+                float o[1];
+                o[0] = fmaf(dsk, sel4(u4, g), kk + __shfl_xor_sync(0xffffffffu, ss, 1));
+                if (cval) store_row<T, 1>(yrow + l0 + t0 + g, o, nvalid - t0 - g, false);
+            }
+        }
+    }
+    cp_async_wait<0>();
+}
+
 // Launch 2 of the chunked variant: the inclusive state after every chunk,
 // inc_m = 2^(A_n log2 e S_m) inc_{m-1} + H_m from inc_{-1} = 0, for every
 // (channel, state) of a tile.  The chain is short in arithmetic but long in
@@ -1380,14 +1565,28 @@ KernelInfo stream_info() {
     return {attr_err == cudaSuccess ? fn : nullptr, LY::bytes, LY::G, LY::DT, LY::THREADS, LY::TS};
 }
 
+template <typename T, class PS>
+KernelInfo packed_info() {
+    using LY = PackedLayout<T, PS>;
+    const void* fn = reinterpret_cast<const void*>(&full_packed_kernel<T, PS>);
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [&] {
+        attr_err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LY::bytes);
+    });
+    return {attr_err == cudaSuccess ? fn : nullptr, LY::bytes, LY::G, LY::DT, LY::THREADS, LY::TS};
+}
+
 // Tile shapes per padded state count, in order of preference (fewest lanes
 // per channel first).  The zero-order-hold variant uses the first shape.
-int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 16; }
+int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 19; }
 constexpr int kLanesShape = 7;   // index of the lane-per-state variant (N <= 16 padded to 16)
 constexpr int kChunkShape = 8;   // first index of the three-launch chunked variant (shapes 8 to 11)
 bool is_chunk_shape(int np, int shape) { return np == 16 && shape >= kChunkShape && shape < kChunkShape + 4; }
 constexpr int kStreamShape = 12;  // first index of the streaming one-lane variant (shapes 12 to 15)
 bool is_stream_shape(int np, int shape) { return np == 16 && shape >= kStreamShape && shape < kStreamShape + 4; }
+constexpr int kPackedShape = 16;  // first index of the packed streaming variant (shapes 16 to 18: G = 1, 2, 4)
+bool is_packed_shape(int np, int shape) { return np == 16 && shape >= kPackedShape && shape < kPackedShape + 3; }
 
 template <typename T, bool ZOH>
 KernelInfo pick_t(int np, int shape) {
@@ -1416,6 +1615,9 @@ KernelInfo pick_t(int np, int shape) {
         case 13: return stream_info<T, StreamShape<1, 64, 8, 8, 0>>();
         case 14: return stream_info<T, StreamShape<1, 128, 8, 4, 2>>();
         case 15: return stream_info<T, StreamShape<2, 64, 8, 6, 2>>();
+        case 16: return packed_info<T, PackedShape<1, 128, 5, 8, 3>>();
+        case 17: return packed_info<T, PackedShape<2, 64, 5, 8, 3>>();
+        case 18: return packed_info<T, PackedShape<4, 32, 5, 8, 3>>();
         default: return info_for<T, 16, Shape<1, 128, 0, 3, 7>, ZOH>();
         }
     }
@@ -1469,7 +1671,7 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
         return VMB_OK;
     };
     // Rules measured on GB300 over the benchmark workloads: 16 states, at least
-    // 256 channel rows per SM and L >= 128 -> the streaming kernel; otherwise plenty of
+    // 256 channel rows per SM and L >= 128 -> the packed streaming kernel; otherwise plenty of
     // rows -> one lane per channel; a fair number -> two lanes; too few -> cut L into
     // chunks: the three-launch variant (two lanes per channel, 32-step chunks)
     // while a grid of 64-step one-lane chunks would fit in two waves, else
@@ -1491,9 +1693,9 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
             n_chunks = (int)(want < mx ? want : mx);
         }
     } else if (np == 16 && rows >= 256LL * sms && a.L >= 128) {
-        // many rows: the streaming one-lane kernel, one pass over L (on very
-        // short sequences its stage prologue does not pay off)
-        shape = kStreamShape;
+        // many rows: the packed streaming one-lane kernel, one pass over L (on
+        // very short sequences its stage prologue does not pay off)
+        shape = kPackedShape;
         if ((st = info(shape, &ki, &res)) != VMB_OK) return st;
     } else {
         const ShapeRoles r = roles(np);
@@ -1561,7 +1763,7 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
         }
     }
     if (is_chunk_shape(np, shape)) n_chunks = (a.L + ki.ts - 1) / ki.ts;  // chunks of exactly ts steps
-    if (is_stream_shape(np, shape)) n_chunks = 1;                       // one pass over L
+    if (is_stream_shape(np, shape) || is_packed_shape(np, shape)) n_chunks = 1;  // one pass over L
     if (n_chunks < 1) n_chunks = 1;
     ScanPlan p{};
     p.np = np;

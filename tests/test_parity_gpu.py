@@ -179,7 +179,7 @@ def test_lookback_wait_times_out_cleanly(mean, force_plan):
 
 
 @pytest.mark.parametrize("plan", ["0", "1", "2", "3", "4", "5", "6", "7", "8", "9", "10", "11", "12", "13", "14", "15",
-                                  "0,3", "3,5", "4,2", "5,4", "6,7", "7,3", "7,6"])
+                                  "16", "17", "18", "0,3", "3,5", "4,2", "5,4", "6,7", "7,3", "7,6"])
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
 def test_every_tile_shape(plan, dt, force_plan):
     """Each tile shape of the full scan (and forced L-chunking) against the oracle."""
