@@ -657,7 +657,7 @@ def selection_summary(us, wl, peak, R=6):
     bytes_ = s * (2 * wl.B * 4 * wl.D * wl.L + 2 * wl.B * 4 * wl.N * wl.L) + 4 * 4 * (2 * wl.N + 2 * R) * wl.D
     gbs = bytes_ / (us / 1e6) / 1e9
     return {"us": us, "algorithmic_bytes": bytes_, "gbs": gbs, "frac_of_peak": gbs / peak, "rank": R,
-            "kernel": "CUDA-core FMA (no tensor cores yet)"}
+            "kernel": "tcgen05.mma kind::tf32 (three-product tf32 split for fp32 accuracy), accumulator in TMEM"}
 
 
 def paper_style_summary(ps, peak):

@@ -5,12 +5,21 @@
 //   z[r] = sum_d Wz[k,r,d] u[b,k,d,l],          delta_raw[b,k,d,l] = sum_r Wup[k,d,r] z[r]
 // (the printed s_Delta = Broadcast_D(Linear_1(u)) is R = 1 with unit Wup).
 //
-// CUDA-core version: a thread owns one step of one (b, k) and accumulates the
-// 2N + R projections over the channels (u read coalesced across the steps of a
-// warp; the weights of a block of channels staged in shared memory, transposed
-// so that one channel's N or R weights are one broadcast 128-bit read), then
-// writes B and C and expands z into the D raw Deltas.
+// Per (b, k) this is one dense contraction, P = W u with W = [WB; WC; Wz]
+// ([2N + R, D]) and u ([D, L]), followed by a rank-R expansion.  It runs on the
+// fifth-generation tensor cores: a CTA of 128 threads owns 128 steps of one
+// (b, k) (the MMA's M = 128 rows are steps, one TMEM lane each), the output
+// columns are B (0..15), C (16..31) and z (32..47) (N = 48), and the D channels
+// are the reduction dimension, staged 32 at a time.  Operands are fp32 in the
+// tensor cores' tf32 format; to keep fp32 accuracy each value is split into a
+// tf32 head and a tf32 tail (x = hi + lo, both exact in fp32) and the product is
+// accumulated as hi.hi + hi.lo + lo.hi in fp32 (the lo.lo term is below fp32
+// resolution).  bf16 inputs are exact in tf32 and need no tail.  The
+// accumulator lives in TMEM; each thread reads back its step's 48 values and
+// writes B, C and the D raw Deltas (z expanded through Wup in registers).
 #include <stdint.h>
+
+#include <mutex>
 
 #include "vmb_common.cuh"
 #include "vmb_internal.h"
@@ -18,9 +27,13 @@
 namespace vmb {
 namespace {
 
-constexpr int kSelThreads = 128;  // steps per CTA
-constexpr int kSelChunk = 64;     // channels whose weights are staged at a time
-constexpr int kSelMaxN = 16, kSelMaxR = 16;
+constexpr int kSelThreads = 128;  // steps per CTA = MMA rows = TMEM lanes
+constexpr int kSelKC = 32;        // channels per staged chunk (four MMA k-steps of 8)
+constexpr int kSelCols = 48;      // MMA N: B at columns 0..15, C at 16..31, z at 32..47
+constexpr int kSelTmemCols = 64;  // TMEM allocation (a power of two >= 32)
+constexpr int kSelRP = 16;        // z values per step held in registers (R <= 16)
+constexpr int kSelDB = 256;       // Wup rows staged at a time in the epilogue
+constexpr int kSelDrain = 8;      // chunks (256 channels) accumulated in TMEM before a drain to registers
 
 struct SelParams {
     const void* u;
@@ -35,122 +48,258 @@ struct SelParams {
     int nlb;  // step blocks per (b, k)
 };
 
-template <typename T, int NP, int RP>
-__global__ void __launch_bounds__(kSelThreads) selection_kernel(const SelParams p) {
-    pdl_wait();
-    pdl_launch_dependents();
-    // [chunk][NP] transposed B and C weights, [chunk][RP] transposed Wz, [chunk][RP] Wup
-    __shared__ __align__(16) float sB[kSelChunk][NP];
-    __shared__ __align__(16) float sC[kSelChunk][NP];
-    __shared__ __align__(16) float sZ[kSelChunk][RP];
-    __shared__ __align__(16) float sU[kSelChunk][RP];
-    const long long bk = blockIdx.x / p.nlb;
-    const int k = (int)(bk % p.K);
-    const int l = (int)(blockIdx.x % p.nlb) * kSelThreads + threadIdx.x;
-    const bool lv = l < p.L;
-    const int D = p.D, N = p.N, R = p.R, L = p.L;
-    const T* ucol = static_cast<const T*>(p.u) + (size_t)bk * D * L + (lv ? l : 0);
-    float aB[NP], aC[NP], aZ[RP];
-#pragma unroll
-    for (int n = 0; n < NP; ++n) aB[n] = aC[n] = 0.0f;
-#pragma unroll
-    for (int r = 0; r < RP; ++r) aZ[r] = 0.0f;
-    for (int d0 = 0; d0 < D; d0 += kSelChunk) {
-        const int dn = min(kSelChunk, D - d0);
-        __syncthreads();  // the previous chunk's weights are no longer read
-        for (int i = threadIdx.x; i < kSelChunk * NP; i += kSelThreads) {
-            const int j = i / NP, n = i % NP;
-            const bool ok = j < dn && n < N;
-            sB[j][n] = ok ? p.WB[((size_t)k * N + n) * D + d0 + j] : 0.0f;
-            sC[j][n] = ok ? p.WC[((size_t)k * N + n) * D + d0 + j] : 0.0f;
-        }
-        for (int i = threadIdx.x; i < kSelChunk * RP; i += kSelThreads) {
-            const int j = i / RP, r = i % RP;
-            const bool ok = j < dn && r < R;
-            sZ[j][r] = ok ? p.Wz[((size_t)k * R + r) * D + d0 + j] : 0.0f;
-        }
-        __syncthreads();
-        if (lv) {
-            for (int j = 0; j < dn; ++j) {
-                const float x = io<T>::ld(ucol + (size_t)(d0 + j) * L);
-#pragma unroll
-                for (int n = 0; n < NP; n += 4) {
-                    const float4 wb = *reinterpret_cast<const float4*>(&sB[j][n]);
-                    const float4 wc = *reinterpret_cast<const float4*>(&sC[j][n]);
-                    aB[n] = fmaf(wb.x, x, aB[n]);
-                    aB[n + 1] = fmaf(wb.y, x, aB[n + 1]);
-                    aB[n + 2] = fmaf(wb.z, x, aB[n + 2]);
-                    aB[n + 3] = fmaf(wb.w, x, aB[n + 3]);
-                    aC[n] = fmaf(wc.x, x, aC[n]);
-                    aC[n + 1] = fmaf(wc.y, x, aC[n + 1]);
-                    aC[n + 2] = fmaf(wc.z, x, aC[n + 2]);
-                    aC[n + 3] = fmaf(wc.w, x, aC[n + 3]);
-                }
-#pragma unroll
-                for (int r = 0; r < RP; r += 4) {
-                    const float4 wz = *reinterpret_cast<const float4*>(&sZ[j][r]);
-                    aZ[r] = fmaf(wz.x, x, aZ[r]);
-                    aZ[r + 1] = fmaf(wz.y, x, aZ[r + 1]);
-                    aZ[r + 2] = fmaf(wz.z, x, aZ[r + 2]);
-                    aZ[r + 3] = fmaf(wz.w, x, aZ[r + 3]);
-                }
-            }
-        }
-    }
-    if (lv) {
-        T* ob = static_cast<T*>(p.Bs) + (size_t)bk * N * L + l;
-        T* oc = static_cast<T*>(p.Cs) + (size_t)bk * N * L + l;
-#pragma unroll
-        for (int n = 0; n < NP; ++n) {
-            if (n < N) {
-                ob[(size_t)n * L] = io<T>::to(aB[n]);
-                oc[(size_t)n * L] = io<T>::to(aC[n]);
-            }
-        }
-    }
-    // the raw Deltas: expand z through Wup, a block of channels at a time
-    T* od = static_cast<T*>(p.dr) + (size_t)bk * D * L + (lv ? l : 0);
-    for (int d0 = 0; d0 < D; d0 += kSelChunk) {
-        const int dn = min(kSelChunk, D - d0);
-        __syncthreads();
-        for (int i = threadIdx.x; i < kSelChunk * RP; i += kSelThreads) {
-            const int j = i / RP, r = i % RP;
-            sU[j][r] = (j < dn && r < R) ? p.Wup[((size_t)k * D + d0 + j) * R + r] : 0.0f;
-        }
-        __syncthreads();
-        if (lv) {
-            for (int j = 0; j < dn; ++j) {
-                float s = 0.0f;
-#pragma unroll
-                for (int r = 0; r < RP; r += 4) {
-                    const float4 w = *reinterpret_cast<const float4*>(&sU[j][r]);
-                    s = fmaf(w.x, aZ[r], s);
-                    s = fmaf(w.y, aZ[r + 1], s);
-                    s = fmaf(w.z, aZ[r + 2], s);
-                    s = fmaf(w.w, aZ[r + 3], s);
-                }
-                od[(size_t)(d0 + j) * L] = io<T>::to(s);
-            }
-        }
-    }
+// Shared memory: the two operands of one chunk in the tensor cores' K-major
+// layout without swizzle.  A core matrix is 8 rows x 16 bytes (4 tf32) stored
+// as 128 contiguous bytes; core matrix (row group g, channel quad c) of an
+// operand with G row groups sits at ((c * G) + g) * 128 bytes, so the stride
+// between row groups is 128 bytes and between channel quads G * 128 bytes.
+struct SelLayout {
+    static constexpr size_t a_bytes = (size_t)kSelThreads * kSelKC * 4;  // u^T rows (steps): 16 KB
+    static constexpr size_t b_bytes = (size_t)kSelCols * kSelKC * 4;     // W rows (outputs): 6 KB
+    static constexpr size_t a_hi = 0, a_lo = a_bytes, b_hi = 2 * a_bytes, b_lo = 2 * a_bytes + b_bytes;
+    static constexpr size_t bytes = 2 * a_bytes + 2 * b_bytes;
+    static_assert((size_t)kSelDB * kSelRP * 4 <= bytes, "the epilogue's Wup rows reuse the operand area");
+};
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+// Round to the nearest tf32 value (10 stored mantissa bits; the low 13 bits become zero).
+__device__ __forceinline__ float to_tf32(float x) {
+    uint32_t r;
+    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+    return __uint_as_float(r);
 }
 
-template <typename T, int NP>
-const void* sel_fn_r(int rp) {
-    switch (rp) {
-    case 4: return reinterpret_cast<const void*>(&selection_kernel<T, NP, 4>);
-    case 8: return reinterpret_cast<const void*>(&selection_kernel<T, NP, 8>);
-    default: return reinterpret_cast<const void*>(&selection_kernel<T, NP, 16>);
+// Shared-memory matrix descriptor of the tensor cores: start address, leading
+// (channel-quad) and stride (row-group) byte offsets, all in 16-byte units,
+// descriptor version 1, no swizzle.
+__device__ __forceinline__ uint64_t mma_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((saddr >> 4) & 0x3FFF) | ((uint64_t)((lbo >> 4) & 0x3FFF) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3FFF) << 32) | ((uint64_t)1 << 46);
+}
+
+// Instruction descriptor of kind::tf32: fp32 accumulator, tf32 A and B, both
+// K-major, N = kSelCols, M = kSelThreads.
+constexpr uint32_t kSelIdesc = (1u << 4) | (2u << 7) | (2u << 10) | ((uint32_t)(kSelCols >> 3) << 17) |
+                               ((uint32_t)(kSelThreads >> 4) << 24);
+
+__device__ __forceinline__ void mma_tf32(uint32_t tmem, uint64_t da, uint64_t db, uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem),
+        "l"(da), "l"(db), "r"(kSelIdesc), "r"(accumulate));
+}
+
+// Wait (bounded by 1 s of wall time) for the given phase of an mbarrier.
+__device__ __forceinline__ bool mbar_wait(uint32_t mbar, uint32_t phase) {
+    const uint64_t t0 = globaltimer_ns();
+    for (;;) {
+        uint32_t done;
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(done)
+            : "r"(mbar), "r"(phase)
+            : "memory");
+        if (done) return true;
+        if (globaltimer_ns() - t0 > 1000000000ull) return false;
     }
 }
 
 template <typename T>
-const void* sel_fn(int np, int rp) {
-    switch (np) {
-    case 4: return sel_fn_r<T, 4>(rp);
-    case 8: return sel_fn_r<T, 8>(rp);
-    default: return sel_fn_r<T, 16>(rp);
+__global__ void __launch_bounds__(kSelThreads) selection_kernel(const SelParams p) {
+    using LY = SelLayout;
+    constexpr bool F32 = sizeof(T) == 4;
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ uint32_t s_tmem;
+    __shared__ __align__(8) uint64_t s_mbar;
+    pdl_wait();
+    pdl_launch_dependents();
+    const int tid = threadIdx.x, warp = tid / 32;
+    const long long bk = blockIdx.x / p.nlb;
+    const int k = (int)(bk % p.K);
+    const int l = (int)(blockIdx.x % p.nlb) * kSelThreads + tid;
+    const bool lv = l < p.L;
+    const int D = p.D, N = p.N, R = p.R, L = p.L;
+
+    // TMEM accumulator (warp 0 allocates) and the MMA-completion barrier
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_addr(&s_tmem)),
+                     "n"(kSelTmemCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
     }
+    const uint32_t mbar = smem_addr(&s_mbar);
+    if (tid == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar));
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = s_tmem;
+
+    const uint32_t sbase = smem_addr(smem);
+    float* sAhi = reinterpret_cast<float*>(smem + LY::a_hi);
+    float* sAlo = reinterpret_cast<float*>(smem + LY::a_lo);
+    float* sBhi = reinterpret_cast<float*>(smem + LY::b_hi);
+    float* sBlo = reinterpret_cast<float*>(smem + LY::b_lo);
+    const T* ucol = static_cast<const T*>(p.u) + (size_t)bk * D * L + (lv ? l : 0);
+    // this thread's row of A (its step): row group tid / 8, row tid % 8
+    const int arow = (tid / 8) * 128 + (tid % 8) * 16;  // bytes within a channel quad's block
+    constexpr int AG = kSelThreads / 8, BG = kSelCols / 8;
+    bool ok = true;
+    uint32_t phase = 0;
+    // The tensor cores accumulate a run of kSelDrain chunks in TMEM; each run's
+    // sums are then added to fp32 registers, which keeps the accumulation chain
+    // inside the tensor cores short for wide maps (D up to 1536).
+    float acc[kSelCols];
+#pragma unroll
+    for (int j = 0; j < kSelCols; ++j) acc[j] = 0.0f;
+    auto drain = [&]() {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll
+        for (int c0 = 0; c0 < kSelCols; c0 += 16) {
+            uint32_t r[16];
+            const uint32_t taddr = tmem + ((uint32_t)(32 * warp) << 16) + (uint32_t)c0;
+            asm volatile(
+                "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, "
+                "[%16];"
+                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+                  "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+                : "r"(taddr));
+            asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+            for (int j = 0; j < 16; ++j) acc[c0 + j] += __uint_as_float(r[j]);
+        }
+        // the next run's first MMA overwrites the accumulator only after every warp has read it
+        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+        __syncthreads();
+    };
+    const int nchunks = (D + kSelKC - 1) / kSelKC;
+    for (int chunk = 0; chunk < nchunks; ++chunk) {
+        const int d0 = chunk * kSelKC;
+        const int dn = min(kSelKC, D - d0);
+        // u of this step over the chunk's channels (coalesced across the steps of a warp)
+        float v[kSelKC];
+#pragma unroll
+        for (int j = 0; j < kSelKC; ++j) v[j] = (lv && j < dn) ? io<T>::ld(ucol + (size_t)(d0 + j) * L) : 0.0f;
+#pragma unroll
+        for (int c = 0; c < kSelKC / 4; ++c) {
+            float hi[4], lo[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                hi[e] = F32 ? to_tf32(v[4 * c + e]) : v[4 * c + e];  // bf16 values are exact in tf32
+                lo[e] = to_tf32(v[4 * c + e] - hi[e]);
+            }
+            const int off = (c * AG * 128 + arow) / 4;
+            *reinterpret_cast<float4*>(sAhi + off) = make_float4(hi[0], hi[1], hi[2], hi[3]);
+            if constexpr (F32) *reinterpret_cast<float4*>(sAlo + off) = make_float4(lo[0], lo[1], lo[2], lo[3]);
+        }
+        // the weight rows of the chunk: B (rows 0..15), C (16..31), z (32..47), zero past N / R / D
+        for (int i = tid; i < kSelCols * kSelKC; i += kSelThreads) {
+            const int m = i / kSelKC, j = i % kSelKC;
+            float wv = 0.0f;
+            if (j < dn) {
+                if (m < 16) {
+                    if (m < N) wv = __ldg(p.WB + ((size_t)k * N + m) * D + d0 + j);
+                } else if (m < 32) {
+                    if (m - 16 < N) wv = __ldg(p.WC + ((size_t)k * N + (m - 16)) * D + d0 + j);
+                } else if (m - 32 < R) {
+                    wv = __ldg(p.Wz + ((size_t)k * R + (m - 32)) * D + d0 + j);
+                }
+            }
+            const float hi = to_tf32(wv);
+            const int off = ((j / 4) * BG * 128 + (m / 8) * 128 + (m % 8) * 16) / 4 + (j % 4);
+            sBhi[off] = hi;
+            sBlo[off] = to_tf32(wv - hi);
+        }
+        // the generic-proxy stores become visible to the tensor cores' async proxy
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncthreads();
+        if (tid == 0) {
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const int ksteps = (dn + 7) / 8;
+            for (int ks = 0; ks < ksteps; ++ks) {
+                // k-step ks covers channel quads 2 ks and 2 ks + 1
+                const uint32_t ao = (uint32_t)(2 * ks * AG * 128), bo = (uint32_t)(2 * ks * BG * 128);
+                const uint64_t ahi = mma_desc(sbase + (uint32_t)LY::a_hi + ao, AG * 128, 128);
+                const uint64_t bhi = mma_desc(sbase + (uint32_t)LY::b_hi + bo, BG * 128, 128);
+                const uint64_t blo = mma_desc(sbase + (uint32_t)LY::b_lo + bo, BG * 128, 128);
+                mma_tf32(tmem, ahi, bhi, (chunk % kSelDrain != 0 || ks > 0) ? 1u : 0u);
+                mma_tf32(tmem, ahi, blo, 1u);
+                if constexpr (F32) {
+                    const uint64_t alo = mma_desc(sbase + (uint32_t)LY::a_lo + ao, AG * 128, 128);
+                    mma_tf32(tmem, alo, bhi, 1u);
+                }
+            }
+            asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar)
+                         : "memory");
+        }
+        // the chunk's MMAs have read the operands before they are overwritten
+        // (after a wait that gave up, the rest of the tile is not waited for)
+        if (ok) ok = mbar_wait(mbar, phase);
+        phase ^= 1u;
+        // this step's sums of the run: warp w reads TMEM lanes 32 w .. 32 w + 31
+        if (chunk % kSelDrain == kSelDrain - 1 || chunk == nchunks - 1) drain();
+    }
+    if (!ok) {
+#pragma unroll
+        for (int j = 0; j < kSelCols; ++j) acc[j] = __int_as_float(0x7fffffff);  // a wait gave up: NaN outputs
+    }
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(kSelTmemCols));
+
+    if (lv) {
+        T* ob = static_cast<T*>(p.Bs) + (size_t)bk * N * L + l;
+        T* oc = static_cast<T*>(p.Cs) + (size_t)bk * N * L + l;
+#pragma unroll
+        for (int n = 0; n < 16; ++n) {
+            if (n < N) {
+                ob[(size_t)n * L] = io<T>::to(acc[n]);
+                oc[(size_t)n * L] = io<T>::to(acc[16 + n]);
+            }
+        }
+    }
+    // the raw Deltas: z expanded through Wup, kSelDB channels' rows staged at a
+    // time over the operand area (rows padded to kSelRP with zeros)
+    float* sW = reinterpret_cast<float*>(smem);
+    T* od = static_cast<T*>(p.dr) + (size_t)bk * D * L + (lv ? l : 0);
+    for (int c0 = 0; c0 < D; c0 += kSelDB) {
+        const int cn = min(kSelDB, D - c0);
+        __syncthreads();  // the previous rows are no longer read
+        for (int i = tid; i < kSelDB * kSelRP; i += kSelThreads) {
+            const int j = i / kSelRP, r = i % kSelRP;
+            sW[i] = (j < cn && r < R) ? __ldg(p.Wup + ((size_t)k * D + c0 + j) * R + r) : 0.0f;
+        }
+        __syncthreads();
+        if (lv) {
+            for (int j = 0; j < cn; ++j) {
+                const float4* w4 = reinterpret_cast<const float4*>(sW + j * kSelRP);
+                float s = 0.0f;
+#pragma unroll
+                for (int q = 0; q < kSelRP / 4; ++q) {
+                    if (4 * q < R) {
+                        const float4 w = w4[q];
+                        s = fmaf(w.x, acc[32 + 4 * q], s);
+                        s = fmaf(w.y, acc[33 + 4 * q], s);
+                        s = fmaf(w.z, acc[34 + 4 * q], s);
+                        s = fmaf(w.w, acc[35 + 4 * q], s);
+                    }
+                }
+                od[(size_t)(c0 + j) * L] = io<T>::to(s);
+            }
+        }
+    }
+}
+
+template <typename T>
+const void* sel_fn() {
+    const void* fn = reinterpret_cast<const void*>(&selection_kernel<T>);
+    static std::once_flag once;
+    static cudaError_t err = cudaSuccess;
+    std::call_once(once, [&] {
+        err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)SelLayout::bytes);
+    });
+    return err == cudaSuccess ? fn : nullptr;
 }
 
 }  // namespace
@@ -171,14 +320,14 @@ vmb_status launch_selection(const SelArgs& a, cudaStream_t stream) {
     p.R = a.R;
     p.L = a.L;
     p.nlb = (a.L + kSelThreads - 1) / kSelThreads;
-    const int np = a.N <= 4 ? 4 : a.N <= 8 ? 8 : 16;
-    const int rp = a.R <= 4 ? 4 : a.R <= 8 ? 8 : 16;
     const long long grid = (long long)a.B * a.K * p.nlb;
     if (grid > INT32_MAX) return VMB_ERR_UNSUPPORTED;
-    const void* fn = a.dtype == VMB_BF16 ? sel_fn<__nv_bfloat16>(np, rp) : sel_fn<float>(np, rp);
+    const void* fn = a.dtype == VMB_BF16 ? sel_fn<__nv_bfloat16>() : sel_fn<float>();
+    if (!fn) return VMB_ERR_CUDA;
     void* args[] = {&p};
-    return launch_kernel(fn, dim3((unsigned)grid), dim3(kSelThreads), 0, args, stream) == cudaSuccess ? VMB_OK
-                                                                                                       : VMB_ERR_CUDA;
+    return launch_kernel(fn, dim3((unsigned)grid), dim3(kSelThreads), SelLayout::bytes, args, stream) == cudaSuccess
+               ? VMB_OK
+               : VMB_ERR_CUDA;
 }
 
 }  // namespace vmb

@@ -35,6 +35,9 @@ CASES = [
     (1, 4, 200, 16, 16, 12, 11, "f32", False),  # four channel blocks, R = 16, L = 132 (two step blocks)
     (2, 4, 48, 8, 3, 9, 9, "bf16", False),
     (1, 1, 3, 1, 1, 1, 5, "f32", False),       # tiny
+    (2, 4, 256, 16, 6, 56, 56, "f32", False),  # the batch-128 workload's shape at batch 2 (8 chunks, 25 step blocks)
+    (1, 4, 192, 16, 6, 128, 128, "bf16", False),  # the 512^2 map's stage-1 shape, bf16
+    (1, 2, 1536, 16, 16, 7, 7, "f32", False),  # stage-4 width: 48 channel chunks, R = 16
 ]
 
 
