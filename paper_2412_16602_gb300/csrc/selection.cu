@@ -10,7 +10,8 @@
 // fifth-generation tensor cores: a CTA of 128 threads owns 128 steps of one
 // (b, k) (the MMA's M = 128 rows are steps, one TMEM lane each), the output
 // columns are B (0..15), C (16..31) and z (32..47) (N = 48), and the D channels
-// are the reduction dimension, staged 32 at a time.  Operands are fp32 in the
+// are the reduction dimension, staged 16 at a time (the next chunk's loads are
+// in flight while the tensor cores work on the current one).  Operands are fp32 in the
 // tensor cores' tf32 format; to keep fp32 accuracy each value is split into a
 // tf32 head and a tf32 tail (x = hi + lo, both exact in fp32) and the product is
 // accumulated as hi.hi + hi.lo + lo.hi in fp32 (the lo.lo term is below fp32
@@ -28,12 +29,12 @@ namespace vmb {
 namespace {
 
 constexpr int kSelThreads = 128;  // steps per CTA = MMA rows = TMEM lanes
-constexpr int kSelKC = 32;        // channels per staged chunk (four MMA k-steps of 8)
+constexpr int kSelKC = 16;        // channels per staged chunk (two MMA k-steps of 8)
 constexpr int kSelCols = 48;      // MMA N: B at columns 0..15, C at 16..31, z at 32..47
 constexpr int kSelTmemCols = 64;  // TMEM allocation (a power of two >= 32)
 constexpr int kSelRP = 16;        // z values per step held in registers (R <= 16)
 constexpr int kSelDB = 256;       // Wup rows staged at a time in the epilogue
-constexpr int kSelDrain = 8;      // chunks (256 channels) accumulated in TMEM before a drain to registers
+constexpr int kSelDrain = 16;     // chunks (256 channels) accumulated in TMEM before a drain to registers
 
 struct SelParams {
     const void* u;
@@ -106,7 +107,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t mbar, uint32_t phase) {
 }
 
 template <typename T>
-__global__ void __launch_bounds__(kSelThreads) selection_kernel(const SelParams p) {
+__global__ void __launch_bounds__(kSelThreads, 5) selection_kernel(const SelParams p) {
     using LY = SelLayout;
     constexpr bool F32 = sizeof(T) == 4;
     extern __shared__ __align__(128) unsigned char smem[];
@@ -175,13 +176,31 @@ __global__ void __launch_bounds__(kSelThreads) selection_kernel(const SelParams 
         __syncthreads();
     };
     const int nchunks = (D + kSelKC - 1) / kSelKC;
+    // u of this step over a chunk's channels (coalesced across the steps of a
+    // warp) and this thread's share of the chunk's weights (B rows 0..15, C rows
+    // 16..31, z rows 32..47, zero past N / R / D), all loads in flight
+    // together; the next chunk's loads are issued while the tensor cores work
+    // on the current one
+    constexpr int kWPT = kSelCols * kSelKC / kSelThreads;  // weights per thread and chunk
+    float v[kSelKC], wv[kWPT];
+    auto load_chunk = [&](int c0) {
+        const int cn = min(kSelKC, D - c0);
+#pragma unroll
+        for (int j = 0; j < kSelKC; ++j) v[j] = (lv && j < cn) ? io<T>::ld(ucol + (size_t)(c0 + j) * L) : 0.0f;
+#pragma unroll
+        for (int q = 0; q < kWPT; ++q) {
+            const int i = tid + q * kSelThreads, m = i / kSelKC, j = i % kSelKC;
+            const float* src = m < 16 ? p.WB + ((size_t)k * N + m) * D
+                                      : m < 32 ? p.WC + ((size_t)k * N + (m - 16)) * D
+                                               : p.Wz + ((size_t)k * R + (m - 32)) * D;
+            const bool in = j < cn && (m < 16 ? m < N : m < 32 ? m - 16 < N : m - 32 < R);
+            wv[q] = in ? __ldg(src + c0 + j) : 0.0f;
+        }
+    };
+    load_chunk(0);
     for (int chunk = 0; chunk < nchunks; ++chunk) {
         const int d0 = chunk * kSelKC;
         const int dn = min(kSelKC, D - d0);
-        // u of this step over the chunk's channels (coalesced across the steps of a warp)
-        float v[kSelKC];
-#pragma unroll
-        for (int j = 0; j < kSelKC; ++j) v[j] = (lv && j < dn) ? io<T>::ld(ucol + (size_t)(d0 + j) * L) : 0.0f;
 #pragma unroll
         for (int c = 0; c < kSelKC / 4; ++c) {
             float hi[4], lo[4];
@@ -194,23 +213,14 @@ __global__ void __launch_bounds__(kSelThreads) selection_kernel(const SelParams 
             *reinterpret_cast<float4*>(sAhi + off) = make_float4(hi[0], hi[1], hi[2], hi[3]);
             if constexpr (F32) *reinterpret_cast<float4*>(sAlo + off) = make_float4(lo[0], lo[1], lo[2], lo[3]);
         }
-        // the weight rows of the chunk: B (rows 0..15), C (16..31), z (32..47), zero past N / R / D
-        for (int i = tid; i < kSelCols * kSelKC; i += kSelThreads) {
-            const int m = i / kSelKC, j = i % kSelKC;
-            float wv = 0.0f;
-            if (j < dn) {
-                if (m < 16) {
-                    if (m < N) wv = __ldg(p.WB + ((size_t)k * N + m) * D + d0 + j);
-                } else if (m < 32) {
-                    if (m - 16 < N) wv = __ldg(p.WC + ((size_t)k * N + (m - 16)) * D + d0 + j);
-                } else if (m - 32 < R) {
-                    wv = __ldg(p.Wz + ((size_t)k * R + (m - 32)) * D + d0 + j);
-                }
-            }
-            const float hi = to_tf32(wv);
+        // the chunk's weight rows in the same layout
+#pragma unroll
+        for (int q = 0; q < kWPT; ++q) {
+            const int i = tid + q * kSelThreads, m = i / kSelKC, j = i % kSelKC;
+            const float hi = to_tf32(wv[q]);
             const int off = ((j / 4) * BG * 128 + (m / 8) * 128 + (m % 8) * 16) / 4 + (j % 4);
             sBhi[off] = hi;
-            sBlo[off] = to_tf32(wv - hi);
+            sBlo[off] = to_tf32(wv[q] - hi);
         }
         // the generic-proxy stores become visible to the tensor cores' async proxy
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -234,6 +244,7 @@ __global__ void __launch_bounds__(kSelThreads) selection_kernel(const SelParams 
             asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar)
                          : "memory");
         }
+        if (chunk + 1 < nchunks) load_chunk(d0 + kSelKC);
         // the chunk's MMAs have read the operands before they are overwritten
         // (after a wait that gave up, the rest of the tile is not waited for)
         if (ok) ok = mbar_wait(mbar, phase);
@@ -272,6 +283,7 @@ __global__ void __launch_bounds__(kSelThreads) selection_kernel(const SelParams 
         }
         __syncthreads();
         if (lv) {
+#pragma unroll 4
             for (int j = 0; j < cn; ++j) {
                 const float4* w4 = reinterpret_cast<const float4*>(sW + j * kSelRP);
                 float s = 0.0f;
