@@ -240,6 +240,11 @@ class Step:
         self.fused = ("mean_scan_merge", lib.vmb_mean_scan_merge_fwd,
                       (P(outs["xs"]), P(g["draw"]), P(g["A"]), P(g["Bs"]), P(g["Cs"]), P(g["Dskip"]), P(g["bias"]),
                        P(g["x"]), P(outs["ofused"]), P(outs["ybar"]), B, D, N, H, W, fl, dt, P(wsm), wsm.numel(), s))
+        # the scan side of the block straight from the map (no cross-scan, no y)
+        self.gathered = ("ss2d_mean", lib.vmb_ss2d_mean_fwd,
+                         (P(g["x"]), P(outs["xt"]), P(g["draw"]), P(g["A"]), P(g["Bs"]), P(g["Cs"]), P(g["Dskip"]),
+                          P(g["bias"]), P(outs["ofused"]), P(outs["ybar"]), B, D, N, H, W, fl, dt, P(wsm),
+                          wsm.numel(), s))
         # kernels each call launches (the chunked full scan launches three)
         self.launches = sum(int(lib.vmb_scan_kernel_count(path, B, K, D, N, H, W, dt)) if path >= 0 else 1
                             for path in (-1, 0, 1, -1, -1))
@@ -247,6 +252,12 @@ class Step:
 
     def run_fused(self):
         name, fn, args = self.fused
+        st = fn(*args)
+        if st != 0:
+            raise RuntimeError(f"{name}: {self.vmb.status_string(st)}")
+
+    def run_gathered(self):
+        name, fn, args = self.gathered
         st = fn(*args)
         if st != 0:
             raise RuntimeError(f"{name}: {self.vmb.status_string(st)}")
@@ -327,6 +338,7 @@ def make_outs(wl, dev, tdt, vmb):
         "ws_mean": torch.zeros(vmb.vmb_scan_workspace_bytes(1, B, 4, D, N, H, W, tdt), dtype=torch.uint8, device=dev),
         "ofused": torch.empty((B, D, H, W), dtype=tdt, device=dev),
         "ybar": torch.empty((B, 4, L), dtype=torch.float32, device=dev),
+        "xt": torch.empty((B, D, W, H), dtype=tdt, device=dev),
     }
 
 
@@ -336,8 +348,9 @@ def check_status(vmb, outs, where):
 
 
 def time_breakdown(step, n, prelude):
-    """n steps with an event after every call: per-kernel durations (ms lists)
-    and the fused channel-mean path timed alone (ms list)."""
+    """n steps with an event after every call: per-kernel durations (ms lists),
+    the fused channel-mean path and the gathered one (from the map) timed alone
+    (ms lists)."""
     import torch
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(KERNELS) + 1)] for _ in range(n)]
     for i in range(n):
@@ -350,12 +363,19 @@ def time_breakdown(step, n, prelude):
         fev[i][0].record()
         step.run_fused()
         fev[i][1].record()
+    gev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(n)]
+    for i in range(n):
+        prelude()
+        gev[i][0].record()
+        step.run_gathered()
+        gev[i][1].record()
     torch.cuda.synchronize()
     per_kernel = {k: [e[j].elapsed_time(e[j + 1]) for e in evs] for j, k in enumerate(KERNELS)}
-    return per_kernel, [e[0].elapsed_time(e[1]) for e in fev]
+    return per_kernel, ([e[0].elapsed_time(e[1]) for e in fev], [e[0].elapsed_time(e[1]) for e in gev])
 
 
-def kernel_table(wl, per_kernel_ms, fused_ms, peak):
+def kernel_table(wl, per_kernel_ms, fused_pair, peak):
+    fused_ms, gathered_ms = fused_pair
     kb = kernel_bytes(wl)
     per = {}
     for k in KERNELS:
@@ -369,6 +389,16 @@ def kernel_table(wl, per_kernel_ms, fused_ms, peak):
              "unfused_us": per["mean_scan"]["us"] + per["cross_merge_mean"]["us"],
              "speedup_over_unfused": (per["mean_scan"]["us"] + per["cross_merge_mean"]["us"]) / fused_us,
              "speedup_over_full_path": (per["full_scan"]["us"] + per["cross_merge_full"]["us"]) / fused_us}
+    g_us = 1e3 * statistics.mean(gathered_ms)
+    gb = wl.gathered_mean_bytes()
+    unfused_all = per["cross_scan"]["us"] + per["mean_scan"]["us"] + per["cross_merge_mean"]["us"]
+    fused["gathered_from_map"] = {
+        "us": g_us, "algorithmic_bytes": gb, "gbs": gb / (g_us / 1e6) / 1e9,
+        "frac_of_peak": gb / (g_us / 1e6) / 1e9 / peak,
+        "calls": "vmb_ss2d_mean_fwd: cross-scan, channel-mean scan and cross-merge, no xs and no y",
+        "speedup_over_cross_scan_plus_fused": (per["cross_scan"]["us"] + fused_us) / g_us,
+        "speedup_over_unfused_mean_path": unfused_all / g_us,
+        "speedup_over_full_path": (per["cross_scan"]["us"] + per["full_scan"]["us"] + per["cross_merge_full"]["us"]) / g_us}
     return per, fused
 
 
@@ -390,6 +420,7 @@ def sweep_configs(vmb, dev, peak, prelude_flush, warmup):
             prelude()
             step.run()
             step.run_fused()
+            step.run_gathered()
         torch.cuda.synchronize()
         est_s = sum(kernel_bytes(wl).values()) / 3e12
         n = int(min(50, max(5, 0.05 / est_s)))
@@ -474,6 +505,7 @@ def run_ours(args, wl, rank, world, local_rank):
     for _ in range(2):
         prelude()
         step.run_fused()
+        step.run_gathered()
     per_kernel, fused_ms = time_breakdown(step, min(args.steps, 50), prelude)
     check_status(vmb, outs, "during the breakdown steps")
 
@@ -736,11 +768,7 @@ def main():
     config["timed_region_s"] = res["total_ms"] / 1e3
     kb = kernel_bytes(wl)
     peak, peak_src = measured_peaks()
-    per = {}
-    for k in KERNELS:
-        avg = statistics.mean(res["per_kernel"][k])
-        per[k] = {"us": avg * 1e3, "gbs": kb[k] / (avg / 1e3) / 1e9, "frac_of_peak": kb[k] / (avg / 1e3) / 1e9 / peak}
-    fused_us = 1e3 * statistics.mean(res["fused_ms"])
+    per, fused_table = kernel_table(wl, res["per_kernel"], res["fused_ms"], peak)
     dominant = max(KERNELS, key=lambda k: statistics.mean(res["per_kernel"][k]))
     dom_ms = statistics.mean(res["per_kernel"][dominant])
     achieved = kb[dominant] / (dom_ms / 1e3) / 1e9
@@ -766,14 +794,9 @@ def main():
                      else "fallback 6.8 TB/s", "unit": "GB/s", "frac": achieved / peak,
                      "algorithmic_bytes_per_launch": kb[dominant], "traffic": traffic,
                      "alu_view": alu_view(dominant, wl, dom_ms)},
-        # the fused channel-mean path (broadcast inside the merge), timed separately
-        "mean_path_fused": {
-            "us": fused_us, "gbs": wl.fused_mean_bytes() / (fused_us / 1e6) / 1e9,
-            "frac_of_peak": wl.fused_mean_bytes() / (fused_us / 1e6) / 1e9 / peak,
-            "algorithmic_bytes": wl.fused_mean_bytes(),
-            "unfused_us": per["mean_scan"]["us"] + per["cross_merge_mean"]["us"],
-            "speedup_over_unfused": (per["mean_scan"]["us"] + per["cross_merge_mean"]["us"]) / fused_us,
-            "speedup_over_full_path": (per["full_scan"]["us"] + per["cross_merge_full"]["us"]) / fused_us},
+        # the fused channel-mean path (broadcast inside the merge) and the same
+        # from the map (no cross-scan either), timed separately
+        "mean_path_fused": fused_table,
         "gpu_launches": res["launches_per_step"] * args.steps,
         "paper_style": paper_style_summary(res["paper_style"], peak),
         # grouped basis: d channel groups per direction, each its own channel mean

@@ -223,6 +223,34 @@ vmb_status vmb_mean_scan_merge_fwd(const void* u, const void* delta, const float
                                    size_t workspace_bytes, cudaStream_t stream);
 
 /*
+ * vmb_ss2d_mean_fwd - the scan side of a VMeanba SS2D block in one call: the
+ * App. A cross-scan, the channel-mean scan (Sec. 2.2, Eq. 9) and the App. A
+ * cross-merge, without the cross-scanned sequences xs [B, 4, D, L] or the
+ * per-channel output y ever being written.  Direction k's step l reads the
+ * value the cross-scan would have put there: directions 0 and 2 read the
+ * (b, d) planes of x row by row (forward and reversed), directions 1 and 3 the
+ * rows of xt, the transpose of every plane (xt[b,d,w,h] = x[b,d,h,w], written
+ * by this call); the merge applies the broadcast and the skip term:
+ *   out = vmb_mean_scan_merge_fwd(vmb_cross_scan(x), delta, ..., x)
+ *   x, out [B, D, H, W] (dtype), out must not alias x;
+ *   xt [B, D, W, H] (dtype), caller-owned scratch (overwritten), aliasing
+ *   neither x nor out;
+ *   delta [B, 4, D, L], Bs, Cs [B, 4, N, L] (dtype); A [4*D, N], Dskip [4*D],
+ *   delta_bias [4*D] (fp32); ybar [B, 4, L] fp32, required (as in
+ *   vmb_mean_scan_merge_fwd); flags and workspace as vmb_mean_scan_fwd with
+ *   K = 4 (vmb_scan_workspace_bytes(VMB_PATH_MEAN, B, 4, D, N, H, W, dtype)).
+ * Moves 2 B*D*L elements for the map instead of the cross-scan's 5 B*D*L.
+ * The same fp32 operations in the same order as that pair of calls, so fp32
+ * results are bit-identical to it.  Not in the paper as such: its kernels keep
+ * the steps apart.
+ */
+vmb_status vmb_ss2d_mean_fwd(const void* x, void* xt, const void* delta, const float* A,
+                             const void* Bs, const void* Cs, const float* Dskip,
+                             const float* delta_bias, void* out, float* ybar, int B, int D, int N,
+                             int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,
+                             size_t workspace_bytes, cudaStream_t stream);
+
+/*
  * vmb_selective_scan_fwd_noalloc - vmb_selective_scan_fwd for callers that
  * cannot allocate device memory (for example plugin code inside a framework
  * whose memory pool owns the device and forbids allocations of its own, or a

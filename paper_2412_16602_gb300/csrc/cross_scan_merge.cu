@@ -616,7 +616,52 @@ vmb_status launch_mean_merge_t(const void* x, const float* ybar, const float* Ds
                ? VMB_OK
                : VMB_ERR_CUDA;
 }
+// ------------------------------------------------------------ map transpose
+// xt[b, d, w, h] = x[b, d, h, w]: the column-major order of every (b, d) plane,
+// which the column-major directions of the cross-scan (1 and 3) read as
+// contiguous rows.  32 x 32 tiles through shared memory (one padded column so
+// the transposed reads hit distinct banks), coalesced on both sides.
+constexpr int kTT = 32, kTR = 8;  // tile edge, rows per thread pass
+
+template <typename T>
+__global__ void __launch_bounds__(kTT * kTR) map_transpose_kernel(const T* x, T* xt, int H, int W, int tiles_w,
+                                                                  int tiles_per_plane) {
+    __shared__ T tile[kTT][kTT + 1];
+    pdl_wait();
+    pdl_launch_dependents();
+    const long long plane = blockIdx.x / tiles_per_plane;
+    const int t = blockIdx.x % tiles_per_plane;
+    const int h0 = (t / tiles_w) * kTT, w0 = (t % tiles_w) * kTT;
+    const T* src = x + plane * (long long)H * W;
+    T* dst = xt + plane * (long long)H * W;
+    const int tx = threadIdx.x % kTT, ty = threadIdx.x / kTT;
+#pragma unroll
+    for (int r = ty; r < kTT; r += kTR) {
+        const int h = h0 + r, w = w0 + tx;
+        if (h < H && w < W) tile[r][tx] = src[(long long)h * W + w];
+    }
+    __syncthreads();
+#pragma unroll
+    for (int r = ty; r < kTT; r += kTR) {
+        const int w = w0 + r, h = h0 + tx;
+        if (h < H && w < W) dst[(long long)w * H + h] = tile[tx][r];
+    }
+}
+
 }  // namespace
+
+vmb_status launch_map_transpose(const void* x, void* xt, int B, int D, int H, int W, vmb_dtype dt, cudaStream_t stream) {
+    const int tiles_h = (H + kTT - 1) / kTT, tiles_w = (W + kTT - 1) / kTT;
+    const long long grid = (long long)B * D * tiles_h * tiles_w;
+    if (grid > INT32_MAX) return VMB_ERR_UNSUPPORTED;
+    int tpp = tiles_h * tiles_w, tw = tiles_w;
+    const void* xp = x;
+    void* args[] = {&xp, &xt, &H, &W, &tw, &tpp};
+    const void* fn = dt == VMB_BF16 ? reinterpret_cast<const void*>(&map_transpose_kernel<__nv_bfloat16>)
+                                    : reinterpret_cast<const void*>(&map_transpose_kernel<float>);
+    return launch_kernel(fn, dim3((unsigned)grid), dim3(kTT * kTR), 0, args, stream) == cudaSuccess ? VMB_OK
+                                                                                                  : VMB_ERR_CUDA;
+}
 
 vmb_status launch_mean_merge(const void* x, const float* ybar, const float* Dskip, void* out, int B, int D, int H,
                              int W, bool per_channel_skip, vmb_dtype dt, cudaStream_t stream) {

@@ -55,6 +55,10 @@ struct MeanParams {
     int no_bcast;  // fused with the cross-merge: no y; ybar (+ the broadcast skip term) only
     int cvec;      // u / y rows allow 4-step vector access (L % 4 == 0, 4-element aligned)
     int bc_group;  // sequences per B / C row block: 1, or G for the grouped basis (K, D are K*G, D/G)
+    int gather_h;  // > 0: u is the map x [B, D, H, W] with H = gather_h and u_t its transpose
+                   // [B, D, W, H] (K = 4, ybar only): direction k's step l reads the value the
+                   // cross-scan would have put there, from x (k = 0, 2) or u_t (k = 1, 3)
+    const void* u_t;
     WsHeader* hdr;
     unsigned* flags;
     float* aggP;
@@ -269,6 +273,14 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
     const size_t col = (size_t)l0 + (tv ? rt : 0);
     const T* dcol = dlr + urow0 * (size_t)L + col;
     const T* ucol = u + urow0 * (size_t)L + col;
+    if (p.gather_h > 0) {
+        // the value the App. A cross-scan puts at step l of direction k: 0 reads
+        // the (b, d) plane of x row by row, 1 column by column (the rows of its
+        // transpose u_t), 2 and 3 the same in reverse; the planes have the same
+        // channel stride L as the rows of u
+        const int lr = (k >= 2) ? L - 1 - (int)col : (int)col;
+        ucol = ((k & 1) ? static_cast<const T*>(p.u_t) : u) + (size_t)(seq / p.K) * D * (size_t)L + lr;
+    }
     // u is read again by the broadcast pass: keep it in L2; delta streams through
     const uint64_t keep = l2_evict_last(), stream = l2_evict_first();
     float* s_a2 = reinterpret_cast<float*>(smb + LY::tab0);
@@ -761,6 +773,8 @@ vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     p.cvec = (a.L % 4 == 0) && al4e(a.u) && (a.y == nullptr || al4e(a.y));
     p.no_bcast = a.no_bcast ? 1 : 0;
     p.bc_group = a.bc_group;
+    p.gather_h = a.gather_h;
+    p.u_t = a.u_t;
     p.tabvec = al16(a.A) && al16(a.bias) && al16(a.Dskip);
     const WsLayout w = ws_layout(plan);
     unsigned char* ws = static_cast<unsigned char*>(a.ws);

@@ -276,6 +276,41 @@ vmb_status vmb_mean_scan_merge_fwd(const void* u, const void* delta, const float
     return launch_mean_merge(x, ybar, Dskip, out, B, D, H, W, (flags & VMB_FLAG_SKIP_MEAN) == 0, dtype, stream);
 }
 
+vmb_status vmb_ss2d_mean_fwd(const void* x, void* xt, const void* delta, const float* A, const void* Bs,
+                             const void* Cs, const float* Dskip, const float* delta_bias, void* out, float* ybar,
+                             int B, int D, int N, int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,
+                             size_t workspace_bytes, cudaStream_t stream) {
+    bool empty = false;
+    vmb_status s = check_csm(x, out, B, D, H, W, dtype, &empty);
+    if (s != VMB_OK || empty) return s;
+    if (x == out || !xt || xt == x || xt == out) return VMB_ERR_INVALID_ARG;
+    if (!aligned(xt, esize(dtype))) return VMB_ERR_MISALIGNED;
+    // the channel-mean scan reads each direction's steps straight from the map
+    // (rows of x) or its transpose (rows of xt), with no materialised
+    // cross-scan; it stops at ybar, and the merge applies the broadcast and the
+    // skip term
+    ScanArgs a{x, delta, A, Bs, Cs, Dskip, delta_bias, nullptr, ybar, B, 4, D, N, H * W, flags, dtype,
+               workspace, workspace_bytes};
+    a.no_bcast = true;
+    a.gather_h = H;
+    a.u_t = xt;
+    // every check (arguments, plan, workspace size) before the first launch
+    bool scan_empty = false;
+    s = check_scan(a, true, &scan_empty);
+    if (s != VMB_OK) return s;
+    if (!workspace) return VMB_ERR_WORKSPACE;
+    if (!aligned(workspace, 256)) return VMB_ERR_MISALIGNED;
+    ScanPlan plan{};
+    s = plan_mean(a, &plan);
+    if (s != VMB_OK) return s;
+    if (workspace_bytes < plan.ws_bytes) return VMB_ERR_WORKSPACE;
+    s = launch_map_transpose(x, xt, B, D, H, W, dtype, stream);
+    if (s != VMB_OK) return s;
+    s = launch_mean(a, plan, stream);
+    if (s != VMB_OK) return s;
+    return launch_mean_merge(x, ybar, Dskip, out, B, D, H, W, (flags & VMB_FLAG_SKIP_MEAN) == 0, dtype, stream);
+}
+
 vmb_status vmb_discretise_fwd(const void* u, const void* delta, const float* A, const void* Bs,
                               const float* delta_bias, float* dA, float* dBu, int B, int K, int D, int N, int H,
                               int W, unsigned flags, vmb_dtype dtype, cudaStream_t stream) {

@@ -28,6 +28,10 @@ struct ScanArgs {
     size_t ws_bytes;
     bool no_bcast = false;  // mean path fused with the cross-merge: ybar only, no y
     int bc_group = 1;       // grouped basis: K and D above are K*G and D/G; B / C rows per G sequences
+    int gather_h = 0;       // > 0: u is the map x [B, D, H, W] (H = gather_h, K = 4) and u_t its transpose
+                            // [B, D, W, H]; directions 0 / 2 read x, 1 / 3 read u_t (no materialised
+                            // cross-scan)
+    const void* u_t = nullptr;
 };
 
 // Execution plan of an L-chunked scan: how the (sequence, chunk) grid is cut
@@ -120,6 +124,8 @@ vmb_status launch_cross_scan(const void* x, void* xs, int B, int D, int H, int W
                              cudaStream_t stream);
 vmb_status launch_cross_merge(const void* ys, void* out, int B, int D, int H, int W, vmb_dtype dt,
                               cudaStream_t stream);
+vmb_status launch_map_transpose(const void* x, void* xt, int B, int D, int H, int W, vmb_dtype dt,
+                                cudaStream_t stream);
 vmb_status launch_discretise(const DiscArgs& a, bool mean, cudaStream_t stream);
 vmb_status launch_selection(const SelArgs& a, cudaStream_t stream);
 vmb_status launch_scan_only(const OnlyArgs& a, cudaStream_t stream);

@@ -1,6 +1,8 @@
 """The channel-mean path with the broadcast fused into the cross-merge
-(vmb_mean_scan_merge_fwd) against the fp64 oracle's unfused chain, and bit for
-bit against the library's own unfused pair for fp32 storage."""
+(vmb_mean_scan_merge_fwd), and the whole scan side of the block from the map
+(vmb_ss2d_mean_fwd: no materialised cross-scan either), against the fp64
+oracle's unfused chain, and bit for bit against the library's own unfused
+calls for fp32 storage."""
 import numpy as np
 import pytest
 
@@ -40,7 +42,10 @@ def _run(inp, flags=vmb.VMB_FLAG_SOFTPLUS):
     ym, yb_plain = vmb.vmb_mean_scan_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W,
                                          want_ybar=True, flags=flags)
     om = vmb.vmb_cross_merge(ym, wl.H, wl.W)
+    og, ybg = vmb.vmb_ss2d_mean_fwd(g["x"], g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], flags=flags)
     assert vmb.vmb_read_status() == vmb.VMB_OK
+    # gathered from the map: the same values and operations as the fused pair
+    assert torch.equal(og, out) and torch.equal(ybg, ybar), "the gathered path must match the fused pair bit for bit"
     return out, ybar, om, yb_plain
 
 

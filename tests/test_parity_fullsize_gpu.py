@@ -117,8 +117,11 @@ def test_fullsize_fused_and_grouped():
                                             wl.H, wl.W)
     grouped = {G: vmb.vmb_mean_scan_grouped_fwd(xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"],
                                                 wl.H, wl.W, G, want_ybar=True) for G in (4, 16)}
+    og, ybg = vmb.vmb_ss2d_mean_fwd(g["x"], g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"])
     assert vmb.vmb_read_status() == vmb.VMB_OK
     torch.cuda.synchronize()
+    # the same block from the map (no cross-scan): bit-identical to the fused pair
+    assert torch.equal(og, out) and torch.equal(ybg, ybar)
     rng = np.random.default_rng(77)
     D, K, dt = wl.D, 4, wl.dtype
     u_ref = oracle.cross_scan(inp.x[0:1])

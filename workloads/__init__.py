@@ -83,6 +83,21 @@ class Workload:
         params = self.K * self.D * (self.N + 2) * 4
         return s * (2 * bkdl + 2 * bknl + 2 * bdl) + 2 * 4 * self.B * self.K * self.L + params
 
+    def gathered_mean_bytes(self) -> int:
+        """Algorithmic bytes of the scan side of the block from the map (cross-scan,
+        channel-mean scan and cross-merge in one call, vmb_ss2d_mean_fwd): delta
+        read once, Bs and Cs read once, the map x read once (every direction
+        reads the same map) and the merged map written once, ybar (fp32,
+        [B, K, L]) written and read back once, plus the per-channel parameters.
+        (The implementation also writes and reads a transposed copy of the map
+        for the column-major directions; that is not counted.)"""
+        s = self.esize
+        bkdl = self.B * self.K * self.D * self.L
+        bknl = self.B * self.K * self.N * self.L
+        bdl = self.B * self.D * self.L
+        params = self.K * self.D * (self.N + 2) * 4
+        return s * (bkdl + 2 * bknl + 2 * bdl) + 2 * 4 * self.B * self.K * self.L + params
+
     def replace(self, **kw) -> "Workload":
         d = dict(self.__dict__)
         d.update(kw)
