@@ -90,6 +90,8 @@ class Oracle:
         lib.oracle_mean_scan_grouped.restype = i
         lib.oracle_selection.argtypes = [P] * 8 + [lg] * 6
         lib.oracle_selection.restype = None
+        lib.oracle_mean_scan_bwd.argtypes = [P] * 15 + [lg] * 6 + [i]
+        lib.oracle_mean_scan_bwd.restype = None
         self.lib = lib
         self.path = lib_path
 
@@ -166,6 +168,25 @@ class Oracle:
         if rc:
             raise ValueError("groups must divide D")
         return y, ybar
+
+    def mean_scan_bwd(self, u, delta, A, Bs, Cs, Dskip, bias, gy, *, groups: int = 1, softplus_on=True):
+        """Gradients of the (grouped) channel-mean scan with the Euler Bbar and the per-channel
+        skip term (the adjoint of Eq. 9's forward), given gy = dLoss/dy [B, K, D, L]: returns
+        dict(u, delta, A, Bs, Cs, Dskip, bias) of gradients with the inputs' shapes (delta is
+        the raw Delta before bias and softplus)."""
+        arrs, (B, K, D, N, L) = self._scan_args(u, delta, A, Bs, Cs, Dskip, bias)
+        gy = _f64(gy)
+        if gy.shape != (B, K, D, L):
+            raise ValueError("gy must be [B, K, D, L]")
+        if groups < 1 or D % groups:
+            raise ValueError("groups must divide D")
+        out = dict(u=np.empty((B, K, D, L)), delta=np.empty((B, K, D, L)), A=np.empty((K * D, N)),
+                   Bs=np.empty((B, K, N, L)), Cs=np.empty((B, K, N, L)), Dskip=np.empty(K * D),
+                   bias=np.empty(K * D))
+        self.lib.oracle_mean_scan_bwd(*(_ptr(a) for a in arrs), _ptr(gy), _ptr(out["u"]), _ptr(out["delta"]),
+                                      _ptr(out["A"]), _ptr(out["Bs"]), _ptr(out["Cs"]), _ptr(out["Dskip"]),
+                                      _ptr(out["bias"]), B, K, D, N, L, int(groups), int(bool(softplus_on)))
+        return out
 
     def selection(self, u, WB, WC, Wz, Wup):
         """Eq. 6 selection functions: u [B, K, D, L], WB and WC [K, N, D], Wz [K, R, D],
@@ -287,6 +308,10 @@ def discretise(*a, **kw):
 
 def discretise_mean(*a, **kw):
     return get().discretise_mean(*a, **kw)
+
+
+def mean_scan_bwd(*a, **kw):
+    return get().mean_scan_bwd(*a, **kw)
 
 
 def scan_only(*a, **kw):

@@ -20,6 +20,11 @@
  *   scan-only kernel setting ....... Sec. 4, "Kernel Implementation" (discretisation done
  *                                     before the scan; the scan reads materialised Abar,
  *                                     Bbar u with D channels, or one channel after T)
+ *   backward of the mean scan ...... the adjoint (reverse-mode derivative) of Eq. 9's forward
+ *                                     (Euler Bbar, per-channel skip) for the grouped basis of
+ *                                     Sec. 2.1 / Eq. 8 (one group = VMeanba); the paper trains
+ *                                     no VMeanba layer, so this is the plain chain rule of the
+ *                                     forward above, pinned by finite differences
  *
  * Readings of points the paper leaves open (each is listed in the design notes):
  *   - scan directions: 0 row-major, 1 column-major, 2 = reverse of 0, 3 = reverse of 1;
@@ -433,4 +438,112 @@ void oracle_selection(const double* u, const double* WB, const double* WC, const
 /* Eq. 6 softplus, exposed so that tests can pin it against known values. */
 void oracle_softplus(const double* x, double* out, long n) {
     for (long i = 0; i < n; ++i) out[i] = softplus(x[i]);
+}
+
+/* ------------------------------------------------------ mean-scan backward */
+
+/*
+ * Gradients of the grouped channel-mean scan (Euler Bbar, per-channel skip) with
+ * respect to every input, given gy = dLoss/dy.  Per (b, k, group g) with the
+ * group's channels d and M = D / groups of them:
+ *   delta_d = softplus(raw_d + bias_c), e_dn = exp(delta_d A_cn),
+ *   Abar_n = (1/M) sum_d e_dn, s = (1/M) sum_d delta_d u_d,
+ *   h_n(t) = Abar_n(t) h_n(t-1) + B_n(t) s(t), ybar = sum_n C_n h_n,
+ *   y_d = ybar + Dskip_c u_d.
+ * Reverse mode, backward in time, with lam_n(t) = dLoss/dh_n(t):
+ *   gybar(t) = sum_d gy_d(t),  lam_n(t) = C_n(t) gybar(t) + Abar_n(t+1) lam_n(t+1),
+ *   gC_n(t) += gybar(t) h_n(t),  gB_n(t) += lam_n(t) s(t),
+ *   gAbar_n(t) = lam_n(t) h_n(t-1),  gs(t) = sum_n lam_n(t) B_n(t),
+ * then through the channel mean and the softplus, per channel d:
+ *   gu_d = Dskip_c gy_d + gs delta_d / M,
+ *   gdelta_d = gs u_d / M + sum_n gAbar_n A_cn e_dn / M,
+ *   graw_d = gdelta_d softplus'(raw_d + bias_c)   (softplus' = the logistic function),
+ *   gA_cn += gAbar_n delta_d e_dn / M, gDskip_c += gy_d u_d, gbias_c += graw_d.
+ * B and C have no channel axis, so the groups of a (b, k) add into the same gB, gC.
+ * Sequential, one (b, k, g) after another; gA, gDskip, gbias, gB and gC are
+ * zeroed here and accumulated.
+ */
+void oracle_mean_scan_bwd(const double* u, const double* raw, const double* A, const double* Bs,
+                          const double* Cs, const double* Dskip, const double* bias, const double* gy,
+                          double* gu, double* graw, double* gA, double* gB, double* gC, double* gDskip,
+                          double* gbias, long B, long K, long D, long N, long L, long groups,
+                          int softplus_on) {
+    long M = D / groups;
+    for (long i = 0; i < K * D * N; ++i) gA[i] = 0.0;
+    for (long i = 0; i < K * D; ++i) { gDskip[i] = 0.0; gbias[i] = 0.0; }
+    for (long i = 0; i < B * K * N * L; ++i) { gB[i] = 0.0; gC[i] = 0.0; }
+    double* h = (double*)calloc((size_t)(L + 1) * N, sizeof(double));  /* h[(t + 1) N + n], h(-1) = 0 */
+    double* abar = (double*)malloc((size_t)L * N * sizeof(double));
+    double* sm = (double*)malloc((size_t)L * sizeof(double));
+    double* gab = (double*)malloc((size_t)L * N * sizeof(double));
+    double* gs = (double*)malloc((size_t)L * sizeof(double));
+    double* lam = (double*)malloc((size_t)N * sizeof(double));
+    for (long b = 0; b < B; ++b)
+        for (long k = 0; k < K; ++k)
+            for (long g = 0; g < groups; ++g) {
+                long row0 = (b * K + k) * D + g * M; /* first (b, k, d) row of the group */
+                const double* Bk = Bs + (b * K + k) * N * L;
+                const double* Ck = Cs + (b * K + k) * N * L;
+                double* gBk = gB + (b * K + k) * N * L;
+                double* gCk = gC + (b * K + k) * N * L;
+                /* forward: the group's means and the states */
+                for (long t = 0; t < L; ++t) {
+                    double s = 0.0;
+                    for (long n = 0; n < N; ++n) abar[t * N + n] = 0.0;
+                    for (long j = 0; j < M; ++j) {
+                        long c = k * D + g * M + j;
+                        double v = raw[(row0 + j) * L + t] + bias[c];
+                        double delta = softplus_on ? softplus(v) : v;
+                        for (long n = 0; n < N; ++n) abar[t * N + n] += exp(delta * A[c * N + n]);
+                        s += delta * u[(row0 + j) * L + t];
+                    }
+                    for (long n = 0; n < N; ++n) abar[t * N + n] /= (double)M;
+                    sm[t] = s / (double)M;
+                    for (long n = 0; n < N; ++n)
+                        h[(t + 1) * N + n] = abar[t * N + n] * h[t * N + n] + Bk[n * L + t] * sm[t];
+                }
+                /* backward in time */
+                for (long n = 0; n < N; ++n) lam[n] = 0.0;
+                for (long t = L - 1; t >= 0; --t) {
+                    double gyb = 0.0;
+                    for (long j = 0; j < M; ++j) gyb += gy[(row0 + j) * L + t];
+                    double gst = 0.0;
+                    for (long n = 0; n < N; ++n) {
+                        /* lam holds Abar_n(t+1) lam_n(t+1) from the previous iteration */
+                        lam[n] += Ck[n * L + t] * gyb;
+                        gCk[n * L + t] += gyb * h[(t + 1) * N + n];
+                        gBk[n * L + t] += lam[n] * sm[t];
+                        gab[t * N + n] = lam[n] * h[t * N + n];
+                        gst += lam[n] * Bk[n * L + t];
+                        lam[n] *= abar[t * N + n];
+                    }
+                    gs[t] = gst;
+                }
+                /* through the channel mean and the softplus */
+                for (long j = 0; j < M; ++j) {
+                    long c = k * D + g * M + j;
+                    for (long t = 0; t < L; ++t) {
+                        long i = (row0 + j) * L + t;
+                        double v = raw[i] + bias[c];
+                        double delta = softplus_on ? softplus(v) : v;
+                        double gd = gs[t] * u[i] / (double)M;
+                        for (long n = 0; n < N; ++n) {
+                            double e = exp(delta * A[c * N + n]);
+                            gd += gab[t * N + n] * A[c * N + n] * e / (double)M;
+                            gA[c * N + n] += gab[t * N + n] * delta * e / (double)M;
+                        }
+                        gu[i] = Dskip[c] * gy[i] + gs[t] * delta / (double)M;
+                        double gv = softplus_on ? gd / (1.0 + exp(-v)) : gd;
+                        graw[i] = gv;
+                        gDskip[c] += gy[i] * u[i];
+                        gbias[c] += gv;
+                    }
+                }
+            }
+    free(h);
+    free(abar);
+    free(sm);
+    free(gab);
+    free(gs);
+    free(lam);
 }

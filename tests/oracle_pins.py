@@ -534,4 +534,46 @@ def pin_discretise_mean_identical_channels(orc):
     _close(dBum, dBu[:, :, 2], rtol=1e-13, atol=1e-15, what="dBu mean")
 
 
+def _fd_gradients(orc, inputs, gy, groups, softplus_on, eps=1e-6):
+    """Central finite differences of the loss sum(gy * y) of the forward grouped
+    channel-mean scan, with respect to every input element."""
+    def loss(**kw):
+        a = dict(inputs)
+        a.update(kw)
+        y, _ = orc.mean_scan_grouped(a["u"], a["delta"], a["A"], a["Bs"], a["Cs"], a["Dskip"], a["bias"], groups,
+                                     softplus_on=softplus_on)
+        return float(np.sum(y * gy))
+    out = {}
+    for name, arr in inputs.items():
+        g = np.zeros_like(arr)
+        for i in np.ndindex(arr.shape):
+            plus, minus = arr.copy(), arr.copy()
+            plus[i] += eps
+            minus[i] -= eps
+            g[i] = (loss(**{name: plus}) - loss(**{name: minus})) / (2 * eps)
+        out[name] = g
+    return out
+
+
+def pin_mean_backward_finite_differences(orc):
+    """The backward of the (grouped) channel-mean scan equals central finite
+    differences of the forward, for every input, with one and two groups and
+    the softplus on and off (the chain rule itself, independent of how the
+    backward is organised)."""
+    rng = np.random.default_rng(91)
+    for groups, softplus_on in [(1, True), (2, True), (1, False)]:
+        u, draw, A, Bs, Cs, Dskip, bias = _rand_problem(rng, B=1, K=2, D=4, N=3, L=5)
+        if not softplus_on:
+            bias = np.abs(bias) + 0.5  # keep delta positive without the softplus
+            draw = 0.05 * np.abs(draw)
+        gy = rng.standard_normal(u.shape)
+        inputs = dict(u=u, delta=draw, A=A, Bs=Bs, Cs=Cs, Dskip=Dskip, bias=bias)
+        got = orc.mean_scan_bwd(u, draw, A, Bs, Cs, Dskip, bias, gy, groups=groups, softplus_on=softplus_on)
+        ref = _fd_gradients(orc, inputs, gy, groups, softplus_on)
+        for name in inputs:
+            scale = max(1e-12, float(np.max(np.abs(ref[name]))))
+            err = float(np.max(np.abs(got[name] - ref[name]))) / scale
+            assert err < 1e-6, f"gradient of {name} (groups {groups}, softplus {softplus_on}): rel err {err:.2e}"
+
+
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_")]

@@ -50,6 +50,12 @@ MUTANTS = {
     "selection_up_transposed": ("sd += Wup[(k * D + d) * R + r] * z[r];", "sd += Wup[(k * R + r) * D + d] * z[r];"),
     "selection_first_direction_weights": ("sz += Wz[(k * R + r) * D + d] * uk[d * L + l];",
                                           "sz += Wz[r * D + d] * uk[d * L + l];"),
+    "bwd_carry_uses_previous_abar": ("lam[n] *= abar[t * N + n];", "lam[n] *= abar[(t > 0 ? t - 1 : 0) * N + n];"),
+    "bwd_gu_without_mean_factor": ("gu[i] = Dskip[c] * gy[i] + gs[t] * delta / (double)M;",
+                                   "gu[i] = Dskip[c] * gy[i] + gs[t] * delta;"),
+    "bwd_without_softplus_derivative": ("double gv = softplus_on ? gd / (1.0 + exp(-v)) : gd;", "double gv = gd;"),
+    "bwd_gabar_with_current_state": ("gab[t * N + n] = lam[n] * h[t * N + n];",
+                                     "gab[t * N + n] = lam[n] * h[(t + 1) * N + n];"),
     "scan_only_drops_decay": ("h[n] = dA[(row * N + n) * L + l] * h[n] + dBu[(row * N + n) * L + l];",
                               "h[n] = h[n] + dBu[(row * N + n) * L + l];"),
     "scan_only_output_before_update": ("h[n] = dA[(row * N + n) * L + l] * h[n] + dBu[(row * N + n) * L + l];\n                        acc += Cs[((b * K + k) * N + n) * L + l] * h[n];",
