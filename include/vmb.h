@@ -339,6 +339,36 @@ vmb_status vmb_selection_fwd(const void* u, const float* WB, const float* WC, co
                              int D, int N, int R, int H, int W, vmb_dtype dtype, cudaStream_t stream);
 
 /*
+ * vmb_mean_scan_bwd - gradients of the channel-mean scan (Sec. 2.2, Eq. 9) or,
+ * with groups > 1, of the grouped basis (Sec. 2.1, Eq. 8; vmb_mean_scan_grouped_fwd),
+ * for the Euler Bbar and the per-channel skip term: the reverse-mode
+ * derivative of the forward, given gy = dLoss/dy [B, K, D, L] (dtype).  Per
+ * sequence (b, k, group) the states are recomputed forward, the adjoint
+ *   lam_n(t) = C_n(t) sum_d gy_d(t) + Abar_n(t+1) lam_n(t+1)
+ * runs backward in time, and the chain rule goes through the group mean and
+ * the softplus.  Outputs (every one written, none accumulated into):
+ *   gu, gdelta [B, K, D, L] (dtype): d/du and d/d(raw delta);
+ *   gA [K*D, N], gDskip [K*D], gdelta_bias [K*D] (fp32), summed over the batch;
+ *   gBs, gCs [B, K, N, L] (dtype), summed over the groups of each (b, k).
+ * Same inputs as vmb_mean_scan_grouped_fwd (delta is the raw Delta); flags:
+ * VMB_FLAG_SOFTPLUS (VMB_FLAG_B_ZOH and VMB_FLAG_SKIP_MEAN: VMB_ERR_UNSUPPORTED).
+ * workspace: >= vmb_mean_scan_bwd_workspace_bytes(...) bytes, 256-B aligned,
+ * any contents (the forward states, group means and adjoints of every
+ * sequence, fp32: about 3 x 64 bytes per (b, k, group, step)).  Every
+ * reduction runs in a fixed order: results are deterministic.  The paper
+ * trains no VMeanba layer (it replaces layers of a trained model); this is the
+ * chain rule of the forward defined there.
+ */
+vmb_status vmb_mean_scan_bwd(const void* u, const void* delta, const float* A, const void* Bs,
+                             const void* Cs, const float* Dskip, const float* delta_bias,
+                             const void* gy, void* gu, void* gdelta, float* gA, void* gBs,
+                             void* gCs, float* gDskip, float* gdelta_bias, int B, int K, int D,
+                             int N, int H, int W, int groups, unsigned flags, vmb_dtype dtype,
+                             void* workspace, size_t workspace_bytes, cudaStream_t stream);
+size_t vmb_mean_scan_bwd_workspace_bytes(int B, int K, int D, int N, int H, int W, int groups,
+                                         vmb_dtype dtype);
+
+/*
  * vmb_read_status - synchronise `stream`, then return and clear the device
  * error word of `workspace` (VMB_OK, VMB_ERR_TIMEOUT or VMB_ERR_BOUNDS).  A
  * device-side error leaves the outputs of that call undefined but the CUDA

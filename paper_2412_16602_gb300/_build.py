@@ -21,7 +21,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libvmb.so")
 BUILD_DIR = os.path.join(PKG, "_build")
-SOURCES = ["vmb_abi.cu", "cross_scan_merge.cu", "full_scan.cu", "mean_scan.cu", "noalloc.cu", "scan_only.cu", "selection.cu"]
+SOURCES = ["vmb_abi.cu", "cross_scan_merge.cu", "full_scan.cu", "mean_scan.cu", "mean_backward.cu", "noalloc.cu",
+           "scan_only.cu", "selection.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

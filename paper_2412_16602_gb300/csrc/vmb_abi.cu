@@ -311,6 +311,35 @@ vmb_status vmb_ss2d_mean_fwd(const void* x, void* xt, const void* delta, const f
     return launch_mean_merge(x, ybar, Dskip, out, B, D, H, W, (flags & VMB_FLAG_SKIP_MEAN) == 0, dtype, stream);
 }
 
+// Checks of the backward call; sets *empty for a problem with no elements.
+static vmb_status check_bwd(const MeanBwdArgs& a, bool* empty) {
+    if (!dtype_ok(a.dtype) || a.B < 0 || a.K < 0 || a.D < 0 || a.N < 0 || a.L < 0) return VMB_ERR_INVALID_ARG;
+    if (a.flags & ~(unsigned)(VMB_FLAG_SOFTPLUS | VMB_FLAG_B_ZOH | VMB_FLAG_SKIP_MEAN)) return VMB_ERR_INVALID_ARG;
+    long long n = 0, nbc = 0;
+    if (!count(&n, {a.B, a.K, a.D, a.L}) || !count(&nbc, {a.B, a.K, a.N > 0 ? a.N : 1, a.L}))
+        return VMB_ERR_INVALID_ARG;
+    *empty = n == 0;
+    if (*empty) return VMB_OK;
+    if (a.N < 1 || a.groups < 1 || a.D % a.groups != 0) return VMB_ERR_INVALID_ARG;
+    if (a.N > 16) return VMB_ERR_UNSUPPORTED;
+    if (a.flags & (VMB_FLAG_B_ZOH | VMB_FLAG_SKIP_MEAN)) return VMB_ERR_UNSUPPORTED;  // Euler Bbar, per-channel skip
+    long long rows = 0;
+    if (!count(&rows, {a.B, a.K, a.D}) || rows > INT_MAX / 2 || (long long)a.B * a.K * a.groups > INT_MAX / 16)
+        return VMB_ERR_UNSUPPORTED;
+    const void* ptrs[] = {a.u, a.delta, a.A, a.Bs, a.Cs, a.Dskip, a.bias, a.gy, a.gu, a.gdelta, a.gA, a.gBs, a.gCs,
+                          a.gDskip, a.gbias};
+    for (const void* q : ptrs)
+        if (!q) return VMB_ERR_INVALID_ARG;
+    const size_t es = esize(a.dtype);
+    const void* elems[] = {a.u, a.delta, a.Bs, a.Cs, a.gy, a.gu, a.gdelta, a.gBs, a.gCs};
+    for (const void* q : elems)
+        if (!aligned(q, es)) return VMB_ERR_MISALIGNED;
+    const void* params[] = {a.A, a.Dskip, a.bias, a.gA, a.gDskip, a.gbias};
+    for (const void* q : params)
+        if (!aligned(q, 4)) return VMB_ERR_MISALIGNED;
+    return VMB_OK;
+}
+
 vmb_status vmb_discretise_fwd(const void* u, const void* delta, const float* A, const void* Bs,
                               const float* delta_bias, float* dA, float* dBu, int B, int K, int D, int N, int H,
                               int W, unsigned flags, vmb_dtype dtype, cudaStream_t stream) {
@@ -365,6 +394,36 @@ vmb_status vmb_selection_fwd(const void* u, const float* WB, const float* WC, co
         return VMB_ERR_MISALIGNED;
     SelArgs a{u, WB, WC, Wz, Wup, Bs, Cs, delta_raw, B, K, D, N, R, H * W, dtype};
     return launch_selection(a, stream);
+}
+
+size_t vmb_mean_scan_bwd_workspace_bytes(int B, int K, int D, int N, int H, int W, int groups, vmb_dtype dtype) {
+    if (H < 0 || W < 0 || (long long)H * W > INT_MAX) return 0;
+    static const float dummy[4] = {0, 0, 0, 0};
+    float* dm = const_cast<float*>(dummy);
+    MeanBwdArgs a{dummy, dummy, dummy, dummy, dummy, dummy, dummy, dummy, dm, dm, dm, dm, dm, dm, dm,
+                  B, K, D, N, H * W, groups, VMB_FLAG_SOFTPLUS, dtype, nullptr, 0};
+    bool empty = false;
+    if (check_bwd(a, &empty) != VMB_OK) return 0;
+    if (empty) return 256;
+    return mean_bwd_workspace_bytes(B, K, D, (long long)H * W, groups);
+}
+
+vmb_status vmb_mean_scan_bwd(const void* u, const void* delta, const float* A, const void* Bs, const void* Cs,
+                             const float* Dskip, const float* delta_bias, const void* gy, void* gu, void* gdelta,
+                             float* gA, void* gBs, void* gCs, float* gDskip, float* gdelta_bias, int B, int K, int D,
+                             int N, int H, int W, int groups, unsigned flags, vmb_dtype dtype, void* workspace,
+                             size_t workspace_bytes, cudaStream_t stream) {
+    if (H < 0 || W < 0) return VMB_ERR_INVALID_ARG;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    MeanBwdArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, gy, gu, gdelta, gA, gBs, gCs, gDskip, gdelta_bias,
+                  B, K, D, N, H * W, groups, flags, dtype, workspace, workspace_bytes};
+    bool empty = false;
+    vmb_status s = check_bwd(a, &empty);
+    if (s != VMB_OK || empty) return s;
+    if (!workspace) return VMB_ERR_WORKSPACE;
+    if (!aligned(workspace, 256)) return VMB_ERR_MISALIGNED;
+    if (workspace_bytes < mean_bwd_workspace_bytes(B, K, D, (long long)H * W, groups)) return VMB_ERR_WORKSPACE;
+    return launch_mean_bwd(a, stream);
 }
 
 vmb_status vmb_read_status(void* workspace, cudaStream_t stream) {

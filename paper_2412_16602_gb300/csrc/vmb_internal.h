@@ -105,6 +105,30 @@ struct SelArgs {
     vmb_dtype dtype;
 };
 
+// Gradients of the (grouped) channel-mean scan.
+struct MeanBwdArgs {
+    const void* u;
+    const void* delta;  // raw Delta (before bias and softplus)
+    const float* A;
+    const void* Bs;
+    const void* Cs;
+    const float* Dskip;
+    const float* bias;
+    const void* gy;
+    void* gu;
+    void* gdelta;
+    float* gA;
+    void* gBs;
+    void* gCs;
+    float* gDskip;
+    float* gbias;
+    int B, K, D, N, L, groups;
+    unsigned flags;
+    vmb_dtype dtype;
+    void* ws;
+    size_t ws_bytes;
+};
+
 int device_sm_count();
 
 // The argument checks of the scan entry points (shapes, flags, pointers,
@@ -128,6 +152,8 @@ vmb_status launch_map_transpose(const void* x, void* xt, int B, int D, int H, in
                                 cudaStream_t stream);
 vmb_status launch_discretise(const DiscArgs& a, bool mean, cudaStream_t stream);
 vmb_status launch_selection(const SelArgs& a, cudaStream_t stream);
+size_t mean_bwd_workspace_bytes(long long B, long long K, long long D, long long L, long long G);
+vmb_status launch_mean_bwd(const MeanBwdArgs& a, cudaStream_t stream);
 vmb_status launch_scan_only(const OnlyArgs& a, cudaStream_t stream);
 vmb_status launch_mean_merge(const void* x, const float* ybar, const float* Dskip, void* out, int B, int D, int H,
                              int W, bool per_channel_skip, vmb_dtype dt, cudaStream_t stream);

@@ -41,7 +41,8 @@ EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb
            "vmb_selective_scan_fwd",
            "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_ss2d_mean_fwd",
            "vmb_discretise_fwd", "vmb_discretise_mean_fwd",
-           "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_read_status", "vmb_status_string", "vmb_version"]
+           "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_mean_scan_bwd", "vmb_mean_scan_bwd_workspace_bytes",
+           "vmb_read_status", "vmb_status_string", "vmb_version"]
 
 
 class VmbError(RuntimeError):
@@ -70,13 +71,16 @@ def _load() -> ctypes.CDLL:
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
     lib.vmb_selection_fwd.argtypes = [vp] * 8 + [i] * 7 + [i, vp]
+    lib.vmb_mean_scan_bwd.argtypes = [vp] * 15 + [i] * 7 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_bwd_workspace_bytes.argtypes = [i] * 8
+    lib.vmb_mean_scan_bwd_workspace_bytes.restype = sz
     lib.vmb_read_status.argtypes = [vp, vp]
     lib.vmb_status_string.argtypes = [i]
     lib.vmb_status_string.restype = ctypes.c_char_p
     lib.vmb_version.argtypes = []
     for name in ["vmb_cross_scan", "vmb_cross_merge", "vmb_selective_scan_fwd", "vmb_mean_scan_fwd",
                  "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_ss2d_mean_fwd", "vmb_discretise_fwd",
-                 "vmb_discretise_mean_fwd", "vmb_scan_only_fwd", "vmb_selection_fwd",
+                 "vmb_discretise_mean_fwd", "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_mean_scan_bwd",
                  "vmb_read_status", "vmb_version"]:
         getattr(lib, name).restype = i
     return lib
@@ -466,6 +470,34 @@ def vmb_selection_fwd(u, WB, WC, Wz, Wup, H: int, W: int, *, delta_raw=None, Bs=
                                  _ptr(delta_raw), B, K, D, N, R, H, W, _dtype_code(u.dtype), _stream(stream)),
            "vmb_selection_fwd")
     return delta_raw, Bs, Cs
+
+
+def vmb_mean_scan_bwd_workspace_bytes(B: int, K: int, D: int, N: int, H: int, W: int, groups: int = 1,
+                                      dtype: torch.dtype = torch.float32) -> int:
+    return int(lib.vmb_mean_scan_bwd_workspace_bytes(B, K, D, N, H, W, groups, _dtype_code(dtype)))
+
+
+def vmb_mean_scan_bwd(u, delta, A, Bs, Cs, Dskip, delta_bias, gy, H: int, W: int, *, groups: int = 1,
+                      flags: int = VMB_FLAG_SOFTPLUS, workspace=None, stream=None) -> dict:
+    """Gradients of the (grouped) channel-mean scan given gy = dLoss/dy [B, K, D, H*W]: returns
+    dict(u, delta, A, Bs, Cs, Dskip, delta_bias) with the inputs' shapes (delta: the raw Delta)."""
+    B, K, D, N, L = _scan_shapes(u, delta, A, Bs, Cs, Dskip, delta_bias, H, W)
+    _dev(gy, "gy")
+    if gy.shape != u.shape or gy.dtype != u.dtype:
+        raise ValueError("gy must match u")
+    if groups < 1 or D % groups:
+        raise ValueError("groups must be >= 1 and divide D")
+    out = dict(u=torch.empty_like(u), delta=torch.empty_like(u), A=torch.empty_like(A), Bs=torch.empty_like(Bs),
+               Cs=torch.empty_like(Cs), Dskip=torch.empty_like(Dskip), delta_bias=torch.empty_like(delta_bias))
+    ws_bytes = vmb_mean_scan_bwd_workspace_bytes(B, K, D, N, H, W, groups, u.dtype)
+    if workspace is None:
+        workspace = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=u.device)
+    _check(lib.vmb_mean_scan_bwd(_ptr(u), _ptr(delta), _ptr(A), _ptr(Bs), _ptr(Cs), _ptr(Dskip), _ptr(delta_bias),
+                                 _ptr(gy), _ptr(out["u"]), _ptr(out["delta"]), _ptr(out["A"]), _ptr(out["Bs"]),
+                                 _ptr(out["Cs"]), _ptr(out["Dskip"]), _ptr(out["delta_bias"]), B, K, D, N, H, W,
+                                 groups, flags, _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
+                                 _stream(stream)), "vmb_mean_scan_bwd")
+    return out
 
 
 def vmb_read_status(workspace=None, device=None, stream=None) -> int:
