@@ -62,6 +62,7 @@ def parse():
                     help="skip the timing of the paper's split (discretise, then scan alone)")
     ap.add_argument("--no-grouped", action="store_true", help="skip the timing of the grouped basis")
     ap.add_argument("--no-selection", action="store_true", help="skip the timing of the Eq. 6 selection functions")
+    ap.add_argument("--no-backward", action="store_true", help="skip the timing of the mean scan's backward")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-configs", action="store_true", help="skip the per-workload timing table")
     ap.add_argument("--extra-steps", type=int, default=20,
@@ -617,6 +618,29 @@ def run_ours(args, wl, rank, world, local_rank):
         def sel():
             vmb.vmb_selection_fwd(outs["xs"], *sw, wl.H, wl.W, delta_raw=sdr, Bs=sB, Cs=sC, stream=stream)
         sel_us = time_alone(sel)
+    # the backward of the channel-mean scan on the step's inputs (dLoss/dy drawn
+    # on the device), with its workspace allocated once
+    bwd_us = None
+    if not args.no_backward:
+        gy = torch.randn(outs["ym"].shape, device=dev, dtype=torch.float32).to(tdt)
+        bws = torch.empty(max(256, vmb.vmb_mean_scan_bwd_workspace_bytes(wl.B, 4, wl.D, wl.N, wl.H, wl.W, 1, tdt)),
+                          dtype=torch.uint8, device=dev)
+        gouts = dict(u=torch.empty_like(outs["xs"]), delta=torch.empty_like(outs["xs"]),
+                     A=torch.empty_like(g["A"]), Bs=torch.empty_like(g["Bs"]), Cs=torch.empty_like(g["Cs"]),
+                     Dskip=torch.empty_like(g["Dskip"]), bias=torch.empty_like(g["bias"]))
+        PP = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
+
+        def bwd():
+            st = vmb.lib.vmb_mean_scan_bwd(
+                PP(outs["xs"]), PP(g["draw"]), PP(g["A"]), PP(g["Bs"]), PP(g["Cs"]), PP(g["Dskip"]), PP(g["bias"]),
+                PP(gy), PP(gouts["u"]), PP(gouts["delta"]), PP(gouts["A"]), PP(gouts["Bs"]), PP(gouts["Cs"]),
+                PP(gouts["Dskip"]), PP(gouts["bias"]), wl.B, 4, wl.D, wl.N, wl.H, wl.W, 1, vmb.VMB_FLAG_SOFTPLUS,
+                vmb.VMB_BF16 if wl.dtype == "bf16" else vmb.VMB_F32, PP(bws), bws.numel(),
+                ctypes.c_void_p(stream.cuda_stream))
+            if st != 0:
+                raise RuntimeError(f"vmb_mean_scan_bwd: {vmb.status_string(st)}")
+        bwd_us = time_alone(bwd)
+        del gy, bws, gouts
     # the materialised operands of the bench workload: 2 x B*4*D*N*L fp32
     small_enough = 8 * wl.B * 4 * wl.D * wl.N * wl.L <= (32 << 30)
     paper = None if args.no_paper_style else {
@@ -632,7 +656,7 @@ def run_ours(args, wl, rank, world, local_rank):
            "paper_style": paper, "grouped_us": grouped, "selection_us": sel_us,
            "h2d": h2d, "d2h": d2h, "clocks": clk.summary(), "fused_ms": fused_ms,
            "launches_per_step": step.launches, "fused_launches": step.fused_launches,
-           "flushed": flush}
+           "flushed": flush, "backward_us": bwd_us}
     del g, outs, step, flush_buf
     torch.cuda.empty_cache()
     peak, _ = measured_peaks()
@@ -690,6 +714,19 @@ def selection_summary(us, wl, peak, R=6):
     gbs = bytes_ / (us / 1e6) / 1e9
     return {"us": us, "algorithmic_bytes": bytes_, "gbs": gbs, "frac_of_peak": gbs / peak, "rank": R,
             "kernel": "tcgen05.mma kind::tf32 (three-product tf32 split for fp32 accuracy), accumulator in TMEM"}
+
+
+def backward_summary(us, wl, peak):
+    """The channel-mean scan's backward: reads u, the raw Delta, dLoss/dy, B and C,
+    writes the gradients of u, Delta, B and C (and the small parameter gradients)."""
+    if us is None:
+        return None
+    s = 2 if wl.dtype == "bf16" else 4
+    bkdl = wl.B * 4 * wl.D * wl.L
+    bknl = wl.B * 4 * wl.N * wl.L
+    bytes_ = s * (5 * bkdl + 4 * bknl) + 2 * 4 * 4 * wl.D * (wl.N + 2)
+    gbs = bytes_ / (us / 1e6) / 1e9
+    return {"us": us, "algorithmic_bytes": bytes_, "gbs": gbs, "frac_of_peak": gbs / peak, "launches": 4}
 
 
 def paper_style_summary(ps, peak):
@@ -802,6 +839,7 @@ def main():
         # grouped basis: d channel groups per direction, each its own channel mean
         # and recurrence (same algorithmic bytes as the mean scan)
         "selection": selection_summary(res["selection_us"], wl, peak),
+        "mean_backward": backward_summary(res["backward_us"], wl, peak),
         "mean_grouped": {str(G): {"groups": G, "us": us, "gbs": kb["mean_scan"] / (us / 1e6) / 1e9,
                                   "frac_of_peak": kb["mean_scan"] / (us / 1e6) / 1e9 / peak}
                          for G, us in res["grouped_us"].items()},
