@@ -48,8 +48,7 @@ __device__ __forceinline__ float rcp(float x) {
 // (Abramowitz & Stegun 4.1.27), truncated after z^12/13: truncation error below
 // (1/3)^14 / 15 ~ 1.4e-8 relative, so the result keeps the relative accuracy of
 // e^-|v| even where log1p(e) is tiny.  No cut-off for large |v|.
-__device__ __forceinline__ float softplus(float v) {
-    float e = ex2(-fabsf(v) * kLog2e);
+__device__ __forceinline__ float softplus_from_e(float v, float e) {
     float z = e * rcp(2.0f + e);
     float w = z * z;
     float p = 1.0f / 13.0f;
@@ -60,6 +59,16 @@ __device__ __forceinline__ float softplus(float v) {
     p = fmaf(p, w, 1.0f / 3.0f);
     p = fmaf(p, w, 1.0f);
     return fmaxf(v, 0.0f) + 2.0f * z * p;
+}
+// e = e^-|v| (ex2.approx), shared with the derivative below
+__device__ __forceinline__ float softplus_e(float v) { return ex2(-fabsf(v) * kLog2e); }
+__device__ __forceinline__ float softplus(float v) { return softplus_from_e(v, softplus_e(v)); }
+
+// softplus'(v) = the logistic function 1 / (1 + e^-v), from e = e^-|v| (no
+// overflow): 1 / (1 + e) for v >= 0, e / (1 + e) otherwise.
+__device__ __forceinline__ float softplus_grad_from_e(float v, float e) {
+    const float r = rcp(1.0f + e);
+    return v >= 0.0f ? r : e * r;
 }
 
 // softplus of two values with the packed f32x2 operations (the same operations

@@ -28,6 +28,9 @@ CASES = [
     (1, 256, 16, 14, 14, "f32", 1),  # two channel blocks of launch 3
     (1, 48, 16, 16, 16, "bf16", 1),
     (2, 32, 8, 6, 10, "bf16", 2),
+    (1, 128, 16, 8, 8, "f32", 2),    # two groups of 64 channels: whole channel blocks per group
+    (1, 96, 16, 12, 12, "bf16", 2),  # groups of 48 channels: a partial channel block per group
+    (1, 64, 16, 40, 40, "f32", 1),   # L = 1600: several step spans of launch 5, chunks of the scans
 ]
 
 
