@@ -628,19 +628,33 @@ def run_ours(args, wl, rank, world, local_rank):
         gouts = dict(u=torch.empty_like(outs["xs"]), delta=torch.empty_like(outs["xs"]),
                      A=torch.empty_like(g["A"]), Bs=torch.empty_like(g["Bs"]), Cs=torch.empty_like(g["Cs"]),
                      Dskip=torch.empty_like(g["Dskip"]), bias=torch.empty_like(g["bias"]))
-        PP = lambda t: ctypes.c_void_p(t.data_ptr())  # noqa: E731
+        PP = lambda t: ctypes.c_void_p(t.data_ptr()) if t is not None else ctypes.c_void_p(0)  # noqa: E731
+        # the training forward: the mean scan that also keeps its group means
+        saved = torch.empty((wl.B, 4, 1, wl.N + 1, wl.L), dtype=torch.float32, device=dev)
+        wst = vmb.default_workspace(dev)
 
-        def bwd():
-            st = vmb.lib.vmb_mean_scan_bwd(
-                PP(outs["xs"]), PP(g["draw"]), PP(g["A"]), PP(g["Bs"]), PP(g["Cs"]), PP(g["Dskip"]), PP(g["bias"]),
-                PP(gy), PP(gouts["u"]), PP(gouts["delta"]), PP(gouts["A"]), PP(gouts["Bs"]), PP(gouts["Cs"]),
-                PP(gouts["Dskip"]), PP(gouts["bias"]), wl.B, 4, wl.D, wl.N, wl.H, wl.W, 1, vmb.VMB_FLAG_SOFTPLUS,
-                vmb.VMB_BF16 if wl.dtype == "bf16" else vmb.VMB_F32, PP(bws), bws.numel(),
-                ctypes.c_void_p(stream.cuda_stream))
-            if st != 0:
-                raise RuntimeError(f"vmb_mean_scan_bwd: {vmb.status_string(st)}")
-        bwd_us = time_alone(bwd)
-        del gy, bws, gouts
+        def train_fwd():
+            vmb.vmb_mean_scan_train_fwd(outs["xs"], g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"],
+                                        wl.H, wl.W, y=outs["ym"], saved=saved, stream=stream)
+        train_us = time_alone(train_fwd)
+
+        def bwd_with(sv):
+            def bwd():
+                st = vmb.lib.vmb_mean_scan_bwd(
+                    PP(outs["xs"]), PP(g["draw"]), PP(g["A"]), PP(g["Bs"]), PP(g["Cs"]), PP(g["Dskip"]),
+                    PP(g["bias"]), PP(gy), PP(sv), PP(gouts["u"]), PP(gouts["delta"]), PP(gouts["A"]),
+                    PP(gouts["Bs"]), PP(gouts["Cs"]), PP(gouts["Dskip"]), PP(gouts["bias"]), wl.B, 4, wl.D, wl.N,
+                    wl.H, wl.W, 1, vmb.VMB_FLAG_SOFTPLUS, vmb.VMB_BF16 if wl.dtype == "bf16" else vmb.VMB_F32,
+                    PP(bws), bws.numel(), ctypes.c_void_p(stream.cuda_stream))
+                if st != 0:
+                    raise RuntimeError(f"vmb_mean_scan_bwd: {vmb.status_string(st)}")
+            return bwd
+        train_fwd()
+        bwd_us = {"saved": time_alone(bwd_with(saved)), "recompute": time_alone(bwd_with(None)),
+                  "train_fwd": train_us}
+        if vmb.vmb_read_status(wst) != 0:
+            raise RuntimeError("device error word set in the training forward")
+        del gy, bws, gouts, saved
     # the materialised operands of the bench workload: 2 x B*4*D*N*L fp32
     small_enough = 8 * wl.B * 4 * wl.D * wl.N * wl.L <= (32 << 30)
     paper = None if args.no_paper_style else {
@@ -718,15 +732,22 @@ def selection_summary(us, wl, peak, R=6):
 
 def backward_summary(us, wl, peak):
     """The channel-mean scan's backward: reads u, the raw Delta, dLoss/dy, B and C,
-    writes the gradients of u, Delta, B and C (and the small parameter gradients)."""
+    writes the gradients of u, Delta, B and C (and the small parameter gradients).
+    "us": given the group means the training forward kept (which it also reads,
+    fp32 [B, K, N + 1, L]); "us_recompute": recomputing them (N exponentials per
+    element).  "train_fwd_us": that forward (the mean scan plus the kept means)."""
     if us is None:
         return None
     s = 2 if wl.dtype == "bf16" else 4
     bkdl = wl.B * 4 * wl.D * wl.L
     bknl = wl.B * 4 * wl.N * wl.L
-    bytes_ = s * (5 * bkdl + 4 * bknl) + 2 * 4 * 4 * wl.D * (wl.N + 2)
-    gbs = bytes_ / (us / 1e6) / 1e9
-    return {"us": us, "algorithmic_bytes": bytes_, "gbs": gbs, "frac_of_peak": gbs / peak, "launches": 4}
+    base = s * (5 * bkdl + 4 * bknl) + 2 * 4 * 4 * wl.D * (wl.N + 2)
+    bytes_ = base + 4 * wl.B * 4 * (wl.N + 1) * wl.L
+    gbs = bytes_ / (us["saved"] / 1e6) / 1e9
+    return {"us": us["saved"], "algorithmic_bytes": bytes_, "gbs": gbs, "frac_of_peak": gbs / peak,
+            "launches": 6, "us_recompute": us["recompute"],
+            "frac_of_peak_recompute": base / (us["recompute"] / 1e6) / 1e9 / peak,
+            "train_fwd_us": us["train_fwd"]}
 
 
 def paper_style_summary(ps, peak):

@@ -339,6 +339,25 @@ vmb_status vmb_selection_fwd(const void* u, const float* WB, const float* WC, co
                              int D, int N, int R, int H, int W, vmb_dtype dtype, cudaStream_t stream);
 
 /*
+ * vmb_mean_scan_train_fwd - vmb_mean_scan_grouped_fwd (groups = 1: the
+ * channel-mean scan of Eq. 9) that also keeps, for vmb_mean_scan_bwd, the
+ * group means it forms on the way:
+ *   saved [B, K, groups, N + 1, L] fp32 out: rows n < N are Abar_n(t) (the
+ *   mean of exp(delta A) over the group), row N is the mean of delta u.
+ * The backward then skips recomputing them (N exponentials per element).
+ * Same arguments and workspace as vmb_mean_scan_grouped_fwd plus `saved`
+ * (not NULL, 4-byte aligned, 16-byte aligned for the backward's vector
+ * loads); flags: VMB_FLAG_SOFTPLUS only (the backward covers Euler Bbar and
+ * the per-channel skip term: VMB_FLAG_B_ZOH and VMB_FLAG_SKIP_MEAN give
+ * VMB_ERR_UNSUPPORTED).  y and ybar are the grouped forward's, bit for bit.
+ */
+vmb_status vmb_mean_scan_train_fwd(const void* u, const void* delta, const float* A, const void* Bs,
+                                   const void* Cs, const float* Dskip, const float* delta_bias,
+                                   void* y, float* ybar, float* saved, int B, int K, int D, int N,
+                                   int H, int W, int groups, unsigned flags, vmb_dtype dtype,
+                                   void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
  * vmb_mean_scan_bwd - gradients of the channel-mean scan (Sec. 2.2, Eq. 9) or,
  * with groups > 1, of the grouped basis (Sec. 2.1, Eq. 8; vmb_mean_scan_grouped_fwd),
  * for the Euler Bbar and the per-channel skip term: the reverse-mode
@@ -352,19 +371,22 @@ vmb_status vmb_selection_fwd(const void* u, const float* WB, const float* WC, co
  *   gBs, gCs [B, K, N, L] (dtype), summed over the groups of each (b, k).
  * Same inputs as vmb_mean_scan_grouped_fwd (delta is the raw Delta); flags:
  * VMB_FLAG_SOFTPLUS (VMB_FLAG_B_ZOH and VMB_FLAG_SKIP_MEAN: VMB_ERR_UNSUPPORTED).
+ * saved: the means vmb_mean_scan_train_fwd wrote for the same inputs,
+ * groups and flags (4-byte aligned), or NULL to recompute them here.
  * workspace: >= vmb_mean_scan_bwd_workspace_bytes(...) bytes, 256-B aligned,
- * any contents (the forward states, group means and adjoints of every
- * sequence, fp32: about 3 x 64 bytes per (b, k, group, step)).  Every
+ * any contents (the group means, chunk carries and adjoints of every
+ * sequence, fp32: about 2 x (N + 2) x 4 bytes per (b, k, group, step)).  Every
  * reduction runs in a fixed order: results are deterministic.  The paper
  * trains no VMeanba layer (it replaces layers of a trained model); this is the
  * chain rule of the forward defined there.
  */
 vmb_status vmb_mean_scan_bwd(const void* u, const void* delta, const float* A, const void* Bs,
                              const void* Cs, const float* Dskip, const float* delta_bias,
-                             const void* gy, void* gu, void* gdelta, float* gA, void* gBs,
-                             void* gCs, float* gDskip, float* gdelta_bias, int B, int K, int D,
-                             int N, int H, int W, int groups, unsigned flags, vmb_dtype dtype,
-                             void* workspace, size_t workspace_bytes, cudaStream_t stream);
+                             const void* gy, const float* saved, void* gu, void* gdelta, float* gA,
+                             void* gBs, void* gCs, float* gDskip, float* gdelta_bias, int B, int K,
+                             int D, int N, int H, int W, int groups, unsigned flags,
+                             vmb_dtype dtype, void* workspace, size_t workspace_bytes,
+                             cudaStream_t stream);
 size_t vmb_mean_scan_bwd_workspace_bytes(int B, int K, int D, int N, int H, int W, int groups,
                                          vmb_dtype dtype);
 

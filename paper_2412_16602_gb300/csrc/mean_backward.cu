@@ -82,9 +82,9 @@ struct BwdParams {
     int nch;                  // scan chunks per sequence
     int nspan, span_len;      // launch-5 spans of the steps
     int vec;                  // rows of Abar, sm, gyb, B, C allow 4-step vector loads
+    bool saved;               // ms holds the forward's means: launch 1 sums gy only
     // workspace arrays (fp32)
-    float* abar;  // [S][kNP][L]
-    float* sm;    // [S][L]
+    float* ms;    // [S][N + 1][L]: Abar_n rows, then sm (the forward's saved means, or launch 1's)
     float* gyb;   // [S][L]
     float* sumP;  // [S][nch][kNP] product of the chunk's Abar
     float* sumH;  // [S][nch][kNP] forward state from zero; after launch 3 the state entering the chunk
@@ -114,10 +114,10 @@ void bwd_spans(long long B, long long K, long long D, long long L, long long G, 
 
 // Workspace layout (256-byte aligned arrays).
 struct BwdLayout {
-    size_t abar, sm, gyb, sumP, sumH, sumV, gab, gs, gBw, gCw, pA, pD, pb, total;
+    size_t ms, gyb, sumP, sumH, sumV, gab, gs, gBw, gCw, pA, pD, pb, total;
     int nch, nspan, span_len;
 };
-BwdLayout bwd_layout(long long B, long long K, long long D, long long L, long long G) {
+BwdLayout bwd_layout(long long B, long long K, long long D, long long N, long long L, long long G) {
     const long long S = B * K * G;
     BwdLayout w{};
     w.nch = (int)((L + kLC - 1) / kLC);
@@ -128,8 +128,7 @@ BwdLayout bwd_layout(long long B, long long K, long long D, long long L, long lo
         o = align_up(o + bytes, 256);
         return at;
     };
-    w.abar = take((size_t)S * kNP * L * 4);
-    w.sm = take((size_t)S * L * 4);
+    w.ms = take((size_t)S * (N + 1) * L * 4);
     w.gyb = take((size_t)S * L * 4);
     w.sumP = take((size_t)S * w.nch * kNP * 4);
     w.sumH = take((size_t)S * w.nch * kNP * 4);
@@ -272,14 +271,53 @@ __global__ void __launch_bounds__(kRThreads, 3) bwd_reduce_kernel(const BwdParam
     for (int i = threadIdx.x; i < (kNP + 2) * kRT; i += kRThreads) {
         const int r = i / kRT, tt = i % kRT;
         if (t0 + tt >= L) continue;
+        if (r >= N && r < kNP) continue;  // padding states
         const float v = red[0][r][tt] + red[1][r][tt];
         if (r < kNP)
-            p.abar[((size_t)seq * kNP + r) * L + t0 + tt] = v * inv;
+            p.ms[((size_t)seq * (N + 1) + r) * L + t0 + tt] = v * inv;
         else if (r == kNP)
-            p.sm[(size_t)seq * L + t0 + tt] = v * inv;
+            p.ms[((size_t)seq * (N + 1) + N) * L + t0 + tt] = v * inv;
         else
             p.gyb[(size_t)seq * L + t0 + tt] = v;
     }
+}
+
+// Launch 1 when the forward kept its means: only gyb = sum_d gy_d per step
+// (CTA = one sequence x kRT steps, the group's channels split in two halves,
+// kPF2 channels in flight per thread).
+constexpr int kPF2 = 8;
+template <typename T>
+__global__ void __launch_bounds__(kRThreads) bwd_gysum_kernel(const BwdParams p) {
+    __shared__ float red[2][kRT];
+    pdl_wait();
+    pdl_launch_dependents();
+    const int L = p.L, M = p.M;
+    const int nlb = (L + kRT - 1) / kRT;
+    const int seq = blockIdx.x / nlb;
+    const int t0 = (blockIdx.x % nlb) * kRT;
+    const int rt = threadIdx.x % kRT, half = threadIdx.x / kRT;
+    const int t = t0 + rt;
+    const bool tv = t < L;
+    const int bk = seq / p.G, g = seq % p.G;
+    const T* gy = static_cast<const T*>(p.gy) + ((size_t)bk * p.D + (size_t)g * M + half) * L + (tv ? t : 0);
+    const uint64_t stream = l2_evict_first();
+    const int nj = (M - half + 1) / 2;  // channels half + 2 i, i < nj
+    const int cs = 2 * L;
+    float s = 0.0f;
+    if (tv) {
+        int i0 = 0;
+        for (; i0 + kPF2 <= nj; i0 += kPF2) {
+            float v[kPF2];
+#pragma unroll
+            for (int q = 0; q < kPF2; ++q) v[q] = ld_hint(gy + (i0 + q) * cs, stream);
+#pragma unroll
+            for (int q = 0; q < kPF2; ++q) s += v[q];
+        }
+        for (; i0 < nj; ++i0) s += ld_hint(gy + i0 * cs, stream);
+    }
+    red[half][rt] = s;
+    __syncthreads();
+    if (half == 0 && tv) p.gyb[(size_t)seq * L + t] = red[0][rt] + red[1][rt];
 }
 
 // One step of either chunk recurrence, in a form both halves of a warp run:
@@ -302,7 +340,8 @@ __device__ __forceinline__ float4 ld4v(const __nv_bfloat16* q) {
 
 // Steps ts .. ts + kSB - 1 of a lane's rows, all loads issued before any is
 // used: Abar_n(t) and the input term (B_n sm forward, C_n gyb adjoint).  Steps
-// at or past tend read nothing and give the identity step (a = 1, term 0).
+// at or past tend, and padding states (n >= N), give the identity step
+// (a = 1, term 0) and read no Abar.
 // With vec (rows 4-element aligned, ts a multiple of 4) whole quads are read
 // as vectors.  rev: the adjoint lanes get the batch in reverse step order.
 template <typename T>
@@ -313,7 +352,7 @@ __device__ __forceinline__ void batch_load(const float* ab, const T* pr, const f
     for (int q = 0; q < kSB / 4; ++q) {
         const int t = ts + 4 * q;
         if (vec && t + 4 <= tend) {
-            const float4 av = ld4v(ab + t), qq = ld4v(qr + t);
+            const float4 av = nv ? ld4v(ab + t) : make_float4(1.0f, 1.0f, 1.0f, 1.0f), qq = ld4v(qr + t);
             const float4 pp = nv ? ld4v(pr + t) : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
             a[4 * q] = av.x, a[4 * q + 1] = av.y, a[4 * q + 2] = av.z, a[4 * q + 3] = av.w;
             qv[4 * q] = qq.x, qv[4 * q + 1] = qq.y, qv[4 * q + 2] = qq.z, qv[4 * q + 3] = qq.w;
@@ -322,7 +361,7 @@ __device__ __forceinline__ void batch_load(const float* ab, const T* pr, const f
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const bool ok = t + i < tend;
-                a[4 * q + i] = ok ? ab[t + i] : 1.0f;
+                a[4 * q + i] = (ok && nv) ? ab[t + i] : 1.0f;
                 pv[4 * q + i] = (ok && nv) ? io<T>::ld(pr + t + i) : 0.0f;
                 qv[4 * q + i] = ok ? qr[t + i] : 0.0f;
             }
@@ -354,9 +393,9 @@ __global__ void __launch_bounds__(32 * kSWarps) bwd_summary_kernel(const BwdPara
     const int seq = pair / p.nch, ch = pair % p.nch;
     const int t0 = ch * kLC, len = min(kLC, L - t0);
     const bool nv = n < N;
-    const float* ab = p.abar + ((size_t)seq * kNP + n) * L;
+    const float* ab = p.ms + ((size_t)seq * (N + 1) + (nv ? n : 0)) * L;
     const T* pr = static_cast<const T*>(dir ? p.Cs : p.Bs) + ((size_t)(seq / p.G) * N + (nv ? n : 0)) * L;
-    const float* qr = (dir ? p.gyb : p.sm) + (size_t)seq * L;
+    const float* qr = dir ? p.gyb + (size_t)seq * L : p.ms + ((size_t)seq * (N + 1) + N) * L;
     // forward lanes take the chunk's batches in order, adjoint lanes in reverse
     const int nb = (len + kSB - 1) / kSB;
     float x = 0.0f, P = 1.0f;
@@ -436,9 +475,9 @@ __global__ void __launch_bounds__(32 * kSWarps) bwd_chunk_kernel(const BwdParams
     float(*hs)[kNP + 1] = s_h[w];
     float(*ls)[kNP + 1] = s_l[w];
     {
-        const float* ab = p.abar + ((size_t)seq * kNP + n) * L;
+        const float* ab = p.ms + ((size_t)seq * (N + 1) + (nv ? n : 0)) * L;
         const T* pr = static_cast<const T*>(dir ? p.Cs : p.Bs) + ((size_t)bk * N + (nv ? n : 0)) * L;
-        const float* qr = (dir ? p.gyb : p.sm) + (size_t)seq * L;
+        const float* qr = dir ? p.gyb + (size_t)seq * L : p.ms + ((size_t)seq * (N + 1) + N) * L;
         const size_t idx = (size_t)pair * kNP + n;
         float x = dir ? p.sumV[idx] : p.sumH[idx];
         if (dir == 0) hs[0][n] = x;
@@ -467,7 +506,7 @@ __global__ void __launch_bounds__(32 * kSWarps) bwd_chunk_kernel(const BwdParams
         gab[j] = m < N ? ls[i][m] * hs[i][m] * invM : 0.0f;
     }
     const T* Bb = static_cast<const T*>(p.Bs) + (size_t)bk * N * L;
-    const float* smv = p.sm + (size_t)seq * L;
+    const float* smv = p.ms + ((size_t)seq * (N + 1) + N) * L;
     const float* gybv = p.gyb + (size_t)seq * L;
     for (int i = lane; i < len; i += 32) {
         const int t = t0 + i;
@@ -642,7 +681,7 @@ __global__ void __launch_bounds__(kCThreads, 4) bwd_channel_kernel(const BwdPara
     const float bias = __ldg(p.bias + c);
     const float dsk = __ldg(p.Dskip + c);
     const int sp = p.softplus_on;
-    float gD = 0.0f, gbs = 0.0f;
+    float2 gD2 = make_float2(0.0f, 0.0f), gbs2 = make_float2(0.0f, 0.0f);  // per step of the pair
     const int ntile = (l1 - l0 + kTS - 1) / kTS;
 #pragma unroll
     for (int j = 0; j < kNS - 1; ++j) {
@@ -665,40 +704,47 @@ __global__ void __launch_bounds__(kCThreads, 4) bwd_channel_kernel(const BwdPara
             const float2 rv = lds2(reinterpret_cast<const T*>(st) + ch * kRowE + lt);
             const float2 uv = lds2(reinterpret_cast<const T*>(st + CS::in) + ch * kRowE + lt);
             const float2 gv = lds2(reinterpret_cast<const T*>(st + 2 * CS::in) + ch * kRowE + lt);
-            float o_gu[2], o_gr[2];
+            // the slot's two steps side by side in the packed f32x2 operations
+            const float2 v2 = __fadd2_rn(rv, make_float2(bias, bias));
+            float2 dl2 = v2, sg2 = make_float2(1.0f, 1.0f);
+            if (sp) {
+                const float2 e2 = softplus2_e(v2);  // e^-|v|, shared with the derivative
+                dl2 = softplus2_from_e(v2, e2);
+                const float2 d1 = __fadd2_rn(e2, make_float2(1.0f, 1.0f));
+                const float2 r2 = make_float2(rcp(d1.x), rcp(d1.y));
+                const float2 er = __fmul2_rn(e2, r2);
+                sg2 = make_float2(v2.x >= 0.0f ? r2.x : er.x, v2.y >= 0.0f ? r2.y : er.y);  // softplus'
+            }
+            const float2 gst2 = *reinterpret_cast<const float2*>(sgs + lt);
+            float sum[2];
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
-                const float r_ = e ? rv.y : rv.x, u_ = e ? uv.y : uv.x, g_ = e ? gv.y : gv.x;
-                const float v = r_ + bias;
-                float dl = v, sgr = 1.0f;
-                if (sp) {
-                    const float ev = softplus_e(v);
-                    dl = softplus_from_e(v, ev);
-                    sgr = softplus_grad_from_e(v, ev);
-                }
-                const float gst = sgs[lt + e];
+                const float dl = e ? dl2.y : dl2.x;
                 const float* w = sgab + (lt + e) * kGabE;
-                const float2 dl2 = make_float2(dl, dl);
+                const float2 dlv = make_float2(dl, dl);
                 float2 acc0 = make_float2(0.0f, 0.0f), acc1 = make_float2(0.0f, 0.0f);
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     const float4 w4 = *reinterpret_cast<const float4*>(w + 4 * q);
                     // states (4q, 4q + 1) and (4q + 2, 4q + 3)
-                    const float2 x01 = __fmul2_rn(dl2, A2[2 * q]), x23 = __fmul2_rn(dl2, A2[2 * q + 1]);
+                    const float2 x01 = __fmul2_rn(dlv, A2[2 * q]), x23 = __fmul2_rn(dlv, A2[2 * q + 1]);
                     const float2 we01 = __fmul2_rn(make_float2(w4.x, w4.y), make_float2(ex2(x01.x), ex2(x01.y)));
                     const float2 we23 = __fmul2_rn(make_float2(w4.z, w4.w), make_float2(ex2(x23.x), ex2(x23.y)));
                     acc0 = __ffma2_rn(we01, A2[2 * q], acc0);
                     acc1 = __ffma2_rn(we23, A2[2 * q + 1], acc1);
-                    gA[2 * q] = __ffma2_rn(we01, dl2, gA[2 * q]);
-                    gA[2 * q + 1] = __ffma2_rn(we23, dl2, gA[2 * q + 1]);
+                    gA[2 * q] = __ffma2_rn(we01, dlv, gA[2 * q]);
+                    gA[2 * q + 1] = __ffma2_rn(we23, dlv, gA[2 * q + 1]);
                 }
-                // sum_n gAbar_n A_n e_n / M = ln 2 sum_n (gAbar_n / M) (A_n log2 e) e_n
-                const float gd = fmaf(gst, u_, ((acc0.x + acc0.y) + (acc1.x + acc1.y)) * kLn2);
-                o_gr[e] = gd * sgr;
-                o_gu[e] = fmaf(dsk, g_, gst * dl);
-                gD = fmaf(g_, u_, gD);
-                gbs += o_gr[e];
+                const float2 s2 = __fadd2_rn(acc0, acc1);
+                sum[e] = s2.x + s2.y;
             }
+            // sum_n gAbar_n A_n e_n / M = ln 2 sum_n (gAbar_n / M) (A_n log2 e) e_n
+            const float2 gd2 = __ffma2_rn(gst2, uv, __fmul2_rn(make_float2(sum[0], sum[1]), make_float2(kLn2, kLn2)));
+            const float2 gr2 = __fmul2_rn(gd2, sg2);
+            const float2 gu2 = __ffma2_rn(make_float2(dsk, dsk), gv, __fmul2_rn(gst2, dl2));
+            gD2 = __ffma2_rn(gv, uv, gD2);
+            gbs2 = __fadd2_rn(gbs2, gr2);
+            const float o_gu[2] = {gu2.x, gu2.y}, o_gr[2] = {gr2.x, gr2.y};
             const int t = ts + lt;
             if (cv) {
                 if (VEC) {
@@ -719,6 +765,7 @@ __global__ void __launch_bounds__(kCThreads, 4) bwd_channel_kernel(const BwdPara
         }
     }
     cp_async_wait<0>();
+    float gD = gD2.x + gD2.y, gbs = gbs2.x + gbs2.y;
     // the slots' sums: (s0 + s1) + (s2 + s3) in every slot
 #pragma unroll
     for (int m = 1; m < kSlots; m *= 2) {
@@ -815,8 +862,9 @@ vmb_status launch_t(const BwdParams& p, cudaStream_t stream) {
         return VMB_ERR_UNSUPPORTED;
     BwdParams q = p;
     void* a1[] = {&q};
-    if (launch_kernel(reinterpret_cast<const void*>(&bwd_reduce_kernel<T>), dim3((unsigned)(S * nlb)), dim3(kRThreads),
-                      0, a1, stream) != cudaSuccess)
+    const void* k1 = p.saved ? reinterpret_cast<const void*>(&bwd_gysum_kernel<T>)
+                             : reinterpret_cast<const void*>(&bwd_reduce_kernel<T>);
+    if (launch_kernel(k1, dim3((unsigned)(S * nlb)), dim3(kRThreads), 0, a1, stream) != cudaSuccess)
         return VMB_ERR_CUDA;
     int np = (int)n_pairs;
     void* a2[] = {&q, &np};
@@ -853,8 +901,8 @@ vmb_status launch_t(const BwdParams& p, cudaStream_t stream) {
 
 }  // namespace
 
-size_t mean_bwd_workspace_bytes(long long B, long long K, long long D, long long L, long long G) {
-    return bwd_layout(B, K, D, L, G).total;
+size_t mean_bwd_workspace_bytes(long long B, long long K, long long D, long long N, long long L, long long G) {
+    return bwd_layout(B, K, D, N, L, G).total;
 }
 
 vmb_status launch_mean_bwd(const MeanBwdArgs& a, cudaStream_t stream) {
@@ -882,20 +930,21 @@ vmb_status launch_mean_bwd(const MeanBwdArgs& a, cudaStream_t stream) {
     p.G = a.groups;
     p.M = a.D / a.groups;
     p.softplus_on = (a.flags & VMB_FLAG_SOFTPLUS) ? 1 : 0;
-    const BwdLayout w = bwd_layout(a.B, a.K, a.D, a.L, a.groups);
+    const BwdLayout w = bwd_layout(a.B, a.K, a.D, a.N, a.L, a.groups);
     p.nch = w.nch;
     p.nspan = w.nspan;
     p.span_len = w.span_len;
+    unsigned char* ws = static_cast<unsigned char*>(a.ws);
+    p.ms = a.saved ? const_cast<float*>(a.saved) : reinterpret_cast<float*>(ws + w.ms);
+    p.saved = a.saved != nullptr;
     {
         const size_t bal = a.dtype == VMB_BF16 ? 8 : 16;
+        // (the caller's saved means need only 4-byte alignment)
         p.vec = (a.L % 4 == 0 && reinterpret_cast<uintptr_t>(a.Bs) % bal == 0 &&
-                 reinterpret_cast<uintptr_t>(a.Cs) % bal == 0)
+                 reinterpret_cast<uintptr_t>(a.Cs) % bal == 0 && reinterpret_cast<uintptr_t>(p.ms) % 16 == 0)
                     ? 1
                     : 0;
     }
-    unsigned char* ws = static_cast<unsigned char*>(a.ws);
-    p.abar = reinterpret_cast<float*>(ws + w.abar);
-    p.sm = reinterpret_cast<float*>(ws + w.sm);
     p.gyb = reinterpret_cast<float*>(ws + w.gyb);
     p.sumP = reinterpret_cast<float*>(ws + w.sumP);
     p.sumH = reinterpret_cast<float*>(ws + w.sumH);

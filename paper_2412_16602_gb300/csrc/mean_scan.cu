@@ -59,6 +59,8 @@ struct MeanParams {
                    // [B, D, W, H] (K = 4, ybar only): direction k's step l reads the value the
                    // cross-scan would have put there, from x (k = 0, 2) or u_t (k = 1, 3)
     const void* u_t;
+    float* save;   // not null: the group means kept for the backward, [n_seq][N + 1][L] fp32
+                   // (rows 0 .. N-1 Abar_n, row N the mean of delta u)
     WsHeader* hdr;
     unsigned* flags;
     float* aggP;
@@ -430,6 +432,11 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
         }
         abar[t * NP + n] = sa * invD;
         bubar[t * NP + n] = io<T>::cvt(sB[n * BCS + t]) * (ZOH ? sb : su) * invD;
+        if (p.save && t < nvalid) {
+            float* sv = p.save + (size_t)seq * (N + 1) * L + l0 + t;
+            if (n < N) sv[(size_t)n * L] = sa * invD;
+            if (n == 0) sv[(size_t)N * L] = su * invD;
+        }
     }
     for (int t = tid; t < TC; t += kThreads) {
         float sd = 0.0f;
@@ -775,6 +782,7 @@ vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     p.bc_group = a.bc_group;
     p.gather_h = a.gather_h;
     p.u_t = a.u_t;
+    p.save = a.saved;
     p.tabvec = al16(a.A) && al16(a.bias) && al16(a.Dskip);
     const WsLayout w = ws_layout(plan);
     unsigned char* ws = static_cast<unsigned char*>(a.ws);

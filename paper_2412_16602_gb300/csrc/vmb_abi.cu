@@ -260,6 +260,33 @@ vmb_status vmb_mean_scan_grouped_fwd(const void* u, const void* delta, const flo
     return run_scan(a, true, stream);
 }
 
+vmb_status vmb_mean_scan_train_fwd(const void* u, const void* delta, const float* A, const void* Bs, const void* Cs,
+                                   const float* Dskip, const float* delta_bias, void* y, float* ybar, float* saved,
+                                   int B, int K, int D, int N, int H, int W, int groups, unsigned flags,
+                                   vmb_dtype dtype, void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+    if (H < 0 || W < 0 || groups < 1) return VMB_ERR_INVALID_ARG;
+    if (D % groups != 0) return VMB_ERR_INVALID_ARG;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    if (flags & (VMB_FLAG_B_ZOH | VMB_FLAG_SKIP_MEAN)) {
+        // the backward covers Euler Bbar and the per-channel skip term; anything
+        // else is rejected after the shape checks the other entry points make
+        if (!dtype_ok(dtype) || B < 0 || K < 0 || D < 0 || N < 0) return VMB_ERR_INVALID_ARG;
+        return VMB_ERR_UNSUPPORTED;
+    }
+    long long kg = 0;
+    if (!count(&kg, {K, groups}) || kg > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    ScanArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, y, ybar, B, (int)kg, D / groups, N, H * W, flags, dtype,
+               workspace, workspace_bytes};
+    a.bc_group = groups;
+    bool empty = false;
+    vmb_status s = validate_scan(a, true, &empty);
+    if (s != VMB_OK || empty) return s;
+    if (!saved) return VMB_ERR_INVALID_ARG;
+    if (!aligned(saved, 4)) return VMB_ERR_MISALIGNED;
+    a.saved = saved;
+    return run_scan(a, true, stream);
+}
+
 vmb_status vmb_mean_scan_merge_fwd(const void* u, const void* delta, const float* A, const void* Bs, const void* Cs,
                                    const float* Dskip, const float* delta_bias, const void* x, void* out, float* ybar,
                                    int B, int D, int N, int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,
@@ -330,6 +357,7 @@ static vmb_status check_bwd(const MeanBwdArgs& a, bool* empty) {
                           a.gDskip, a.gbias};
     for (const void* q : ptrs)
         if (!q) return VMB_ERR_INVALID_ARG;
+    if (a.saved && !aligned(a.saved, 4)) return VMB_ERR_MISALIGNED;
     const size_t es = esize(a.dtype);
     const void* elems[] = {a.u, a.delta, a.Bs, a.Cs, a.gy, a.gu, a.gdelta, a.gBs, a.gCs};
     for (const void* q : elems)
@@ -400,29 +428,30 @@ size_t vmb_mean_scan_bwd_workspace_bytes(int B, int K, int D, int N, int H, int 
     if (H < 0 || W < 0 || (long long)H * W > INT_MAX) return 0;
     static const float dummy[4] = {0, 0, 0, 0};
     float* dm = const_cast<float*>(dummy);
-    MeanBwdArgs a{dummy, dummy, dummy, dummy, dummy, dummy, dummy, dummy, dm, dm, dm, dm, dm, dm, dm,
+    MeanBwdArgs a{dummy, dummy, dummy, dummy, dummy, dummy, dummy, dummy, nullptr, dm, dm, dm, dm, dm, dm, dm,
                   B, K, D, N, H * W, groups, VMB_FLAG_SOFTPLUS, dtype, nullptr, 0};
     bool empty = false;
     if (check_bwd(a, &empty) != VMB_OK) return 0;
     if (empty) return 256;
-    return mean_bwd_workspace_bytes(B, K, D, (long long)H * W, groups);
+    return mean_bwd_workspace_bytes(B, K, D, N, (long long)H * W, groups);
 }
 
 vmb_status vmb_mean_scan_bwd(const void* u, const void* delta, const float* A, const void* Bs, const void* Cs,
-                             const float* Dskip, const float* delta_bias, const void* gy, void* gu, void* gdelta,
+                             const float* Dskip, const float* delta_bias, const void* gy, const float* saved,
+                             void* gu, void* gdelta,
                              float* gA, void* gBs, void* gCs, float* gDskip, float* gdelta_bias, int B, int K, int D,
                              int N, int H, int W, int groups, unsigned flags, vmb_dtype dtype, void* workspace,
                              size_t workspace_bytes, cudaStream_t stream) {
     if (H < 0 || W < 0) return VMB_ERR_INVALID_ARG;
     if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
-    MeanBwdArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, gy, gu, gdelta, gA, gBs, gCs, gDskip, gdelta_bias,
+    MeanBwdArgs a{u, delta, A, Bs, Cs, Dskip, delta_bias, gy, saved, gu, gdelta, gA, gBs, gCs, gDskip, gdelta_bias,
                   B, K, D, N, H * W, groups, flags, dtype, workspace, workspace_bytes};
     bool empty = false;
     vmb_status s = check_bwd(a, &empty);
     if (s != VMB_OK || empty) return s;
     if (!workspace) return VMB_ERR_WORKSPACE;
     if (!aligned(workspace, 256)) return VMB_ERR_MISALIGNED;
-    if (workspace_bytes < mean_bwd_workspace_bytes(B, K, D, (long long)H * W, groups)) return VMB_ERR_WORKSPACE;
+    if (workspace_bytes < mean_bwd_workspace_bytes(B, K, D, N, (long long)H * W, groups)) return VMB_ERR_WORKSPACE;
     return launch_mean_bwd(a, stream);
 }
 

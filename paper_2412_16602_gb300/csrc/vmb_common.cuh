@@ -73,12 +73,14 @@ __device__ __forceinline__ float softplus_grad_from_e(float v, float e) {
 
 // softplus of two values with the packed f32x2 operations (the same operations
 // as softplus() applied to each value, issued as one instruction per pair
-// where the FMA pipe allows it).
-__device__ __forceinline__ float2 softplus2(float2 v) {
+// where the FMA pipe allows it); softplus2_from_e takes e = e^-|v| of both.
+__device__ __forceinline__ float2 softplus2_e(float2 v) {
     const float2 av = make_float2(__int_as_float(__float_as_int(v.x) & 0x7fffffff),
                                   __int_as_float(__float_as_int(v.y) & 0x7fffffff));
     const float2 m = __fmul2_rn(av, make_float2(-kLog2e, -kLog2e));
-    const float2 e = make_float2(ex2(m.x), ex2(m.y));
+    return make_float2(ex2(m.x), ex2(m.y));
+}
+__device__ __forceinline__ float2 softplus2_from_e(float2 v, float2 e) {
     const float2 den = __fadd2_rn(e, make_float2(2.0f, 2.0f));
     const float2 z = __fmul2_rn(e, make_float2(rcp(den.x), rcp(den.y)));
     const float2 w = __fmul2_rn(z, z);
@@ -92,6 +94,7 @@ __device__ __forceinline__ float2 softplus2(float2 v) {
     const float2 z2 = __fadd2_rn(z, z);
     return __ffma2_rn(z2, q, make_float2(fmaxf(v.x, 0.0f), fmaxf(v.y, 0.0f)));
 }
+__device__ __forceinline__ float2 softplus2(float2 v) { return softplus2_from_e(v, softplus2_e(v)); }
 
 // ------------------------------------------- programmatic dependent launch
 

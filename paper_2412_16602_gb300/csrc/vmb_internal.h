@@ -32,6 +32,7 @@ struct ScanArgs {
                             // [B, D, W, H]; directions 0 / 2 read x, 1 / 3 read u_t (no materialised
                             // cross-scan)
     const void* u_t = nullptr;
+    float* saved = nullptr;  // mean path: the group means kept for the backward, [B*K][N + 1][L] fp32
 };
 
 // Execution plan of an L-chunked scan: how the (sequence, chunk) grid is cut
@@ -115,6 +116,7 @@ struct MeanBwdArgs {
     const float* Dskip;
     const float* bias;
     const void* gy;
+    const float* saved;  // the forward's group means, or null (recomputed)
     void* gu;
     void* gdelta;
     float* gA;
@@ -152,7 +154,7 @@ vmb_status launch_map_transpose(const void* x, void* xt, int B, int D, int H, in
                                 cudaStream_t stream);
 vmb_status launch_discretise(const DiscArgs& a, bool mean, cudaStream_t stream);
 vmb_status launch_selection(const SelArgs& a, cudaStream_t stream);
-size_t mean_bwd_workspace_bytes(long long B, long long K, long long D, long long L, long long G);
+size_t mean_bwd_workspace_bytes(long long B, long long K, long long D, long long N, long long L, long long G);
 vmb_status launch_mean_bwd(const MeanBwdArgs& a, cudaStream_t stream);
 vmb_status launch_scan_only(const OnlyArgs& a, cudaStream_t stream);
 vmb_status launch_mean_merge(const void* x, const float* ybar, const float* Dskip, void* out, int B, int D, int H,

@@ -41,7 +41,8 @@ EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb
            "vmb_selective_scan_fwd",
            "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_ss2d_mean_fwd",
            "vmb_discretise_fwd", "vmb_discretise_mean_fwd",
-           "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_mean_scan_bwd", "vmb_mean_scan_bwd_workspace_bytes",
+           "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_mean_scan_train_fwd", "vmb_mean_scan_bwd",
+           "vmb_mean_scan_bwd_workspace_bytes",
            "vmb_read_status", "vmb_status_string", "vmb_version"]
 
 
@@ -71,7 +72,8 @@ def _load() -> ctypes.CDLL:
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
     lib.vmb_selection_fwd.argtypes = [vp] * 8 + [i] * 7 + [i, vp]
-    lib.vmb_mean_scan_bwd.argtypes = [vp] * 15 + [i] * 7 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_train_fwd.argtypes = [vp] * 10 + [i] * 7 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_bwd.argtypes = [vp] * 16 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_bwd_workspace_bytes.argtypes = [i] * 8
     lib.vmb_mean_scan_bwd_workspace_bytes.restype = sz
     lib.vmb_read_status.argtypes = [vp, vp]
@@ -297,6 +299,38 @@ def vmb_mean_scan_grouped_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, H: int, W:
     return y, ybar
 
 
+def vmb_mean_scan_train_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, H: int, W: int, *, groups: int = 1,
+                            y=None, ybar=None, saved=None, flags: int = VMB_FLAG_SOFTPLUS, workspace=None,
+                            stream=None):
+    """The (grouped) channel-mean scan that also keeps its group means for the backward: returns
+    (y [B, K, D, L], saved [B, K, groups, N + 1, L] fp32, ybar or None)."""
+    B, K, D, N, L = _scan_shapes(u, delta, A, Bs, Cs, Dskip, delta_bias, H, W)
+    if groups < 1 or D % groups:
+        raise ValueError("groups must be >= 1 and divide D")
+    if y is None:
+        y = torch.empty_like(u)
+    _dev(y, "y")
+    if y.shape != u.shape or y.dtype != u.dtype:
+        raise ValueError("y must match u")
+    if saved is None:
+        saved = torch.empty((B, K, groups, N + 1, L), dtype=torch.float32, device=u.device)
+    _dev(saved, "saved")
+    if tuple(saved.shape) != (B, K, groups, N + 1, L) or saved.dtype != torch.float32:
+        raise ValueError("saved must be float32 [B, K, groups, N + 1, L]")
+    if ybar is not None:
+        _dev(ybar, "ybar")
+        if ybar.shape != (B, K, groups, L) or ybar.dtype != torch.float32:
+            raise ValueError("ybar must be float32 [B, K, groups, L]")
+    ws_bytes = vmb_scan_workspace_bytes(VMB_PATH_MEAN, B, K * groups, D // groups, N, H, W, u.dtype)
+    if workspace is None:
+        workspace = _default_ws.get(ws_bytes, u.device)
+    _check(lib.vmb_mean_scan_train_fwd(_ptr(u), _ptr(delta), _ptr(A), _ptr(Bs), _ptr(Cs), _ptr(Dskip),
+                                       _ptr(delta_bias), _ptr(y), _ptr(ybar), _ptr(saved), B, K, D, N, H, W, groups,
+                                       flags, _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
+                                       _stream(stream)), "vmb_mean_scan_train_fwd")
+    return y, saved, ybar
+
+
 def vmb_mean_scan_merge_fwd(u, delta, A, Bs, Cs, Dskip, delta_bias, x, H: int, W: int, *,
                             out=None, ybar=None, flags: int = VMB_FLAG_SOFTPLUS, workspace=None, stream=None):
     """Channel-mean path with the broadcast fused into the cross-merge:
@@ -478,22 +512,27 @@ def vmb_mean_scan_bwd_workspace_bytes(B: int, K: int, D: int, N: int, H: int, W:
 
 
 def vmb_mean_scan_bwd(u, delta, A, Bs, Cs, Dskip, delta_bias, gy, H: int, W: int, *, groups: int = 1,
-                      flags: int = VMB_FLAG_SOFTPLUS, workspace=None, stream=None) -> dict:
+                      saved=None, flags: int = VMB_FLAG_SOFTPLUS, workspace=None, stream=None) -> dict:
     """Gradients of the (grouped) channel-mean scan given gy = dLoss/dy [B, K, D, H*W]: returns
-    dict(u, delta, A, Bs, Cs, Dskip, delta_bias) with the inputs' shapes (delta: the raw Delta)."""
+    dict(u, delta, A, Bs, Cs, Dskip, delta_bias) with the inputs' shapes (delta: the raw Delta).
+    saved: the group means vmb_mean_scan_train_fwd kept for these inputs, or None (recomputed)."""
     B, K, D, N, L = _scan_shapes(u, delta, A, Bs, Cs, Dskip, delta_bias, H, W)
     _dev(gy, "gy")
     if gy.shape != u.shape or gy.dtype != u.dtype:
         raise ValueError("gy must match u")
     if groups < 1 or D % groups:
         raise ValueError("groups must be >= 1 and divide D")
+    if saved is not None:
+        _dev(saved, "saved")
+        if tuple(saved.shape) != (B, K, groups, N + 1, L) or saved.dtype != torch.float32:
+            raise ValueError("saved must be float32 [B, K, groups, N + 1, L]")
     out = dict(u=torch.empty_like(u), delta=torch.empty_like(u), A=torch.empty_like(A), Bs=torch.empty_like(Bs),
                Cs=torch.empty_like(Cs), Dskip=torch.empty_like(Dskip), delta_bias=torch.empty_like(delta_bias))
     ws_bytes = vmb_mean_scan_bwd_workspace_bytes(B, K, D, N, H, W, groups, u.dtype)
     if workspace is None:
         workspace = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=u.device)
     _check(lib.vmb_mean_scan_bwd(_ptr(u), _ptr(delta), _ptr(A), _ptr(Bs), _ptr(Cs), _ptr(Dskip), _ptr(delta_bias),
-                                 _ptr(gy), _ptr(out["u"]), _ptr(out["delta"]), _ptr(out["A"]), _ptr(out["Bs"]),
+                                 _ptr(gy), _ptr(saved), _ptr(out["u"]), _ptr(out["delta"]), _ptr(out["A"]), _ptr(out["Bs"]),
                                  _ptr(out["Cs"]), _ptr(out["Dskip"]), _ptr(out["delta_bias"]), B, K, D, N, H, W,
                                  groups, flags, _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
                                  _stream(stream)), "vmb_mean_scan_bwd")

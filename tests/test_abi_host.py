@@ -31,7 +31,8 @@ def lib():
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
     lib.vmb_selection_fwd.argtypes = [vp] * 8 + [i] * 7 + [i, vp]
-    lib.vmb_mean_scan_bwd.argtypes = [vp] * 15 + [i] * 7 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_bwd.argtypes = [vp] * 16 + [i] * 7 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_train_fwd.argtypes = [vp] * 10 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_bwd_workspace_bytes.argtypes = [i] * 8
     lib.vmb_mean_scan_bwd_workspace_bytes.restype = sz
     lib.vmb_status_string.argtypes = [i]
@@ -239,7 +240,7 @@ def test_selection_validation(lib):
 
 def bwd_call(lib, *, ptrs=None, B=1, K=4, D=8, N=16, H=4, W=4, groups=1, flags=1, dtype=0, ws=0x100000,
              ws_bytes=1 << 30):
-    p = [FAKE] * 15 if ptrs is None else ptrs
+    p = [FAKE] * 16 if ptrs is None else ptrs
     return lib.vmb_mean_scan_bwd(*p, B, K, D, N, H, W, groups, flags, dtype, ws, ws_bytes, S)
 
 
@@ -247,8 +248,9 @@ def test_mean_backward_validation(lib):
     """The backward rejects invalid arguments and the flags it does not
     implement before any launch."""
     assert bwd_call(lib, B=-1) == 1
-    assert bwd_call(lib, ptrs=[FAKE] * 14 + [0]) == 1                # a null gradient output
-    assert bwd_call(lib, ptrs=[FAKE + 2] + [FAKE] * 14) == 2         # misaligned fp32 input
+    assert bwd_call(lib, ptrs=[FAKE] * 15 + [0]) == 1                # a null gradient output
+    assert bwd_call(lib, ptrs=[FAKE + 2] + [FAKE] * 15) == 2         # misaligned fp32 input
+    assert bwd_call(lib, ptrs=[FAKE] * 8 + [FAKE + 2] + [FAKE] * 7) == 2  # misaligned saved means
     assert bwd_call(lib, groups=3) == 1                              # groups must divide D
     assert bwd_call(lib, groups=0) == 1
     assert bwd_call(lib, N=17) == 3
@@ -257,7 +259,21 @@ def test_mean_backward_validation(lib):
     assert bwd_call(lib, flags=0x100) == 1
     assert bwd_call(lib, ws=0) == 4
     assert bwd_call(lib, ws_bytes=256) == 4
-    assert bwd_call(lib, ptrs=[0] * 15, B=0, ws=0) == 0             # empty problem
+    assert bwd_call(lib, ptrs=[0] * 16, B=0, ws=0) == 0             # empty problem
     assert lib.vmb_mean_scan_bwd_workspace_bytes(1, 4, 8, 16, 4, 4, 3, 0) == 0
     assert lib.vmb_mean_scan_bwd_workspace_bytes(0, 4, 8, 16, 4, 4, 1, 0) == 256
     assert lib.vmb_mean_scan_bwd_workspace_bytes(2, 4, 8, 16, 4, 4, 2, 0) > 256
+
+
+def test_train_forward_validation(lib):
+    """The training forward (mean scan keeping its group means) rejects a
+    missing or misaligned buffer and the forms the backward does not cover."""
+    def call(ptrs=None, B=1, K=4, D=8, N=16, H=4, W=4, groups=1, flags=1, dtype=0):
+        p = [FAKE] * 10 if ptrs is None else ptrs
+        return lib.vmb_mean_scan_train_fwd(*p, B, K, D, N, H, W, groups, flags, dtype, 0x100000, 1 << 30, S)
+    assert call(ptrs=[FAKE] * 9 + [0]) == 1          # no buffer for the means
+    assert call(ptrs=[FAKE] * 9 + [FAKE + 2]) == 2   # misaligned means
+    assert call(flags=1 | 2) == 3                    # zero-order hold: the backward does not cover it
+    assert call(flags=1 | 4) == 3                    # mean skip term: likewise
+    assert call(groups=3) == 1                       # groups must divide D
+    assert call(B=0, ptrs=[0] * 10) == 0             # empty problem

@@ -59,6 +59,36 @@ def test_mean_backward_matches_oracle(case):
         assert torch.equal(got[gname], got2[gname]), f"grad {gname} must be deterministic"
 
 
+@pytest.mark.parametrize("case", CASES, ids=[f"B{c[0]}_D{c[1]}_N{c[2]}_{c[3]}x{c[4]}_{c[5]}_G{c[6]}" for c in CASES])
+def test_mean_backward_from_saved_means(case):
+    """The training pair: vmb_mean_scan_train_fwd (y bit-identical to the
+    grouped forward) keeps the group means, and the backward given them matches
+    the oracle's gradients."""
+    B, D, N, H, W, dt, G = case
+    wl = workloads.small_case(B=B, D=D, N=N, H=H, W=W, dtype=dt, seed=940 + D + N + G)
+    inp = workloads.make_inputs(wl, params="random")
+    g = to_device(inp, DEV)
+    xs = vmb.vmb_cross_scan(g["x"])
+    args = (xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"])
+    y, saved, _ = vmb.vmb_mean_scan_train_fwd(*args, H, W, groups=G)
+    y_ref, _ = vmb.vmb_mean_scan_grouped_fwd(*args, H, W, G)
+    assert torch.equal(y, y_ref), "the training forward's y must be the grouped forward's"
+    rng = np.random.default_rng(941 + D)
+    gy_np = rng.standard_normal((B, 4, D, H * W)).astype(np.float32)
+    if dt == "bf16":
+        gy_np = workloads.round_to_bf16(gy_np)
+    gy = torch.from_numpy(gy_np).to(xs.dtype).to(DEV)
+    got = vmb.vmb_mean_scan_bwd(*args, gy, H, W, groups=G, saved=saved)
+    torch.cuda.synchronize()
+    assert vmb.vmb_read_status() == vmb.VMB_OK
+    ref = oracle.mean_scan_bwd(oracle.cross_scan(inp.x), inp.draw, inp.A, inp.Bs, inp.Cs, inp.Dskip, inp.bias, gy_np,
+                               groups=G)
+    names = {"u": "u", "delta": "delta", "A": "A", "Bs": "Bs", "Cs": "Cs", "Dskip": "Dskip", "delta_bias": "bias"}
+    for gname, rname in names.items():
+        kind = dt if gname in ("u", "delta", "Bs", "Cs") else ("f32" if dt == "f32" else "bf16")
+        check(to_numpy(got[gname]), ref[rname], kind, f"grad {gname} (saved means)")
+
+
 def test_mean_backward_softplus_off():
     wl = workloads.small_case(B=1, D=20, N=16, H=6, W=9, seed=931)
     inp = workloads.make_inputs(wl, params="random")
