@@ -46,8 +46,8 @@ constexpr int kRT = 128;          // steps per CTA of launch 1
 constexpr int kRThreads = 2 * kRT;
 constexpr int kCG = 256;          // channels whose A rows are staged at a time (launch 1)
 constexpr int kPF = 4;            // channels a launch-1 thread has in flight
-constexpr int kLC = 64;           // steps per scan chunk (launches 2-4)
-constexpr int kSWarps = 4;        // chunks per CTA of launches 2 and 4
+constexpr int kLC = 32;           // steps per scan chunk (launches 2-4)
+constexpr int kSWarps = 8;        // chunks per CTA of launches 2 and 4
 constexpr int kSB = 16;           // steps whose loads a launch-2/4 lane issues together
 constexpr int kCThreads = 128;    // threads per CTA of launch 5
 constexpr int kSlots = 4;         // launch-5 threads per channel
@@ -369,13 +369,12 @@ __device__ __forceinline__ void batch_load(const float* ab, const T* pr, const f
     }
 #pragma unroll
     for (int i = 0; i < kSB; ++i) pq[i] = pv[i] * qv[i];
-    if (rev) {
+    // the two halves of a warp differ in rev: selects, not a branch
 #pragma unroll
-        for (int i = 0; i < kSB / 2; ++i) {
-            const float x = a[i], y = pq[i];
-            a[i] = a[kSB - 1 - i], pq[i] = pq[kSB - 1 - i];
-            a[kSB - 1 - i] = x, pq[kSB - 1 - i] = y;
-        }
+    for (int i = 0; i < kSB / 2; ++i) {
+        const float x = a[i], y = pq[i], xr = a[kSB - 1 - i], yr = pq[kSB - 1 - i];
+        a[i] = rev ? xr : x, pq[i] = rev ? yr : y;
+        a[kSB - 1 - i] = rev ? x : xr, pq[kSB - 1 - i] = rev ? y : yr;
     }
 }
 
@@ -482,18 +481,18 @@ __global__ void __launch_bounds__(32 * kSWarps) bwd_chunk_kernel(const BwdParams
         float x = dir ? p.sumV[idx] : p.sumH[idx];
         if (dir == 0) hs[0][n] = x;
         const int nb = (len + kSB - 1) / kSB;
+        // the row a lane stores step i of a batch in: forward h(t) at hs row
+        // b0 + i + 1, adjoint lam(t) at ls row b0 + kSB - 1 - i (one store, no branch)
+        const int rstep = dir ? -(kNP + 1) : kNP + 1;
         for (int bi = 0; bi < nb; ++bi) {
             const int b0 = kSB * (dir ? nb - 1 - bi : bi);  // first step of the batch within the chunk
             float a[kSB], pq[kSB];
             batch_load<T>(ab, pr, qr, nv, p.vec, dir, t0 + b0, t0 + len, a, pq);
+            float* rowp = dir ? &ls[b0 + kSB - 1][n] : &hs[b0 + 1][n];
 #pragma unroll
             for (int i = 0; i < kSB; ++i) {
                 // steps past the chunk are identity steps; their rows (< kLC) are never read
-                const float r = chunk_step(dir, a[i], pq[i], x);
-                if (dir)
-                    ls[b0 + kSB - 1 - i][n] = r;
-                else
-                    hs[b0 + i + 1][n] = r;
+                rowp[i * rstep] = chunk_step(dir, a[i], pq[i], x);
             }
         }
     }
