@@ -21,6 +21,9 @@
 // carry-in state; the second pass recomputes the chunk from that state and
 // writes y.  Chunk order follows a ticket counter, so a CTA only waits on
 // CTAs that started before it; every wait is bounded.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include <mutex>
 #include <type_traits>
 
@@ -1439,6 +1442,209 @@ __global__ void __launch_bounds__(PackedLayout<T, PS>::THREADS, PS::MINB) full_p
     cp_async_wait<0>();
 }
 
+// ------------------------------------- warp-specialised variant (tensor copies)
+// The packed state update of the streaming variant, with the tile movement
+// taken off the compute warps.  A CTA is CW consumer warps (one channel per
+// lane, all 16 states in registers) and one producer warp.  The producer
+// issues, per stage of TS steps, four tiled tensor copies (u and delta:
+// DT rows x TS steps, B and C: 16 rows x TS steps) into an NSTG-deep ring
+// and, once a stage has landed, converts its B and C rows into fp32
+// [t][B0..15, C0..15] rows for broadcast reads.  Stages are handed over with
+// mbarriers (landed / ready / released), so no barrier spans the CTA and the
+// copies of the next stages overlap the consumers' arithmetic.  Each
+// consumer lane computes delta = softplus(raw + bias) of its own row of the
+// stage, runs the packed update (the same operations, in the same order, as
+// full_packed_kernel: its y is bit-identical) and stores y from registers.
+// Requires rows of 16-byte multiples and 16-byte aligned tensors (the host
+// picks this variant only then); every wait is bounded.
+template <int CW_, int TS_, int NSTG_, int MINB_>
+struct WsShape {
+    static constexpr int CW = CW_, TS = TS_, NSTG = NSTG_, MINB = MINB_;
+};
+
+struct TensorMaps {
+    CUtensorMap u, dl, B, C;  // [B*K][D][L] (u, delta) and [B*K][N][L] (B, C)
+};
+
+template <typename T, class WS>
+struct WsTileLayout {
+    static constexpr int CW = WS::CW, DT = 32 * CW, NP = 16, TS = WS::TS, NSTG = WS::NSTG;
+    static constexpr int THREADS = DT + 32;
+    static constexpr int U_BYTES = DT * TS * (int)sizeof(T);   // one u (or delta) box
+    static constexpr int BC_BYTES = NP * TS * (int)sizeof(T);  // one B (or C) box
+    static constexpr int RAW_STAGE = 2 * U_BYTES + 2 * BC_BYTES;
+    static constexpr int BCT_STAGE = TS * 2 * NP * 4;           // fp32 [TS][B0..15, C0..15]
+    static constexpr size_t bct_off = (size_t)NSTG * RAW_STAGE;
+    static constexpr size_t bar_off = bct_off + (size_t)NSTG * BCT_STAGE;
+    static constexpr size_t bytes = bar_off + (size_t)3 * NSTG * 8;
+    static_assert(U_BYTES % 128 == 0 && BC_BYTES % 128 == 0 && TS % 4 == 0 && TS * sizeof(T) % 16 == 0,
+                  "tensor-copy boxes: 16-byte rows, 128-byte aligned boxes");
+};
+
+constexpr uint64_t kStageWaitNs = 1000000000ull;  // 1 s per stage hand-over
+
+template <typename T, class WS>
+__global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
+    full_ws_kernel(const FullParams p, const __grid_constant__ TensorMaps tm) {
+    pdl_wait();
+    pdl_launch_dependents();
+    using LY = WsTileLayout<T, WS>;
+    constexpr int DT = LY::DT, NP = 16, TS = LY::TS, NSTG = LY::NSTG, NPR = NP / 2;
+    extern __shared__ __align__(128) unsigned char smem_ws[];
+    unsigned char* smem = smem_ws;
+    const uint32_t sbase = smem_u32(smem);
+    const uint32_t bar0 = sbase + (uint32_t)LY::bar_off;
+    // landed[i]: the four copies of the stage in slot i arrived; ready[i]: its
+    // B/C rows are converted; released[i]: every consumer warp is done with it
+    auto landed = [&](int i) { return bar0 + 8u * i; };
+    auto ready = [&](int i) { return bar0 + 8u * (NSTG + i); };
+    auto released = [&](int i) { return bar0 + 8u * (2 * NSTG + i); };
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int tile = blockIdx.x;
+    const int bk = tile / p.tiles_per_bk;
+    const int d0 = (tile % p.tiles_per_bk) * DT;
+    const int k = bk % p.K;
+    const int L = p.L;
+    const int nst = (L + TS - 1) / TS;
+    const int cwarps = min(LY::CW, (p.D - d0 + 31) / 32);  // consumer warps with at least one channel
+    if (tid == 0) {
+        for (int i = 0; i < NSTG; ++i) {
+            mbarrier_init(landed(i), 1);
+            mbarrier_init(ready(i), 32);
+            mbarrier_init(released(i), cwarps);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    __syncthreads();
+    if (warp == LY::CW) {
+        // ------------------------------------------------------ producer warp
+        auto issue = [&](int s) {
+            const int slot = s % NSTG;
+            const uint32_t dst = sbase + (uint32_t)(slot * LY::RAW_STAGE);
+            mbarrier_expect_tx(landed(slot), (unsigned)LY::RAW_STAGE);
+            tma_load_3d(dst, &tm.u, s * TS, d0, bk, landed(slot));
+            tma_load_3d(dst + LY::U_BYTES, &tm.dl, s * TS, d0, bk, landed(slot));
+            tma_load_3d(dst + 2 * LY::U_BYTES, &tm.B, s * TS, 0, bk, landed(slot));
+            tma_load_3d(dst + 2 * LY::U_BYTES + LY::BC_BYTES, &tm.C, s * TS, 0, bk, landed(slot));
+        };
+        if (lane == 0)
+            for (int s = 0; s < NSTG && s < nst; ++s) issue(s);
+        int seen = 0;  // stages whose copies this warp has seen land
+        bool ok = true;
+        for (int s = 0; s < nst; ++s) {
+            const int slot = s % NSTG;
+            if (!(ok = mbarrier_wait(landed(slot), (s / NSTG) & 1, kStageWaitNs))) break;
+            seen = s + 1;
+            // lane r converts row r of [B rows 0..15, C rows 0..15] into column r
+            const T* rb = reinterpret_cast<const T*>(smem + slot * LY::RAW_STAGE + 2 * LY::U_BYTES) + lane * TS;
+            float* bo = reinterpret_cast<float*>(smem + LY::bct_off + slot * LY::BCT_STAGE);
+#pragma unroll
+            for (int t = 0; t < TS; ++t) bo[t * 2 * NP + lane] = io<T>::cvt(rb[t]);
+            __syncwarp();
+            mbarrier_arrive(ready(slot));
+            // refill the slot of stage s - 1 once the consumers released it
+            if (s >= 1 && s - 1 + NSTG < nst) {
+                const int ps = (s - 1) % NSTG;
+                if (!(ok = mbarrier_wait(released(ps), ((s - 1) / NSTG) & 1, kStageWaitNs))) break;
+                if (lane == 0) issue(s - 1 + NSTG);
+            }
+        }
+        if (!ok) {
+            if (lane == 0) atomicOr(&p.hdr->err, kErrTimeout);
+            // every copy issued must land before the CTA exits
+            const int issued = min(nst, seen + NSTG);
+            for (int s = seen; s < issued; ++s) mbarrier_wait(landed(s % NSTG), (s / NSTG) & 1, kStageWaitNs);
+        }
+        return;
+    }
+    if (warp >= cwarps) return;  // a tile's channels past D: no work, not counted by `released`
+    // -------------------------------------------------------- consumer warps
+    const int c = tid;
+    const int d = d0 + c;
+    const bool cval = d < p.D;
+    const size_t row0 = (size_t)bk * p.D + d0;
+    const float bias = cval ? p.bias[(size_t)k * p.D + d] : 0.0f;
+    const float dsk = cval ? p.Dskip[(size_t)k * p.D + d] : 0.0f;
+    const float* Ad = p.A + ((size_t)k * p.D + d) * p.N;
+    float2 A2[NPR], h[NPR];
+#pragma unroll
+    for (int i = 0; i < NPR; ++i) {
+        const int n = 2 * i;
+        A2[i] = make_float2((cval && n < p.N) ? Ad[n] * kLog2e : 0.0f, (cval && n + 1 < p.N) ? Ad[n + 1] * kLog2e : 0.0f);
+        h[i] = make_float2(0.0f, 0.0f);
+    }
+    T* yrow = static_cast<T*>(p.y) + (row0 + c) * (size_t)L;
+    for (int s = 0; s < nst; ++s) {
+        const int slot = s % NSTG;
+        if (!mbarrier_wait(ready(slot), (s / NSTG) & 1, kStageWaitNs)) {
+            atomicOr(&p.hdr->err, kErrTimeout);
+            return;
+        }
+        const int l0 = s * TS;
+        const int nvalid = min(TS, L - l0);
+        const T* ru = reinterpret_cast<const T*>(smem + slot * LY::RAW_STAGE) + c * TS;
+        const T* rd = reinterpret_cast<const T*>(smem + slot * LY::RAW_STAGE + LY::U_BYTES) + c * TS;
+        float uv[TS], dv[TS];
+#pragma unroll
+        for (int j = 0; j < TS; j += 4) {
+            float q[4], w[4];
+            load4(ru + j, q);
+            load4(rd + j, w);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                uv[j + e] = q[e];
+                dv[j + e] = w[e] + bias;
+            }
+        }
+        if (p.softplus_on) {
+#pragma unroll
+            for (int j = 0; j < TS; j += 2) {
+                const float2 v = softplus2(make_float2(dv[j], dv[j + 1]));
+                dv[j] = v.x;
+                dv[j + 1] = v.y;
+            }
+        }
+        const float* bct = reinterpret_cast<const float*>(smem + LY::bct_off + slot * LY::BCT_STAGE);
+#pragma unroll
+        for (int t0 = 0; t0 < TS; t0 += 4) {
+            float yp[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float2 dd = make_float2(dv[t0 + j], dv[t0 + j]);
+                const float du = dv[t0 + j] * uv[t0 + j];
+                const float2 uu = make_float2(du, du);
+                const float* bt = bct + (t0 + j) * 2 * NP;
+                float2 ya = make_float2(0.0f, 0.0f);
+#pragma unroll
+                for (int q = 0; q < NP / 4; ++q) {
+                    const float4 b = *reinterpret_cast<const float4*>(bt + 4 * q);
+                    const float4 cc = *reinterpret_cast<const float4*>(bt + NP + 4 * q);
+                    {
+                        const float2 x = __fmul2_rn(dd, A2[2 * q]);
+                        const float2 a = make_float2(ex2(x.x), ex2(x.y));
+                        h[2 * q] = __ffma2_rn(a, h[2 * q], __fmul2_rn(uu, make_float2(b.x, b.y)));
+                        ya = __ffma2_rn(make_float2(cc.x, cc.y), h[2 * q], ya);
+                    }
+                    {
+                        const float2 x = __fmul2_rn(dd, A2[2 * q + 1]);
+                        const float2 a = make_float2(ex2(x.x), ex2(x.y));
+                        h[2 * q + 1] = __ffma2_rn(a, h[2 * q + 1], __fmul2_rn(uu, make_float2(b.z, b.w)));
+                        ya = __ffma2_rn(make_float2(cc.z, cc.w), h[2 * q + 1], ya);
+                    }
+                }
+                yp[j] = ya.x + ya.y;
+            }
+            float o[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) o[j] = fmaf(dsk, uv[t0 + j], yp[j]);
+            if (cval) store_row<T, 4>(yrow + l0 + t0, o, nvalid - t0, true);
+        }
+        __syncwarp();
+        if (lane == 0) mbarrier_arrive(released(slot));
+    }
+}
+
 // Launch 2 of the chunked variant: the inclusive state after every chunk,
 // inc_m = 2^(A_n log2 e S_m) inc_{m-1} + H_m from inc_{-1} = 0, for every
 // (channel, state) of a tile.  The chain is short in arithmetic but long in
@@ -1511,6 +1717,7 @@ struct KernelInfo {
     size_t smem;
     int G, DT, threads, ts;
     const void* agg = nullptr;  // chunked variant: the aggregate kernel (launch 1)
+    bool tma = false;           // warp-specialised variant: takes the tensor maps of u, delta, B and C
 };
 
 template <typename T, int NP, class SH, bool ZOH>
@@ -1577,9 +1784,54 @@ KernelInfo packed_info() {
     return {attr_err == cudaSuccess ? fn : nullptr, LY::bytes, LY::G, LY::DT, LY::THREADS, LY::TS};
 }
 
+template <typename T, class WS>
+KernelInfo ws_info() {
+    using LY = WsTileLayout<T, WS>;
+    const void* fn = reinterpret_cast<const void*>(&full_ws_kernel<T, WS>);
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [&] {
+        attr_err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)LY::bytes);
+    });
+    KernelInfo ki{attr_err == cudaSuccess ? fn : nullptr, LY::bytes, 1, LY::DT, LY::THREADS, LY::TS};
+    ki.tma = true;
+    return ki;
+}
+
+// The driver's tensor-map encoder, looked up once (null when unavailable).
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static std::once_flag once;
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    std::call_once(once, [] {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    });
+    return fn;
+}
+
+// Tensor map of `planes` row-major [rows][L] slabs of u, delta, B or C, read
+// in boxes of box_rows rows x box_ts steps (rows past `rows` and steps past L
+// read as zero).
+bool encode_rows(CUtensorMap* m, const void* base, vmb_dtype dt, int L, int rows, long long planes, int box_ts,
+                 int box_rows) {
+    const PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+    if (!enc) return false;
+    const cuuint64_t es = dt == VMB_BF16 ? 2 : 4;
+    const cuuint64_t dims[3] = {(cuuint64_t)L, (cuuint64_t)rows, (cuuint64_t)planes};
+    const cuuint64_t strides[2] = {(cuuint64_t)L * es, (cuuint64_t)rows * L * es};
+    const cuuint32_t box[3] = {(cuuint32_t)box_ts, (cuuint32_t)box_rows, 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return enc(m, dt == VMB_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3,
+               const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Tile shapes per padded state count, in order of preference (fewest lanes
 // per channel first).  The zero-order-hold variant uses the first shape.
-int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 19; }
+int shape_count(int np) { return np <= 4 ? 1 : np == 8 ? 2 : 20; }
 constexpr int kLanesShape = 7;   // index of the lane-per-state variant (N <= 16 padded to 16)
 constexpr int kChunkShape = 8;   // first index of the three-launch chunked variant (shapes 8 to 11)
 bool is_chunk_shape(int np, int shape) { return np == 16 && shape >= kChunkShape && shape < kChunkShape + 4; }
@@ -1587,6 +1839,8 @@ constexpr int kStreamShape = 12;  // first index of the streaming one-lane varia
 bool is_stream_shape(int np, int shape) { return np == 16 && shape >= kStreamShape && shape < kStreamShape + 4; }
 constexpr int kPackedShape = 16;  // first index of the packed streaming variant (shapes 16 to 18: G = 1, 2, 4)
 bool is_packed_shape(int np, int shape) { return np == 16 && shape >= kPackedShape && shape < kPackedShape + 3; }
+constexpr int kWsShape = 19;  // the warp-specialised variant (tensor copies; 16-byte rows and aligned tensors)
+bool is_ws_shape(int np, int shape) { return np == 16 && shape == kWsShape; }
 
 template <typename T, bool ZOH>
 KernelInfo pick_t(int np, int shape) {
@@ -1618,6 +1872,7 @@ KernelInfo pick_t(int np, int shape) {
         case 16: return packed_info<T, PackedShape<1, 128, 5, 8, 3>>();
         case 17: return packed_info<T, PackedShape<2, 64, 5, 8, 3>>();
         case 18: return packed_info<T, PackedShape<4, 32, 5, 8, 3>>();
+        case 19: return ws_info<T, WsShape<4, 8, 4, 4>>();
         default: return info_for<T, 16, Shape<1, 128, 0, 3, 7>, ZOH>();
         }
     }
@@ -1677,12 +1932,19 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     // while a grid of 64-step one-lane chunks would fit in two waves, else
     // look-back chunks with one lane per channel when they stay long (>= 256
     // steps) and the widest split otherwise (>= 128 steps).
+    // the warp-specialised variant needs 16-byte rows and 16-byte aligned
+    // tensors (tiled tensor copies) and the driver's tensor-map encoder
+    const size_t es = a.dtype == VMB_BF16 ? 2 : 4;
+    const auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
+    const bool tma_ok = np == 16 && (size_t)a.L * es % 16 == 0 && al16(a.u) && al16(a.delta) && al16(a.Bs) &&
+                        al16(a.Cs) && al16(a.y) && tensor_map_encoder() != nullptr;
     int shape = 0, n_chunks = 1, forced_chunks = 0, forced_shape = 0;
     KernelInfo ki{};
     long long res = 0;
     vmb_status st;
     if (!zoh && forced_plan(&forced_shape, &forced_chunks)) {
         shape = forced_shape % shape_count(np);
+        if (is_ws_shape(np, shape) && !tma_ok) shape = kPackedShape;
         if ((st = info(shape, &ki, &res)) != VMB_OK) return st;
         n_chunks = forced_chunks > 1 ? forced_chunks : 1;
     } else if (zoh) {
@@ -1695,7 +1957,8 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     } else if (np == 16 && rows >= 256LL * sms && a.L >= 128) {
         // many rows: the packed streaming one-lane kernel, one pass over L (on
         // very short sequences its stage prologue does not pay off)
-        shape = kPackedShape;
+        // (warp-specialised, with tensor copies, when the tensors allow it)
+        shape = tma_ok ? kWsShape : kPackedShape;
         if ((st = info(shape, &ki, &res)) != VMB_OK) return st;
     } else {
         const ShapeRoles r = roles(np);
@@ -1763,7 +2026,8 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
         }
     }
     if (is_chunk_shape(np, shape)) n_chunks = (a.L + ki.ts - 1) / ki.ts;  // chunks of exactly ts steps
-    if (is_stream_shape(np, shape) || is_packed_shape(np, shape)) n_chunks = 1;  // one pass over L
+    if (is_stream_shape(np, shape) || is_packed_shape(np, shape) || is_ws_shape(np, shape))
+        n_chunks = 1;  // one pass over L
     if (n_chunks < 1) n_chunks = 1;
     ScanPlan p{};
     p.np = np;
@@ -1833,6 +2097,22 @@ vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
         // launch 3 loads its tile and applies the softplus before it waits for the carry
         return launch_kernel(ki.fn, dim3(grid), dim3(ki.threads), ki.smem, args, stream) == cudaSuccess ? VMB_OK
                                                                                                        : VMB_ERR_CUDA;
+    }
+    if (ki.tma) {
+        TensorMaps tm;
+        const long long planes = (long long)a.B * a.K;
+        if (encode_rows(&tm.u, a.u, a.dtype, a.L, a.D, planes, ki.ts, ki.DT) &&
+            encode_rows(&tm.dl, a.delta, a.dtype, a.L, a.D, planes, ki.ts, ki.DT) &&
+            encode_rows(&tm.B, a.Bs, a.dtype, a.L, a.N, planes, ki.ts, 16) &&
+            encode_rows(&tm.C, a.Cs, a.dtype, a.L, a.N, planes, ki.ts, 16)) {
+            void* targs[] = {&p, &tm};
+            return launch_kernel(ki.fn, dim3(grid), dim3(ki.threads), ki.smem, targs, stream) == cudaSuccess
+                       ? VMB_OK
+                       : VMB_ERR_CUDA;
+        }
+        // the encoder refused the tensors: the packed streaming variant (same tiles, same results)
+        ki = pick(a.dtype, plan.np, kPackedShape, false);
+        if (!ki.fn) return VMB_ERR_CUDA;
     }
     return launch_kernel(ki.fn, dim3(grid), dim3(ki.threads), ki.smem, args, stream) == cudaSuccess ? VMB_OK
                                                                                                    : VMB_ERR_CUDA;

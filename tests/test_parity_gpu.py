@@ -179,7 +179,7 @@ def test_lookback_wait_times_out_cleanly(mean, force_plan):
 
 
 @pytest.mark.parametrize("plan", ["0", "1", "2", "3", "4", "5", "6", "7", "8", "9", "10", "11", "12", "13", "14", "15",
-                                  "16", "17", "18", "0,3", "3,5", "4,2", "5,4", "6,7", "7,3", "7,6"])
+                                  "16", "17", "18", "19", "0,3", "3,5", "4,2", "5,4", "6,7", "7,3", "7,6"])
 @pytest.mark.parametrize("dt", ["f32", "bf16"])
 def test_every_tile_shape(plan, dt, force_plan):
     """Each tile shape of the full scan (and forced L-chunking) against the oracle."""
@@ -192,6 +192,39 @@ def test_every_tile_shape(plan, dt, force_plan):
     assert vmb.vmb_read_status() == vmb.VMB_OK
     _, ref, _ = oracle.ss2d_full(inp)
     check(to_numpy(y), ref, dt, f"full y plan {plan}")
+
+
+WS_CASES = [
+    # (B, D, N, H, W, dtype)
+    (1, 256, 16, 9, 12, "f32"),   # L = 108: the last 8-step stage half full; two full channel tiles
+    (2, 72, 16, 16, 24, "bf16"),  # bf16 rows of 16-byte multiples; a tile with three consumer warps
+    (1, 200, 13, 8, 10, "f32"),   # 13 states: B/C rows past N read as zero; a 72-channel tile
+    (1, 128, 16, 56, 56, "f32"),  # 392 stages: the 4-slot ring wraps around many times
+    (1, 64, 16, 7, 7, "f32"),     # L = 49: rows not 16-byte multiples -> the packed variant instead
+]
+
+
+@pytest.mark.parametrize("case", WS_CASES, ids=[f"B{s[0]}_D{s[1]}_N{s[2]}_{s[3]}x{s[4]}_{s[5]}" for s in WS_CASES])
+def test_warp_specialised_full_scan(case, force_plan):
+    """The warp-specialised full scan (tensor copies, mbarrier hand-over) against
+    the oracle, deterministic, and bit-identical to the packed streaming variant
+    whose arithmetic it shares."""
+    B, D, N, H, W, dt = case
+    wl = workloads.small_case(B=B, D=D, N=N, H=H, W=W, dtype=dt, seed=71 + D + N)
+    inp = workloads.make_inputs(wl, params="random")
+    g = to_device(inp, DEV)
+    xs = vmb.vmb_cross_scan(g["x"])
+    args = (xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], wl.H, wl.W)
+    force_plan.full("19")
+    y = vmb.vmb_selective_scan_fwd(*args)
+    y2 = vmb.vmb_selective_scan_fwd(*args)
+    force_plan.full("16")
+    yp = vmb.vmb_selective_scan_fwd(*args)
+    assert vmb.vmb_read_status() == vmb.VMB_OK
+    _, ref, _ = oracle.ss2d_full(inp)
+    check(to_numpy(y), ref, dt, "warp-specialised full y")
+    assert torch.equal(y, y2), "the warp-specialised scan must be deterministic"
+    assert torch.equal(y, yp), "the warp-specialised scan must match the packed variant bit for bit"
 
 
 CHUNKED_CASES = [
