@@ -1925,8 +1925,9 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
         *resident = (long long)(per_sm < 1 ? 1 : per_sm) * sms;
         return VMB_OK;
     };
-    // Rules measured on GB300 over the benchmark workloads: 16 states, at least
-    // 256 channel rows per SM and L >= 128 -> the packed streaming kernel; otherwise plenty of
+    // Rules measured on GB300 over the benchmark workloads: 16 states, L >= 128 and
+    // at least 128 channel rows per SM -> the warp-specialised kernel when the tensors
+    // allow tensor copies, else (at least 256 rows per SM) the packed streaming kernel; otherwise plenty of
     // rows -> one lane per channel; a fair number -> two lanes; too few -> cut L into
     // chunks: the three-launch variant (two lanes per channel, 32-step chunks)
     // while a grid of 64-step one-lane chunks would fit in two waves, else
@@ -1954,11 +1955,16 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
             const long long want = (res + tiles - 1) / tiles, mx = (a.L + 255) / 256;
             n_chunks = (int)(want < mx ? want : mx);
         }
+    } else if (tma_ok && rows >= 128LL * sms && a.L >= 128) {
+        // a fair number of rows and tensors the tensor copies can read: the
+        // warp-specialised kernel, one pass over L (measured on GB300: fastest
+        // from the batch-32 56x56 map, under a third of a wave of its tiles, up)
+        shape = kWsShape;
+        if ((st = info(shape, &ki, &res)) != VMB_OK) return st;
     } else if (np == 16 && rows >= 256LL * sms && a.L >= 128) {
         // many rows: the packed streaming one-lane kernel, one pass over L (on
         // very short sequences its stage prologue does not pay off)
-        // (warp-specialised, with tensor copies, when the tensors allow it)
-        shape = tma_ok ? kWsShape : kPackedShape;
+        shape = kPackedShape;
         if ((st = info(shape, &ki, &res)) != VMB_OK) return st;
     } else {
         const ShapeRoles r = roles(np);
