@@ -246,6 +246,11 @@ class Step:
                          (P(g["x"]), P(outs["xt"]), P(g["draw"]), P(g["A"]), P(g["Bs"]), P(g["Cs"]), P(g["Dskip"]),
                           P(g["bias"]), P(outs["ofused"]), P(outs["ybar"]), B, D, N, H, W, fl, dt, P(wsm),
                           wsm.numel(), s))
+        # the full-channel scan side of the block from the map (no cross-scan)
+        self.gathered_full = ("ss2d_full", lib.vmb_ss2d_full_fwd,
+                              (P(g["x"]), P(outs["xt"]), P(g["draw"]), P(g["A"]), P(g["Bs"]), P(g["Cs"]),
+                               P(g["Dskip"]), P(g["bias"]), P(outs["yf"]), P(outs["of"]), B, D, N, H, W, fl, dt,
+                               P(wsf), wsf.numel(), s))
         # kernels each call launches (the chunked full scan launches three)
         self.launches = sum(int(lib.vmb_scan_kernel_count(path, B, K, D, N, H, W, dt)) if path >= 0 else 1
                             for path in (-1, 0, 1, -1, -1))
@@ -259,6 +264,12 @@ class Step:
 
     def run_gathered(self):
         name, fn, args = self.gathered
+        st = fn(*args)
+        if st != 0:
+            raise RuntimeError(f"{name}: {self.vmb.status_string(st)}")
+
+    def run_gathered_full(self):
+        name, fn, args = self.gathered_full
         st = fn(*args)
         if st != 0:
             raise RuntimeError(f"{name}: {self.vmb.status_string(st)}")
@@ -370,13 +381,20 @@ def time_breakdown(step, n, prelude):
         gev[i][0].record()
         step.run_gathered()
         gev[i][1].record()
+    hev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(n)]
+    for i in range(n):
+        prelude()
+        hev[i][0].record()
+        step.run_gathered_full()
+        hev[i][1].record()
     torch.cuda.synchronize()
     per_kernel = {k: [e[j].elapsed_time(e[j + 1]) for e in evs] for j, k in enumerate(KERNELS)}
-    return per_kernel, ([e[0].elapsed_time(e[1]) for e in fev], [e[0].elapsed_time(e[1]) for e in gev])
+    return per_kernel, ([e[0].elapsed_time(e[1]) for e in fev], [e[0].elapsed_time(e[1]) for e in gev],
+                        [e[0].elapsed_time(e[1]) for e in hev])
 
 
 def kernel_table(wl, per_kernel_ms, fused_pair, peak):
-    fused_ms, gathered_ms = fused_pair
+    fused_ms, gathered_ms, gathered_full_ms = fused_pair
     kb = kernel_bytes(wl)
     per = {}
     for k in KERNELS:
@@ -400,6 +418,15 @@ def kernel_table(wl, per_kernel_ms, fused_pair, peak):
         "speedup_over_cross_scan_plus_fused": (per["cross_scan"]["us"] + fused_us) / g_us,
         "speedup_over_unfused_mean_path": unfused_all / g_us,
         "speedup_over_full_path": (per["cross_scan"]["us"] + per["full_scan"]["us"] + per["cross_merge_full"]["us"]) / g_us}
+    h_us = 1e3 * statistics.mean(gathered_full_ms)
+    hb = wl.gathered_full_bytes()
+    three = per["cross_scan"]["us"] + per["full_scan"]["us"] + per["cross_merge_full"]["us"]
+    fused["full_path_from_map"] = {
+        "us": h_us, "algorithmic_bytes": hb, "gbs": hb / (h_us / 1e6) / 1e9,
+        "frac_of_peak": hb / (h_us / 1e6) / 1e9 / peak,
+        "calls": "vmb_ss2d_full_fwd: cross-scan, full scan and cross-merge, no xs",
+        "three_calls_us": three, "speedup_over_three_calls": three / h_us,
+        "gathered_mean_speedup_over_it": h_us / g_us}
     return per, fused
 
 
@@ -432,6 +459,7 @@ def sweep_configs(vmb, dev, peak, prelude_flush, warmup):
                        "sigma": wl.sigma, "calls": n, "l2": "flushed before every step" if flush else
                        "not flushed (inputs far larger than L2)",
                        "kernels": per, "mean_speedup_over_full": per["full_scan"]["us"] / per["mean_scan"]["us"],
+                       "full_path_from_map": fused.pop("full_path_from_map"),
                        "mean_path_fused": fused, "gpu_launches_per_step": step.launches}
         del g, outs, step
         torch.cuda.empty_cache()
@@ -854,6 +882,7 @@ def main():
                      "alu_view": alu_view(dominant, wl, dom_ms)},
         # the fused channel-mean path (broadcast inside the merge) and the same
         # from the map (no cross-scan either), timed separately
+        "full_path_from_map": fused_table.pop("full_path_from_map"),
         "mean_path_fused": fused_table,
         "gpu_launches": res["launches_per_step"] * args.steps,
         "paper_style": paper_style_summary(res["paper_style"], peak),

@@ -223,6 +223,35 @@ vmb_status vmb_mean_scan_merge_fwd(const void* u, const void* delta, const float
                                    size_t workspace_bytes, cudaStream_t stream);
 
 /*
+ * vmb_ss2d_full_fwd - the scan side of a full-channel SS2D block in one call
+ * (App. A: cross-scan, the selective scan of Eqs. 3, 4 and 6, cross-merge)
+ * without the cross-scanned sequences xs [B, 4, D, L] being written:
+ *   y   = vmb_selective_scan_fwd(vmb_cross_scan(x), delta, ...) with K = 4,
+ *   out = vmb_cross_merge(y)
+ *   x, out [B, D, H, W] (dtype); y [B, 4, D, L] (dtype), written (the
+ *   per-direction output); xt [B, D, W, H] (dtype), caller-owned scratch
+ *   (overwritten); none of x, xt, y, out may alias another;
+ *   delta [B, 4, D, L], Bs, Cs [B, 4, N, L] (dtype); A [4*D, N], Dskip [4*D],
+ *   delta_bias [4*D] (fp32); flags and workspace as vmb_selective_scan_fwd with
+ *   K = 4 (vmb_scan_workspace_bytes(VMB_PATH_FULL, B, 4, D, N, H, W, dtype)).
+ * Where the warp-specialised scan kernel runs (16 states, rows of 16-byte
+ * multiples, 16-byte aligned tensors, enough channel rows) direction k's step
+ * l reads the value the cross-scan would have put there: directions 0 and 2
+ * the (b, d) planes of x row by row (forward and reversed), directions 1 and 3
+ * the rows of xt, the transpose of every plane (written by this call), so the
+ * map moves 2 B*D*L elements instead of the cross-scan's 5 B*D*L.  Otherwise
+ * the cross-scan is written into y and the scan runs in place.  Either way
+ * the values and operations are those of the three separate calls, so y and
+ * out are bit-identical to them.  Not in the paper as such: its kernels keep
+ * the steps apart.
+ */
+vmb_status vmb_ss2d_full_fwd(const void* x, void* xt, const void* delta, const float* A,
+                             const void* Bs, const void* Cs, const float* Dskip,
+                             const float* delta_bias, void* y, void* out, int B, int D, int N,
+                             int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,
+                             size_t workspace_bytes, cudaStream_t stream);
+
+/*
  * vmb_ss2d_mean_fwd - the scan side of a VMeanba SS2D block in one call: the
  * App. A cross-scan, the channel-mean scan (Sec. 2.2, Eq. 9) and the App. A
  * cross-merge, without the cross-scanned sequences xs [B, 4, D, L] or the

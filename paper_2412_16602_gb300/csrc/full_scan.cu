@@ -47,6 +47,7 @@ struct FullParams {
     int tiles_per_bk, n_tiles, n_chunks, chunk_len;
     int vec;       // rows are 16-byte aligned: cp.async 16-byte path and vector stores
     int suppress;  // test hook: chunk 0 does not publish
+    int gather_h;  // > 0: u is gathered from the map x and its transpose (warp-specialised variant only)
     WsHeader* hdr;
     unsigned* flags;
     float* aggP;   // per chunk: sum of delta per channel (DT floats, rest unused)
@@ -1457,6 +1458,12 @@ __global__ void __launch_bounds__(PackedLayout<T, PS>::THREADS, PS::MINB) full_p
 // full_packed_kernel: its y is bit-identical) and stores y from registers.
 // Requires rows of 16-byte multiples and 16-byte aligned tensors (the host
 // picks this variant only then); every wait is bounded.
+// Gathering from the map (p.gather_h > 0, App. A cross-scan without the
+// cross-scanned sequences): direction k's u rows are the (b, d) planes of x
+// (k = 0, 2) or of its transpose xt (k = 1, 3), and the reversed directions
+// (k = 2, 3) load the mirrored box, steps [L - (s+1) TS, L - s TS), and read
+// it from the end, so each step sees the value the cross-scan would have put
+// there (the same operations: y is bit-identical to the scan of xs).
 template <int CW_, int TS_, int NSTG_, int MINB_>
 struct WsShape {
     static constexpr int CW = CW_, TS = TS_, NSTG = NSTG_, MINB = MINB_;
@@ -1464,6 +1471,7 @@ struct WsShape {
 
 struct TensorMaps {
     CUtensorMap u, dl, B, C;  // [B*K][D][L] (u, delta) and [B*K][N][L] (B, C)
+    CUtensorMap u2;           // gathering from the map: u is x [B][D][L] and u2 its transpose xt
 };
 
 template <typename T, class WS>
@@ -1519,11 +1527,16 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
     __syncthreads();
     if (warp == LY::CW) {
         // ------------------------------------------------------ producer warp
+        // u: the rows of (b, k), or gathered from x / xt (see above)
+        const bool gather = p.gather_h > 0;
+        const CUtensorMap* um = (gather && (k & 1)) ? &tm.u2 : &tm.u;
+        const int uz = gather ? bk / p.K : bk;
+        const bool urev = gather && k >= 2;
         auto issue = [&](int s) {
             const int slot = s % NSTG;
             const uint32_t dst = sbase + (uint32_t)(slot * LY::RAW_STAGE);
             mbarrier_expect_tx(landed(slot), (unsigned)LY::RAW_STAGE);
-            tma_load_3d(dst, &tm.u, s * TS, d0, bk, landed(slot));
+            tma_load_3d(dst, um, urev ? L - (s + 1) * TS : s * TS, d0, uz, landed(slot));
             tma_load_3d(dst + LY::U_BYTES, &tm.dl, s * TS, d0, bk, landed(slot));
             tma_load_3d(dst + 2 * LY::U_BYTES, &tm.B, s * TS, 0, bk, landed(slot));
             tma_load_3d(dst + 2 * LY::U_BYTES + LY::BC_BYTES, &tm.C, s * TS, 0, bk, landed(slot));
@@ -1560,6 +1573,7 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
     }
     if (warp >= cwarps) return;  // a tile's channels past D: no work, not counted by `released`
     // -------------------------------------------------------- consumer warps
+    const bool urev = p.gather_h > 0 && k >= 2;  // u arrives mirrored (see above)
     const int c = tid;
     const int d = d0 + c;
     const bool cval = d < p.D;
@@ -1589,13 +1603,19 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
 #pragma unroll
         for (int j = 0; j < TS; j += 4) {
             float q[4], w[4];
-            load4(ru + j, q);
+            if (urev) {
+                // the mirrored box, read from its end
+                load4(ru + TS - 4 - j, q);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) uv[j + e] = q[3 - e];
+            } else {
+                load4(ru + j, q);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) uv[j + e] = q[e];
+            }
             load4(rd + j, w);
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                uv[j + e] = q[e];
-                dv[j + e] = w[e] + bias;
-            }
+            for (int e = 0; e < 4; ++e) dv[j + e] = w[e] + bias;
         }
         if (p.softplus_on) {
 #pragma unroll
@@ -1938,7 +1958,8 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     const size_t es = a.dtype == VMB_BF16 ? 2 : 4;
     const auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
     const bool tma_ok = np == 16 && (size_t)a.L * es % 16 == 0 && al16(a.u) && al16(a.delta) && al16(a.Bs) &&
-                        al16(a.Cs) && al16(a.y) && tensor_map_encoder() != nullptr;
+                        al16(a.Cs) && al16(a.y) && (a.gather_h == 0 || al16(a.u_t)) &&
+                        tensor_map_encoder() != nullptr;
     int shape = 0, n_chunks = 1, forced_chunks = 0, forced_shape = 0;
     KernelInfo ki{};
     long long res = 0;
@@ -2047,9 +2068,18 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
     p.chunk_len = chunk_len;
     p.state_floats = (size_t)ki.DT * np;
     p.ws_bytes = ws_layout(p).total;
+    // the warp-specialised kernel's CTAs each stream a whole sequence: a grid of
+    // less than one wave launched early would be placed on the SMs that the
+    // previous kernel frees first, up to the per-SM limit, and leave the others
+    // idle for its whole life (measured on GB300, batch-32 56x56 map after the
+    // map transpose: 514 us alone, about 900 us launched early); from a full
+    // wave up the early launch is about 3% faster (batch-128 map)
+    if (is_ws_shape(np, shape)) p.early = (long long)p.n_seq * p.n_chunks >= res;
     *plan = p;
     return VMB_OK;
 }
+
+bool full_plan_gathers(const ScanPlan& plan) { return is_ws_shape(plan.np, plan.split); }
 
 int full_plan_launches(const ScanPlan& plan) {
     return (is_chunk_shape(plan.np, plan.split) && plan.n_chunks > 1) ? 3 : 1;
@@ -2080,6 +2110,8 @@ vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     const auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
     p.vec = ((size_t)a.L * es % 16 == 0) && al16(a.u) && al16(a.delta) && al16(a.Bs) && al16(a.Cs) && al16(a.y);
     p.suppress = (a.flags & VMB_FLAG_TEST_SUPPRESS_PUBLISH) ? 1 : 0;
+    p.gather_h = a.gather_h;
+    if (a.gather_h > 0 && !ki.tma) return VMB_ERR_UNSUPPORTED;  // only the warp-specialised kernel gathers
     const WsLayout w = ws_layout(plan);
     unsigned char* ws = static_cast<unsigned char*>(a.ws);
     p.hdr = reinterpret_cast<WsHeader*>(ws);
@@ -2107,16 +2139,24 @@ vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     if (ki.tma) {
         TensorMaps tm;
         const long long planes = (long long)a.B * a.K;
-        if (encode_rows(&tm.u, a.u, a.dtype, a.L, a.D, planes, ki.ts, ki.DT) &&
-            encode_rows(&tm.dl, a.delta, a.dtype, a.L, a.D, planes, ki.ts, ki.DT) &&
+        const bool gather = a.gather_h > 0;
+        // gathering: u and u2 are the map x and its transpose, [B][D][L] each
+        bool ok = gather ? encode_rows(&tm.u, a.u, a.dtype, a.L, a.D, a.B, ki.ts, ki.DT) &&
+                               encode_rows(&tm.u2, a.u_t, a.dtype, a.L, a.D, a.B, ki.ts, ki.DT)
+                         : encode_rows(&tm.u, a.u, a.dtype, a.L, a.D, planes, ki.ts, ki.DT);
+        if (!gather) tm.u2 = tm.u;
+        if (ok && encode_rows(&tm.dl, a.delta, a.dtype, a.L, a.D, planes, ki.ts, ki.DT) &&
             encode_rows(&tm.B, a.Bs, a.dtype, a.L, a.N, planes, ki.ts, 16) &&
             encode_rows(&tm.C, a.Cs, a.dtype, a.L, a.N, planes, ki.ts, 16)) {
             void* targs[] = {&p, &tm};
-            return launch_kernel(ki.fn, dim3(grid), dim3(ki.threads), ki.smem, targs, stream) == cudaSuccess
+            return launch_kernel(ki.fn, dim3(grid), dim3(ki.threads), ki.smem, targs, stream, plan.early) ==
+                           cudaSuccess
                        ? VMB_OK
                        : VMB_ERR_CUDA;
         }
-        // the encoder refused the tensors: the packed streaming variant (same tiles, same results)
+        // the encoder refused the tensors: the packed streaming variant (same tiles, same
+        // results), which reads materialised sequences only
+        if (gather) return VMB_ERR_UNSUPPORTED;
         ki = pick(a.dtype, plan.np, kPackedShape, false);
         if (!ki.fn) return VMB_ERR_CUDA;
     }

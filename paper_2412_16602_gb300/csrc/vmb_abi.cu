@@ -338,6 +338,56 @@ vmb_status vmb_ss2d_mean_fwd(const void* x, void* xt, const void* delta, const f
     return launch_mean_merge(x, ybar, Dskip, out, B, D, H, W, (flags & VMB_FLAG_SKIP_MEAN) == 0, dtype, stream);
 }
 
+vmb_status vmb_ss2d_full_fwd(const void* x, void* xt, const void* delta, const float* A, const void* Bs,
+                             const void* Cs, const float* Dskip, const float* delta_bias, void* y, void* out, int B,
+                             int D, int N, int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,
+                             size_t workspace_bytes, cudaStream_t stream) {
+    bool empty = false;
+    vmb_status s = check_csm(x, out, B, D, H, W, dtype, &empty);
+    if (s != VMB_OK || empty) return s;
+    if (x == out || !xt || !y || xt == x || xt == out || xt == y || y == x || y == out) return VMB_ERR_INVALID_ARG;
+    if (!aligned(xt, esize(dtype))) return VMB_ERR_MISALIGNED;
+    // the full scan reads each direction's steps from the map (rows of x) or its
+    // transpose (rows of xt), with no materialised cross-scan, and writes y;
+    // the merge then sums the four directions
+    ScanArgs a{x, delta, A, Bs, Cs, Dskip, delta_bias, y, nullptr, B, 4, D, N, H * W, flags, dtype,
+               workspace, workspace_bytes};
+    a.gather_h = H;
+    a.u_t = xt;
+    // every check (arguments, plan, workspace size) before the first launch
+    bool scan_empty = false;
+    s = check_scan(a, false, &scan_empty);
+    if (s != VMB_OK) return s;
+    if (!workspace) return VMB_ERR_WORKSPACE;
+    if (!aligned(workspace, 256)) return VMB_ERR_MISALIGNED;
+    ScanPlan plan{};
+    s = plan_full(a, &plan);
+    if (s != VMB_OK) return s;
+    if (workspace_bytes < plan.ws_bytes) return VMB_ERR_WORKSPACE;
+    if (full_plan_gathers(plan)) {
+        s = launch_map_transpose(x, xt, B, D, H, W, dtype, stream);
+        if (s != VMB_OK) return s;
+        s = launch_full(a, plan, stream);
+    } else {
+        // a plan whose kernel reads materialised sequences: the cross-scan goes
+        // into y and the scan runs in place (each of its CTAs reads the steps of
+        // its own rows before it writes them, and no other CTA touches them)
+        ScanArgs m = a;
+        m.u = y;
+        m.gather_h = 0;
+        m.u_t = nullptr;
+        ScanPlan mplan{};
+        s = plan_full(m, &mplan);
+        if (s != VMB_OK) return s;
+        if (workspace_bytes < mplan.ws_bytes) return VMB_ERR_WORKSPACE;
+        s = launch_cross_scan(x, y, B, D, H, W, dtype, stream);
+        if (s != VMB_OK) return s;
+        s = launch_full(m, mplan, stream);
+    }
+    if (s != VMB_OK) return s;
+    return launch_cross_merge(y, out, B, D, H, W, dtype, stream);
+}
+
 // Checks of the backward call; sets *empty for a problem with no elements.
 static vmb_status check_bwd(const MeanBwdArgs& a, bool* empty) {
     if (!dtype_ok(a.dtype) || a.B < 0 || a.K < 0 || a.D < 0 || a.N < 0 || a.L < 0) return VMB_ERR_INVALID_ARG;

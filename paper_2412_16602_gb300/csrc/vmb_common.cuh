@@ -112,8 +112,13 @@ __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepc
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 // Host side: launch `fn` with the programmatic attribute set.
+// programmatic = false: an ordinary launch (the kernel starts after the
+// previous one has completed; its pdl_wait returns at once).  Used for grids
+// of long-lived CTAs: launched early, they are placed on the SMs that the
+// previous kernel frees first, up to the per-SM limit, and leave the others
+// idle for their whole life.
 inline cudaError_t launch_kernel(const void* fn, dim3 grid, dim3 block, size_t smem, void** args,
-                                 cudaStream_t stream) {
+                                 cudaStream_t stream, bool programmatic = true) {
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = grid;
     cfg.blockDim = block;
@@ -122,8 +127,8 @@ inline cudaError_t launch_kernel(const void* fn, dim3 grid, dim3 block, size_t s
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.attrs = programmatic ? attr : nullptr;
+    cfg.numAttrs = programmatic ? 1 : 0;
     return cudaLaunchKernelExC(&cfg, fn, args);
 }
 

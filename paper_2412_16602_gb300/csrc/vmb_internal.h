@@ -48,6 +48,7 @@ struct ScanPlan {
     int chunk_len;     // steps per chunk (a multiple of the stage length)
     size_t state_floats;  // floats of one chunk's published state (per array)
     size_t ws_bytes;      // total workspace bytes
+    bool early = true;    // may be launched before the previous kernel of the stream completes
 };
 
 inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
@@ -145,6 +146,8 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan);
 vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan);
 vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream);
 int full_plan_launches(const ScanPlan& plan);  // kernels launch_full starts for this plan
+// Whether launch_full can read the plan's u gathered from the map (ScanArgs::gather_h).
+bool full_plan_gathers(const ScanPlan& plan);
 vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream);
 vmb_status launch_cross_scan(const void* x, void* xs, int B, int D, int H, int W, vmb_dtype dt,
                              cudaStream_t stream);

@@ -40,7 +40,7 @@ VMB_PATH_MEAN = 1
 EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb_scan_kernel_count",
            "vmb_selective_scan_fwd",
            "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_ss2d_mean_fwd",
-           "vmb_discretise_fwd", "vmb_discretise_mean_fwd",
+           "vmb_ss2d_full_fwd", "vmb_discretise_fwd", "vmb_discretise_mean_fwd",
            "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_mean_scan_train_fwd", "vmb_mean_scan_bwd",
            "vmb_mean_scan_bwd_workspace_bytes",
            "vmb_read_status", "vmb_status_string", "vmb_version"]
@@ -67,6 +67,7 @@ def _load() -> ctypes.CDLL:
     lib.vmb_mean_scan_fwd.argtypes = [vp] * 9 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_merge_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
     lib.vmb_ss2d_mean_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
+    lib.vmb_ss2d_full_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_grouped_fwd.argtypes = [vp] * 9 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_discretise_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
@@ -81,7 +82,8 @@ def _load() -> ctypes.CDLL:
     lib.vmb_status_string.restype = ctypes.c_char_p
     lib.vmb_version.argtypes = []
     for name in ["vmb_cross_scan", "vmb_cross_merge", "vmb_selective_scan_fwd", "vmb_mean_scan_fwd",
-                 "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_ss2d_mean_fwd", "vmb_discretise_fwd",
+                 "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_ss2d_mean_fwd", "vmb_ss2d_full_fwd",
+                 "vmb_discretise_fwd",
                  "vmb_discretise_mean_fwd", "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_mean_scan_bwd",
                  "vmb_read_status", "vmb_version"]:
         getattr(lib, name).restype = i
@@ -404,6 +406,50 @@ def vmb_ss2d_mean_fwd(x, delta, A, Bs, Cs, Dskip, delta_bias, *, out=None, ybar=
                                  _ptr(out), _ptr(ybar), B, D, N, H, W, flags, _dtype_code(x.dtype), _ptr(workspace),
                                  workspace.numel(), _stream(stream)), "vmb_ss2d_mean_fwd")
     return out, ybar
+
+
+def vmb_ss2d_full_fwd(x, delta, A, Bs, Cs, Dskip, delta_bias, *, out=None, y=None, xt=None,
+                      flags: int = VMB_FLAG_SOFTPLUS, workspace=None, stream=None):
+    """The scan side of a full-channel SS2D block from the map: cross-scan, selective scan and
+    cross-merge in one call, xs never written.  x [B, D, H, W]; delta [B, 4, D, H*W], Bs, Cs
+    [B, 4, N, H*W]; xt [B, D, W, H] scratch for the map's transpose (allocated when not given);
+    returns (out [B, D, H, W], y [B, 4, D, H*W])."""
+    _dev(x, "x")
+    B, D, H, W = x.shape
+    if xt is None:
+        xt = torch.empty((B, D, W, H), dtype=x.dtype, device=x.device)
+    _dev(xt, "xt")
+    if tuple(xt.shape) != (B, D, W, H) or xt.dtype != x.dtype:
+        raise ValueError("xt must be [B, D, W, H] in the dtype of x")
+    L = H * W
+    for t, n in [(delta, "delta"), (A, "A"), (Bs, "Bs"), (Cs, "Cs"), (Dskip, "Dskip"), (delta_bias, "delta_bias")]:
+        _dev(t, n)
+    N = Bs.shape[2]
+    if tuple(delta.shape) != (B, 4, D, L) or tuple(Bs.shape) != (B, 4, N, L) or tuple(Cs.shape) != (B, 4, N, L):
+        raise ValueError("delta [B,4,D,H*W], Bs and Cs [B,4,N,H*W] expected")
+    if len({x.dtype, delta.dtype, Bs.dtype, Cs.dtype}) != 1:
+        raise ValueError("x, delta, Bs, Cs must share one dtype")
+    if tuple(A.shape) != (4 * D, N) or tuple(Dskip.shape) != (4 * D,) or tuple(delta_bias.shape) != (4 * D,):
+        raise ValueError("A [4*D, N], Dskip [4*D], delta_bias [4*D] expected")
+    if A.dtype != torch.float32 or Dskip.dtype != torch.float32 or delta_bias.dtype != torch.float32:
+        raise ValueError("A, Dskip, delta_bias must be float32")
+    if out is None:
+        out = torch.empty_like(x)
+    _dev(out, "out")
+    if out.shape != x.shape or out.dtype != x.dtype:
+        raise ValueError("out must match x")
+    if y is None:
+        y = torch.empty((B, 4, D, L), dtype=x.dtype, device=x.device)
+    _dev(y, "y")
+    if tuple(y.shape) != (B, 4, D, L) or y.dtype != x.dtype:
+        raise ValueError("y must be [B, 4, D, H*W] in the dtype of x")
+    ws_bytes = vmb_scan_workspace_bytes(VMB_PATH_FULL, B, 4, D, N, H, W, x.dtype)
+    if workspace is None:
+        workspace = _default_ws.get(ws_bytes, x.device)
+    _check(lib.vmb_ss2d_full_fwd(_ptr(x), _ptr(xt), _ptr(delta), _ptr(A), _ptr(Bs), _ptr(Cs), _ptr(Dskip),
+                                 _ptr(delta_bias), _ptr(y), _ptr(out), B, D, N, H, W, flags, _dtype_code(x.dtype),
+                                 _ptr(workspace), workspace.numel(), _stream(stream)), "vmb_ss2d_full_fwd")
+    return out, y
 
 
 # ------------------------------------------- the paper's scan-only kernel setting

@@ -26,6 +26,7 @@ def lib():
     lib.vmb_mean_scan_fwd.argtypes = [vp] * 9 + [i] * 6 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_merge_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
     lib.vmb_ss2d_mean_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
+    lib.vmb_ss2d_full_fwd.argtypes = [vp] * 10 + [i] * 5 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_grouped_fwd.argtypes = [vp] * 9 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_discretise_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
@@ -166,6 +167,31 @@ def test_ss2d_mean_validation(lib):
     assert ss2d_call(lib, flags=0x100) == 1
     assert ss2d_call(lib, ws=0) == 4
     assert ss2d_call(lib, ptrs=[0] * 10, B=0, ws=0) == 0                       # empty problem
+
+
+def ss2d_full_call(lib, *, ptrs=None, B=1, D=8, N=16, H=4, W=4, flags=1, dtype=0, ws=0x100000, ws_bytes=1 << 20):
+    p = [FAKE, FAKE + 0x3000] + [FAKE] * 6 + [FAKE + 0x4000, FAKE + 0x1000] if ptrs is None else ptrs
+    return lib.vmb_ss2d_full_fwd(*p, B, D, N, H, W, flags, dtype, ws, ws_bytes, S)
+
+
+def test_ss2d_full_validation(lib):
+    """The full-channel scan side of the block from the map: x, xt, y and out
+    must be distinct and aligned, the scan inputs are checked like the full
+    scan's, all before any launch."""
+    base = [FAKE, FAKE + 0x3000] + [FAKE] * 6 + [FAKE + 0x4000, FAKE + 0x1000]
+    assert ss2d_full_call(lib, B=-1) == 1
+    assert ss2d_full_call(lib, ptrs=[0] + base[1:]) == 1                       # null map
+    assert ss2d_full_call(lib, ptrs=base[:1] + [0] + base[2:]) == 1            # null transpose scratch
+    assert ss2d_full_call(lib, ptrs=base[:8] + [0] + base[9:]) == 1            # null y
+    assert ss2d_full_call(lib, ptrs=base[:1] + [FAKE] + base[2:]) == 1         # transpose aliases x
+    assert ss2d_full_call(lib, ptrs=base[:8] + [FAKE + 0x1000] + base[9:]) == 1  # y aliases out
+    assert ss2d_full_call(lib, ptrs=base[:9] + [FAKE]) == 1                    # out aliases x
+    assert ss2d_full_call(lib, ptrs=[FAKE + 2] + base[1:]) == 2                # misaligned fp32 map
+    assert ss2d_full_call(lib, ptrs=base[:1] + [FAKE + 0x3002] + base[2:]) == 2  # misaligned transpose
+    assert ss2d_full_call(lib, N=17) == 3
+    assert ss2d_full_call(lib, flags=0x100) == 1
+    assert ss2d_full_call(lib, ws=0) == 4
+    assert ss2d_full_call(lib, ptrs=[0] * 10, B=0, ws=0) == 0                  # empty problem
 
 
 def disc_call(fn, *, ptrs=None, B=1, K=4, D=8, N=16, H=4, W=4, flags=1, dtype=0):

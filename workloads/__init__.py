@@ -98,6 +98,21 @@ class Workload:
         params = self.K * self.D * (self.N + 2) * 4
         return s * (bkdl + 2 * bknl + 2 * bdl) + 2 * 4 * self.B * self.K * self.L + params
 
+    def gathered_full_bytes(self) -> int:
+        """Algorithmic bytes of the full-channel scan side of the block from the
+        map (vmb_ss2d_full_fwd: selective scan reading the map, then the
+        cross-merge): delta read once, Bs and Cs read once, the map x read once
+        (every direction reads the same map), y written once and read back by
+        the merge, the merged map written once, plus the per-channel
+        parameters.  (The transposed copy of the map the column-major
+        directions read is not counted, as in gathered_mean_bytes.)"""
+        s = self.esize
+        bkdl = self.B * self.K * self.D * self.L
+        bknl = self.B * self.K * self.N * self.L
+        bdl = self.B * self.D * self.L
+        params = self.K * self.D * (self.N + 2) * 4
+        return s * (3 * bkdl + 2 * bknl + 2 * bdl) + params
+
     def replace(self, **kw) -> "Workload":
         d = dict(self.__dict__)
         d.update(kw)
