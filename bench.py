@@ -646,6 +646,27 @@ def run_ours(args, wl, rank, world, local_rank):
         def sel():
             vmb.vmb_selection_fwd(outs["xs"], *sw, wl.H, wl.W, delta_raw=sdr, Bs=sB, Cs=sC, stream=stream)
         sel_us = time_alone(sel)
+        # the same with the Delta branch left low-rank: the selection writes z
+        # [B, 4, R, L] and the full scan forms the raw Deltas Wup z itself
+        sz = torch.empty((wl.B, 4, R, wl.L), dtype=torch.float32, device=dev)
+        ylr = outs["ym"]
+        wsf = outs["ws_full"]
+
+        def sel_lr():
+            vmb.vmb_selection_lowrank_fwd(outs["xs"], sw[0], sw[1], sw[2], wl.H, wl.W, z=sz, Bs=sB, Cs=sC,
+                                          stream=stream)
+
+        def scan_lr():
+            vmb.vmb_selective_scan_lowrank_fwd(outs["xs"], sz, sw[3], g["A"], sB, sC, g["Dskip"], g["bias"],
+                                               wl.H, wl.W, y=ylr, workspace=wsf, stream=stream)
+
+        def scan_raw():
+            vmb.vmb_selective_scan_fwd(outs["xs"], sdr, g["A"], sB, sC, g["Dskip"], g["bias"], wl.H, wl.W,
+                                       y=ylr, workspace=wsf, stream=stream)
+        sel()
+        lowrank = {"selection_us": time_alone(sel_lr), "scan_us": time_alone(scan_lr),
+                   "scan_raw_deltas_us": time_alone(scan_raw), "rank": R}
+        sel_us = (sel_us, lowrank)
     # the backward of the channel-mean scan on the step's inputs (dLoss/dy drawn
     # on the device), with its workspace allocated once
     bwd_us = None
@@ -747,15 +768,32 @@ def alu_view(kernel, wl, ms):
             "basis": ALU_BASIS[kernel]}
 
 
-def selection_summary(us, wl, peak, R=6):
-    """Eq. 6 selection on the step's input: reads u, writes B, C and the raw Delta."""
-    if us is None:
+def selection_summary(us_pair, wl, peak, R=6):
+    """Eq. 6 selection on the step's input: reads u, writes B, C and the raw Delta.
+    "lowrank": the same with the Delta branch left low-rank (the selection writes
+    z, fp32 [B, 4, R, L]; the full scan forms the raw Deltas Wup z itself),
+    timed next to the selection + full scan on its raw Deltas."""
+    if us_pair is None:
         return None
+    us, lr = us_pair
     s = 2 if wl.dtype == "bf16" else 4
-    bytes_ = s * (2 * wl.B * 4 * wl.D * wl.L + 2 * wl.B * 4 * wl.N * wl.L) + 4 * 4 * (2 * wl.N + 2 * R) * wl.D
+    bkdl, bknl, bkrl = wl.B * 4 * wl.D * wl.L, wl.B * 4 * wl.N * wl.L, wl.B * 4 * R * wl.L
+    bytes_ = s * (2 * bkdl + 2 * bknl) + 4 * 4 * (2 * wl.N + 2 * R) * wl.D
     gbs = bytes_ / (us / 1e6) / 1e9
+    sel_lr_bytes = s * (bkdl + 2 * bknl) + 4 * bkrl + 4 * 4 * (2 * wl.N + R) * wl.D
+    scan_lr_bytes = s * (2 * bkdl + 2 * bknl) + 4 * bkrl + 4 * 4 * wl.D * (wl.N + 2 + R)
+    pair_lr = lr["selection_us"] + lr["scan_us"]
+    pair_raw = us + lr["scan_raw_deltas_us"]
+    lowrank = {"rank": R, "selection_us": lr["selection_us"], "scan_us": lr["scan_us"],
+               "scan_algorithmic_bytes": scan_lr_bytes,
+               "scan_gbs": scan_lr_bytes / (lr["scan_us"] / 1e6) / 1e9,
+               "scan_frac_of_peak": scan_lr_bytes / (lr["scan_us"] / 1e6) / 1e9 / peak,
+               "pair_us": pair_lr, "pair_bytes": sel_lr_bytes + scan_lr_bytes,
+               "raw_deltas_pair_us": pair_raw, "raw_deltas_pair_bytes": bytes_ + wl.scan_bytes(),
+               "speedup_over_raw_deltas": pair_raw / pair_lr}
     return {"us": us, "algorithmic_bytes": bytes_, "gbs": gbs, "frac_of_peak": gbs / peak, "rank": R,
-            "kernel": "tcgen05.mma kind::tf32 (three-product tf32 split for fp32 accuracy), accumulator in TMEM"}
+            "kernel": "tcgen05.mma kind::tf32 (three-product tf32 split for fp32 accuracy), accumulator in TMEM",
+            "lowrank": lowrank}
 
 
 def backward_summary(us, wl, peak):

@@ -368,6 +368,38 @@ vmb_status vmb_selection_fwd(const void* u, const float* WB, const float* WC, co
                              int D, int N, int R, int H, int W, vmb_dtype dtype, cudaStream_t stream);
 
 /*
+ * The selection functions with the Delta branch left in its low-rank form
+ * (Eq. 6, App. A: s_Delta = Linear_D(Linear_R(u))), so the raw Deltas
+ * [B,K,D,L] are never written: the scan expands them itself.
+ *
+ * vmb_selection_lowrank_fwd - as vmb_selection_fwd, but writes the rank-R
+ *   intermediate z[b,k,r,l] = sum_d Wz[k,r,d] u[b,k,d,l] (fp32 [B,K,R,L],
+ *   4-byte aligned) instead of delta_raw; no Wup.  Bs, Cs as there.
+ *
+ * vmb_selective_scan_lowrank_fwd - vmb_selective_scan_fwd with
+ *   delta_raw[b,k,d,l] = sum_r Wup[k,d,r] z[b,k,r,l] (r in order, fp32)
+ *   formed inside the scan from z [B,K,R,L] fp32 and Wup [K,D,R] fp32 (R in
+ *   1..16; VMB_ERR_UNSUPPORTED above); every other argument, flag and the
+ *   workspace (vmb_scan_workspace_bytes(VMB_PATH_FULL, ...)) as there; y must
+ *   not alias u.  The warp-specialised scan (16 states, rows of 16-byte
+ *   multiples, 16-byte aligned tensors, enough channel rows, Euler Bbar) reads
+ *   z instead of the raw Deltas, i.e. R instead of D values per step and
+ *   direction; for other plans the raw Deltas are written into y (rounded to
+ *   the storage type) and the scan runs in place.  In fp32 the result is
+ *   bit-identical to vmb_selection_fwd's raw Deltas fed to
+ *   vmb_selective_scan_fwd; with bf16 storage the warp-specialised scan keeps
+ *   the raw Deltas in fp32 (that pair rounds them to bf16 first).
+ */
+vmb_status vmb_selection_lowrank_fwd(const void* u, const float* WB, const float* WC, const float* Wz,
+                                     void* Bs, void* Cs, float* z, int B, int K, int D, int N, int R, int H,
+                                     int W, vmb_dtype dtype, cudaStream_t stream);
+vmb_status vmb_selective_scan_lowrank_fwd(const void* u, const float* z, const float* Wup, const float* A,
+                                          const void* Bs, const void* Cs, const float* Dskip,
+                                          const float* delta_bias, void* y, int B, int K, int D, int N,
+                                          int R, int H, int W, unsigned flags, vmb_dtype dtype,
+                                          void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
  * vmb_mean_scan_train_fwd - vmb_mean_scan_grouped_fwd (groups = 1: the
  * channel-mean scan of Eq. 9) that also keeps, for vmb_mean_scan_bwd, the
  * group means it forms on the way:

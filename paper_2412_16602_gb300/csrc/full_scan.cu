@@ -48,6 +48,8 @@ struct FullParams {
     int vec;       // rows are 16-byte aligned: cp.async 16-byte path and vector stores
     int suppress;  // test hook: chunk 0 does not publish
     int gather_h;  // > 0: u is gathered from the map x and its transpose (warp-specialised variant only)
+    const float* Wup;  // low-rank Delta (warp-specialised variant only): dl is z [B*K][R][L] fp32 and
+    int R;             // delta_raw[b,k,d,l] = sum_r Wup[k,d,r] z[b,k,r,l]
     WsHeader* hdr;
     unsigned* flags;
     float* aggP;   // per chunk: sum of delta per channel (DT floats, rest unused)
@@ -1464,9 +1466,16 @@ __global__ void __launch_bounds__(PackedLayout<T, PS>::THREADS, PS::MINB) full_p
 // (k = 2, 3) load the mirrored box, steps [L - (s+1) TS, L - s TS), and read
 // it from the end, so each step sees the value the cross-scan would have put
 // there (the same operations: y is bit-identical to the scan of xs).
-template <int CW_, int TS_, int NSTG_, int MINB_>
+// Low-rank Delta (RP > 0, Eq. 6's s_Delta = Linear_D(Linear_R(u)) with the
+// rank-R expansion fused into the scan): the second box of a stage is z
+// (16 rows x TS steps, fp32, rows past R zero) instead of the raw Deltas, and
+// each consumer lane forms its channel's raw Delta per step as
+// sum_r Wup[k,d,r] z_r (r in order, as the selection kernel's epilogue does,
+// so fp32 results are bit-identical to selection -> raw Deltas -> scan), with
+// its Wup row (RP >= R values, zero-padded) in registers.
+template <int CW_, int TS_, int NSTG_, int MINB_, int RP_ = 0>
 struct WsShape {
-    static constexpr int CW = CW_, TS = TS_, NSTG = NSTG_, MINB = MINB_;
+    static constexpr int CW = CW_, TS = TS_, NSTG = NSTG_, MINB = MINB_, RP = RP_;
 };
 
 struct TensorMaps {
@@ -1479,11 +1488,14 @@ struct WsTileLayout {
     static constexpr int CW = WS::CW, DT = 32 * CW, NP = 16, TS = WS::TS, NSTG = WS::NSTG;
     static constexpr int THREADS = DT + 32;
     static constexpr int U_BYTES = DT * TS * (int)sizeof(T);   // one u (or delta) box
+    static constexpr int DL_BYTES = WS::RP ? NP * TS * 4 : U_BYTES;  // the delta box, or the z box (fp32)
     static constexpr int BC_BYTES = NP * TS * (int)sizeof(T);  // one B (or C) box
-    static constexpr int RAW_STAGE = 2 * U_BYTES + 2 * BC_BYTES;
+    static constexpr int B_OFF = U_BYTES + DL_BYTES;            // B box within a stage (C follows)
+    static constexpr int RAW_STAGE = U_BYTES + DL_BYTES + 2 * BC_BYTES;
     static constexpr int BCT_STAGE = TS * 2 * NP * 4;           // fp32 [TS][B0..15, C0..15]
     static constexpr size_t bct_off = (size_t)NSTG * RAW_STAGE;
-    static constexpr size_t bar_off = bct_off + (size_t)NSTG * BCT_STAGE;
+    static constexpr size_t wup_off = bct_off + (size_t)NSTG * BCT_STAGE;  // low rank: fp32 [DT][RP + 1] Wup rows
+    static constexpr size_t bar_off = wup_off + (WS::RP ? (size_t)DT * (WS::RP + 1) * 4 : 0);
     static constexpr size_t bytes = bar_off + (size_t)3 * NSTG * 8;
     static_assert(U_BYTES % 128 == 0 && BC_BYTES % 128 == 0 && TS % 4 == 0 && TS * sizeof(T) % 16 == 0,
                   "tensor-copy boxes: 16-byte rows, 128-byte aligned boxes");
@@ -1537,9 +1549,9 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
             const uint32_t dst = sbase + (uint32_t)(slot * LY::RAW_STAGE);
             mbarrier_expect_tx(landed(slot), (unsigned)LY::RAW_STAGE);
             tma_load_3d(dst, um, urev ? L - (s + 1) * TS : s * TS, d0, uz, landed(slot));
-            tma_load_3d(dst + LY::U_BYTES, &tm.dl, s * TS, d0, bk, landed(slot));
-            tma_load_3d(dst + 2 * LY::U_BYTES, &tm.B, s * TS, 0, bk, landed(slot));
-            tma_load_3d(dst + 2 * LY::U_BYTES + LY::BC_BYTES, &tm.C, s * TS, 0, bk, landed(slot));
+            tma_load_3d(dst + LY::U_BYTES, &tm.dl, s * TS, WS::RP ? 0 : d0, bk, landed(slot));
+            tma_load_3d(dst + LY::B_OFF, &tm.B, s * TS, 0, bk, landed(slot));
+            tma_load_3d(dst + LY::B_OFF + LY::BC_BYTES, &tm.C, s * TS, 0, bk, landed(slot));
         };
         if (lane == 0)
             for (int s = 0; s < NSTG && s < nst; ++s) issue(s);
@@ -1550,7 +1562,7 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
             if (!(ok = mbarrier_wait(landed(slot), (s / NSTG) & 1, kStageWaitNs))) break;
             seen = s + 1;
             // lane r converts row r of [B rows 0..15, C rows 0..15] into column r
-            const T* rb = reinterpret_cast<const T*>(smem + slot * LY::RAW_STAGE + 2 * LY::U_BYTES) + lane * TS;
+            const T* rb = reinterpret_cast<const T*>(smem + slot * LY::RAW_STAGE + LY::B_OFF) + lane * TS;
             float* bo = reinterpret_cast<float*>(smem + LY::bct_off + slot * LY::BCT_STAGE);
 #pragma unroll
             for (int t = 0; t < TS; ++t) bo[t * 2 * NP + lane] = io<T>::cvt(rb[t]);
@@ -1589,6 +1601,14 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
         h[i] = make_float2(0.0f, 0.0f);
     }
     T* yrow = static_cast<T*>(p.y) + (row0 + c) * (size_t)L;
+    constexpr int RP = WS::RP > 0 ? WS::RP : 1;
+    // low rank: this channel's Wup row, in the lane's own shared-memory row (a
+    // padded stride: conflict-free) to leave the registers to the states
+    float* wr = reinterpret_cast<float*>(smem + LY::wup_off) + c * (RP + 1);
+    if constexpr (WS::RP > 0) {
+#pragma unroll
+        for (int r = 0; r < RP; ++r) wr[r] = (cval && r < p.R) ? p.Wup[((size_t)k * p.D + d) * p.R + r] : 0.0f;
+    }
     for (int s = 0; s < nst; ++s) {
         const int slot = s % NSTG;
         if (!mbarrier_wait(ready(slot), (s / NSTG) & 1, kStageWaitNs)) {
@@ -1613,9 +1633,36 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) uv[j + e] = q[e];
             }
-            load4(rd + j, w);
+            if constexpr (WS::RP == 0) {
+                load4(rd + j, w);
 #pragma unroll
-            for (int e = 0; e < 4; ++e) dv[j + e] = w[e] + bias;
+                for (int e = 0; e < 4; ++e) dv[j + e] = w[e] + bias;
+            }
+        }
+        if constexpr (WS::RP > 0) {
+            // raw Delta = sum_r Wup[r] z_r, r in order (the z rows are broadcast reads)
+            const float* zr = reinterpret_cast<const float*>(smem + slot * LY::RAW_STAGE + LY::U_BYTES);
+            // (packed: each lane of a pair is the same fused multiply-add as fmaf)
+            float2 raw[TS / 2];
+#pragma unroll
+            for (int j = 0; j < TS / 2; ++j) raw[j] = make_float2(0.0f, 0.0f);
+#pragma unroll
+            for (int r = 0; r < RP; ++r) {
+                if (r < p.R) {
+                    const float2 w2 = make_float2(wr[r], wr[r]);
+#pragma unroll
+                    for (int j = 0; j < TS; j += 4) {
+                        const float4 z4 = *reinterpret_cast<const float4*>(zr + r * TS + j);
+                        raw[j / 2] = __ffma2_rn(w2, make_float2(z4.x, z4.y), raw[j / 2]);
+                        raw[j / 2 + 1] = __ffma2_rn(w2, make_float2(z4.z, z4.w), raw[j / 2 + 1]);
+                    }
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < TS; j += 2) {
+                dv[j] = raw[j / 2].x + bias;
+                dv[j + 1] = raw[j / 2].y + bias;
+            }
         }
         if (p.softplus_on) {
 #pragma unroll
@@ -1816,6 +1863,13 @@ KernelInfo ws_info() {
     KernelInfo ki{attr_err == cudaSuccess ? fn : nullptr, LY::bytes, 1, LY::DT, LY::THREADS, LY::TS};
     ki.tma = true;
     return ki;
+}
+
+// The low-rank-Delta instance of the warp-specialised kernel for rank <= RP.
+KernelInfo ws_lowrank_info(vmb_dtype dt, int R) {
+    if (dt == VMB_BF16)
+        return R <= 8 ? ws_info<__nv_bfloat16, WsShape<4, 8, 4, 4, 8>>() : ws_info<__nv_bfloat16, WsShape<4, 8, 4, 4, 16>>();
+    return R <= 8 ? ws_info<float, WsShape<4, 8, 4, 4, 8>>() : ws_info<float, WsShape<4, 8, 4, 4, 16>>();
 }
 
 // The driver's tensor-map encoder, looked up once (null when unavailable).
@@ -2081,12 +2135,49 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan) {
 
 bool full_plan_gathers(const ScanPlan& plan) { return is_ws_shape(plan.np, plan.split); }
 
+// Raw Deltas of the low-rank form written out (for plans whose kernels read
+// materialised Deltas): out[b,k,d,l] = sum_r Wup[k,d,r] z[b,k,r,l], r in order
+// (the selection kernel's epilogue order), rounded to the storage type.
+template <typename T>
+__global__ void __launch_bounds__(256) lowrank_expand_kernel(const float* __restrict__ z, const float* __restrict__ Wup,
+                                                             T* __restrict__ out, int K, int D, int R, int L,
+                                                             long long total) {
+    pdl_wait();
+    pdl_launch_dependents();
+    for (long long i = blockIdx.x * 256LL + threadIdx.x; i < total; i += (long long)gridDim.x * 256) {
+        const int l = (int)(i % L);
+        const long long rowi = i / L;  // (b, k, d)
+        const int d = (int)(rowi % D);
+        const long long bk = rowi / D;
+        const int k = (int)(bk % K);
+        const float* w = Wup + ((size_t)k * D + d) * R;
+        const float* zz = z + (size_t)bk * R * L + l;
+        float s = 0.0f;
+        for (int r = 0; r < R; ++r) s = fmaf(__ldg(w + r), __ldg(zz + (size_t)r * L), s);
+        out[i] = io<T>::to(s);
+    }
+}
+
+vmb_status launch_lowrank_expand(const float* z, const float* Wup, void* out, int B, int K, int D, int R, int L,
+                                 vmb_dtype dt, cudaStream_t stream) {
+    long long total = (long long)B * K * D * L;
+    int K_ = K, D_ = D, R_ = R, L_ = L;
+    const long long want = (total + 255) / 256;
+    const unsigned grid = (unsigned)(want < 152LL * 64 ? want : 152LL * 64);
+    void* args[] = {(void*)&z, (void*)&Wup, &out, &K_, &D_, &R_, &L_, &total};
+    const void* fn = dt == VMB_BF16 ? reinterpret_cast<const void*>(&lowrank_expand_kernel<__nv_bfloat16>)
+                                    : reinterpret_cast<const void*>(&lowrank_expand_kernel<float>);
+    return launch_kernel(fn, dim3(grid), dim3(256), 0, args, stream) == cudaSuccess ? VMB_OK : VMB_ERR_CUDA;
+}
+
 int full_plan_launches(const ScanPlan& plan) {
     return (is_chunk_shape(plan.np, plan.split) && plan.n_chunks > 1) ? 3 : 1;
 }
 
 vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream) {
-    KernelInfo ki = pick(a.dtype, plan.np, plan.split, (a.flags & VMB_FLAG_B_ZOH) != 0);
+    const bool lowrank = a.R > 0;
+    if (lowrank && !is_ws_shape(plan.np, plan.split)) return VMB_ERR_UNSUPPORTED;
+    KernelInfo ki = lowrank ? ws_lowrank_info(a.dtype, a.R) : pick(a.dtype, plan.np, plan.split, (a.flags & VMB_FLAG_B_ZOH) != 0);
     if (!ki.fn) return VMB_ERR_CUDA;
     const size_t es = a.dtype == VMB_BF16 ? 2 : 4;
     FullParams p{};
@@ -2112,6 +2203,8 @@ vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     p.suppress = (a.flags & VMB_FLAG_TEST_SUPPRESS_PUBLISH) ? 1 : 0;
     p.gather_h = a.gather_h;
     if (a.gather_h > 0 && !ki.tma) return VMB_ERR_UNSUPPORTED;  // only the warp-specialised kernel gathers
+    p.Wup = a.Wup;
+    p.R = a.R;
     const WsLayout w = ws_layout(plan);
     unsigned char* ws = static_cast<unsigned char*>(a.ws);
     p.hdr = reinterpret_cast<WsHeader*>(ws);
@@ -2145,7 +2238,10 @@ vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
                                encode_rows(&tm.u2, a.u_t, a.dtype, a.L, a.D, a.B, ki.ts, ki.DT)
                          : encode_rows(&tm.u, a.u, a.dtype, a.L, a.D, planes, ki.ts, ki.DT);
         if (!gather) tm.u2 = tm.u;
-        if (ok && encode_rows(&tm.dl, a.delta, a.dtype, a.L, a.D, planes, ki.ts, ki.DT) &&
+        // the delta box: DT rows of raw Deltas, or (low rank) the 16 rows of z, fp32
+        ok = ok && (lowrank ? encode_rows(&tm.dl, a.delta, VMB_F32, a.L, a.R, planes, ki.ts, 16)
+                            : encode_rows(&tm.dl, a.delta, a.dtype, a.L, a.D, planes, ki.ts, ki.DT));
+        if (ok &&
             encode_rows(&tm.B, a.Bs, a.dtype, a.L, a.N, planes, ki.ts, 16) &&
             encode_rows(&tm.C, a.Cs, a.dtype, a.L, a.N, planes, ki.ts, 16)) {
             void* targs[] = {&p, &tm};
@@ -2156,7 +2252,7 @@ vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
         }
         // the encoder refused the tensors: the packed streaming variant (same tiles, same
         // results), which reads materialised sequences only
-        if (gather) return VMB_ERR_UNSUPPORTED;
+        if (gather || lowrank) return VMB_ERR_UNSUPPORTED;
         ki = pick(a.dtype, plan.np, kPackedShape, false);
         if (!ki.fn) return VMB_ERR_CUDA;
     }

@@ -45,6 +45,7 @@ struct SelParams {
     void* Bs;
     void* Cs;
     void* dr;
+    float* z;  // not null: the rank-R intermediate z [B,K,R,L] fp32 is written instead of dr
     int K, D, N, R, L;
     int nlb;  // step blocks per (b, k)
 };
@@ -270,6 +271,16 @@ __global__ void __launch_bounds__(kSelThreads, 5) selection_kernel(const SelPara
             }
         }
     }
+    if (p.z) {
+        // the low-rank form: z itself, for a scan that expands it through Wup
+        if (lv) {
+            float* oz = p.z + (size_t)bk * R * L + l;
+#pragma unroll
+            for (int r = 0; r < 16; ++r)
+                if (r < R) oz[(size_t)r * L] = acc[32 + r];
+        }
+        return;
+    }
     // the raw Deltas: z expanded through Wup, kSelDB channels' rows staged at a
     // time over the operand area (rows padded to kSelRP with zeros)
     float* sW = reinterpret_cast<float*>(smem);
@@ -326,6 +337,7 @@ vmb_status launch_selection(const SelArgs& a, cudaStream_t stream) {
     p.Bs = a.Bs;
     p.Cs = a.Cs;
     p.dr = a.delta_raw;
+    p.z = a.z;
     p.K = a.K;
     p.D = a.D;
     p.N = a.N;

@@ -338,6 +338,46 @@ vmb_status vmb_ss2d_mean_fwd(const void* x, void* xt, const void* delta, const f
     return launch_mean_merge(x, ybar, Dskip, out, B, D, H, W, (flags & VMB_FLAG_SKIP_MEAN) == 0, dtype, stream);
 }
 
+vmb_status vmb_selective_scan_lowrank_fwd(const void* u, const float* z, const float* Wup, const float* A,
+                                          const void* Bs, const void* Cs, const float* Dskip, const float* delta_bias,
+                                          void* y, int B, int K, int D, int N, int R, int H, int W, unsigned flags,
+                                          vmb_dtype dtype, void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+    if (H < 0 || W < 0 || R < 0) return VMB_ERR_INVALID_ARG;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    ScanArgs a{u, z, A, Bs, Cs, Dskip, delta_bias, y, nullptr, B, K, D, N, H * W, flags, dtype, workspace,
+               workspace_bytes};
+    a.Wup = Wup;
+    a.R = R;
+    bool empty = false;
+    vmb_status s = check_scan(a, false, &empty);
+    if (s != VMB_OK || empty) return s;
+    if (R < 1) return VMB_ERR_INVALID_ARG;
+    if (R > 16) return VMB_ERR_UNSUPPORTED;
+    if (!Wup || u == y) return VMB_ERR_INVALID_ARG;
+    if (!aligned(z, 4) || !aligned(Wup, 4)) return VMB_ERR_MISALIGNED;
+    if (!workspace) return VMB_ERR_WORKSPACE;
+    if (!aligned(workspace, 256)) return VMB_ERR_MISALIGNED;
+    ScanPlan plan{};
+    s = plan_full(a, &plan);
+    if (s != VMB_OK) return s;
+    if (workspace_bytes < plan.ws_bytes) return VMB_ERR_WORKSPACE;
+    if (full_plan_gathers(plan)) return launch_full(a, plan, stream);
+    // a plan whose kernel reads materialised raw Deltas: they are written into
+    // y and the scan runs in place (each of its CTAs reads the steps of its own
+    // rows before it writes them, and no other CTA touches them)
+    ScanArgs m = a;
+    m.delta = y;
+    m.Wup = nullptr;
+    m.R = 0;
+    ScanPlan mplan{};
+    s = plan_full(m, &mplan);
+    if (s != VMB_OK) return s;
+    if (workspace_bytes < mplan.ws_bytes) return VMB_ERR_WORKSPACE;
+    s = launch_lowrank_expand(z, Wup, y, B, K, D, R, H * W, dtype, stream);
+    if (s != VMB_OK) return s;
+    return launch_full(m, mplan, stream);
+}
+
 vmb_status vmb_ss2d_full_fwd(const void* x, void* xt, const void* delta, const float* A, const void* Bs,
                              const void* Cs, const float* Dskip, const float* delta_bias, void* y, void* out, int B,
                              int D, int N, int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,
@@ -471,6 +511,28 @@ vmb_status vmb_selection_fwd(const void* u, const float* WB, const float* WC, co
         !aligned(WC, 4) || !aligned(Wz, 4) || !aligned(Wup, 4))
         return VMB_ERR_MISALIGNED;
     SelArgs a{u, WB, WC, Wz, Wup, Bs, Cs, delta_raw, B, K, D, N, R, H * W, dtype};
+    return launch_selection(a, stream);
+}
+
+vmb_status vmb_selection_lowrank_fwd(const void* u, const float* WB, const float* WC, const float* Wz, void* Bs,
+                                     void* Cs, float* z, int B, int K, int D, int N, int R, int H, int W,
+                                     vmb_dtype dtype, cudaStream_t stream) {
+    if (!dtype_ok(dtype) || B < 0 || K < 0 || D < 0 || N < 0 || R < 0 || H < 0 || W < 0) return VMB_ERR_INVALID_ARG;
+    long long n = 0, nbc = 0;
+    if (!count(&n, {B, K, D, H, W}) || !count(&nbc, {B, K, N > 0 ? N : 1, H, W})) return VMB_ERR_INVALID_ARG;
+    if (n == 0) return VMB_OK;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    if (N < 1 || R < 1) return VMB_ERR_INVALID_ARG;
+    if (N > 16 || R > 16) return VMB_ERR_UNSUPPORTED;
+    long long rows = 0;
+    if (!count(&rows, {B, K, D}) || rows > INT_MAX / 2) return VMB_ERR_UNSUPPORTED;
+    if (!u || !WB || !WC || !Wz || !Bs || !Cs || !z) return VMB_ERR_INVALID_ARG;
+    const size_t es = esize(dtype);
+    if (!aligned(u, es) || !aligned(Bs, es) || !aligned(Cs, es) || !aligned(z, 4) || !aligned(WB, 4) ||
+        !aligned(WC, 4) || !aligned(Wz, 4))
+        return VMB_ERR_MISALIGNED;
+    SelArgs a{u, WB, WC, Wz, nullptr, Bs, Cs, nullptr, B, K, D, N, R, H * W, dtype};
+    a.z = z;
     return launch_selection(a, stream);
 }
 

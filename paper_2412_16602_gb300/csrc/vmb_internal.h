@@ -33,6 +33,8 @@ struct ScanArgs {
                             // cross-scan)
     const void* u_t = nullptr;
     float* saved = nullptr;  // mean path: the group means kept for the backward, [B*K][N + 1][L] fp32
+    const float* Wup = nullptr;  // full path, low-rank Delta: delta is z [B*K][R][L] fp32 and
+    int R = 0;                   // delta_raw = Wup z (Wup [K][D][R]); warp-specialised plans only
 };
 
 // Execution plan of an L-chunked scan: how the (sequence, chunk) grid is cut
@@ -105,6 +107,7 @@ struct SelArgs {
     void* delta_raw;   // [B][K][D][L], dtype
     int B, K, D, N, R, L;
     vmb_dtype dtype;
+    float* z = nullptr;  // not null: z [B][K][R][L] fp32 written instead of delta_raw (Wup unused)
 };
 
 // Gradients of the (grouped) channel-mean scan.
@@ -146,8 +149,12 @@ vmb_status plan_full(const ScanArgs& a, ScanPlan* plan);
 vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan);
 vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream);
 int full_plan_launches(const ScanPlan& plan);  // kernels launch_full starts for this plan
-// Whether launch_full can read the plan's u gathered from the map (ScanArgs::gather_h).
+// Whether launch_full can read the plan's u gathered from the map (ScanArgs::gather_h)
+// or expand a low-rank Delta (ScanArgs::R): the warp-specialised plans.
 bool full_plan_gathers(const ScanPlan& plan);
+// out [B,K,D,L] (dtype) = Wup z, the raw Deltas of the low-rank form.
+vmb_status launch_lowrank_expand(const float* z, const float* Wup, void* out, int B, int K, int D, int R, int L,
+                                 vmb_dtype dt, cudaStream_t stream);
 vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream);
 vmb_status launch_cross_scan(const void* x, void* xs, int B, int D, int H, int W, vmb_dtype dt,
                              cudaStream_t stream);

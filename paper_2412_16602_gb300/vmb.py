@@ -41,7 +41,8 @@ EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb
            "vmb_selective_scan_fwd",
            "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_ss2d_mean_fwd",
            "vmb_ss2d_full_fwd", "vmb_discretise_fwd", "vmb_discretise_mean_fwd",
-           "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_mean_scan_train_fwd", "vmb_mean_scan_bwd",
+           "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_selection_lowrank_fwd", "vmb_selective_scan_lowrank_fwd",
+           "vmb_mean_scan_train_fwd", "vmb_mean_scan_bwd",
            "vmb_mean_scan_bwd_workspace_bytes",
            "vmb_read_status", "vmb_status_string", "vmb_version"]
 
@@ -73,6 +74,8 @@ def _load() -> ctypes.CDLL:
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
     lib.vmb_selection_fwd.argtypes = [vp] * 8 + [i] * 7 + [i, vp]
+    lib.vmb_selection_lowrank_fwd.argtypes = [vp] * 7 + [i] * 7 + [i, vp]
+    lib.vmb_selective_scan_lowrank_fwd.argtypes = [vp] * 9 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_train_fwd.argtypes = [vp] * 10 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_bwd.argtypes = [vp] * 16 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_bwd_workspace_bytes.argtypes = [i] * 8
@@ -85,6 +88,7 @@ def _load() -> ctypes.CDLL:
                  "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_ss2d_mean_fwd", "vmb_ss2d_full_fwd",
                  "vmb_discretise_fwd",
                  "vmb_discretise_mean_fwd", "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_mean_scan_bwd",
+                 "vmb_selection_lowrank_fwd", "vmb_selective_scan_lowrank_fwd",
                  "vmb_read_status", "vmb_version"]:
         getattr(lib, name).restype = i
     return lib
@@ -550,6 +554,59 @@ def vmb_selection_fwd(u, WB, WC, Wz, Wup, H: int, W: int, *, delta_raw=None, Bs=
                                  _ptr(delta_raw), B, K, D, N, R, H, W, _dtype_code(u.dtype), _stream(stream)),
            "vmb_selection_fwd")
     return delta_raw, Bs, Cs
+
+
+def vmb_selection_lowrank_fwd(u, WB, WC, Wz, H: int, W: int, *, z=None, Bs=None, Cs=None, stream=None):
+    """Eq. 6 selection functions with the Delta branch left low-rank: u [B, K, D, H*W] ->
+    (z [B, K, R, L] float32, Bs, Cs [B, K, N, L] in u's dtype); WB, WC [K, N, D], Wz [K, R, D]."""
+    for t, n in [(u, "u"), (WB, "WB"), (WC, "WC"), (Wz, "Wz")]:
+        _dev(t, n)
+    B, K, D, L = u.shape
+    N, R = WB.shape[1], Wz.shape[1]
+    if L != H * W or tuple(WB.shape) != (K, N, D) or tuple(WC.shape) != (K, N, D) or tuple(Wz.shape) != (K, R, D):
+        raise ValueError("u [B,K,D,H*W], WB/WC [K,N,D], Wz [K,R,D] expected")
+    if any(w.dtype != torch.float32 for w in (WB, WC, Wz)):
+        raise ValueError("weights must be float32")
+    z = torch.empty((B, K, R, L), dtype=torch.float32, device=u.device) if z is None else z
+    Bs = torch.empty((B, K, N, L), dtype=u.dtype, device=u.device) if Bs is None else Bs
+    Cs = torch.empty((B, K, N, L), dtype=u.dtype, device=u.device) if Cs is None else Cs
+    for t, n, shp, dt in [(z, "z", (B, K, R, L), torch.float32), (Bs, "Bs", (B, K, N, L), u.dtype),
+                          (Cs, "Cs", (B, K, N, L), u.dtype)]:
+        _dev(t, n)
+        if tuple(t.shape) != shp or t.dtype != dt:
+            raise ValueError(f"{n} must be {dt} {shp}")
+    _check(lib.vmb_selection_lowrank_fwd(_ptr(u), _ptr(WB), _ptr(WC), _ptr(Wz), _ptr(Bs), _ptr(Cs), _ptr(z),
+                                         B, K, D, N, R, H, W, _dtype_code(u.dtype), _stream(stream)),
+           "vmb_selection_lowrank_fwd")
+    return z, Bs, Cs
+
+
+def vmb_selective_scan_lowrank_fwd(u, z, Wup, A, Bs, Cs, Dskip, delta_bias, H: int, W: int, *, y=None,
+                                   flags: int = VMB_FLAG_SOFTPLUS, workspace=None, stream=None) -> torch.Tensor:
+    """Full-channel selective scan whose raw Deltas are Wup z, formed inside the scan:
+    z [B, K, R, H*W] float32, Wup [K, D, R] float32; returns y [B, K, D, H*W] (dtype of u)."""
+    for t, n in [(z, "z"), (Wup, "Wup")]:
+        _dev(t, n)
+    B, K, D, L = u.shape
+    R = z.shape[2]
+    if tuple(z.shape) != (B, K, R, L) or z.dtype != torch.float32:
+        raise ValueError("z must be float32 [B, K, R, H*W]")
+    if tuple(Wup.shape) != (K, D, R) or Wup.dtype != torch.float32:
+        raise ValueError("Wup must be float32 [K, D, R]")
+    B, K, D, N, L = _scan_shapes(u, u, A, Bs, Cs, Dskip, delta_bias, H, W)
+    if y is None:
+        y = torch.empty_like(u)
+    _dev(y, "y")
+    if y.shape != u.shape or y.dtype != u.dtype:
+        raise ValueError("y must match u")
+    ws_bytes = vmb_scan_workspace_bytes(VMB_PATH_FULL, B, K, D, N, H, W, u.dtype)
+    if workspace is None:
+        workspace = _default_ws.get(ws_bytes, u.device)
+    _check(lib.vmb_selective_scan_lowrank_fwd(_ptr(u), _ptr(z), _ptr(Wup), _ptr(A), _ptr(Bs), _ptr(Cs), _ptr(Dskip),
+                                              _ptr(delta_bias), _ptr(y), B, K, D, N, R, H, W, flags,
+                                              _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
+                                              _stream(stream)), "vmb_selective_scan_lowrank_fwd")
+    return y
 
 
 def vmb_mean_scan_bwd_workspace_bytes(B: int, K: int, D: int, N: int, H: int, W: int, groups: int = 1,

@@ -32,6 +32,8 @@ def lib():
     lib.vmb_discretise_mean_fwd.argtypes = [vp] * 7 + [i] * 6 + [u, i, vp]
     lib.vmb_scan_only_fwd.argtypes = [vp] * 4 + [i] * 6 + [i, vp]
     lib.vmb_selection_fwd.argtypes = [vp] * 8 + [i] * 7 + [i, vp]
+    lib.vmb_selection_lowrank_fwd.argtypes = [vp] * 7 + [i] * 7 + [i, vp]
+    lib.vmb_selective_scan_lowrank_fwd.argtypes = [vp] * 9 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_bwd.argtypes = [vp] * 16 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_train_fwd.argtypes = [vp] * 10 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_bwd_workspace_bytes.argtypes = [i] * 8
@@ -192,6 +194,47 @@ def test_ss2d_full_validation(lib):
     assert ss2d_full_call(lib, flags=0x100) == 1
     assert ss2d_full_call(lib, ws=0) == 4
     assert ss2d_full_call(lib, ptrs=[0] * 10, B=0, ws=0) == 0                  # empty problem
+
+
+def sel_lr_call(lib, *, ptrs=None, B=1, K=4, D=8, N=16, R=6, H=4, W=4, dtype=0):
+    p = [FAKE] * 4 + [FAKE + 0x1000, FAKE + 0x2000, FAKE + 0x3000] if ptrs is None else ptrs
+    return lib.vmb_selection_lowrank_fwd(*p, B, K, D, N, R, H, W, dtype, S)
+
+
+def test_selection_lowrank_validation(lib):
+    base = [FAKE] * 4 + [FAKE + 0x1000, FAKE + 0x2000, FAKE + 0x3000]
+    assert sel_lr_call(lib, B=-1) == 1
+    assert sel_lr_call(lib, N=0) == 1
+    assert sel_lr_call(lib, R=0) == 1
+    assert sel_lr_call(lib, R=17) == 3
+    assert sel_lr_call(lib, ptrs=base[:6] + [0]) == 1                          # null z
+    assert sel_lr_call(lib, ptrs=base[:6] + [FAKE + 0x3002]) == 2              # misaligned z (fp32)
+    assert sel_lr_call(lib, dtype=5) == 1
+    assert sel_lr_call(lib, ptrs=[0] * 7, B=0) == 0                            # empty problem
+
+
+def scan_lr_call(lib, *, ptrs=None, B=1, K=4, D=8, N=16, R=6, H=4, W=4, flags=1, dtype=0, ws=0x100000,
+                 ws_bytes=1 << 20):
+    p = [FAKE, FAKE + 0x1000] + [FAKE] * 6 + [FAKE + 0x2000] if ptrs is None else ptrs
+    return lib.vmb_selective_scan_lowrank_fwd(*p, B, K, D, N, R, H, W, flags, dtype, ws, ws_bytes, S)
+
+
+def test_selective_scan_lowrank_validation(lib):
+    """Rank, the low-rank operands and the usual scan arguments are checked
+    before any launch."""
+    base = [FAKE, FAKE + 0x1000] + [FAKE] * 6 + [FAKE + 0x2000]
+    assert scan_lr_call(lib, B=-1) == 1
+    assert scan_lr_call(lib, R=-1) == 1
+    assert scan_lr_call(lib, R=0) == 1
+    assert scan_lr_call(lib, R=17) == 3
+    assert scan_lr_call(lib, N=17) == 3
+    assert scan_lr_call(lib, ptrs=base[:2] + [0] + base[3:]) == 1              # null Wup
+    assert scan_lr_call(lib, ptrs=base[:1] + [0] + base[2:]) == 1              # null z
+    assert scan_lr_call(lib, ptrs=base[:1] + [FAKE + 0x1002] + base[2:]) == 2  # misaligned z
+    assert scan_lr_call(lib, ptrs=base[:8] + [FAKE]) == 1                      # y aliases u
+    assert scan_lr_call(lib, flags=0x100) == 1
+    assert scan_lr_call(lib, ws=0) == 4
+    assert scan_lr_call(lib, ptrs=[0] * 9, B=0, ws=0) == 0                     # empty problem
 
 
 def disc_call(fn, *, ptrs=None, B=1, K=4, D=8, N=16, H=4, W=4, flags=1, dtype=0):
