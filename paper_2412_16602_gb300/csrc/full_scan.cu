@@ -1473,9 +1473,10 @@ __global__ void __launch_bounds__(PackedLayout<T, PS>::THREADS, PS::MINB) full_p
 // sum_r Wup[k,d,r] z_r (r in order, as the selection kernel's epilogue does,
 // so fp32 results are bit-identical to selection -> raw Deltas -> scan), with
 // its Wup row (RP >= R values, zero-padded) in registers.
-template <int CW_, int TS_, int NSTG_, int MINB_, int RP_ = 0>
+template <int CW_, int TS_, int NSTG_, int MINB_, int RP_ = 0, bool GATHER_ = false>
 struct WsShape {
     static constexpr int CW = CW_, TS = TS_, NSTG = NSTG_, MINB = MINB_, RP = RP_;
+    static constexpr bool GATHER = GATHER_;  // u gathered from the map (see above)
 };
 
 struct TensorMaps {
@@ -1540,7 +1541,7 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
     if (warp == LY::CW) {
         // ------------------------------------------------------ producer warp
         // u: the rows of (b, k), or gathered from x / xt (see above)
-        const bool gather = p.gather_h > 0;
+        constexpr bool gather = WS::GATHER;
         const CUtensorMap* um = (gather && (k & 1)) ? &tm.u2 : &tm.u;
         const int uz = gather ? bk / p.K : bk;
         const bool urev = gather && k >= 2;
@@ -1585,7 +1586,7 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
     }
     if (warp >= cwarps) return;  // a tile's channels past D: no work, not counted by `released`
     // -------------------------------------------------------- consumer warps
-    const bool urev = p.gather_h > 0 && k >= 2;  // u arrives mirrored (see above)
+    const bool urev = WS::GATHER && k >= 2;  // u arrives mirrored (see above)
     const int c = tid;
     const int d = d0 + c;
     const bool cval = d < p.D;
@@ -1863,6 +1864,12 @@ KernelInfo ws_info() {
     KernelInfo ki{attr_err == cudaSuccess ? fn : nullptr, LY::bytes, 1, LY::DT, LY::THREADS, LY::TS};
     ki.tma = true;
     return ki;
+}
+
+// The gathering instance of the warp-specialised kernel (u from the map).
+KernelInfo ws_gather_info(vmb_dtype dt) {
+    return dt == VMB_BF16 ? ws_info<__nv_bfloat16, WsShape<4, 8, 4, 4, 0, true>>()
+                          : ws_info<float, WsShape<4, 8, 4, 4, 0, true>>();
 }
 
 // The low-rank-Delta instance of the warp-specialised kernel for rank <= RP.
@@ -2176,8 +2183,11 @@ int full_plan_launches(const ScanPlan& plan) {
 
 vmb_status launch_full(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream) {
     const bool lowrank = a.R > 0;
-    if (lowrank && !is_ws_shape(plan.np, plan.split)) return VMB_ERR_UNSUPPORTED;
-    KernelInfo ki = lowrank ? ws_lowrank_info(a.dtype, a.R) : pick(a.dtype, plan.np, plan.split, (a.flags & VMB_FLAG_B_ZOH) != 0);
+    if ((lowrank || a.gather_h > 0) && !is_ws_shape(plan.np, plan.split)) return VMB_ERR_UNSUPPORTED;
+    if (lowrank && a.gather_h > 0) return VMB_ERR_UNSUPPORTED;
+    KernelInfo ki = lowrank ? ws_lowrank_info(a.dtype, a.R)
+                    : a.gather_h > 0 ? ws_gather_info(a.dtype)
+                                     : pick(a.dtype, plan.np, plan.split, (a.flags & VMB_FLAG_B_ZOH) != 0);
     if (!ki.fn) return VMB_ERR_CUDA;
     const size_t es = a.dtype == VMB_BF16 ? 2 : 4;
     FullParams p{};
