@@ -663,9 +663,19 @@ def run_ours(args, wl, rank, world, local_rank):
         def scan_raw():
             vmb.vmb_selective_scan_fwd(outs["xs"], sdr, g["A"], sB, sC, g["Dskip"], g["bias"], wl.H, wl.W,
                                        y=ylr, workspace=wsf, stream=stream)
+        wsm = outs["ws_mean"]
+
+        def mean_lr():
+            vmb.vmb_mean_scan_lowrank_fwd(outs["xs"], sz, sw[3], g["A"], sB, sC, g["Dskip"], g["bias"],
+                                          wl.H, wl.W, y=ylr, workspace=wsm, stream=stream)
+
+        def mean_raw():
+            vmb.vmb_mean_scan_fwd(outs["xs"], sdr, g["A"], sB, sC, g["Dskip"], g["bias"], wl.H, wl.W,
+                                  y=ylr, workspace=wsm, stream=stream)
         sel()
         lowrank = {"selection_us": time_alone(sel_lr), "scan_us": time_alone(scan_lr),
-                   "scan_raw_deltas_us": time_alone(scan_raw), "rank": R}
+                   "scan_raw_deltas_us": time_alone(scan_raw), "rank": R,
+                   "mean_scan_us": time_alone(mean_lr), "mean_scan_raw_deltas_us": time_alone(mean_raw)}
         sel_us = (sel_us, lowrank)
     # the backward of the channel-mean scan on the step's inputs (dLoss/dy drawn
     # on the device), with its workspace allocated once
@@ -790,7 +800,12 @@ def selection_summary(us_pair, wl, peak, R=6):
                "scan_frac_of_peak": scan_lr_bytes / (lr["scan_us"] / 1e6) / 1e9 / peak,
                "pair_us": pair_lr, "pair_bytes": sel_lr_bytes + scan_lr_bytes,
                "raw_deltas_pair_us": pair_raw, "raw_deltas_pair_bytes": bytes_ + wl.scan_bytes(),
-               "speedup_over_raw_deltas": pair_raw / pair_lr}
+               "speedup_over_raw_deltas": pair_raw / pair_lr,
+               "mean_scan_us": lr["mean_scan_us"], "mean_scan_raw_deltas_us": lr["mean_scan_raw_deltas_us"],
+               "mean_pair_us": lr["selection_us"] + lr["mean_scan_us"],
+               "mean_raw_deltas_pair_us": us + lr["mean_scan_raw_deltas_us"],
+               "mean_speedup_over_raw_deltas": (us + lr["mean_scan_raw_deltas_us"]) /
+                                               (lr["selection_us"] + lr["mean_scan_us"])}
     return {"us": us, "algorithmic_bytes": bytes_, "gbs": gbs, "frac_of_peak": gbs / peak, "rank": R,
             "kernel": "tcgen05.mma kind::tf32 (three-product tf32 split for fp32 accuracy), accumulator in TMEM",
             "lowrank": lowrank}

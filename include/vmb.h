@@ -400,6 +400,24 @@ vmb_status vmb_selective_scan_lowrank_fwd(const void* u, const float* z, const f
                                           void* workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /*
+ * vmb_mean_scan_lowrank_fwd - vmb_mean_scan_fwd (the channel-mean scan of
+ *   Sec. 2.2, Eq. 9) with delta_raw = Wup z formed inside the scan, as in
+ *   vmb_selective_scan_lowrank_fwd: z [B,K,R,L] fp32, Wup [K,D,R] fp32, R in
+ *   1..16; every other argument (ybar optional), flag and the workspace
+ *   (vmb_scan_workspace_bytes(VMB_PATH_MEAN, ...)) as vmb_mean_scan_fwd; y
+ *   must not alias u.  For ranks up to 8 with the Euler Bbar each thread of
+ *   the reduction forms the raw Delta of its step and channel (R FMAs) instead
+ *   of reading it; otherwise the raw Deltas are written into y (rounded to the
+ *   storage type) and the scan runs in place.  In fp32 the result is
+ *   bit-identical to vmb_selection_fwd's raw Deltas fed to vmb_mean_scan_fwd.
+ */
+vmb_status vmb_mean_scan_lowrank_fwd(const void* u, const float* z, const float* Wup, const float* A,
+                                     const void* Bs, const void* Cs, const float* Dskip,
+                                     const float* delta_bias, void* y, float* ybar, int B, int K, int D,
+                                     int N, int R, int H, int W, unsigned flags, vmb_dtype dtype,
+                                     void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
  * vmb_mean_scan_train_fwd - vmb_mean_scan_grouped_fwd (groups = 1: the
  * channel-mean scan of Eq. 9) that also keeps, for vmb_mean_scan_bwd, the
  * group means it forms on the way:

@@ -61,6 +61,9 @@ struct MeanParams {
     const void* u_t;
     float* save;   // not null: the group means kept for the backward, [n_seq][N + 1][L] fp32
                    // (rows 0 .. N-1 Abar_n, row N the mean of delta u)
+    const float* z;    // low-rank Delta (LR kernels): z [n_seq][R][L] fp32 and Wup [K][D][R] fp32,
+    const float* Wup;  // delta_raw[d, l] = sum_r Wup[k, d, r] z[r, l] (r in order)
+    int R;
     WsHeader* hdr;
     unsigned* flags;
     float* aggP;
@@ -68,11 +71,13 @@ struct MeanParams {
     float* incH;
 };
 
-template <typename T, int NP, int TC, bool ZOH>
+template <typename T, int NP, int TC, bool ZOH, bool LR = false>
 struct MLayout {
     static constexpr int S = kThreads / TC;  // channel groups
     static constexpr int NMC = TC / kMC;
-    static constexpr int CG = 256;           // channels whose A / bias / Dskip are staged at a time
+    // channels whose A / bias / Dskip (and, low rank, Wup rows) are staged at a time
+    static constexpr int CG = LR ? 128 : 256;
+    static constexpr int WR = 8;             // low rank: staged Wup row length (ranks up to 8, zero-padded)
     static constexpr int BCS = TC + 16 / (int)sizeof(T);  // raw B / C row stride (elements), rows 16-byte aligned
     // shared memory, byte offsets
     static constexpr size_t red = 0;                                            // f32 [S][NP][TC] partial sums of Abar
@@ -89,7 +94,7 @@ struct MLayout {
     // channel tables of one group of CG channels: A [CG][NP] (scaled by log2 e
     // in place unless ZOH), delta bias [CG], Dskip [CG]
     static constexpr size_t tab0 = a16(bc + (size_t)2 * NP * BCS * sizeof(T));
-    static constexpr size_t tab_bytes = (size_t)CG * NP * 4 + 2 * (size_t)CG * 4;
+    static constexpr size_t tab_bytes = (size_t)CG * NP * 4 + 2 * (size_t)CG * 4 + (LR ? (size_t)CG * WR * 4 : 0);
     static constexpr size_t bytes1 = tab0 + tab_bytes;
     static constexpr size_t bytes2 = bytes1;
     static_assert(kThreads % TC == 0 && TC % 32 == 0, "a warp covers 32 consecutive steps");
@@ -100,9 +105,9 @@ struct MLayout {
 // Stage group g0 of the channel tables (raw A rows, delta bias, Dskip) into
 // buffer `tb`: 16-byte async copies where rows are aligned, element loads
 // otherwise; channels past the group are zero.
-template <typename T, int NP, int TC, bool ZOH>
+template <typename T, int NP, int TC, bool ZOH, bool LR = false>
 __device__ __forceinline__ void stage_tables(const MeanParams& p, unsigned char* tb, int k, int g0, int gn) {
-    using LY = MLayout<T, NP, TC, ZOH>;
+    using LY = MLayout<T, NP, TC, ZOH, LR>;
     constexpr int CG = LY::CG;
     float* ta = reinterpret_cast<float*>(tb);
     float* tbias = ta + CG * NP;
@@ -140,6 +145,15 @@ __device__ __forceinline__ void stage_tables(const MeanParams& p, unsigned char*
             tdsk[i] = i < gn ? __ldg(dg + i) : 0.0f;
         }
     }
+    if constexpr (LR) {
+        // Wup rows of the group, [CG][WR] fp32, zero past R and past the group
+        float* tw = reinterpret_cast<float*>(tb) + CG * NP + 2 * CG;
+        const float* wg = p.Wup + ((size_t)k * p.D + g0) * p.R;
+        for (int i = tid; i < CG * LY::WR; i += kThreads) {
+            const int r = i / LY::WR, q = i % LY::WR;
+            tw[i] = (r < gn && q < p.R) ? __ldg(wg + (size_t)r * p.R + q) : 0.0f;
+        }
+    }
 }
 
 // Four consecutive elements with an L2 eviction policy (16 bytes fp32, 8 bytes bf16).
@@ -169,9 +183,16 @@ __device__ __forceinline__ void st4_hint(__nv_bfloat16* q, const float (&v)[4], 
     asm volatile("st.global.L2::cache_hint.v2.b32 [%0], {%1, %2}, %3;" ::"l"(q), "r"(a), "r"(b), "l"(pol) : "memory");
 }
 
-template <typename T, int NP, int TC, bool ZOH>
+// LR: the raw Deltas are formed from the low-rank form of Eq. 6 (z, Wup) at
+// the thread's step instead of being read: R FMAs per channel, r in order (the
+// selection kernel's epilogue order, so fp32 results are bit-identical to
+// selection -> raw Deltas -> this scan), z of the step in registers, the Wup
+// row read through L1 (every lane of a warp has the same channel).
+constexpr int kLRMax = 8;  // ranks the LR kernels hold in registers
+
+template <typename T, int NP, int TC, bool ZOH, bool LR = false>
 __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const MeanParams p) {
-    using LY = MLayout<T, NP, TC, ZOH>;
+    using LY = MLayout<T, NP, TC, ZOH, LR>;
     constexpr int S = LY::S, NMC = LY::NMC, CG = LY::CG, BCS = LY::BCS;
     extern __shared__ __align__(16) unsigned char smb[];
     float* red = reinterpret_cast<float*>(smb + LY::red);
@@ -253,7 +274,7 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
         }
     }
     const int ngroups = (D + CG - 1) / CG;
-    stage_tables<T, NP, TC, ZOH>(p, smb + LY::tab0, k, 0, min(CG, D));
+    stage_tables<T, NP, TC, ZOH, LR>(p, smb + LY::tab0, k, 0, min(CG, D));
     cp_async_commit();
 
     // ---------------------------------------------------------------- phase A
@@ -288,10 +309,18 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
     float* s_a2 = reinterpret_cast<float*>(smb + LY::tab0);
     const float* s_bias = s_a2 + CG * NP;
     const float* s_dsk = s_bias + CG;
+    const float* s_wup = s_dsk + CG;  // low rank: the group's Wup rows [CG][WR]
     // Offsets within the (b, k) slab are 32-bit (D * L < 2^31, checked by the
     // planner); a thread's consecutive channels are SL elements apart.
     const int SL = S * L;
     float vd[kPF], vu[kPF];
+    float zr[LR ? kLRMax : 1];  // LR: z of this thread's step
+    if constexpr (LR) {
+#pragma unroll
+        for (int r = 0; r < kLRMax; ++r)
+            zr[r] = (tv && r < p.R) ? __ldg(p.z + ((size_t)seq * p.R + r) * L + col) : 0.0f;
+    }
+    static_assert(!LR || kLRMax == 8, "the staged Wup rows hold 8 ranks");
     {
         // the first group's first channels, requested before the tables are waited on
         const int gn = min(CG, D);
@@ -299,12 +328,27 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
 #pragma unroll
         for (int q = 0; q < kPF; ++q, o += SL) {
             const int d = sg + q * S;
-            vd[q] = (tv && d < gn) ? ld_hint(dcol + o, stream) : 0.0f;
+            vd[q] = (!LR && tv && d < gn) ? ld_hint(dcol + o, stream) : 0.0f;
             vu[q] = (tv && d < gn) ? ld_hint(ucol + o, keep) : 0.0f;
         }
     }
     // one channel's contribution: softplus, the N exponentials of Abar, delta u
     auto reduce_one = [&](float vdq, float vuq, int d) {
+        if constexpr (LR) {
+            // the row is zero past R, as is zr: the padded terms add exact zeros
+            const float4* w4 = reinterpret_cast<const float4*>(s_wup + d * LY::WR);
+            const float4 wa = w4[0], wb = w4[1];
+            float rs = 0.0f;
+            rs = fmaf(wa.x, zr[0], rs);
+            rs = fmaf(wa.y, zr[1], rs);
+            rs = fmaf(wa.z, zr[2], rs);
+            rs = fmaf(wa.w, zr[3], rs);
+            rs = fmaf(wb.x, zr[4], rs);
+            rs = fmaf(wb.y, zr[5], rs);
+            rs = fmaf(wb.z, zr[6], rs);
+            rs = fmaf(wb.w, zr[7], rs);
+            vdq = rs;
+        }
         const float v = vdq + s_bias[d];
         const float dv = p.softplus_on ? softplus(v) : v;
         const float* a2 = s_a2 + d * NP;  // broadcast reads: every lane has the same d
@@ -350,7 +394,7 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
         const int g0 = gi * CG, gn = min(CG, D - g0);
         if (gi > 0) {
             __syncthreads();  // the previous group's tables are no longer read
-            stage_tables<T, NP, TC, ZOH>(p, smb + LY::tab0, k, g0, gn);
+            stage_tables<T, NP, TC, ZOH, LR>(p, smb + LY::tab0, k, g0, gn);
             cp_async_commit();
         }
         cp_async_wait<0>();
@@ -365,7 +409,7 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
 #pragma unroll
             for (int q = 0; q < kPF; ++q, o += SL) {
                 const int d = sg + q * S;
-                vd[q] = d < gn ? ld_hint(dcol + o, stream) : 0.0f;
+                vd[q] = (!LR && d < gn) ? ld_hint(dcol + o, stream) : 0.0f;
                 vu[q] = d < gn ? ld_hint(ucol + o, keep) : 0.0f;
             }
         }
@@ -376,14 +420,14 @@ __global__ void __launch_bounds__(kThreads, ZOH ? 2 : 3) mean_scan_kernel(const 
                 // the next batch is entirely in range: no per-channel checks
 #pragma unroll
                 for (int q = 0; q < kPF; ++q, o += SL) {
-                    nd[q] = ld_hint(dcol + o, stream);
+                    nd[q] = LR ? 0.0f : ld_hint(dcol + o, stream);
                     nu[q] = ld_hint(ucol + o, keep);
                 }
             } else {
 #pragma unroll
                 for (int q = 0; q < kPF; ++q, o += SL) {
                     const int d = d0 + (q + kPF) * S;
-                    nd[q] = d < gn ? ld_hint(dcol + o, stream) : 0.0f;
+                    nd[q] = (!LR && d < gn) ? ld_hint(dcol + o, stream) : 0.0f;
                     nu[q] = d < gn ? ld_hint(ucol + o, keep) : 0.0f;
                 }
             }
@@ -666,10 +710,10 @@ struct KInfo {
     size_t smem2;  // D > 256: two
 };
 
-template <typename T, int NP, int TC, bool ZOH>
+template <typename T, int NP, int TC, bool ZOH, bool LR>
 KInfo minfo() {
-    using LY = MLayout<T, NP, TC, ZOH>;
-    const void* fn = reinterpret_cast<const void*>(&mean_scan_kernel<T, NP, TC, ZOH>);
+    using LY = MLayout<T, NP, TC, ZOH, LR>;
+    const void* fn = reinterpret_cast<const void*>(&mean_scan_kernel<T, NP, TC, ZOH, LR>);
     static std::once_flag once;
     static cudaError_t err = cudaSuccess;
     std::call_once(once, [&] {
@@ -679,29 +723,32 @@ KInfo minfo() {
     return {fn, LY::bytes1, LY::bytes2};
 }
 
-template <typename T, int NP, bool ZOH>
+template <typename T, int NP, bool ZOH, bool LR>
 KInfo pick_tc(int tc) {
     switch (tc) {
-    case 32: return minfo<T, NP, 32, ZOH>();
-    case 128: return minfo<T, NP, 128, ZOH>();
-    default: return minfo<T, NP, 64, ZOH>();
+    case 32: return minfo<T, NP, 32, ZOH, LR>();
+    case 128: return minfo<T, NP, 128, ZOH, LR>();
+    default: return minfo<T, NP, 64, ZOH, LR>();
     }
 }
 
-template <typename T, bool ZOH>
+template <typename T, bool ZOH, bool LR>
 KInfo pick_np(int np, int tc) {
     switch (np) {
-    case 1: return pick_tc<T, 1, ZOH>(tc);
-    case 2: return pick_tc<T, 2, ZOH>(tc);
-    case 4: return pick_tc<T, 4, ZOH>(tc);
-    case 8: return pick_tc<T, 8, ZOH>(tc);
-    default: return pick_tc<T, 16, ZOH>(tc);
+    case 1: return pick_tc<T, 1, ZOH, LR>(tc);
+    case 2: return pick_tc<T, 2, ZOH, LR>(tc);
+    case 4: return pick_tc<T, 4, ZOH, LR>(tc);
+    case 8: return pick_tc<T, 8, ZOH, LR>(tc);
+    default: return pick_tc<T, 16, ZOH, LR>(tc);
     }
 }
 
-KInfo mpick(vmb_dtype dt, int np, int tc, bool zoh) {
-    if (dt == VMB_BF16) return zoh ? pick_np<__nv_bfloat16, true>(np, tc) : pick_np<__nv_bfloat16, false>(np, tc);
-    return zoh ? pick_np<float, true>(np, tc) : pick_np<float, false>(np, tc);
+// lr: the low-rank-Delta kernels (Euler Bbar only)
+KInfo mpick(vmb_dtype dt, int np, int tc, bool zoh, bool lr = false) {
+    if (lr) return dt == VMB_BF16 ? pick_np<__nv_bfloat16, false, true>(np, tc) : pick_np<float, false, true>(np, tc);
+    if (dt == VMB_BF16)
+        return zoh ? pick_np<__nv_bfloat16, true, false>(np, tc) : pick_np<__nv_bfloat16, false, false>(np, tc);
+    return zoh ? pick_np<float, true, false>(np, tc) : pick_np<float, false, false>(np, tc);
 }
 
 }  // namespace
@@ -751,7 +798,9 @@ vmb_status plan_mean(const ScanArgs& a, ScanPlan* plan) {
 }
 
 vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t stream) {
-    KInfo ki = mpick(a.dtype, plan.np, plan.chunk_len, (a.flags & VMB_FLAG_B_ZOH) != 0);
+    const bool lr = a.R > 0;
+    if (lr && ((a.flags & VMB_FLAG_B_ZOH) || a.R > kLRMax || a.bc_group != 1)) return VMB_ERR_UNSUPPORTED;
+    KInfo ki = mpick(a.dtype, plan.np, plan.chunk_len, (a.flags & VMB_FLAG_B_ZOH) != 0, lr);
     if (!ki.fn) return VMB_ERR_CUDA;
     MeanParams p{};
     p.u = a.u;
@@ -783,6 +832,9 @@ vmb_status launch_mean(const ScanArgs& a, const ScanPlan& plan, cudaStream_t str
     p.gather_h = a.gather_h;
     p.u_t = a.u_t;
     p.save = a.saved;
+    p.z = lr ? static_cast<const float*>(a.delta) : nullptr;
+    p.Wup = a.Wup;
+    p.R = a.R;
     p.tabvec = al16(a.A) && al16(a.bias) && al16(a.Dskip);
     const WsLayout w = ws_layout(plan);
     unsigned char* ws = static_cast<unsigned char*>(a.ws);

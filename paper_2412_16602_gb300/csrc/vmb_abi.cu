@@ -378,6 +378,43 @@ vmb_status vmb_selective_scan_lowrank_fwd(const void* u, const float* z, const f
     return launch_full(m, mplan, stream);
 }
 
+vmb_status vmb_mean_scan_lowrank_fwd(const void* u, const float* z, const float* Wup, const float* A,
+                                     const void* Bs, const void* Cs, const float* Dskip, const float* delta_bias,
+                                     void* y, float* ybar, int B, int K, int D, int N, int R, int H, int W,
+                                     unsigned flags, vmb_dtype dtype, void* workspace, size_t workspace_bytes,
+                                     cudaStream_t stream) {
+    if (H < 0 || W < 0 || R < 0) return VMB_ERR_INVALID_ARG;
+    if ((long long)H * W > INT_MAX) return VMB_ERR_UNSUPPORTED;
+    ScanArgs a{u, z, A, Bs, Cs, Dskip, delta_bias, y, ybar, B, K, D, N, H * W, flags, dtype, workspace,
+               workspace_bytes};
+    a.Wup = Wup;
+    a.R = R;
+    bool empty = false;
+    vmb_status s = check_scan(a, true, &empty);
+    if (s != VMB_OK || empty) return s;
+    if (R < 1) return VMB_ERR_INVALID_ARG;
+    if (R > 16) return VMB_ERR_UNSUPPORTED;
+    if (!Wup || u == y) return VMB_ERR_INVALID_ARG;
+    if (!aligned(z, 4) || !aligned(Wup, 4)) return VMB_ERR_MISALIGNED;
+    if (!workspace) return VMB_ERR_WORKSPACE;
+    if (!aligned(workspace, 256)) return VMB_ERR_MISALIGNED;
+    ScanPlan plan{};
+    s = plan_mean(a, &plan);
+    if (s != VMB_OK) return s;
+    if (workspace_bytes < plan.ws_bytes) return VMB_ERR_WORKSPACE;
+    if (!(flags & VMB_FLAG_B_ZOH) && R <= 8) return launch_mean(a, plan, stream);
+    // ranks above 8 and the ZOH form: the raw Deltas are written into y and
+    // the scan runs in place (a CTA reads the Deltas of its chunk before it
+    // writes that chunk's y, and no other CTA touches them)
+    ScanArgs m = a;
+    m.delta = y;
+    m.Wup = nullptr;
+    m.R = 0;
+    s = launch_lowrank_expand(z, Wup, y, B, K, D, R, H * W, dtype, stream);
+    if (s != VMB_OK) return s;
+    return launch_mean(m, plan, stream);
+}
+
 vmb_status vmb_ss2d_full_fwd(const void* x, void* xt, const void* delta, const float* A, const void* Bs,
                              const void* Cs, const float* Dskip, const float* delta_bias, void* y, void* out, int B,
                              int D, int N, int H, int W, unsigned flags, vmb_dtype dtype, void* workspace,

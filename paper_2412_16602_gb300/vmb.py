@@ -42,7 +42,7 @@ EXPORTS = ["vmb_cross_scan", "vmb_cross_merge", "vmb_scan_workspace_bytes", "vmb
            "vmb_mean_scan_fwd", "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_ss2d_mean_fwd",
            "vmb_ss2d_full_fwd", "vmb_discretise_fwd", "vmb_discretise_mean_fwd",
            "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_selection_lowrank_fwd", "vmb_selective_scan_lowrank_fwd",
-           "vmb_mean_scan_train_fwd", "vmb_mean_scan_bwd",
+           "vmb_mean_scan_lowrank_fwd", "vmb_mean_scan_train_fwd", "vmb_mean_scan_bwd",
            "vmb_mean_scan_bwd_workspace_bytes",
            "vmb_read_status", "vmb_status_string", "vmb_version"]
 
@@ -76,6 +76,7 @@ def _load() -> ctypes.CDLL:
     lib.vmb_selection_fwd.argtypes = [vp] * 8 + [i] * 7 + [i, vp]
     lib.vmb_selection_lowrank_fwd.argtypes = [vp] * 7 + [i] * 7 + [i, vp]
     lib.vmb_selective_scan_lowrank_fwd.argtypes = [vp] * 9 + [i] * 7 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_lowrank_fwd.argtypes = [vp] * 10 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_train_fwd.argtypes = [vp] * 10 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_bwd.argtypes = [vp] * 16 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_bwd_workspace_bytes.argtypes = [i] * 8
@@ -88,7 +89,7 @@ def _load() -> ctypes.CDLL:
                  "vmb_mean_scan_merge_fwd", "vmb_mean_scan_grouped_fwd", "vmb_ss2d_mean_fwd", "vmb_ss2d_full_fwd",
                  "vmb_discretise_fwd",
                  "vmb_discretise_mean_fwd", "vmb_scan_only_fwd", "vmb_selection_fwd", "vmb_mean_scan_bwd",
-                 "vmb_selection_lowrank_fwd", "vmb_selective_scan_lowrank_fwd",
+                 "vmb_selection_lowrank_fwd", "vmb_selective_scan_lowrank_fwd", "vmb_mean_scan_lowrank_fwd",
                  "vmb_read_status", "vmb_version"]:
         getattr(lib, name).restype = i
     return lib
@@ -607,6 +608,40 @@ def vmb_selective_scan_lowrank_fwd(u, z, Wup, A, Bs, Cs, Dskip, delta_bias, H: i
                                               _dtype_code(u.dtype), _ptr(workspace), workspace.numel(),
                                               _stream(stream)), "vmb_selective_scan_lowrank_fwd")
     return y
+
+
+def vmb_mean_scan_lowrank_fwd(u, z, Wup, A, Bs, Cs, Dskip, delta_bias, H: int, W: int, *, y=None, ybar=None,
+                              want_ybar: bool = False, flags: int = VMB_FLAG_SOFTPLUS, workspace=None, stream=None):
+    """Channel-mean scan whose raw Deltas are Wup z, formed inside the scan: z [B, K, R, H*W]
+    float32, Wup [K, D, R] float32; returns (y [B, K, D, L], ybar [B, K, L] fp32 or None)."""
+    for t, n in [(z, "z"), (Wup, "Wup")]:
+        _dev(t, n)
+    B, K, D, L = u.shape
+    R = z.shape[2]
+    if tuple(z.shape) != (B, K, R, L) or z.dtype != torch.float32:
+        raise ValueError("z must be float32 [B, K, R, H*W]")
+    if tuple(Wup.shape) != (K, D, R) or Wup.dtype != torch.float32:
+        raise ValueError("Wup must be float32 [K, D, R]")
+    B, K, D, N, L = _scan_shapes(u, u, A, Bs, Cs, Dskip, delta_bias, H, W)
+    if y is None:
+        y = torch.empty_like(u)
+    _dev(y, "y")
+    if y.shape != u.shape or y.dtype != u.dtype:
+        raise ValueError("y must match u")
+    if ybar is None and want_ybar:
+        ybar = torch.empty((B, K, L), dtype=torch.float32, device=u.device)
+    if ybar is not None:
+        _dev(ybar, "ybar")
+        if tuple(ybar.shape) != (B, K, L) or ybar.dtype != torch.float32:
+            raise ValueError("ybar must be float32 [B, K, L]")
+    ws_bytes = vmb_scan_workspace_bytes(VMB_PATH_MEAN, B, K, D, N, H, W, u.dtype)
+    if workspace is None:
+        workspace = _default_ws.get(ws_bytes, u.device)
+    _check(lib.vmb_mean_scan_lowrank_fwd(_ptr(u), _ptr(z), _ptr(Wup), _ptr(A), _ptr(Bs), _ptr(Cs), _ptr(Dskip),
+                                         _ptr(delta_bias), _ptr(y), _ptr(ybar),
+                                         B, K, D, N, R, H, W, flags, _dtype_code(u.dtype), _ptr(workspace),
+                                         workspace.numel(), _stream(stream)), "vmb_mean_scan_lowrank_fwd")
+    return y, ybar
 
 
 def vmb_mean_scan_bwd_workspace_bytes(B: int, K: int, D: int, N: int, H: int, W: int, groups: int = 1,

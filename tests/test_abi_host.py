@@ -34,6 +34,7 @@ def lib():
     lib.vmb_selection_fwd.argtypes = [vp] * 8 + [i] * 7 + [i, vp]
     lib.vmb_selection_lowrank_fwd.argtypes = [vp] * 7 + [i] * 7 + [i, vp]
     lib.vmb_selective_scan_lowrank_fwd.argtypes = [vp] * 9 + [i] * 7 + [u, i, vp, sz, vp]
+    lib.vmb_mean_scan_lowrank_fwd.argtypes = [vp] * 10 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_bwd.argtypes = [vp] * 16 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_train_fwd.argtypes = [vp] * 10 + [i] * 7 + [u, i, vp, sz, vp]
     lib.vmb_mean_scan_bwd_workspace_bytes.argtypes = [i] * 8
@@ -235,6 +236,23 @@ def test_selective_scan_lowrank_validation(lib):
     assert scan_lr_call(lib, flags=0x100) == 1
     assert scan_lr_call(lib, ws=0) == 4
     assert scan_lr_call(lib, ptrs=[0] * 9, B=0, ws=0) == 0                     # empty problem
+
+
+def test_mean_scan_lowrank_validation(lib):
+    base = [FAKE, FAKE + 0x1000] + [FAKE] * 6 + [FAKE + 0x2000, 0]
+
+    def call(ptrs=base, R=6, N=16, flags=1, ws=0x100000, B=1):
+        return lib.vmb_mean_scan_lowrank_fwd(*ptrs, B, 4, 8, N, R, 4, 4, flags, 0, ws, 1 << 20, S)
+    assert call(B=-1) == 1
+    assert call(R=0) == 1
+    assert call(R=17) == 3
+    assert call(N=17) == 3
+    assert call(ptrs=base[:2] + [0] + base[3:]) == 1                  # null Wup
+    assert call(ptrs=base[:1] + [FAKE + 0x1002] + base[2:]) == 2      # misaligned z
+    assert call(ptrs=base[:8] + [FAKE, 0]) == 1                       # y aliases u
+    assert call(flags=0x100) == 1
+    assert call(ws=0) == 4
+    assert call(ptrs=[0] * 10, B=0, ws=0) == 0                        # empty problem
 
 
 def disc_call(fn, *, ptrs=None, B=1, K=4, D=8, N=16, H=4, W=4, flags=1, dtype=0):

@@ -1,11 +1,13 @@
 """The Delta branch of Eq. 6 kept low-rank through the scan: the selection
 functions writing the rank-R intermediate z (vmb_selection_lowrank_fwd) and the
-full scan forming the raw Deltas Wup z itself (vmb_selective_scan_lowrank_fwd),
+full and channel-mean scans forming the raw Deltas Wup z themselves
+(vmb_selective_scan_lowrank_fwd, vmb_mean_scan_lowrank_fwd),
 against the fp64 oracle's selection -> scan chain, and in fp32 bit for bit
 against the library's selection -> raw Deltas -> scan.  Forcing the
 warp-specialised tile shape exercises the fused expansion on small problems;
 the planner's own choice there, 5 states and rows that are not 16-byte
-multiples exercise the expand-into-y fallback."""
+multiples exercise the expand-into-y fallback (for the mean scan: ranks above
+8 and the ZOH form)."""
 import numpy as np
 import pytest
 
@@ -76,6 +78,48 @@ def test_lowrank_selection_and_scan(case, forced, force_plan):
         eye[:, r, r] = 1.0
     rz = oracle.selection(un, Ws[0], Ws[1], Ws[2], eye)[0][:, :, :R, :]
     check(to_numpy(z), rz, "f32", "low-rank selection z")
+
+
+MEAN_CASES = [
+    # (B, D, N, R, H, W, dtype, flags)
+    (1, 64, 16, 6, 16, 24, "f32", 0),
+    (2, 40, 16, 1, 9, 11, "f32", 0),     # odd L, rank 1
+    (1, 300, 16, 8, 8, 8, "f32", 0),     # two channel-table groups; the largest rank held in registers
+    (1, 48, 5, 6, 16, 16, "bf16", 0),    # padded states, bf16 storage, fp32 raw Deltas
+    (1, 32, 16, 12, 8, 8, "f32", 0),     # rank 12: raw Deltas into y, scan in place
+    (1, 24, 8, 6, 9, 9, "f32", 1),       # ZOH: raw Deltas into y, scan in place
+    (2, 40, 16, 6, 12, 10, "f32", 2),    # the mean skip term
+]
+
+
+@pytest.mark.parametrize("case", MEAN_CASES, ids=[f"B{c[0]}_D{c[1]}_N{c[2]}_R{c[3]}_{c[4]}x{c[5]}_{c[6]}_f{c[7]}"
+                                                  for c in MEAN_CASES])
+def test_lowrank_mean_scan(case):
+    B, D, N, R, H, W, dt, fl = case
+    flags = vmb.VMB_FLAG_SOFTPLUS | (vmb.VMB_FLAG_B_ZOH if fl == 1 else 0) | (vmb.VMB_FLAG_SKIP_MEAN if fl == 2 else 0)
+    wl = workloads.small_case(B=B, D=D, N=N, H=H, W=W, dtype=dt, seed=1350 + D + R)
+    inp = workloads.make_inputs(wl, params="random")
+    g = to_device(inp, DEV)
+    u = vmb.vmb_cross_scan(g["x"])
+    rng = np.random.default_rng(1351 + D + R)
+    gw = [torch.from_numpy(w).float().to(DEV) for w in _weights(rng, 4, D, N, R)]
+    WB, WC, Wz, Wup = gw
+    z, Bs, Cs = vmb.vmb_selection_lowrank_fwd(u, WB, WC, Wz, H, W)
+    y, yb = vmb.vmb_mean_scan_lowrank_fwd(u, z, Wup, g["A"], Bs, Cs, g["Dskip"], g["bias"], H, W, want_ybar=True,
+                                          flags=flags)
+    dr, _, _ = vmb.vmb_selection_fwd(u, WB, WC, Wz, Wup, H, W)
+    y_u, yb_u = vmb.vmb_mean_scan_fwd(u, dr, g["A"], Bs, Cs, g["Dskip"], g["bias"], H, W, want_ybar=True,
+                                      flags=flags)
+    assert vmb.vmb_read_status() == vmb.VMB_OK
+    if dt == "f32":
+        assert torch.equal(y, y_u) and torch.equal(yb, yb_u), "fp32: bit-identical to raw Deltas -> mean scan"
+    un = to_numpy(u).astype(np.float64)
+    Ws = [w.double().cpu().numpy() for w in gw]
+    rdr, rB, rC = oracle.selection(un, *Ws)
+    y_ref, yb_ref = oracle.mean_scan(un, rdr, inp.A, rB, rC, inp.Dskip, inp.bias, b_mode=1 if fl == 1 else 0,
+                                     skip_mode=oracle.SKIP_MEAN if fl == 2 else oracle.SKIP_PER_CHANNEL)
+    check(to_numpy(y), y_ref, dt, "low-rank mean y")
+    check(to_numpy(yb), yb_ref, "f32" if dt == "f32" else "bf16", "low-rank mean ybar")
 
 
 def test_lowrank_scan_at_the_benchmark_size():
