@@ -34,11 +34,13 @@
  *   - Outputs must not alias inputs.
  *   - Calls are thread-safe.  Scan calls that share one workspace must not
  *     overlap in time (order them on one stream).
- *   - Every kernel is launched with programmatic stream serialization
- *     (programmatic dependent launch): its blocks may be scheduled while the
- *     previous kernel of the stream is finishing, and each waits
+ *   - Kernels are launched with programmatic stream serialization
+ *     (programmatic dependent launch): their blocks may be scheduled while
+ *     the previous kernel of the stream is finishing, and each waits
  *     (griddepcontrol.wait) for that kernel to complete before it reads or
- *     writes global memory.  Stream order is therefore kept for any
+ *     writes global memory.  (The exception: a warp-specialised full scan
+ *     whose grid is smaller than one wave is launched normally, so that its
+ *     blocks spread over every SM.)  Stream order is therefore kept for any
  *     preceding work; a caller's own kernel launched after a vmb call with
  *     the same attribute must likewise wait before touching vmb outputs.
  */
