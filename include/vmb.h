@@ -78,7 +78,10 @@ typedef enum { VMB_F32 = 0, VMB_BF16 = 1 } vmb_dtype;
 /* Test hook, never set in production: the first L-chunk of every sequence of
  * a multi-chunk scan does not publish its state, so that the look-back waits
  * of its successors run out (bounded, about 0.2 s) and the call reports
- * VMB_ERR_TIMEOUT through vmb_read_status.  No effect on single-chunk plans. */
+ * VMB_ERR_TIMEOUT through vmb_read_status; in the warp-specialised full scan
+ * the first stage of every tile is never handed to the compute warps, so
+ * their waits and then the copy warp's run out (bounded, about 1 s each) and
+ * the call reports VMB_ERR_TIMEOUT.  No effect on other single-chunk plans. */
 #define VMB_FLAG_TEST_SUPPRESS_PUBLISH 0x40000000u
 
 /* Scan path selector for vmb_scan_workspace_bytes. */

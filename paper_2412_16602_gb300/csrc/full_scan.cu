@@ -1545,7 +1545,9 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
         const CUtensorMap* um = (gather && (k & 1)) ? &tm.u2 : &tm.u;
         const int uz = gather ? bk / p.K : bk;
         const bool urev = gather && k >= 2;
+        int issued = 0;  // stages whose copies have been issued (0 .. issued-1)
         auto issue = [&](int s) {
+            issued = s + 1;
             const int slot = s % NSTG;
             const uint32_t dst = sbase + (uint32_t)(slot * LY::RAW_STAGE);
             mbarrier_expect_tx(landed(slot), (unsigned)LY::RAW_STAGE);
@@ -1556,11 +1558,14 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
         };
         if (lane == 0)
             for (int s = 0; s < NSTG && s < nst; ++s) issue(s);
+        issued = __shfl_sync(0xffffffffu, issued, 0);
         int seen = 0;  // stages whose copies this warp has seen land
         bool ok = true;
+        // (every wait's outcome is made warp-uniform, so that no lane leaves a
+        // loop whose warp-wide operations the others still execute)
         for (int s = 0; s < nst; ++s) {
             const int slot = s % NSTG;
-            if (!(ok = mbarrier_wait(landed(slot), (s / NSTG) & 1, kStageWaitNs))) break;
+            if (!(ok = __all_sync(0xffffffffu, mbarrier_wait(landed(slot), (s / NSTG) & 1, kStageWaitNs)))) break;
             seen = s + 1;
             // lane r converts row r of [B rows 0..15, C rows 0..15] into column r
             const T* rb = reinterpret_cast<const T*>(smem + slot * LY::RAW_STAGE + LY::B_OFF) + lane * TS;
@@ -1568,18 +1573,20 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
 #pragma unroll
             for (int t = 0; t < TS; ++t) bo[t * 2 * NP + lane] = io<T>::cvt(rb[t]);
             __syncwarp();
-            mbarrier_arrive(ready(slot));
+            // (test hook: the first stage is never handed over, so every wait on it runs out)
+            if (!(p.suppress && s == 0)) mbarrier_arrive(ready(slot));
             // refill the slot of stage s - 1 once the consumers released it
             if (s >= 1 && s - 1 + NSTG < nst) {
                 const int ps = (s - 1) % NSTG;
-                if (!(ok = mbarrier_wait(released(ps), ((s - 1) / NSTG) & 1, kStageWaitNs))) break;
+                if (!(ok = __all_sync(0xffffffffu, mbarrier_wait(released(ps), ((s - 1) / NSTG) & 1, kStageWaitNs))))
+                    break;
                 if (lane == 0) issue(s - 1 + NSTG);
+                issued = __shfl_sync(0xffffffffu, issued, 0);
             }
         }
         if (!ok) {
             if (lane == 0) atomicOr(&p.hdr->err, kErrTimeout);
             // every copy issued must land before the CTA exits
-            const int issued = min(nst, seen + NSTG);
             for (int s = seen; s < issued; ++s) mbarrier_wait(landed(s % NSTG), (s / NSTG) & 1, kStageWaitNs);
         }
         return;
@@ -1612,8 +1619,8 @@ __global__ void __launch_bounds__(WsTileLayout<T, WS>::THREADS, WS::MINB)
     }
     for (int s = 0; s < nst; ++s) {
         const int slot = s % NSTG;
-        if (!mbarrier_wait(ready(slot), (s / NSTG) & 1, kStageWaitNs)) {
-            atomicOr(&p.hdr->err, kErrTimeout);
+        if (!__all_sync(0xffffffffu, mbarrier_wait(ready(slot), (s / NSTG) & 1, kStageWaitNs))) {
+            if (lane == 0) atomicOr(&p.hdr->err, kErrTimeout);
             return;
         }
         const int l0 = s * TS;

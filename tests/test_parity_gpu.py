@@ -194,6 +194,27 @@ def test_every_tile_shape(plan, dt, force_plan):
     check(to_numpy(y), ref, dt, f"full y plan {plan}")
 
 
+def test_warp_specialised_stage_wait_times_out_cleanly(force_plan):
+    """The warp-specialised full scan with the first stage never handed over
+    (test hook): the compute warps' bounded waits and then the copy warp's run
+    out, the call reports VMB_ERR_TIMEOUT, the status clears, and the same
+    workspace then gives correct results."""
+    force_plan.full("19")
+    wl = workloads.small_case(B=1, D=64, N=16, H=16, W=16, seed=88)
+    inp = workloads.make_inputs(wl, params="random")
+    g = to_device(inp, DEV)
+    xs = vmb.vmb_cross_scan(g["x"])
+    ws = torch.zeros(vmb.vmb_scan_workspace_bytes(0, 1, 4, 64, 16, 16, 16), dtype=torch.uint8, device=DEV)
+    args = (xs, g["draw"], g["A"], g["Bs"], g["Cs"], g["Dskip"], g["bias"], 16, 16)
+    vmb.vmb_selective_scan_fwd(*args, flags=vmb.VMB_FLAG_SOFTPLUS | vmb.VMB_FLAG_TEST_SUPPRESS_PUBLISH, workspace=ws)
+    assert vmb.vmb_read_status(ws) == vmb.VMB_ERR_TIMEOUT
+    assert vmb.vmb_read_status(ws) == vmb.VMB_OK  # cleared
+    y = vmb.vmb_selective_scan_fwd(*args, workspace=ws)
+    assert vmb.vmb_read_status(ws) == vmb.VMB_OK
+    _, ref, _ = oracle.ss2d_full(inp)
+    check(to_numpy(y), ref, "f32", "after the stage wait ran out")
+
+
 WS_CASES = [
     # (B, D, N, H, W, dtype)
     (1, 256, 16, 9, 12, "f32"),   # L = 108: the last 8-step stage half full; two full channel tiles
