@@ -7,7 +7,8 @@
 // aligned; the padding keeps the column-major reads free of bank conflicts.
 //
 // Maps of 1024 pixels or more use band kernels instead: one CTA per band of
-// eight rows of one map (see below), which keeps batch-1 problems parallel.
+// rows of one map (eight for the scan, up to 32 for the merge; see below),
+// which keeps batch-1 problems parallel.
 //
 // cross-merge: ys[B,4,D,L] -> out[B,D,H,W], out = (ys0[p0] + ys2[p2]) +
 // (ys1[p1] + ys3[p3]) in fp32 in that order.  Directions 0 and 2 are read
@@ -211,10 +212,14 @@ __global__ void __launch_bounds__(kThreads) cross_merge_kernel(const CsmParams p
 }
 
 // ---------------------------------------------------------------- band kernels
-// Maps of at least kBandMinL pixels: one CTA per band of kRB rows of one map, so
+// Maps of at least kBandMinL pixels: one CTA per band of rows of one map, so
 // that even a batch-1 problem has enough CTAs.  Directions 0 and 2 of a band are
-// one contiguous run of the sequence; directions 1 and 3 are W runs of kRB
-// steps, written from a [kRB][W+1] shared tile.
+// one contiguous run of the sequence; directions 1 and 3 are W runs of one step
+// per row of the band, written from (scan) or read into (merge) a [rows][W+1]
+// shared tile.  The scan takes bands of kRB rows; the merge takes taller bands
+// (mrb rows, chosen on the host), whose runs of directions 1 and 3 are longer
+// reads (measured on GB300: 32-row fp32 bands 305 us against 337 us for 8 rows
+// on the batch-128 56x56 map; 16 rows best for bf16).
 constexpr int kRB = 8;
 constexpr int kBandMinL = 1024;
 constexpr int kBandThreads = 128;
@@ -225,6 +230,7 @@ struct BandParams {
     int D, H, W, L;
     int nbands;  // bands per map
     int vec;     // W and H multiples of the vector width, 16-byte aligned bases
+    int mrb;     // merge: rows per band (a multiple of 8)
 };
 
 template <typename T>
@@ -302,13 +308,13 @@ __global__ void __launch_bounds__(kBandThreads) cross_merge_band_kernel(const Ba
     pdl_launch_dependents();
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const int W = p.W, H = p.H, L = p.L, WP = p.W + 1;
-    T* s1 = reinterpret_cast<T*>(smem_raw);  // [kRB][W+1]: ys1 at pixel (h0 + j, w)
-    T* s3 = s1 + kRB * WP;                     // [kRB][W+1]: ys3 at pixel (h0 + j, w)
+    T* s1 = reinterpret_cast<T*>(smem_raw);  // [mrb][W+1]: ys1 at pixel (h0 + j, w)
+    T* s3 = s1 + p.mrb * WP;                   // [mrb][W+1]: ys3 at pixel (h0 + j, w)
     constexpr int VE = 16 / sizeof(T);
     const long long plane = blockIdx.x / p.nbands;
     const int band = blockIdx.x % p.nbands;
-    const int h0 = band * kRB;
-    const int rb = min(kRB, H - h0);
+    const int h0 = band * p.mrb;
+    const int rb = min(p.mrb, H - h0);
     const int n = rb * W;
     const long long b = plane / p.D, d = plane % p.D;
     const T* ys = static_cast<const T*>(p.in);
@@ -318,8 +324,8 @@ __global__ void __launch_bounds__(kBandThreads) cross_merge_band_kernel(const Ba
     const T* row3 = ys + ((b * 4 + 3) * p.D + d) * L;
     T* out = static_cast<T*>(p.out) + plane * L + (long long)h0 * W;
     // stage directions 1 and 3 of the band's pixels
-    if (p.vec && rb == kRB) {
-        constexpr int RV = kRB / VE;
+    if (p.vec && rb % VE == 0) {
+        const int RV = rb / VE;  // vectors per run
         for (int i = threadIdx.x; i < W * RV; i += kBandThreads) {
             const int w = i / RV, jv = (i - w * RV) * VE;
             const long long pos = (long long)w * H + h0 + jv;
@@ -426,11 +432,16 @@ vmb_status launch_csm(bool merge, const void* in, void* outp, int B, int D, int 
         bp.H = H;
         bp.W = W;
         bp.L = L;
-        bp.nbands = (H + kRB - 1) / kRB;
+        // merge bands: 32 rows (fp32) or 16 (bf16), fewer while the tiles would
+        // not fit
+        int mrb = es == 4 ? 32 : 16;
+        while (mrb > kRB && (size_t)2 * mrb * (W + 1) * es > kMaxSmem) mrb /= 2;
+        bp.mrb = mrb;
+        bp.nbands = merge ? (H + mrb - 1) / mrb : (H + kRB - 1) / kRB;
         const int VE = (int)(16 / es);
         const auto a16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
         bp.vec = (W % VE == 0) && (H % VE == 0) && a16(in) && a16(outp);
-        const size_t smem = (merge ? 2 : 1) * (size_t)kRB * (W + 1) * es;
+        const size_t smem = merge ? 2 * (size_t)mrb * (W + 1) * es : (size_t)kRB * (W + 1) * es;
         const void* fn = merge ? reinterpret_cast<const void*>(&cross_merge_band_kernel<T>)
                                : reinterpret_cast<const void*>(&cross_scan_band_kernel<T>);
         if (smem > 48 * 1024 &&

@@ -93,12 +93,19 @@ def test_skip_mean_mode():
 
 
 def test_merge_exact_on_integers():
-    """With integer-valued inputs every partial sum is exact: the merge is bit-exact."""
+    """With integer-valued inputs every partial sum is exact: the merge is bit-exact.
+    Maps of 1024 pixels or more take the band kernel (32-row fp32 bands, 16-row
+    bf16 bands): 72 and 40 rows end in a short band on the vector path, 37 x 29
+    on the element path."""
     rng = np.random.default_rng(9)
-    for (B, D, H, W) in [(2, 3, 5, 7), (1, 4, 8, 8), (3, 2, 1, 9)]:
-        ys = rng.integers(-1000, 1000, size=(B, 4, D, H * W)).astype(np.float32)
-        got = vmb.vmb_cross_merge(torch.from_numpy(ys).to(DEV), H, W).cpu().numpy()
-        assert np.array_equal(got.astype(np.float64), oracle.cross_merge(ys, H, W))
+    for (B, D, H, W, dt) in [(2, 3, 5, 7, "f32"), (1, 4, 8, 8, "f32"), (3, 2, 1, 9, "f32"), (1, 3, 72, 40, "f32"),
+                             (1, 2, 37, 29, "f32"), (2, 2, 40, 48, "bf16"), (1, 2, 56, 56, "f32")]:
+        ys = rng.integers(-30, 31, size=(B, 4, D, H * W)).astype(np.float32)
+        t = torch.from_numpy(ys).to(DEV)
+        if dt == "bf16":
+            t = t.to(torch.bfloat16)  # |sums| <= 120: exact in bf16
+        got = vmb.vmb_cross_merge(t, H, W).float().cpu().numpy()
+        assert np.array_equal(got.astype(np.float64), oracle.cross_merge(ys, H, W)), (H, W, dt)
 
 
 def test_misaligned_views_take_element_path():
