@@ -74,3 +74,18 @@ def test_bf16_workloads_hold_bf16_values():
 def test_rejects_unknown_parameter_recipe():
     with pytest.raises(ValueError):
         workloads.make_inputs(_small(), params="nope")
+
+
+def test_algorithmic_bytes_of_the_benchmark_workload():
+    """The per-call byte counts the roofline divides by, against the sizes of
+    the scan's operands written out: a scan call reads u, the raw Deltas, B
+    and C and writes y (plus the per-channel parameters); a cross-scan or
+    cross-merge call moves one map and its four direction rows."""
+    wl = workloads.WORKLOADS["batch128_d256_n16_56x56_sigma0.05_f32"]
+    B, K, D, N, L, s = 128, 4, 256, 16, 56 * 56, 4
+    params = K * D * (N + 2) * 4  # A, Dskip, delta bias in fp32
+    assert wl.scan_bytes() == s * (3 * B * K * D * L + 2 * B * K * N * L) + params
+    assert abs(wl.scan_bytes() / 1e9 - 5.138) < 1e-3
+    assert wl.csm_bytes() == 5 * s * B * D * L
+    assert abs(wl.csm_bytes() / 1e9 - 2.055) < 1e-3
+    assert wl.scan_elements() == B * K * D * L
